@@ -1,0 +1,311 @@
+/*
+ * nld_oracle.c -- plain, slow, fp64 CPU oracle for block attention over a
+ * paged KV cache and for the two token-decision rules of tri-mode decoding.
+ *
+ * TEST INFRASTRUCTURE ONLY. Nothing in the product path may call, link or
+ * load this file; only the tests, the smoke check and the bench's CPU
+ * baseline do. It shares no code, header or table with the CUDA library.
+ *
+ * What it computes, by definition (each function cites its passage):
+ *
+ *  - Block attention (Sec. 2.2 attention pattern; Sec. 3 Mode 2 and Mode 3).
+ *    A block of bl query tokens sits after a cached prefix of L_b tokens.
+ *    Key t is visible to block row i when t < L_b (the clean prefix is fully
+ *    visible), or t = L_b + j with j in J(i): J(i) = {0..bl-1} in the
+ *    diffusion-draft pass (bidirectional inside the block) and {0..i} in the
+ *    AR-verify pass (causal inside the block). Query head h reads KV head
+ *    floor(h / G), G = Hq / Hkv. Logical key t lives in physical page
+ *    page_table[b][t / P] at slot t mod P.
+ *      s_t = scale * <q, k_t>,  m = max s_t,  w_t = exp(s_t - m),
+ *      l = sum w_t,  o = sum w_t v_t / l,  lse = m + ln l.
+ *  - Split-KV combine: partial results over disjoint key ranges merge as
+ *      m* = max_s lse_s, c_s = exp(lse_s - m*), o = sum c_s o_s / sum c_s,
+ *      lse = m* + ln sum c_s.
+ *  - Acceptance (Sec. 3 Mode 3, linear self-speculation): the longest prefix
+ *    of draft tokens equal to the verifier's predictions is accepted; the
+ *    accepted length is the first mismatch index j*, or n if none.
+ *  - Confidence-ranked unmasking (Sec. 3 Mode 2; Sec. 4 serial denoising
+ *    commits the highest-confidence position): the k eligible positions with
+ *    the largest confidence, ordered by (confidence descending, position
+ *    ascending). -inf and NaN mark ineligible positions.
+ *
+ * Build: gcc -O2 -fopenmp -ffp-contract=off -shared -fPIC (see build.py).
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+#define NLDO_OK 0
+#define NLDO_ERR_ARGS -1
+#define NLDO_ERR_PAGE -2
+#define NLDO_ERR_NOMEM -3
+
+/* Exact widening of a bf16 bit pattern: the 16 bits are the top half of an
+ * IEEE binary32, which converts to binary64 exactly. */
+static double bf16_to_f64(uint16_t bits)
+{
+    uint32_t u = ((uint32_t)bits) << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+/* Mask of Sec. 2.2 / Sec. 3 for block row i (0-based) and logical key t. */
+static int key_visible(long t, long L, int bl, int i, int mode)
+{
+    if (t < L) return 1;             /* clean prefix: always visible */
+    long j = t - L;                  /* block slot of key t */
+    if (j >= bl) return 0;           /* slots past the block hold nothing */
+    if (mode == 0) return 1;         /* diffusion draft: bidirectional */
+    return j <= i;                   /* AR verify: causal, self included */
+}
+
+int nldo_max_threads(void)
+{
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+/*
+ * One query row (b, i, h). Keys are restricted to the logical range
+ * [key_begin, key_end) in addition to the mask (key_end < 0: no limit).
+ * Writes o[D], *lse, and, when probs != NULL, probs[t] for t < L_b + bl
+ * (0 for keys that are not used). A row with no usable key gets o = 0 and
+ * lse = -inf.
+ */
+static int attn_row(const uint16_t *q, const uint16_t *k, const uint16_t *v,
+                    const int32_t *page_table, long L, int b, int i, int h,
+                    int Hq, int Hkv, int D, int P, int num_pages, int max_pages,
+                    int bl, int mode, double scale, long key_begin, long key_end,
+                    double *s, char *use, double *o, double *lse, double *probs)
+{
+    const int G = Hq / Hkv;
+    const int g = h / G;
+    const long N = L + bl;
+    const uint16_t *qrow = q + (((long)b * bl + i) * Hq + h) * (long)D;
+    double m = -INFINITY;
+    long nuse = 0;
+
+    for (long t = 0; t < N; ++t) {
+        use[t] = key_visible(t, L, bl, i, mode) && t >= key_begin && (key_end < 0 || t < key_end);
+        if (!use[t]) continue;
+        long lp = t / P;
+        if (lp >= max_pages) return NLDO_ERR_PAGE;
+        int page = page_table[(long)b * max_pages + lp];
+        if (page < 0 || page >= num_pages) return NLDO_ERR_PAGE;
+        const uint16_t *krow = k + (((long)page * Hkv + g) * P + (t % P)) * (long)D;
+        double dot = 0.0;
+        for (int d = 0; d < D; ++d) dot += bf16_to_f64(qrow[d]) * bf16_to_f64(krow[d]);
+        s[t] = scale * dot;
+        if (s[t] > m) m = s[t];
+        ++nuse;
+    }
+    for (int d = 0; d < D; ++d) o[d] = 0.0;
+    if (nuse == 0) {
+        *lse = -INFINITY;
+        if (probs) for (long t = 0; t < N; ++t) probs[t] = 0.0;
+        return NLDO_OK;
+    }
+    double l = 0.0;
+    for (long t = 0; t < N; ++t) {
+        if (!use[t]) continue;
+        double w = exp(s[t] - m);
+        l += w;
+        int page = page_table[(long)b * max_pages + t / P];
+        const uint16_t *vrow = v + (((long)page * Hkv + g) * P + (t % P)) * (long)D;
+        for (int d = 0; d < D; ++d) o[d] += w * bf16_to_f64(vrow[d]);
+    }
+    for (int d = 0; d < D; ++d) o[d] /= l;
+    *lse = m + log(l);
+    if (probs)
+        for (long t = 0; t < N; ++t) probs[t] = use[t] ? exp(s[t] - m) / l : 0.0;
+    return NLDO_OK;
+}
+
+static int check_shape(int B, int Hq, int Hkv, int D, int P, int bl, int mode)
+{
+    if (B < 0 || Hq <= 0 || Hkv <= 0 || D <= 0 || P <= 0 || bl <= 0) return 0;
+    if (Hq % Hkv != 0) return 0;
+    if (mode != 0 && mode != 1) return 0;
+    return 1;
+}
+
+/*
+ * Block attention for every row. q [B, bl, Hq, D]; k, v [num_pages, Hkv, P, D]
+ * (bf16 bits); page_table [B, max_pages]; prefix_lens [B].
+ * out [B, bl, Hq, D], lse [B, Hq, bl] (fp64). probs: NULL, or
+ * [B, Hq, bl, probs_stride] with probs_stride >= max_b (L_b + bl).
+ */
+int nldo_block_attn(const uint16_t *q, const uint16_t *k, const uint16_t *v,
+                    const int32_t *page_table, const int32_t *prefix_lens,
+                    int B, int Hq, int Hkv, int D, int P, int num_pages, int max_pages,
+                    int bl, int mode, double scale, long key_begin, long key_end,
+                    double *out, double *lse, double *probs, long probs_stride)
+{
+    if (!check_shape(B, Hq, Hkv, D, P, bl, mode)) return NLDO_ERR_ARGS;
+    long maxN = 0;
+    for (int b = 0; b < B; ++b) {
+        if (prefix_lens[b] < 0) return NLDO_ERR_ARGS;
+        if ((long)prefix_lens[b] + bl > maxN) maxN = (long)prefix_lens[b] + bl;
+    }
+    if (probs && probs_stride < maxN) return NLDO_ERR_ARGS;
+    int status = NLDO_OK;
+    long nrows = (long)B * Hq;
+#pragma omp parallel
+    {
+        double *s = (double *)malloc(sizeof(double) * (maxN > 0 ? maxN : 1));
+        char *use = (char *)malloc(maxN > 0 ? maxN : 1);
+        double *o = (double *)malloc(sizeof(double) * D);
+        if (!s || !use || !o) {
+#pragma omp atomic write
+            status = NLDO_ERR_NOMEM;
+        } else {
+#pragma omp for schedule(dynamic, 1)
+            for (long bh = 0; bh < nrows; ++bh) {
+                int b = (int)(bh / Hq), h = (int)(bh % Hq);
+                for (int i = 0; i < bl; ++i) {
+                    double l_out;
+                    double *p = probs ? probs + ((bh * bl) + i) * probs_stride : NULL;
+                    int rc = attn_row(q, k, v, page_table, prefix_lens[b], b, i, h, Hq, Hkv, D, P,
+                                      num_pages, max_pages, bl, mode, scale, key_begin, key_end,
+                                      s, use, o, &l_out, p);
+                    if (rc != NLDO_OK) {
+#pragma omp atomic write
+                        status = rc;
+                        continue;
+                    }
+                    double *orow = out + (((long)b * bl + i) * Hq + h) * (long)D;
+                    for (int d = 0; d < D; ++d) orow[d] = o[d];
+                    lse[((long)b * Hq + h) * bl + i] = l_out;
+                }
+            }
+        }
+        free(s); free(use); free(o);
+    }
+    return status;
+}
+
+/*
+ * Block attention for selected rows only: rows[r] = (b, i, h) triples.
+ * out [nrows, D], lse [nrows].
+ */
+int nldo_block_attn_rows(const uint16_t *q, const uint16_t *k, const uint16_t *v,
+                         const int32_t *page_table, const int32_t *prefix_lens,
+                         int B, int Hq, int Hkv, int D, int P, int num_pages, int max_pages,
+                         int bl, int mode, double scale, long nsel, const int32_t *rows,
+                         double *out, double *lse)
+{
+    if (!check_shape(B, Hq, Hkv, D, P, bl, mode)) return NLDO_ERR_ARGS;
+    long maxN = 0;
+    for (int b = 0; b < B; ++b)
+        if ((long)prefix_lens[b] + bl > maxN) maxN = (long)prefix_lens[b] + bl;
+    int status = NLDO_OK;
+#pragma omp parallel
+    {
+        double *s = (double *)malloc(sizeof(double) * (maxN > 0 ? maxN : 1));
+        char *use = (char *)malloc(maxN > 0 ? maxN : 1);
+        if (!s || !use) {
+#pragma omp atomic write
+            status = NLDO_ERR_NOMEM;
+        } else {
+#pragma omp for schedule(dynamic, 1)
+            for (long r = 0; r < nsel; ++r) {
+                int b = rows[3 * r], i = rows[3 * r + 1], h = rows[3 * r + 2];
+                if (b < 0 || b >= B || i < 0 || i >= bl || h < 0 || h >= Hq) {
+#pragma omp atomic write
+                    status = NLDO_ERR_ARGS;
+                    continue;
+                }
+                int rc = attn_row(q, k, v, page_table, prefix_lens[b], b, i, h, Hq, Hkv, D, P,
+                                  num_pages, max_pages, bl, mode, scale, 0, -1,
+                                  s, use, out + r * (long)D, lse + r, NULL);
+                if (rc != NLDO_OK) {
+#pragma omp atomic write
+                    status = rc;
+                }
+            }
+        }
+        free(s); free(use);
+    }
+    return status;
+}
+
+/*
+ * Split-KV combine. o_part [S, R, D], lse_part [S, R] -> out [R, D], lse [R].
+ * Partials with lse = -inf carry no keys and get weight 0.
+ */
+void nldo_combine(const double *o_part, const double *lse_part, int S, long R, int D,
+                  double *out, double *lse)
+{
+    for (long r = 0; r < R; ++r) {
+        double m = -INFINITY;
+        for (int s = 0; s < S; ++s)
+            if (lse_part[(long)s * R + r] > m) m = lse_part[(long)s * R + r];
+        double *orow = out + r * (long)D;
+        for (int d = 0; d < D; ++d) orow[d] = 0.0;
+        if (m == -INFINITY) { lse[r] = -INFINITY; continue; }
+        double csum = 0.0;
+        for (int s = 0; s < S; ++s) {
+            double ls = lse_part[(long)s * R + r];
+            if (ls == -INFINITY) continue;
+            double c = exp(ls - m);
+            csum += c;
+            const double *op = o_part + ((long)s * R + r) * D;
+            for (int d = 0; d < D; ++d) orow[d] += c * op[d];
+        }
+        for (int d = 0; d < D; ++d) orow[d] /= csum;
+        lse[r] = m + log(csum);
+    }
+}
+
+/* Longest accepted prefix: first j with draft[j] != verify[j], else n. */
+void nldo_accept(const int32_t *draft, const int32_t *verify, int B, int n, int32_t *accepted)
+{
+    for (int b = 0; b < B; ++b) {
+        int j = 0;
+        while (j < n && draft[(long)b * n + j] == verify[(long)b * n + j]) ++j;
+        accepted[b] = j;
+    }
+}
+
+/* a ranks before b: larger confidence first; equal confidence -> lower index. */
+static int ranks_before(float ca, int a, float cb, int b)
+{
+    if (ca > cb) return 1;
+    if (ca < cb) return 0;
+    return a < b;
+}
+
+/*
+ * Top-k unmasking by confidence. conf [B, n] fp32. positions [B, k] in rank
+ * order, -1 past the eligible count; num_selected [B] (nullable).
+ * Eligible: not NaN and not -inf. Comparisons are made on the fp32 values
+ * (+0 and -0 compare equal, so they tie and the lower index wins).
+ */
+void nldo_unmask(const float *conf, int B, int n, int k, int32_t *positions, int32_t *num_selected)
+{
+    int *idx = (int *)malloc(sizeof(int) * (n > 0 ? n : 1));
+    for (int b = 0; b < B; ++b) {
+        const float *c = conf + (long)b * n;
+        int m = 0;
+        for (int i = 0; i < n; ++i)
+            if (!isnan(c[i]) && !(isinf(c[i]) && c[i] < 0)) idx[m++] = i;
+        /* insertion sort: stable and obviously correct */
+        for (int a = 1; a < m; ++a) {
+            int x = idx[a], j = a - 1;
+            while (j >= 0 && ranks_before(c[x], x, c[idx[j]], idx[j])) { idx[j + 1] = idx[j]; --j; }
+            idx[j + 1] = x;
+        }
+        int sel = m < k ? m : k;
+        for (int r = 0; r < k; ++r) positions[(long)b * k + r] = r < sel ? idx[r] : -1;
+        if (num_selected) num_selected[b] = sel;
+    }
+    free(idx);
+}

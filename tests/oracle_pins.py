@@ -1,0 +1,419 @@
+"""Pins for the fp64 oracle: checks against things other than the oracle itself.
+
+Each ``pin_*`` takes an oracle handle and raises AssertionError on a mismatch.
+They are run on the real oracle (tests/test_oracle_pins.py) and on copies of
+the oracle with a planted mistake (tests/test_oracle_mutations.py), which
+must each fail at least one pin.
+
+What pins what:
+  - torch's scaled_dot_product_attention (fp64, CPU): bl = 1 decode, the
+    diffusion pass as full attention over prefix + block, the verify pass as
+    the last rows of causal attention, GQA as MHA with repeated KV heads.
+  - scipy.special.logsumexp: the lse output.
+  - Hand-derived golden values (tests/golden/attn_uniform_q0.txt).
+  - Closed forms: constant V, identical keys, one visible key.
+  - Invariants: softmax rows sum to 1, page permutation, block permutation.
+  - Split / combine against the unsplit result.
+  - Brute force and hand-written cases for accept and unmask.
+"""
+from __future__ import annotations
+
+import math
+import os
+
+import numpy as np
+import scipy.special
+import torch
+
+from paper_2607_05722_gb300 import workloads as W
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+DIFF, VER = W.MODE_DIFFUSION, W.MODE_VERIFY
+
+
+# --------------------------------------------------------------------------
+# helpers (independent of the oracle)
+# --------------------------------------------------------------------------
+
+def small_case(seed, B=2, Hq=4, Hkv=2, D=16, P=4, bl=5, prefix=(7, 12), shuffle=True):
+    return W.make_block_attn_case("pin", B, Hq, Hkv, D, bl, P, list(prefix), seed, shuffle_pages=shuffle)
+
+
+def gather_contiguous(case, b):
+    """K, V of sequence b as fp64 [Hkv, L+bl, D], read through the page table
+    with numpy indexing."""
+    kv = case.kv
+    N = int(kv.prefix_lens[b]) + case.block_len
+    t = np.arange(N)
+    pages = kv.page_table[b, t // kv.page_size]
+    slots = t % kv.page_size
+    k = W.bf16_bits_to_f32(kv.k_bits[pages, :, slots, :]).astype(np.float64)  # [N, Hkv, D]
+    v = W.bf16_bits_to_f32(kv.v_bits[pages, :, slots, :]).astype(np.float64)
+    return np.transpose(k, (1, 0, 2)), np.transpose(v, (1, 0, 2))
+
+
+def q_f64(bits):
+    return W.bf16_bits_to_f32(bits).astype(np.float64)
+
+
+def sdpa(q, k, v, scale, causal=False):
+    """torch SDPA in fp64 on CPU. q [H, M, D], k/v [H, N, D]."""
+    out = torch.nn.functional.scaled_dot_product_attention(
+        torch.from_numpy(q)[None], torch.from_numpy(k)[None], torch.from_numpy(v)[None],
+        is_causal=causal, scale=scale)
+    return out[0].numpy()
+
+
+def repeat_heads(x, G):
+    return np.repeat(x, G, axis=0)
+
+
+def assert_close(a, b, tol, what):
+    err = float(np.max(np.abs(np.asarray(a) - np.asarray(b)))) if np.size(a) else 0.0
+    assert err <= tol, f"{what}: max abs err {err:.3e} > {tol:.1e}"
+
+
+# --------------------------------------------------------------------------
+# attention pins
+# --------------------------------------------------------------------------
+
+def pin_decode_bl1(orc):
+    """bl = 1: both modes are single-token decode attention over L + 1 keys."""
+    case = small_case(11, bl=1, prefix=(6, 13))
+    G = case.num_q_heads // case.num_kv_heads
+    for mode in (DIFF, VER):
+        out, lse = orc.block_attn(case.q_draft_bits, case.kv.k_bits, case.kv.v_bits, case.kv.page_table,
+                                  case.kv.prefix_lens, case.num_q_heads, case.num_kv_heads, 1, mode, case.scale)
+        for b in range(case.batch):
+            k, v = gather_contiguous(case, b)
+            q = np.transpose(q_f64(case.q_draft_bits[b]), (1, 0, 2))  # [Hq, 1, D]
+            ref = sdpa(q, repeat_heads(k, G), repeat_heads(v, G), case.scale)
+            assert_close(np.transpose(out[b], (1, 0, 2)), ref, 1e-12, f"decode mode={mode}")
+
+
+def pin_diffusion_full_attention(orc):
+    """Diffusion pass = unmasked attention over prefix + block (L = 0 included)."""
+    for prefix, seed in (((0, 0), 3), ((9, 0), 4), ((7, 12), 5)):
+        case = small_case(seed, prefix=prefix)
+        G = case.num_q_heads // case.num_kv_heads
+        out, _ = orc.block_attn(case.q_draft_bits, case.kv.k_bits, case.kv.v_bits, case.kv.page_table,
+                                case.kv.prefix_lens, case.num_q_heads, case.num_kv_heads, case.block_len,
+                                DIFF, case.scale)
+        for b in range(case.batch):
+            k, v = gather_contiguous(case, b)
+            q = np.transpose(q_f64(case.q_draft_bits[b]), (1, 0, 2))
+            ref = sdpa(q, repeat_heads(k, G), repeat_heads(v, G), case.scale)
+            assert_close(np.transpose(out[b], (1, 0, 2)), ref, 1e-12, f"diffusion prefix={prefix}")
+
+
+def pin_verify_causal_tail(orc):
+    """Verify pass = the last bl rows of causal attention over the L + bl sequence."""
+    rng = np.random.default_rng(77)
+    for prefix, seed in (((0, 3), 6), ((7, 12), 8)):
+        case = small_case(seed, prefix=prefix)
+        G = case.num_q_heads // case.num_kv_heads
+        out, _ = orc.block_attn(case.q_verify_bits, case.kv.k_bits, case.kv.v_bits, case.kv.page_table,
+                                case.kv.prefix_lens, case.num_q_heads, case.num_kv_heads, case.block_len,
+                                VER, case.scale)
+        for b in range(case.batch):
+            L = int(case.kv.prefix_lens[b])
+            k, v = gather_contiguous(case, b)
+            qb = np.transpose(q_f64(case.q_verify_bits[b]), (1, 0, 2))  # [Hq, bl, D]
+            qpre = rng.standard_normal((case.num_q_heads, L, case.head_dim))
+            qfull = np.concatenate([qpre, qb], axis=1)
+            ref = sdpa(qfull, repeat_heads(k, G), repeat_heads(v, G), case.scale, causal=True)[:, L:, :]
+            assert_close(np.transpose(out[b], (1, 0, 2)), ref, 1e-12, f"verify prefix={prefix}")
+
+
+def pin_lse_logsumexp(orc):
+    """lse = logsumexp of the scaled scores over the visible keys."""
+    case = small_case(21, prefix=(5, 10))
+    G = case.num_q_heads // case.num_kv_heads
+    for mode, qbits in ((DIFF, case.q_draft_bits), (VER, case.q_verify_bits)):
+        _, lse = orc.block_attn(qbits, case.kv.k_bits, case.kv.v_bits, case.kv.page_table,
+                                case.kv.prefix_lens, case.num_q_heads, case.num_kv_heads, case.block_len,
+                                mode, case.scale)
+        for b in range(case.batch):
+            L = int(case.kv.prefix_lens[b])
+            k, _ = gather_contiguous(case, b)
+            q = q_f64(qbits[b])  # [bl, Hq, D]
+            for h in range(case.num_q_heads):
+                scores = q[:, h, :] @ k[h // G].T * case.scale  # [bl, N]
+                for i in range(case.block_len):
+                    n_vis = L + (case.block_len if mode == DIFF else i + 1)
+                    ref = scipy.special.logsumexp(scores[i, :n_vis])
+                    assert abs(lse[b, h, i] - ref) <= 1e-12, f"lse b={b} h={h} i={i} mode={mode}"
+
+
+def pin_softmax_rows(orc):
+    """Probabilities are >= 0, sum to 1 per row, and are 0 on masked keys."""
+    case = small_case(31, prefix=(4, 9))
+    for mode in (DIFF, VER):
+        _, _, p = orc.block_attn(case.q_draft_bits, case.kv.k_bits, case.kv.v_bits, case.kv.page_table,
+                                 case.kv.prefix_lens, case.num_q_heads, case.num_kv_heads, case.block_len,
+                                 mode, case.scale, want_probs=True)
+        assert np.all(p >= 0.0)
+        assert_close(p.sum(axis=-1), 1.0, 1e-12, "row sums")
+        for b in range(case.batch):
+            L = int(case.kv.prefix_lens[b])
+            for i in range(case.block_len):
+                n_vis = L + (case.block_len if mode == DIFF else i + 1)
+                assert np.all(p[b, :, i, n_vis:] == 0.0), "probability on a masked key"
+                assert np.all(p[b, :, i, :n_vis] > 0.0), "visible key with zero probability"
+
+
+def pin_page_permutation(orc):
+    """Relabelling physical pages (and moving their contents) changes nothing, bit for bit."""
+    case = small_case(41, prefix=(10, 3))
+    kv = case.kv
+    rng = np.random.default_rng(5)
+    perm = rng.permutation(kv.num_pages)  # new physical index of old page p is perm[p]
+    k2 = np.empty_like(kv.k_bits)
+    v2 = np.empty_like(kv.v_bits)
+    k2[perm] = kv.k_bits
+    v2[perm] = kv.v_bits
+    table2 = np.where(kv.page_table >= 0, perm[np.maximum(kv.page_table, 0)], -1).astype(np.int32)
+    for mode in (DIFF, VER):
+        a = orc.block_attn(case.q_draft_bits, kv.k_bits, kv.v_bits, kv.page_table, kv.prefix_lens,
+                           case.num_q_heads, case.num_kv_heads, case.block_len, mode, case.scale)
+        b = orc.block_attn(case.q_draft_bits, k2, v2, table2, kv.prefix_lens,
+                           case.num_q_heads, case.num_kv_heads, case.block_len, mode, case.scale)
+        assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1])
+
+
+def pin_block_permutation(orc):
+    """Diffusion pass: permuting block tokens (queries and their K/V slots
+    together) permutes the output rows."""
+    case = small_case(51, B=1, prefix=(6,), P=4, bl=5, shuffle=False)
+    kv = case.kv
+    L = int(kv.prefix_lens[0])
+    bl = case.block_len
+    perm = np.random.default_rng(9).permutation(bl)
+    q2 = case.q_draft_bits.copy()
+    q2[0] = case.q_draft_bits[0][perm]
+    k2, v2 = kv.k_bits.copy(), kv.v_bits.copy()
+    P = kv.page_size
+    for j in range(bl):  # slot L + j gets the content of old slot L + perm[j]
+        dst, src = L + j, L + perm[j]
+        dp, ds = kv.page_table[0, dst // P], dst % P
+        sp, ss = kv.page_table[0, src // P], src % P
+        k2[dp, :, ds, :] = kv.k_bits[sp, :, ss, :]
+        v2[dp, :, ds, :] = kv.v_bits[sp, :, ss, :]
+    a, la = orc.block_attn(case.q_draft_bits, kv.k_bits, kv.v_bits, kv.page_table, kv.prefix_lens,
+                           case.num_q_heads, case.num_kv_heads, bl, DIFF, case.scale)
+    b, lb = orc.block_attn(q2, k2, v2, kv.page_table, kv.prefix_lens,
+                           case.num_q_heads, case.num_kv_heads, bl, DIFF, case.scale)
+    assert_close(b[0], a[0][perm], 1e-12, "block permutation (out)")
+    assert_close(lb[0], la[0][:, perm], 1e-12, "block permutation (lse)")
+
+
+def pin_closed_forms(orc):
+    """Constant V gives o = V; identical keys give the mean of the visible V;
+    a single visible key (L = 0, bl = 1) gives that key's V and lse = score."""
+    case = small_case(61, prefix=(5, 11))
+    kv = case.kv
+    G = case.num_q_heads // case.num_kv_heads
+    c_bits = W.f32_to_bf16_bits(np.full(kv.v_bits.shape, 0.75, dtype=np.float32))
+    for mode in (DIFF, VER):
+        out, _ = orc.block_attn(case.q_draft_bits, kv.k_bits, c_bits, kv.page_table, kv.prefix_lens,
+                                case.num_q_heads, case.num_kv_heads, case.block_len, mode, case.scale)
+        assert_close(out, 0.75, 1e-14, "constant V")
+    same_k = np.broadcast_to(kv.k_bits[:1, :, :1, :], kv.k_bits.shape).copy()
+    for mode in (DIFF, VER):
+        out, lse = orc.block_attn(case.q_draft_bits, same_k, kv.v_bits, kv.page_table, kv.prefix_lens,
+                                  case.num_q_heads, case.num_kv_heads, case.block_len, mode, case.scale)
+        for b in range(case.batch):
+            L = int(kv.prefix_lens[b])
+            _, v = gather_contiguous(case, b)
+            k0 = W.bf16_bits_to_f32(kv.k_bits[0, :, 0, :]).astype(np.float64)  # [Hkv, D]
+            q = q_f64(case.q_draft_bits[b])
+            for i in range(case.block_len):
+                n_vis = L + (case.block_len if mode == DIFF else i + 1)
+                for h in range(case.num_q_heads):
+                    ref = v[h // G, :n_vis].mean(axis=0)
+                    assert_close(out[b, i, h], ref, 1e-12, "identical keys")
+                    s = float(q[i, h] @ k0[h // G]) * case.scale
+                    assert abs(lse[b, h, i] - (s + math.log(n_vis))) <= 1e-12, "identical keys lse"
+    one = small_case(62, B=1, prefix=(0,), bl=1)
+    out, lse = orc.block_attn(one.q_draft_bits, one.kv.k_bits, one.kv.v_bits, one.kv.page_table,
+                              one.kv.prefix_lens, one.num_q_heads, one.num_kv_heads, 1, VER, one.scale)
+    k, v = gather_contiguous(one, 0)
+    q = q_f64(one.q_draft_bits[0, 0])
+    G1 = one.num_q_heads // one.num_kv_heads
+    for h in range(one.num_q_heads):
+        assert_close(out[0, 0, h], v[h // G1, 0], 0.0, "single key")
+        assert abs(lse[0, h, 0] - float(q[h] @ k[h // G1, 0]) * one.scale) <= 1e-12
+
+
+def read_golden_uniform():
+    rows = []
+    with open(os.path.join(GOLDEN, "attn_uniform_q0.txt")) as f:
+        for line in f:
+            line = line.strip()
+            if not line or line.startswith("#"):
+                continue
+            mode, i, o, cnt = [x.strip() for x in line.split("|")]
+            rows.append((DIFF if mode == "diffusion" else VER, int(i),
+                         np.array([float(x) for x in o.split()]), int(cnt)))
+    return rows
+
+
+def golden_uniform_inputs():
+    B, Hq, Hkv, D, P, L, bl = 1, 2, 1, 4, 4, 6, 3
+    table = np.array([[2, 0, 1]], dtype=np.int32)
+    v = np.full((3, Hkv, P, D), 1000.0, dtype=np.float32)
+    for t in range(L + bl):
+        page, slot = table[0, t // P], t % P
+        v[page, 0, slot] = [t, 2 * t, -t, 1]
+    k = np.random.default_rng(0).standard_normal((3, Hkv, P, D)).astype(np.float32)
+    q = np.zeros((B, bl, Hq, D), dtype=np.float32)
+    return (W.f32_to_bf16_bits(q), W.f32_to_bf16_bits(k), W.f32_to_bf16_bits(v), table,
+            np.array([L], dtype=np.int32), Hq, Hkv, bl)
+
+
+def pin_golden_uniform(orc):
+    """Hand-derived outputs for all-zero queries (tests/golden/attn_uniform_q0.txt)."""
+    q, k, v, table, pl, Hq, Hkv, bl = golden_uniform_inputs()
+    res = {m: orc.block_attn(q, k, v, table, pl, Hq, Hkv, bl, m, 0.5) for m in (DIFF, VER)}
+    for mode, i, o_ref, cnt in read_golden_uniform():
+        out, lse = res[mode]
+        for h in range(Hq):
+            assert_close(out[0, i, h], o_ref, 1e-12, f"golden mode={mode} i={i}")
+            assert abs(lse[0, h, i] - math.log(cnt)) <= 1e-12
+
+
+def pin_split_combine(orc):
+    """Attention over S disjoint key ranges, merged by the combine rule, equals
+    the unsplit result; empty ranges (lse = -inf) are ignored."""
+    case = small_case(71, prefix=(9, 14), bl=6)
+    kv = case.kv
+    Nmax = int(np.max(kv.prefix_lens)) + case.block_len
+    for mode in (DIFF, VER):
+        full, lse_full = orc.block_attn(case.q_verify_bits, kv.k_bits, kv.v_bits, kv.page_table,
+                                        kv.prefix_lens, case.num_q_heads, case.num_kv_heads,
+                                        case.block_len, mode, case.scale)
+        for cuts in ([0, 4, 11, Nmax], [0, 1, 2, 3, 15, 16, Nmax + 8], [0, Nmax]):
+            parts_o, parts_l = [], []
+            for a, b in zip(cuts[:-1], cuts[1:]):
+                o, l = orc.block_attn(case.q_verify_bits, kv.k_bits, kv.v_bits, kv.page_table,
+                                      kv.prefix_lens, case.num_q_heads, case.num_kv_heads,
+                                      case.block_len, mode, case.scale, key_begin=a, key_end=b)
+                parts_o.append(o.reshape(-1, case.head_dim))
+                # lse is [B, Hq, bl]; reorder to the out row order [B, bl, Hq]
+                parts_l.append(np.transpose(l, (0, 2, 1)).reshape(-1))
+            out, lse = orc.combine(np.stack(parts_o), np.stack(parts_l))
+            assert_close(out, full.reshape(-1, case.head_dim), 1e-12, f"split {cuts}")
+            assert_close(lse, np.transpose(lse_full, (0, 2, 1)).reshape(-1), 1e-12, "split lse")
+
+
+# --------------------------------------------------------------------------
+# decision pins
+# --------------------------------------------------------------------------
+
+def read_golden(name):
+    cases = []
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            line = line.strip()
+            if line and not line.startswith("#"):
+                cases.append([x.strip() for x in line.split("|")])
+    return cases
+
+
+def pin_accept_golden(orc):
+    for d, v, acc in read_golden("accept_cases.txt"):
+        d = np.array([[int(x) for x in d.split()]], dtype=np.int32)
+        v = np.array([[int(x) for x in v.split()]], dtype=np.int32)
+        got = orc.accept(d, v)
+        assert int(got[0]) == int(acc), f"accept {d} {v}: {got[0]} != {acc}"
+
+
+def brute_accept(d, v):
+    out = []
+    for row_d, row_v in zip(d.tolist(), v.tolist()):
+        acc = len(row_d)
+        for j, (a, b) in enumerate(zip(row_d, row_v)):
+            if a != b:
+                acc = j
+                break
+        out.append(acc)
+    return np.array(out, dtype=np.int32)
+
+
+def pin_accept_brute(orc):
+    rng = np.random.default_rng(3)
+    for n in (1, 2, 7, 8, 16, 31, 32):
+        for p in (0.0, 0.5, 0.9, 1.0):
+            d, v = W.make_accept_ids(rng, 64, n, 50, p)
+            assert np.array_equal(orc.accept(d, v), brute_accept(d, v)), f"n={n} p={p}"
+
+
+def pin_accept_statistics(orc):
+    """E[accepted_len] = p (1 - p^n) / (1 - p) for independent agreement with prob p."""
+    rng = np.random.default_rng(2024)
+    for n, p in ((8, 0.8), (16, 0.75), (8, 0.7), (32, 0.75)):
+        B = 40000
+        d, v = W.make_accept_ids(rng, B, n, 131072, p)
+        acc = orc.accept(d, v).astype(np.float64)
+        mean_ref = p * (1 - p ** n) / (1 - p)
+        se = acc.std() / math.sqrt(B)
+        assert abs(acc.mean() - mean_ref) < 5 * se, f"n={n} p={p}: {acc.mean()} vs {mean_ref}"
+
+
+def pin_unmask_golden(orc):
+    for c, k, pos, nsel in read_golden("unmask_cases.txt"):
+        conf = np.array([[float(x) for x in c.split()]], dtype=np.float32)
+        k = int(k)
+        p, s = orc.unmask(conf, k)
+        assert p[0].tolist() == [int(x) for x in pos.split()], f"unmask {c} k={k}: {p[0]}"
+        assert int(s[0]) == int(nsel)
+
+
+def brute_unmask(conf, k):
+    B, n = conf.shape
+    pos = np.full((B, k), -1, dtype=np.int32)
+    nsel = np.zeros(B, dtype=np.int32)
+    for b in range(B):
+        c = [float(x) for x in conf[b]]
+        elig = [i for i in range(n) if not (math.isnan(c[i]) or c[i] == -math.inf)]
+        order = sorted(elig, key=lambda i: (-c[i], i))[:k]
+        pos[b, :len(order)] = order
+        nsel[b] = len(order)
+    return pos, nsel
+
+
+def pin_unmask_brute(orc):
+    rng = np.random.default_rng(8)
+    for n in (1, 2, 8, 16, 32):
+        for k in sorted({1, 2, min(4, n), min(8, n), n}):
+            # few distinct values -> many ties; sprinkle -inf / nan / signed zeros
+            conf = rng.integers(0, 4, size=(50, n)).astype(np.float32) / 4
+            conf[rng.random((50, n)) < 0.15] = -np.inf
+            conf[rng.random((50, n)) < 0.05] = np.nan
+            z = rng.random((50, n)) < 0.1
+            conf[z] = np.where(rng.random(z.sum()) < 0.5, 0.0, -0.0)
+            p, s = orc.unmask(conf, k)
+            bp, bs = brute_unmask(conf, k)
+            assert np.array_equal(p, bp) and np.array_equal(s, bs), f"n={n} k={k}"
+
+
+def pin_unmask_lexsort(orc):
+    """Against numpy's lexsort (key: confidence descending, then index)."""
+    rng = np.random.default_rng(12)
+    conf = rng.random((200, 32), dtype=np.float32)
+    for k in (1, 4, 8, 32):
+        p, s = orc.unmask(conf, k)
+        for b in range(conf.shape[0]):
+            order = np.lexsort((np.arange(32), -conf[b].astype(np.float64)))[:k]
+            assert p[b].tolist() == order.tolist()
+        assert np.all(s == k)
+    p, _ = orc.unmask(conf, 32)
+    assert all(sorted(row) == list(range(32)) for row in p.tolist()), "k = n is a permutation"
+
+
+ATTENTION_PINS = [pin_decode_bl1, pin_diffusion_full_attention, pin_verify_causal_tail, pin_lse_logsumexp,
+                  pin_softmax_rows, pin_page_permutation, pin_block_permutation, pin_closed_forms,
+                  pin_golden_uniform, pin_split_combine]
+DECISION_PINS = [pin_accept_golden, pin_accept_brute, pin_accept_statistics, pin_unmask_golden,
+                 pin_unmask_brute, pin_unmask_lexsort]
+ALL_PINS = ATTENTION_PINS + DECISION_PINS

@@ -1,0 +1,69 @@
+"""Plant plausible mistakes in copies of the oracle; each must fail a pin.
+
+Every mutant is the oracle's C source with one textual change, compiled into a
+temporary library. A mutant that passes every pin would mean the pins cannot
+tell that mistake from the definition.
+"""
+import os
+
+import pytest
+
+import oracle
+import oracle_pins as pins
+
+MUTANTS = {
+    # mask: verify pass loses the diagonal (a token not seeing itself)
+    "verify_excludes_self": ("return j <= i;", "return j < i;"),
+    # mask: the diffusion pass made causal
+    "diffusion_causal": ("if (mode == 0) return 1;", "if (mode == 0) return j <= i;"),
+    # mask: block slots indexed from the wrong origin
+    "block_offset": ("long j = t - L;", "long j = t - L + 1;"),
+    # mask: verify pass made anti-causal (row i sees later block slots)
+    "verify_anticausal": ("return j <= i;", "return j >= i;"),
+    # GQA head mapping interleaved instead of grouped
+    "gqa_interleaved": ("const int g = h / G;", "const int g = h % Hkv;"),
+    # softmax scale dropped
+    "scale_dropped": ("s[t] = scale * dot;", "s[t] = dot;"),
+    # lse without the max shift
+    "lse_missing_max": ("*lse = m + log(l);", "*lse = log(l);"),
+    # page slot from the wrong index (K side only)
+    "slot_index": ("const uint16_t *krow = k + (((long)page * Hkv + g) * P + (t % P)) * (long)D;",
+                   "const uint16_t *krow = k + (((long)page * Hkv + g) * P + (t / P) % P) * (long)D;"),
+    # query layout transposed ([B, Hq, bl, D] instead of [B, bl, Hq, D])
+    "q_layout": ("q + (((long)b * bl + i) * Hq + h) * (long)D;", "q + (((long)b * Hq + h) * bl + i) * (long)D;"),
+    # combine forgets the partial weights
+    "combine_unweighted": ("orow[d] += c * op[d];", "orow[d] += op[d];"),
+    # combine: normaliser dropped
+    "combine_no_norm": ("for (int d = 0; d < D; ++d) orow[d] /= csum;", ""),
+    # accept counts the bonus token
+    "accept_plus_bonus": ("accepted[b] = j;", "accepted[b] = j < n ? j + 1 : j;"),
+    # accept counts all matches instead of the matching prefix
+    "accept_counts_matches": ("while (j < n && draft[(long)b * n + j] == verify[(long)b * n + j]) ++j;",
+                              "for (int t = 0; t < n; ++t) j += draft[(long)b * n + t] == verify[(long)b * n + t];"),
+    # unmask tie-break reversed
+    "unmask_tie_high_index": ("return a < b;", "return a > b;"),
+    # unmask: -inf treated as eligible
+    "unmask_neginf_eligible": ("if (!isnan(c[i]) && !(isinf(c[i]) && c[i] < 0)) idx[m++] = i;",
+                               "if (!isnan(c[i])) idx[m++] = i;"),
+    # unmask: ascending order
+    "unmask_ascending": ("if (ca > cb) return 1;\n    if (ca < cb) return 0;",
+                         "if (ca < cb) return 1;\n    if (ca > cb) return 0;"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_mutant_fails_a_pin(tmp_path, name):
+    old, new = MUTANTS[name]
+    src = open(oracle.SOURCE).read()
+    assert src.count(old) == 1, f"mutation site for {name} not unique"
+    path = tmp_path / "mutant.c"
+    path.write_text(src.replace(old, new))
+    lib = oracle.compile_oracle(str(path), str(tmp_path / "libmutant.so"), openmp=False)
+    orc = oracle.load(lib)
+    failed = []
+    for pin in pins.ALL_PINS:
+        try:
+            pin(orc)
+        except (AssertionError, ValueError):
+            failed.append(pin.__name__)
+    assert failed, f"mutant {name} passed every pin"
