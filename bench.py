@@ -1,0 +1,529 @@
+#!/usr/bin/env python3
+"""Draft+verify decoding step of tri-mode decoding on one GB300, at the 8B shape.
+
+One step = the whole path on one batch of synthetic input:
+  diffusion-draft block attention (bidirectional in-block) over the paged KV
+  cache, top-k unmasking of the draft confidences, AR-verify block attention
+  (causal in-block), and longest-prefix acceptance. Each block-attention pass
+  is the attention kernel plus, when the KV range is split, the combine.
+
+Workload: batch 1, 32 query / 8 KV heads, head_dim 128, 4096-token prefix in
+16-token pages under a random page permutation, block of 16 (the 8B decoder
+shape). Every pass reads its own KV pool from a rotation of pools larger than
+three times L2, so each pass streams its KV from HBM as it would with the other
+layers of a model running between two passes of the same layer.
+
+Output: one JSON line (rank 0). value = KV GB/s over the whole step
+(algorithmic KV bytes of both passes / step time); steps_per_s alongside.
+
+--impl reference times the fp64 CPU oracle on the host cores instead (the
+slow reference program this path is checked against), on a bounded sample of
+the same workload per step.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2607_05722_gb300 import workloads as W  # noqa: E402
+
+METRIC = "block-attn KV GB/s (% of GB300 HBM peak); draft+verify steps/sec at 8B shape"
+WORKLOAD = W.HEADLINE
+PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FALLBACK_HBM_GBS = 6800.0
+TRAFFIC_NOTE = os.path.join(ROOT, "profiles", "block_attn_8b_b1_L4096_bl16.md")
+KERNEL_SOURCES = [os.path.join(ROOT, "paper_2607_05722_gb300", "csrc", f)
+                  for f in ("block_attn.cu", "nld_internal.cuh")]
+
+
+def parse_args():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30000)
+    ap.add_argument("--warmup", type=int, default=300)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--pools", type=int, default=32, help="rotating KV pools (cold-L2 rotation)")
+    ap.add_argument("--splits", type=int, default=0, help="KV splits (0 = automatic)")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--seed", type=int, default=0)
+    return ap.parse_args()
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def hbm_peak():
+    try:
+        with open(PEAKS_PATH) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    for p in KERNEL_SOURCES:
+        with open(p, "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic():
+    """DRAM bytes per launch of the attention kernel from a committed ncu
+    summary, when it was taken on the current kernel source; else None."""
+    try:
+        text = open(TRAFFIC_NOTE).read()
+    except OSError:
+        return None
+    m_src = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]{16})", text)
+    m_tr = re.search(r"dram_bytes_per_launch:\s*([0-9]+)", text)
+    if not m_src or not m_tr or m_src.group(1) != kernel_source_hash():
+        return None
+    return int(m_tr.group(1))
+
+
+# ---------------------------------------------------------------------------
+# clock sampling during the timed region
+# ---------------------------------------------------------------------------
+
+CLOCK_FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+
+class ClockSampler:
+    def __init__(self, device_index: int):
+        self.proc = None
+        self.path = None
+        try:
+            fd, self.path = tempfile.mkstemp(prefix="nld_clocks_", suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={CLOCK_FIELDS}", "--format=csv,noheader,nounits", "-lms", "50",
+                 "-i", str(device_index)], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, ValueError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self, t0: float, t1: float):
+        """Median SM clock and throttle reasons of samples inside [t0, t1] (host
+        time); falls back to all samples while the GPU was busy."""
+        if self.path is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0, "note": "nvidia-smi unavailable"}
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 10:
+                continue
+            try:
+                ts = time.mktime(time.strptime(parts[0].split(".")[0], "%Y/%m/%d %H:%M:%S"))
+                ts += float("0." + parts[0].split(".")[1]) if "." in parts[0] else 0.0
+                rows.append((ts, float(parts[2]), float(parts[3]), parts[6:10]))
+            except (ValueError, IndexError):
+                continue
+        os.unlink(self.path)
+        inside = [r for r in rows if t0 - 0.05 <= r[0] <= t1 + 0.05]
+        note = "samples inside the timed region"
+        if not inside:
+            inside = rows
+            note = "timed region shorter than the sampling period: all samples of the run"
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0, "note": "no samples"}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[j] for r in inside for j, v in enumerate(r[3]) if v.lower() == "active"})
+        return {"sm_mhz": float(np.median([r[1] for r in inside])), "sm_max_mhz": max(r[2] for r in inside),
+                "reasons": reasons, "samples": len(inside), "note": note}
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+
+def run_ours(args, world, rank, local):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2607_05722_gb300 import build as nld_build
+    from paper_2607_05722_gb300 import nld
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    nld_build.build()
+    nld.lib()
+
+    wl = W.make_workload(WORKLOAD, seed=args.seed + rank)
+    c = wl.attn
+    kv = c.kv
+    B, bl, Hq, Hkv, D = c.batch, c.block_len, c.num_q_heads, c.num_kv_heads, c.head_dim
+    kv_bytes = c.kv_bytes_per_pass()
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    npool = max(args.pools, 2)
+    if npool * kv_bytes < 3 * l2:
+        npool = int(np.ceil(3 * l2 / kv_bytes)) + 1
+    npool += npool % 2
+
+    def dev_bf16(bits):
+        return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(dev)
+
+    k0, v0 = dev_bf16(kv.k_bits), dev_bf16(kv.v_bits)
+    pools = [(k0, v0)] + [(k0.clone(), v0.clone()) for _ in range(npool - 1)]
+    table = torch.from_numpy(kv.page_table).to(dev)
+    prefix = torch.from_numpy(kv.prefix_lens).to(dev)
+    q_d, q_v = dev_bf16(c.q_draft_bits), dev_bf16(c.q_verify_bits)
+    params = nld.make_params(B, Hq, Hkv, D, c.page_size, kv.num_pages, kv.max_pages, args.splits, 0.0)
+    splits = nld.nld_block_attn_num_splits(params, bl)
+    ws = torch.empty(max(nld.nld_block_attn_workspace_size(params, bl), 16), dtype=torch.uint8, device=dev)
+    out_d = torch.empty((B, bl, Hq, D), dtype=torch.bfloat16, device=dev)
+    out_v = torch.empty_like(out_d)
+    lse_d = torch.empty((B, Hq, bl), dtype=torch.float32, device=dev)
+    lse_v = torch.empty_like(lse_d)
+    draft = torch.from_numpy(wl.draft_ids).to(dev)
+    verify = torch.from_numpy(wl.verify_ids).to(dev)
+    conf = torch.from_numpy(wl.conf[0]).to(dev)
+    k_unmask = wl.unmask_k[0]
+    acc = torch.empty((B,), dtype=torch.int32, device=dev)
+    pos = torch.empty((B, k_unmask), dtype=torch.int32, device=dev)
+    nsel = torch.empty((B,), dtype=torch.int32, device=dev)
+    launches_per_step = 2 * (1 + (splits > 1)) + 2
+
+    def step(i, kd=None, vd=None, kvv=None, vv=None):
+        kd, vd = (kd, vd) if kd is not None else pools[(2 * i) % npool]
+        kvv, vv = (kvv, vv) if kvv is not None else pools[(2 * i + 1) % npool]
+        nld.nld_block_attn(params, q_d, kd, vd, table, prefix, bl, nld.NLD_MODE_DIFFUSION, out_d, lse_d, ws)
+        nld.nld_unmask(conf, k_unmask, pos, nsel)
+        nld.nld_block_attn(params, q_v, kvv, vv, table, prefix, bl, nld.NLD_MODE_VERIFY, out_v, lse_v, ws)
+        nld.nld_accept(draft, verify, acc)
+
+    # eager run once (also loads per-device state before capture)
+    step(0)
+    torch.cuda.synchronize()
+
+    chunk = 256
+    stream = torch.cuda.Stream(device=dev)
+
+    def capture(nsteps, offset=0):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(stream):
+            with torch.cuda.graph(g, stream=stream):
+                for i in range(nsteps):
+                    step(offset + i)
+        return g
+
+    g_main = capture(chunk)
+    reps, rem = divmod(args.steps, chunk)
+    g_rem = capture(rem, offset=reps * chunk) if rem else None
+    wreps, wrem = divmod(max(args.warmup, 3), chunk)
+    g_wrem = capture(wrem) if wrem else None
+    torch.cuda.synchronize()
+
+    sampler = ClockSampler(local) if rank == 0 else None
+    time.sleep(0.3 if sampler else 0.0)
+    # warm-up steps (untimed)
+    with torch.cuda.stream(stream):
+        for _ in range(wreps):
+            g_main.replay()
+        if g_wrem is not None:
+            g_wrem.replay()
+    torch.cuda.synchronize()
+
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_host0 = time.time()
+    with torch.cuda.stream(stream):
+        ev0.record(stream)
+        for _ in range(reps):
+            g_main.replay()
+        if g_rem is not None:
+            g_rem.replay()
+        ev1.record(stream)
+    torch.cuda.synchronize()
+    t_host1 = time.time()
+    if world > 1:
+        dist.barrier()
+    ms = ev0.elapsed_time(ev1)
+    if world > 1:
+        t = torch.tensor([ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    clocks = None
+    if sampler is not None:
+        time.sleep(0.1)
+        sampler.stop()
+        clocks = sampler.summary(t_host0, t_host1)
+
+    # ---- per-launch duration of the attention kernel (CUDA events on its stream) ----
+    nker = 2 * npool
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(nker)]
+    evc = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(nker)]
+    views = nld.workspace_views(params, bl, ws)
+    with torch.cuda.stream(stream):
+        torch.cuda._sleep(int(60e6))  # queue the launches behind a busy GPU so no host gap enters a bracket
+        for j in range(nker):
+            kp, vp = pools[j % npool]
+            mode = nld.NLD_MODE_VERIFY if j % 2 else nld.NLD_MODE_DIFFUSION
+            evs[j][0].record(stream)
+            nld.nld_block_attn_partials(params, q_v if j % 2 else q_d, kp, vp, table, prefix, bl, mode, out_v,
+                                        lse_v, ws, stream=stream)
+            evs[j][1].record(stream)
+            if views is not None:
+                evc[j][0].record(stream)
+                nld.nld_split_kv_combine(views[0], views[1], out_v, lse_v, stream=stream)
+                evc[j][1].record(stream)
+    torch.cuda.synchronize()
+    attn_ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))
+    comb_ms = float(np.mean([a.elapsed_time(b) for a, b in evc])) if views is not None else 0.0
+
+    # ---- end to end through the API with host buffers ----
+    e2e = run_e2e(args, torch, nld, dev, stream, wl, params, splits, kv_bytes, world)
+
+    if world > 1:
+        dist.barrier()
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+    peak, peak_kind = hbm_peak()
+    ms_step = ms / args.steps
+    total_kv = 2 * kv_bytes * world
+    value = total_kv / (ms_step * 1e-3) / 1e9
+    attn_gbs = kv_bytes / (attn_ms * 1e-3) / 1e9
+    line = {
+        "metric": METRIC,
+        "value": round(value, 2),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms_step,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic",
+        "config": {
+            "workload": WORKLOAD,
+            "batch_per_gpu": B, "q_heads": Hq, "kv_heads": Hkv, "head_dim": D, "prefix": int(kv.prefix_lens[0]),
+            "block_len": bl, "page_size": c.page_size, "page_order": "random permutation",
+            "kv_splits": splits, "unmask_k": k_unmask,
+            "step": "diffusion attention + unmask + verify attention + accept (one attention layer)",
+            "l2": f"cold: each pass reads its own KV pool from a rotation of {npool} pools "
+                  f"({npool * kv_bytes / 2**20:.0f} MiB > 3x L2 {l2 / 2**20:.0f} MiB)",
+            "timing": "CUDA graph of the steps, CUDA events on the launching stream",
+        },
+        "steps_per_s": round(1e3 / ms_step, 1) * world,
+        "pct_of_hbm_peak": round(100.0 * value / world / peak, 2),
+        "clocks": clocks,
+        "e2e": e2e,
+        "gpu_launches": launches_per_step * args.steps,
+        "roofline": {
+            "kernel": "block_attn_mma_kernel (attention, split partials)",
+            "bound": "hbm",
+            "achieved": round(attn_gbs, 1),
+            "peak": peak,
+            "peak_kind": f"{peak_kind} hbm_gbs (burst copy)",
+            "unit": "GB/s",
+            "frac": round(attn_gbs / peak, 4),
+            "traffic": recorded_traffic(),
+            "algorithmic_bytes_per_launch": kv_bytes,
+            "avg_launch_us": round(attn_ms * 1e3, 3),
+            "combine_avg_launch_us": round(comb_ms * 1e3, 3),
+        },
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl, budget_s=12.0)
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def run_e2e(args, torch, nld, dev, stream, wl, params, splits, kv_bytes, world):
+    """The same step through the API, with every input copied in from pinned
+    host memory and the results read back, inside the timed region."""
+    c = wl.attn
+    kv = c.kv
+    B, bl, Hq, D = c.batch, c.block_len, c.num_q_heads, c.head_dim
+
+    def pinned(a):
+        t = torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
+        return t
+
+    h_in = {
+        "q_d": pinned(c.q_draft_bits.view(np.int16)), "q_v": pinned(c.q_verify_bits.view(np.int16)),
+        "k": pinned(kv.k_bits.view(np.int16)), "v": pinned(kv.v_bits.view(np.int16)),
+        "table": pinned(kv.page_table), "prefix": pinned(kv.prefix_lens),
+        "draft": pinned(wl.draft_ids), "verify": pinned(wl.verify_ids), "conf": pinned(wl.conf[0]),
+    }
+    d_in = {k: torch.empty(v.shape, dtype=v.dtype, device=dev) for k, v in h_in.items()}
+    kk = wl.unmask_k[0]
+    d_out = {"out_d": torch.empty((B, bl, Hq, D), dtype=torch.bfloat16, device=dev),
+             "out_v": torch.empty((B, bl, Hq, D), dtype=torch.bfloat16, device=dev),
+             "acc": torch.empty((B,), dtype=torch.int32, device=dev),
+             "pos": torch.empty((B, kk), dtype=torch.int32, device=dev)}
+    h_out = {k: torch.empty(v.shape, dtype=v.dtype).pin_memory() for k, v in d_out.items()}
+    ws = torch.empty(max(nld.nld_block_attn_workspace_size(params, bl), 16), dtype=torch.uint8, device=dev)
+    nsel = torch.empty((B,), dtype=torch.int32, device=dev)
+
+    def bf(t):
+        return t.view(torch.bfloat16)
+
+    def step():
+        for k in h_in:
+            d_in[k].copy_(h_in[k], non_blocking=True)
+        nld.nld_block_attn(params, bf(d_in["q_d"]), bf(d_in["k"]), bf(d_in["v"]), d_in["table"], d_in["prefix"], bl,
+                           nld.NLD_MODE_DIFFUSION, d_out["out_d"], None, ws)
+        nld.nld_unmask(d_in["conf"], kk, d_out["pos"], nsel)
+        nld.nld_block_attn(params, bf(d_in["q_v"]), bf(d_in["k"]), bf(d_in["v"]), d_in["table"], d_in["prefix"], bl,
+                           nld.NLD_MODE_VERIFY, d_out["out_v"], None, ws)
+        nld.nld_accept(d_in["draft"], d_in["verify"], d_out["acc"])
+        for k in d_out:
+            h_out[k].copy_(d_out[k], non_blocking=True)
+
+    nsteps = max(1, min(args.steps, 3000))
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            step()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            step()
+        g.replay()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(nsteps):
+            g.replay()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / nsteps
+    h2d = int(sum(t.numel() * t.element_size() for t in h_in.values()))
+    d2h = int(sum(t.numel() * t.element_size() for t in h_out.values()))
+    return {"value": round(2 * kv_bytes * world / (ms * 1e-3) / 1e9, 2), "unit": "GB/s",
+            "ms_per_step": ms, "steps": nsteps, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "note": "every input copied from pinned host memory and outputs read back each step, in a CUDA graph"}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timings
+# ---------------------------------------------------------------------------
+
+def oracle_step(orc, wl, rows=None):
+    """One draft+verify step on the oracle: both passes (all rows, or the
+    given (b, i, h) rows), unmask and accept."""
+    c = wl.attn
+    kv = c.kv
+    for mode, qb in ((W.MODE_DIFFUSION, c.q_draft_bits), (W.MODE_VERIFY, c.q_verify_bits)):
+        if rows is None:
+            orc.block_attn(qb, kv.k_bits, kv.v_bits, kv.page_table, kv.prefix_lens, c.num_q_heads, c.num_kv_heads,
+                           c.block_len, mode, c.scale)
+        else:
+            orc.block_attn_rows(qb, kv.k_bits, kv.v_bits, kv.page_table, kv.prefix_lens, c.num_q_heads,
+                                c.num_kv_heads, c.block_len, mode, c.scale, rows)
+        if mode == W.MODE_DIFFUSION:
+            orc.unmask(wl.conf[0], wl.unmask_k[0])
+    orc.accept(wl.draft_ids, wl.verify_ids)
+
+
+def cpu_baseline(wl, budget_s: float):
+    import oracle
+    orc = oracle.load()
+    kv_bytes = wl.attn.kv_bytes_per_pass()
+    n = 0
+    t0 = time.perf_counter()
+    while True:
+        oracle_step(orc, wl)
+        n += 1
+        if time.perf_counter() - t0 > budget_s or n >= 50:
+            break
+    dt = time.perf_counter() - t0
+    return {"value": round(2 * kv_bytes * n / dt / 1e9, 4), "unit": "GB/s", "cores": orc.max_threads(),
+            "kind": "oracle", "steps_per_s": round(n / dt, 3),
+            "sample": f"{n} full draft+verify steps (every row of both passes, unmask, accept) of {WORKLOAD}, "
+                      f"fp64, OpenMP over (sequence, query head)"}
+
+
+def run_reference(args, world, rank):
+    if rank != 0:
+        return
+    import oracle
+    orc = oracle.load()
+    wl = W.make_workload(WORKLOAD, seed=args.seed)
+    c = wl.attn
+    kv_bytes = c.kv_bytes_per_pass()
+    total_rows = c.batch * c.block_len * c.num_q_heads
+    rng = np.random.default_rng(7)
+    all_rows = np.array([(b, i, h) for b in range(c.batch) for i in range(c.block_len)
+                         for h in range(c.num_q_heads)], dtype=np.int32)
+    # calibrate the per-row cost, then size each step's sample so the run stays
+    # within about two minutes
+    probe = all_rows[rng.permutation(total_rows)[:64]]
+    t0 = time.perf_counter()
+    oracle_step(orc, wl, probe)
+    per_row = (time.perf_counter() - t0) / (2 * len(probe))
+    budget = 120.0 / max(1, args.steps + args.warmup)
+    nrows = int(np.clip(budget / (2 * per_row), 1, total_rows))
+    sample = all_rows[rng.permutation(total_rows)[:nrows]]
+    for _ in range(args.warmup):
+        oracle_step(orc, wl, sample)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle_step(orc, wl, sample)
+    dt = time.perf_counter() - t0
+    frac = nrows / total_rows
+    value = 2 * kv_bytes * frac * args.steps / dt / 1e9
+    desc = (f"{nrows} of {total_rows} query rows of both passes per step (+ unmask, accept), {WORKLOAD}, "
+            f"fp64 oracle, OpenMP over rows")
+    line = {
+        "metric": METRIC, "value": round(value, 4), "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3 / frac, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+        "config": {"workload": WORKLOAD, "batch_per_gpu": c.batch, "q_heads": c.num_q_heads,
+                   "kv_heads": c.num_kv_heads, "head_dim": c.head_dim, "prefix": int(c.kv.prefix_lens[0]),
+                   "block_len": c.block_len, "page_size": c.page_size},
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": orc.max_threads(), "kind": "oracle",
+                         "sample": desc},
+        "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    world, rank, local = dist_env()
+    if args.gpus != world and world > 1:
+        print(f"--gpus {args.gpus} but WORLD_SIZE {world}", file=sys.stderr)
+    if args.impl == "reference":
+        run_reference(args, world, rank)
+        return
+    run_ours(args, world, rank, local)
+
+
+if __name__ == "__main__":
+    main()

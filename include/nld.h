@@ -1,0 +1,210 @@
+/*
+ * nld.h -- C ABI of libnld: block attention over a paged bf16 KV cache and
+ * the token decisions of tri-mode decoding, on one sm_103a GPU.
+ *
+ * Method (Nemotron-Labs-Diffusion, tri-mode decoding):
+ *   - Sec. 2.2 (attention pattern): noisy block tokens attend bidirectionally
+ *     inside their block and to the whole clean prefix; the clean stream is
+ *     strictly causal.
+ *   - Sec. 3, Mode 2 (block-wise diffusion): a block of mask tokens is
+ *     denoised in parallel against the cached prefix; confident positions are
+ *     committed step by step.
+ *   - Sec. 3, Mode 3 (linear self-speculation): a diffusion draft pass over
+ *     k mask positions, then a causal AR verify pass over the drafts, both
+ *     reusing the prefix KV cache; the longest matching draft prefix is
+ *     accepted.
+ *
+ * Conventions shared by every entry point:
+ *   - All tensor pointers are DEVICE pointers, row-major and contiguous, owned
+ *     by the caller. The library never allocates, frees or synchronises; each
+ *     call enqueues its kernels on `stream` and returns.
+ *   - Arguments that can be checked on the host are checked before anything
+ *     is launched; a failed check returns NLD_ERR_INVALID_ARG,
+ *     NLD_ERR_UNSUPPORTED or NLD_ERR_WORKSPACE and launches nothing. A failed
+ *     launch returns NLD_ERR_CUDA.
+ *   - Values that live on the device (prefix lengths, page ids) are not read
+ *     by the host. Kernels clamp out-of-range values into range (so no access
+ *     leaves the caller's buffers) and record the event in a device error
+ *     word, readable with nld_device_error().
+ *   - Pointers to bf16 and fp32 tensor data and the workspace must be 16-byte
+ *     aligned; int32 arrays must be 4-byte aligned.
+ */
+#ifndef NLD_H
+#define NLD_H
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    NLD_OK = 0,
+    NLD_ERR_INVALID_ARG = 1, /* null/misaligned pointer, bad size or shape   */
+    NLD_ERR_UNSUPPORTED = 2, /* valid but not built: head_dim, block, group  */
+    NLD_ERR_WORKSPACE = 3,   /* workspace missing or smaller than required   */
+    NLD_ERR_CUDA = 4         /* a CUDA runtime/driver call or launch failed  */
+} nld_status_t;
+
+/* Mask inside the block (Sec. 2.2, Sec. 3). The prefix is visible in both. */
+typedef enum {
+    NLD_MODE_DIFFUSION = 0, /* diffusion draft: bidirectional inside the block */
+    NLD_MODE_VERIFY = 1     /* AR verify: causal inside the block, self included */
+} nld_mode_t;
+
+/* Bits of the device error word (nld_device_error). */
+#define NLD_DEVERR_PREFIX_RANGE 0x1u /* a prefix length outside [0, max_pages*P - bl] was clamped */
+#define NLD_DEVERR_PAGE_RANGE 0x2u   /* a page id outside [0, num_pages) was clamped              */
+#define NLD_DEVERR_WAIT_TIMEOUT 0x4u /* a pipeline wait passed its time limit; output is invalid  */
+
+/*
+ * Shape of one block-attention call.
+ *   batch             B, number of sequences (>= 1)
+ *   num_q_heads       Hq; query head h reads KV head h / (Hq / Hkv)
+ *   num_kv_heads      Hkv; Hq % Hkv == 0
+ *   head_dim          D, 64 or 128
+ *   page_size         P, tokens per page: a power of two in [16, 256]
+ *   num_pages         pages in the pool (first dim of k_pages / v_pages)
+ *   max_pages_per_seq second dim of page_table
+ *   num_splits        KV splits per (sequence, KV head); 0 = choose from the
+ *                     SM count. Values above 128 are rejected.
+ *   softmax_scale     score scale; 0 = 1/sqrt(head_dim)
+ */
+typedef struct {
+    int batch;
+    int num_q_heads;
+    int num_kv_heads;
+    int head_dim;
+    int page_size;
+    int num_pages;
+    int max_pages_per_seq;
+    int num_splits;
+    float softmax_scale;
+} nld_attn_params_t;
+
+/*
+ * Number of KV splits nld_block_attn will use for these parameters (>= 1),
+ * or -1 if the parameters are invalid. With num_splits = 0 it queries the
+ * current device's SM count.
+ */
+int nld_block_attn_num_splits(const nld_attn_params_t *params, int block_len);
+
+/*
+ * Workspace bytes nld_block_attn needs (0 when it runs unsplit). The
+ * workspace holds fp32 split partials: O_part [S, B, Hq, bl, D] then
+ * LSE_part [S, B, Hq, bl] at the next 256-byte boundary.
+ * Returns (size_t)-1 if the parameters are invalid.
+ */
+size_t nld_block_attn_workspace_size(const nld_attn_params_t *params, int block_len);
+
+/*
+ * Block attention of a block of `block_len` tokens per sequence against the
+ * paged KV cache (Sec. 2.2 mask; Sec. 3 Modes 2 and 3).
+ *
+ * For sequence b with prefix length L_b = prefix_lens[b], query head h,
+ * block row i (0 <= i < block_len), key t is visible when t < L_b, or
+ * t = L_b + j with j < block_len and (mode == DIFFUSION or j <= i). Key t is
+ * read from physical page page_table[b][t / P], slot t % P, KV head
+ * h / (Hq / Hkv). Then, with s_t = softmax_scale * <q, k_t>:
+ *   out[b, i, h, :] = sum_t softmax(s)_t v_t,   lse[b, h, i] = ln sum_t exp(s_t).
+ *
+ *   q_block     bf16 [B, block_len, Hq, D]
+ *   k_pages     bf16 [num_pages, Hkv, P, D]
+ *   v_pages     bf16 [num_pages, Hkv, P, D]
+ *   page_table  int32 [B, max_pages_per_seq]; entries for logical pages
+ *               0 .. ceil((L_b + block_len) / P) - 1 must be valid page ids
+ *   prefix_lens int32 [B], L_b >= 0 and L_b + block_len <= max_pages_per_seq * P
+ *   block_len   1 .. 32, with (Hq / Hkv) * block_len <= 160
+ *   mode        NLD_MODE_DIFFUSION or NLD_MODE_VERIFY
+ *   out         bf16 [B, block_len, Hq, D]
+ *   lse         fp32 [B, Hq, block_len] (natural log), or NULL
+ *   workspace   device scratch of nld_block_attn_workspace_size() bytes
+ *               (may be NULL when that size is 0)
+ *
+ * The block's own K/V must already be in the paged slots L_b .. L_b+bl-1.
+ * When the call splits the KV range it launches the attention kernel and
+ * then the split combine (the same kernel nld_split_kv_combine runs).
+ */
+nld_status_t nld_block_attn(const nld_attn_params_t *params, const void *q_block,
+                            const void *k_pages, const void *v_pages,
+                            const int32_t *page_table, const int32_t *prefix_lens,
+                            int block_len, nld_mode_t mode, void *out, float *lse,
+                            void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/*
+ * The attention kernel of nld_block_attn alone, same arguments. When the
+ * split plan has one split it writes out and lse exactly as nld_block_attn
+ * does. With S > 1 splits it writes only the fp32 partials into the
+ * workspace (O_part at offset 0, LSE_part at the next 256-byte boundary
+ * after S*B*Hq*bl*D*4 bytes) and leaves out/lse untouched; the caller then
+ * merges them with nld_split_kv_combine (S = nld_block_attn_num_splits()).
+ * This lets a caller time, overlap or reorder the two kernels.
+ */
+nld_status_t nld_block_attn_partials(const nld_attn_params_t *params, const void *q_block,
+                                     const void *k_pages, const void *v_pages,
+                                     const int32_t *page_table, const int32_t *prefix_lens,
+                                     int block_len, nld_mode_t mode, void *out, float *lse,
+                                     void *workspace, size_t workspace_bytes,
+                                     cudaStream_t stream);
+
+/*
+ * Merge split-KV partials (each a softmax-normalised partial output and its
+ * log-sum-exp over one key range) into the full result:
+ *   m = max_s lse_s, c_s = exp(lse_s - m),
+ *   out = sum_s c_s o_s / sum_s c_s,  lse = m + ln sum_s c_s.
+ * A partial with lse_s = -inf carries no keys: it gets weight 0 and its
+ * o_s is not read. A row whose partials are all -inf gets out = 0 and
+ * lse = -inf.
+ *
+ *   o_part   fp32 [S, B, Hq, bl, D]
+ *   lse_part fp32 [S, B, Hq, bl]
+ *   out      bf16 [B, bl, Hq, D]
+ *   lse      fp32 [B, Hq, bl], or NULL
+ *   1 <= num_splits <= 128, head_dim 64 or 128, 1 <= block_len <= 32
+ */
+nld_status_t nld_split_kv_combine(const float *o_part, const float *lse_part, int num_splits,
+                                  int batch, int num_q_heads, int block_len, int head_dim,
+                                  void *out, float *lse, cudaStream_t stream);
+
+/*
+ * Longest-prefix acceptance of linear self-speculation (Sec. 3, Mode 3):
+ * accepted_len[b] = the first j with draft_ids[b][j] != verify_ids[b][j],
+ * or n when all n positions agree. The caller commits draft[0:acc] plus the
+ * verifier's token at the first mismatch, so a step yields 1..n+1 tokens.
+ *
+ *   draft_ids, verify_ids int32 [B, n];  accepted_len int32 [B];  1 <= n <= 32
+ */
+nld_status_t nld_accept(const int32_t *draft_ids, const int32_t *verify_ids, int batch, int n,
+                        int32_t *accepted_len, cudaStream_t stream);
+
+/*
+ * Confidence-ranked unmasking of the diffusion mode (Sec. 3, Mode 2; the
+ * serial denoising of Sec. 4 commits the single most confident position):
+ * the k eligible positions with the largest fp32 confidence, written in rank
+ * order (confidence descending; equal values, +0 and -0 included, by
+ * position ascending). -inf and NaN mark ineligible (already committed)
+ * positions. When fewer than k are eligible the tail of `positions` is -1.
+ *
+ *   confidences fp32 [B, n];  positions int32 [B, k];
+ *   num_selected int32 [B] or NULL;  1 <= k <= n <= 32
+ */
+nld_status_t nld_unmask(const float *confidences, int batch, int n, int k, int32_t *positions,
+                        int32_t *num_selected, cudaStream_t stream);
+
+/* A static, human-readable name for a status code. */
+const char *nld_status_string(nld_status_t status);
+
+/*
+ * Read the current device's error word (NLD_DEVERR_* bits) into *bits;
+ * with clear != 0 reset it to 0. Synchronises the device; meant for tests
+ * and diagnostics, not for the decode loop.
+ */
+nld_status_t nld_device_error(uint32_t *bits, int clear);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* NLD_H */

@@ -1,0 +1,306 @@
+// C ABI of libnld (include/nld.h): host-side argument checks, KV split choice,
+// TMA descriptor encoding and kernel launches. Nothing here allocates device
+// memory or synchronises, except nld_device_error().
+#include <math.h>
+#include <stdio.h>
+
+#include <mutex>
+
+#include "nld_internal.cuh"
+
+namespace {
+
+using nld::AttnArgs;
+
+// Error word the kernels OR their NLD_DEVERR_* bits into.
+__device__ unsigned int g_device_error;
+
+constexpr int kMaxDevices = 64;
+unsigned int* g_err_ptr[kMaxDevices];
+int g_sm_count[kMaxDevices];
+std::mutex g_mu;
+
+bool aligned(const void* p, size_t a) { return p != nullptr && (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// Per-device state: address of the error word and SM count, looked up once.
+nld_status_t device_state(unsigned int** err, int* sms) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return NLD_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_mu);
+  if (g_err_ptr[dev] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_device_error) != cudaSuccess) return NLD_ERR_CUDA;
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return NLD_ERR_CUDA;
+    g_sm_count[dev] = n;
+    g_err_ptr[dev] = static_cast<unsigned int*>(p);
+  }
+  if (err) *err = g_err_ptr[dev];
+  if (sms) *sms = g_sm_count[dev];
+  return NLD_OK;
+}
+
+bool is_pow2(int x) { return x > 0 && (x & (x - 1)) == 0; }
+
+nld_status_t check_params(const nld_attn_params_t* p, int block_len) {
+  if (p == nullptr) return NLD_ERR_INVALID_ARG;
+  if (p->batch < 1 || p->num_q_heads < 1 || p->num_kv_heads < 1 || p->num_pages < 1 ||
+      p->max_pages_per_seq < 1 || p->num_splits < 0 || p->softmax_scale < 0.f || !isfinite(p->softmax_scale))
+    return NLD_ERR_INVALID_ARG;
+  if (p->num_q_heads % p->num_kv_heads != 0) return NLD_ERR_INVALID_ARG;
+  if (block_len < 1 || block_len > nld::kMaxBlock) return NLD_ERR_INVALID_ARG;
+  if (p->num_splits > nld::kMaxSplits) return NLD_ERR_INVALID_ARG;
+  if (!is_pow2(p->page_size) || p->page_size < 16 || p->page_size > 256) return NLD_ERR_INVALID_ARG;
+  if (p->batch > 65535 || p->num_kv_heads > 65535) return NLD_ERR_UNSUPPORTED;
+  if (p->head_dim != 64 && p->head_dim != 128) return NLD_ERR_UNSUPPORTED;
+  if ((p->num_q_heads / p->num_kv_heads) * block_len > nld::kMaxRows) return NLD_ERR_UNSUPPORTED;
+  // logical token positions must fit in int
+  if (static_cast<long long>(p->max_pages_per_seq) * p->page_size > (1ll << 30)) return NLD_ERR_UNSUPPORTED;
+  if (static_cast<long long>(p->max_pages_per_seq) * p->page_size < block_len) return NLD_ERR_INVALID_ARG;
+  return NLD_OK;
+}
+
+// Split plan: S splits of `chunk` tokens (a multiple of 16) over the longest
+// possible sequence, max_pages_per_seq * page_size tokens. Splits past a
+// shorter sequence's end do no work. With num_splits = 0 the count is
+// chosen so that (splits x sequences x KV heads) covers the SMs once.
+struct SplitPlan {
+  int splits;
+  int chunk;
+};
+
+nld_status_t plan_splits(const nld_attn_params_t* p, int block_len, SplitPlan* out) {
+  const long long max_tokens = static_cast<long long>(p->max_pages_per_seq) * p->page_size;
+  int want = p->num_splits;
+  if (want == 0) {
+    int sms = 0;
+    nld_status_t st = device_state(nullptr, &sms);
+    if (st != NLD_OK) return st;
+    const long long units = static_cast<long long>(p->batch) * p->num_kv_heads;
+    long long s = (sms + units - 1) / units;
+    const long long by_tiles = (max_tokens + nld::kTileTok - 1) / nld::kTileTok;  // >= one tile per split
+    if (s > by_tiles) s = by_tiles;
+    if (s > nld::kMaxSplits) s = nld::kMaxSplits;
+    want = static_cast<int>(s < 1 ? 1 : s);
+  }
+  long long chunk = (max_tokens + want - 1) / want;
+  chunk = (chunk + nld::kGroupTok - 1) / nld::kGroupTok * nld::kGroupTok;
+  out->chunk = static_cast<int>(chunk);
+  out->splits = static_cast<int>((max_tokens + chunk - 1) / chunk);
+  (void)block_len;
+  return NLD_OK;
+}
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+size_t partial_o_bytes(const nld_attn_params_t* p, int block_len, int splits) {
+  return static_cast<size_t>(splits) * p->batch * p->num_q_heads * block_len * p->head_dim * sizeof(float);
+}
+size_t partial_lse_bytes(const nld_attn_params_t* p, int block_len, int splits) {
+  return static_cast<size_t>(splits) * p->batch * p->num_q_heads * block_len * sizeof(float);
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(f);
+  });
+  return fn;
+}
+
+// 4-D map over a page pool [num_pages, Hkv, P, D] (innermost first: D, P, Hkv,
+// pages); one box is 64 dims x 16 tokens of one (page, KV head), stored with
+// the 128-byte swizzle. Boxes past num_pages read as zeros.
+nld_status_t encode_pool_map(CUtensorMap* map, const void* base, const nld_attn_params_t* p) {
+  EncodeTiledFn fn = encode_fn();
+  if (fn == nullptr) return NLD_ERR_CUDA;
+  const cuuint64_t D = static_cast<cuuint64_t>(p->head_dim);
+  cuuint64_t dims[4] = {D, static_cast<cuuint64_t>(p->page_size), static_cast<cuuint64_t>(p->num_kv_heads),
+                        static_cast<cuuint64_t>(p->num_pages)};
+  cuuint64_t strides[3] = {D * 2, D * 2 * p->page_size, D * 2 * p->page_size * p->num_kv_heads};
+  cuuint32_t box[4] = {64, static_cast<cuuint32_t>(nld::kGroupTok), 1, 1};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? NLD_OK : NLD_ERR_CUDA;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* nld_status_string(nld_status_t s) {
+  switch (s) {
+    case NLD_OK: return "NLD_OK";
+    case NLD_ERR_INVALID_ARG: return "NLD_ERR_INVALID_ARG";
+    case NLD_ERR_UNSUPPORTED: return "NLD_ERR_UNSUPPORTED";
+    case NLD_ERR_WORKSPACE: return "NLD_ERR_WORKSPACE";
+    case NLD_ERR_CUDA: return "NLD_ERR_CUDA";
+  }
+  return "NLD_ERR_UNKNOWN";
+}
+
+int nld_block_attn_num_splits(const nld_attn_params_t* params, int block_len) {
+  if (check_params(params, block_len) != NLD_OK) return -1;
+  SplitPlan plan;
+  if (plan_splits(params, block_len, &plan) != NLD_OK) return -1;
+  return plan.splits;
+}
+
+size_t nld_block_attn_workspace_size(const nld_attn_params_t* params, int block_len) {
+  if (check_params(params, block_len) != NLD_OK) return static_cast<size_t>(-1);
+  SplitPlan plan;
+  if (plan_splits(params, block_len, &plan) != NLD_OK) return static_cast<size_t>(-1);
+  if (plan.splits == 1) return 0;
+  return align256(partial_o_bytes(params, block_len, plan.splits)) + partial_lse_bytes(params, block_len, plan.splits);
+}
+
+}  // extern "C"
+
+namespace {
+
+nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_block, const void* k_pages,
+                             const void* v_pages, const int32_t* page_table, const int32_t* prefix_lens,
+                             int block_len, nld_mode_t mode, void* out, float* lse, void* workspace,
+                             size_t workspace_bytes, bool run_combine, cudaStream_t stream) {
+  nld_status_t st = check_params(params, block_len);
+  if (st != NLD_OK) return st;
+  if (mode != NLD_MODE_DIFFUSION && mode != NLD_MODE_VERIFY) return NLD_ERR_INVALID_ARG;
+  if (!aligned(q_block, 16) || !aligned(k_pages, 16) || !aligned(v_pages, 16) || !aligned(out, 16) ||
+      !aligned(page_table, 4) || !aligned(prefix_lens, 4))
+    return NLD_ERR_INVALID_ARG;
+  if (lse != nullptr && !aligned(lse, 4)) return NLD_ERR_INVALID_ARG;
+  SplitPlan plan;
+  st = plan_splits(params, block_len, &plan);
+  if (st != NLD_OK) return st;
+  size_t o_bytes = 0;
+  if (plan.splits > 1) {
+    o_bytes = align256(partial_o_bytes(params, block_len, plan.splits));
+    const size_t need = o_bytes + partial_lse_bytes(params, block_len, plan.splits);
+    if (workspace == nullptr || workspace_bytes < need) return NLD_ERR_WORKSPACE;
+    if (!aligned(workspace, 16)) return NLD_ERR_INVALID_ARG;
+  }
+  unsigned int* err = nullptr;
+  st = device_state(&err, nullptr);
+  if (st != NLD_OK) return st;
+
+  CUtensorMap tmk, tmv;
+  if ((st = encode_pool_map(&tmk, k_pages, params)) != NLD_OK) return st;
+  if ((st = encode_pool_map(&tmv, v_pages, params)) != NLD_OK) return st;
+
+  const int G = params->num_q_heads / params->num_kv_heads;
+  const float scale = params->softmax_scale > 0.f ? params->softmax_scale : 1.0f / sqrtf((float)params->head_dim);
+  AttnArgs a{};
+  a.q = static_cast<const __nv_bfloat16*>(q_block);
+  a.page_table = page_table;
+  a.prefix_lens = prefix_lens;
+  a.out = static_cast<__nv_bfloat16*>(out);
+  a.lse = lse;
+  a.err = err;
+  a.B = params->batch;
+  a.Hq = params->num_q_heads;
+  a.Hkv = params->num_kv_heads;
+  a.G = G;
+  a.bl = block_len;
+  a.R = G * block_len;
+  a.page_size = params->page_size;
+  a.log2_page = __builtin_ctz(static_cast<unsigned>(params->page_size));
+  a.num_pages = params->num_pages;
+  a.max_pages = params->max_pages_per_seq;
+  a.num_splits = plan.splits;
+  a.chunk = plan.chunk;
+  a.mode = static_cast<int>(mode);
+  a.scale_log2 = scale * nld::kLog2e;
+  if (plan.splits > 1) {
+    a.o_part = static_cast<float*>(workspace);
+    a.lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) + o_bytes);
+  }
+  if (nld::launch_block_attn(a, tmk, tmv, params->head_dim, stream) != cudaSuccess) return NLD_ERR_CUDA;
+  if (plan.splits > 1 && run_combine) {
+    if (nld::launch_combine(a.o_part, a.lse_part, plan.splits, a.B, a.Hq, block_len, params->head_dim, a.out, lse,
+                            stream) != cudaSuccess)
+      return NLD_ERR_CUDA;
+  }
+  return NLD_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+nld_status_t nld_block_attn(const nld_attn_params_t* params, const void* q_block, const void* k_pages,
+                            const void* v_pages, const int32_t* page_table, const int32_t* prefix_lens,
+                            int block_len, nld_mode_t mode, void* out, float* lse, void* workspace,
+                            size_t workspace_bytes, cudaStream_t stream) {
+  return block_attn_impl(params, q_block, k_pages, v_pages, page_table, prefix_lens, block_len, mode, out, lse,
+                         workspace, workspace_bytes, true, stream);
+}
+
+nld_status_t nld_block_attn_partials(const nld_attn_params_t* params, const void* q_block, const void* k_pages,
+                                     const void* v_pages, const int32_t* page_table, const int32_t* prefix_lens,
+                                     int block_len, nld_mode_t mode, void* out, float* lse, void* workspace,
+                                     size_t workspace_bytes, cudaStream_t stream) {
+  return block_attn_impl(params, q_block, k_pages, v_pages, page_table, prefix_lens, block_len, mode, out, lse,
+                         workspace, workspace_bytes, false, stream);
+}
+
+nld_status_t nld_split_kv_combine(const float* o_part, const float* lse_part, int num_splits, int batch,
+                                  int num_q_heads, int block_len, int head_dim, void* out, float* lse,
+                                  cudaStream_t stream) {
+  if (num_splits < 1 || num_splits > nld::kMaxSplits || batch < 1 || num_q_heads < 1 || block_len < 1 ||
+      block_len > nld::kMaxBlock)
+    return NLD_ERR_INVALID_ARG;
+  if (head_dim != 64 && head_dim != 128) return NLD_ERR_UNSUPPORTED;
+  if (!aligned(o_part, 16) || !aligned(lse_part, 4) || !aligned(out, 16)) return NLD_ERR_INVALID_ARG;
+  if (lse != nullptr && !aligned(lse, 4)) return NLD_ERR_INVALID_ARG;
+  if (nld::launch_combine(o_part, lse_part, num_splits, batch, num_q_heads, block_len, head_dim,
+                          static_cast<__nv_bfloat16*>(out), lse, stream) != cudaSuccess)
+    return NLD_ERR_CUDA;
+  return NLD_OK;
+}
+
+nld_status_t nld_accept(const int32_t* draft_ids, const int32_t* verify_ids, int batch, int n,
+                        int32_t* accepted_len, cudaStream_t stream) {
+  if (batch < 1 || n < 1 || n > nld::kMaxBlock) return NLD_ERR_INVALID_ARG;
+  if (!aligned(draft_ids, 4) || !aligned(verify_ids, 4) || !aligned(accepted_len, 4)) return NLD_ERR_INVALID_ARG;
+  return nld::launch_accept(draft_ids, verify_ids, batch, n, accepted_len, stream) == cudaSuccess ? NLD_OK
+                                                                                                   : NLD_ERR_CUDA;
+}
+
+nld_status_t nld_unmask(const float* confidences, int batch, int n, int k, int32_t* positions,
+                        int32_t* num_selected, cudaStream_t stream) {
+  if (batch < 1 || n < 1 || n > nld::kMaxBlock || k < 1 || k > n) return NLD_ERR_INVALID_ARG;
+  if (!aligned(confidences, 4) || !aligned(positions, 4)) return NLD_ERR_INVALID_ARG;
+  if (num_selected != nullptr && !aligned(num_selected, 4)) return NLD_ERR_INVALID_ARG;
+  return nld::launch_unmask(confidences, batch, n, k, positions, num_selected, stream) == cudaSuccess
+             ? NLD_OK
+             : NLD_ERR_CUDA;
+}
+
+nld_status_t nld_device_error(uint32_t* bits, int clear) {
+  if (bits == nullptr) return NLD_ERR_INVALID_ARG;
+  unsigned int* err = nullptr;
+  nld_status_t st = device_state(&err, nullptr);
+  if (st != NLD_OK) return st;
+  unsigned int v = 0;
+  if (cudaMemcpy(&v, err, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return NLD_ERR_CUDA;
+  *bits = v;
+  if (clear) {
+    const unsigned int zero = 0;
+    if (cudaMemcpy(err, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess) return NLD_ERR_CUDA;
+  }
+  return NLD_OK;
+}
+
+}  // extern "C"

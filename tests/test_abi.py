@@ -1,0 +1,103 @@
+"""The C ABI library without a GPU: it loads, exports every function that
+include/nld.h declares, and rejects bad arguments on the host before any
+CUDA call (the checks below return before the library touches a device)."""
+import ctypes
+import os
+
+import pytest
+
+from paper_2607_05722_gb300 import build, nld
+
+FAKE = ctypes.c_void_p(0x10000)  # aligned, never dereferenced: every call below fails a host check first
+
+
+@pytest.fixture(scope="module")
+def L():
+    build.build()
+    return nld.lib()
+
+
+def test_header_declares_the_abi():
+    names = nld.header_functions()
+    for f in ("nld_block_attn", "nld_block_attn_partials", "nld_block_attn_workspace_size", "nld_block_attn_num_splits",
+              "nld_split_kv_combine", "nld_accept", "nld_unmask", "nld_status_string", "nld_device_error"):
+        assert f in names, f
+
+
+def test_library_exports_every_declared_symbol(L):
+    for f in nld.header_functions():
+        assert hasattr(L, f), f"libnld.so does not export {f}"
+
+
+def test_status_strings(L):
+    for code, name in ((0, "NLD_OK"), (1, "NLD_ERR_INVALID_ARG"), (2, "NLD_ERR_UNSUPPORTED"),
+                       (3, "NLD_ERR_WORKSPACE"), (4, "NLD_ERR_CUDA")):
+        assert nld.nld_status_string(code) == name
+
+
+def params(**kw):
+    base = dict(batch=1, num_q_heads=32, num_kv_heads=8, head_dim=128, page_size=16, num_pages=300,
+                max_pages_per_seq=257, num_splits=4, softmax_scale=0.0)
+    base.update(kw)
+    return nld.make_params(**base)
+
+
+def test_split_plan_and_workspace_size(L):
+    p = params(num_splits=19)
+    assert nld.nld_block_attn_num_splits(p, 16) == 19
+    # 4112 tokens / 19 -> 217 -> 224 per split -> 19 splits
+    S, B, Hq, bl, D = 19, 1, 32, 16, 128
+    o = S * B * Hq * bl * D * 4
+    assert nld.nld_block_attn_workspace_size(p, 16) == ((o + 255) // 256) * 256 + S * B * Hq * bl * 4
+    assert nld.nld_block_attn_workspace_size(params(num_splits=1), 16) == 0
+    assert nld.nld_block_attn_num_splits(params(num_splits=64, max_pages_per_seq=4), 8) == 4  # chunk >= 16
+
+
+@pytest.mark.parametrize("kw,bl,code", [
+    (dict(num_q_heads=30), 16, 1),          # Hq % Hkv != 0
+    (dict(head_dim=96), 16, 2),             # head_dim not built
+    (dict(page_size=24), 16, 1),            # not a power of two
+    (dict(page_size=8), 16, 1),             # below 16
+    (dict(page_size=512), 16, 1),           # above 256
+    (dict(num_splits=129), 16, 1),          # too many splits
+    (dict(), 0, 1),                         # block_len 0
+    (dict(), 33, 1),                        # block_len > 32
+    (dict(num_q_heads=48, num_kv_heads=8), 32, 2),  # 6 * 32 = 192 packed rows > 160
+    (dict(batch=0), 16, 1),
+])
+def test_block_attn_rejects_bad_shapes(L, kw, bl, code):
+    p = params(**kw)
+    st = L.nld_block_attn(ctypes.byref(p), FAKE, FAKE, FAKE, FAKE, FAKE, bl, 0, FAKE, None, None, 0, None)
+    assert st == code
+
+
+def test_block_attn_rejects_bad_pointers_and_workspace(L):
+    p = params()
+    st = L.nld_block_attn(ctypes.byref(p), None, FAKE, FAKE, FAKE, FAKE, 16, 0, FAKE, None, None, 0, None)
+    assert st == 1
+    mis = ctypes.c_void_p(0x10008)  # 8-byte aligned, not 16
+    st = L.nld_block_attn(ctypes.byref(p), FAKE, mis, FAKE, FAKE, FAKE, 16, 0, FAKE, None, None, 0, None)
+    assert st == 1
+    st = L.nld_block_attn(ctypes.byref(p), FAKE, FAKE, FAKE, FAKE, FAKE, 16, 2, FAKE, None, None, 0, None)
+    assert st == 1  # mode
+    need = nld.nld_block_attn_workspace_size(p, 16)
+    st = L.nld_block_attn(ctypes.byref(p), FAKE, FAKE, FAKE, FAKE, FAKE, 16, 0, FAKE, None, FAKE, need - 1, None)
+    assert st == 3
+    st = L.nld_block_attn(ctypes.byref(p), FAKE, FAKE, FAKE, FAKE, FAKE, 16, 0, FAKE, None, None, 0, None)
+    assert st == 3
+
+
+def test_decisions_reject_bad_sizes(L):
+    assert L.nld_accept(FAKE, FAKE, 1, 33, FAKE, None) == 1
+    assert L.nld_accept(FAKE, FAKE, 0, 8, FAKE, None) == 1
+    assert L.nld_accept(None, FAKE, 1, 8, FAKE, None) == 1
+    assert L.nld_unmask(FAKE, 1, 8, 9, FAKE, None, None) == 1
+    assert L.nld_unmask(FAKE, 1, 8, 0, FAKE, None, None) == 1
+    assert L.nld_unmask(FAKE, 1, 40, 4, FAKE, None, None) == 1
+    assert L.nld_split_kv_combine(FAKE, FAKE, 0, 1, 4, 8, 128, FAKE, None, None) == 1
+    assert L.nld_split_kv_combine(FAKE, FAKE, 2, 1, 4, 8, 80, FAKE, None, None) == 2
+
+
+def test_no_cpu_fallback_without_library(tmp_path):
+    with pytest.raises(RuntimeError):
+        nld.lib(str(tmp_path / "missing.so"))

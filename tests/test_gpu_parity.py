@@ -1,0 +1,324 @@
+"""CUDA path vs the fp64 oracle, through the C ABI, on seeded inputs.
+
+Bars: accept/unmask bit-exact; attention max-abs <= 1e-2 and rel-L2 <= 5e-3
+against the fp64 oracle (bf16 inputs, fp32 accumulation), lse within 2e-3.
+Small cases run the oracle on every row; the full-size workloads run in the
+launch configuration the bench times (automatic split count) and compare a
+sample of rows the oracle computes one by one.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle_pins
+from gpu_helpers import DeviceCase, compare_attn, oracle_full, sample_rows
+from paper_2607_05722_gb300 import nld
+from paper_2607_05722_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+DIFF, VER = W.MODE_DIFFUSION, W.MODE_VERIFY
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2607_05722_gb300 import build
+    build.build()
+    nld.lib()
+    nld.nld_device_error(clear=True)
+    yield
+    assert nld.nld_device_error(clear=True) == 0, "a kernel flagged a device error"
+
+
+# ---------------------------------------------------------------------------
+# token decisions: bit-exact
+# ---------------------------------------------------------------------------
+
+def gpu_accept(d, v):
+    dt, vt = torch.from_numpy(d).cuda(), torch.from_numpy(v).cuda()
+    acc = torch.full((d.shape[0],), -7, dtype=torch.int32, device="cuda")
+    nld.nld_accept(dt, vt, acc)
+    return acc.cpu().numpy()
+
+
+def gpu_unmask(conf, k):
+    ct = torch.from_numpy(np.ascontiguousarray(conf)).cuda()
+    pos = torch.full((conf.shape[0], k), -7, dtype=torch.int32, device="cuda")
+    nsel = torch.full((conf.shape[0],), -7, dtype=torch.int32, device="cuda")
+    nld.nld_unmask(ct, k, pos, nsel)
+    return pos.cpu().numpy(), nsel.cpu().numpy()
+
+
+def test_accept_golden_cases():
+    for d, v, acc in oracle_pins.read_golden("accept_cases.txt"):
+        d = np.array([[int(x) for x in d.split()]], dtype=np.int32)
+        v = np.array([[int(x) for x in v.split()]], dtype=np.int32)
+        assert int(gpu_accept(d, v)[0]) == int(acc)
+
+
+@pytest.mark.parametrize("name", sorted(W.WORKLOADS))
+def test_accept_workload_ids(orc, name):
+    cfg = W.WORKLOADS[name]
+    for seed in range(5):
+        rng = np.random.default_rng(seed)
+        d, v = W.make_accept_ids(rng, max(cfg["batch"], 1000), cfg["bl"], cfg["vocab"], cfg["p"])
+        assert np.array_equal(gpu_accept(d, v), orc.accept(d, v))
+
+
+def test_accept_all_widths(orc):
+    rng = np.random.default_rng(1)
+    for n in range(1, 33):
+        for p in (0.0, 0.6, 1.0):
+            d, v = W.make_accept_ids(rng, 77, n, 1000, p)
+            assert np.array_equal(gpu_accept(d, v), orc.accept(d, v)), (n, p)
+
+
+def test_unmask_golden_cases():
+    for c, k, pos, nsel in oracle_pins.read_golden("unmask_cases.txt"):
+        conf = np.array([[float(x) for x in c.split()]], dtype=np.float32)
+        p, s = gpu_unmask(conf, int(k))
+        assert p[0].tolist() == [int(x) for x in pos.split()]
+        assert int(s[0]) == int(nsel)
+
+
+def test_unmask_ties_and_ineligible(orc):
+    rng = np.random.default_rng(2)
+    for n in (1, 2, 3, 8, 16, 31, 32):
+        for k in sorted({1, 2, max(1, n // 2), n}):
+            conf = rng.integers(0, 3, size=(300, n)).astype(np.float32) / 2
+            conf[rng.random((300, n)) < 0.2] = -np.inf
+            conf[rng.random((300, n)) < 0.05] = np.nan
+            z = rng.random((300, n)) < 0.1
+            conf[z] = np.where(rng.random(z.sum()) < 0.5, 0.0, -0.0)
+            conf[rng.random((300, n)) < 0.03] = np.inf
+            p, s = gpu_unmask(conf, k)
+            op, os_ = orc.unmask(conf, k)
+            assert np.array_equal(p, op) and np.array_equal(s, os_), (n, k)
+
+
+def test_unmask_workload_confidences(orc):
+    for name, cfg in W.WORKLOADS.items():
+        wl = W.make_workload(name, seed=0, batch=min(cfg["batch"], 16),
+                             prefix_override=[64] * min(cfg["batch"], 16))
+        for conf in wl.conf:
+            for k in wl.unmask_k:
+                big = np.concatenate([conf, W.make_confidences(np.random.default_rng(5), 500, cfg["bl"], cfg["conf"])])
+                assert all(np.array_equal(a, b) for a, b in zip(gpu_unmask(big, k), orc.unmask(big, k)))
+
+
+def test_unmask_denoising_chain(orc):
+    """Four successive top-8 steps on a 32-position block; committed positions
+    become -inf (the 14B-shape diffusion steps). Each side chains its own result."""
+    rng = np.random.default_rng(14)
+    B, n, k = 16, 32, 8
+    conf_steps = [W.make_confidences(rng, B, n, "uniform") for _ in range(4)]
+    committed_g = np.zeros((B, n), dtype=bool)
+    committed_o = np.zeros((B, n), dtype=bool)
+    for c in conf_steps:
+        cg = np.where(committed_g, -np.inf, c).astype(np.float32)
+        co = np.where(committed_o, -np.inf, c).astype(np.float32)
+        pg, sg = gpu_unmask(cg, k)
+        po, so = orc.unmask(co, k)
+        assert np.array_equal(pg, po) and np.array_equal(sg, so)
+        for b in range(B):
+            committed_g[b, pg[b][pg[b] >= 0]] = True
+            committed_o[b, po[b][po[b] >= 0]] = True
+    assert committed_g.all(), "4 x top-8 fills the 32-token block"
+
+
+# ---------------------------------------------------------------------------
+# split combine
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("S,D", [(1, 128), (2, 64), (7, 128), (64, 128), (128, 64)])
+def test_combine_matches_oracle(orc, S, D):
+    rng = np.random.default_rng(S * 1000 + D)
+    B, Hq, bl = 3, 8, 5
+    o = rng.standard_normal((S, B, Hq, bl, D)).astype(np.float32)
+    l = (rng.standard_normal((S, B, Hq, bl)) * 3).astype(np.float32)
+    l[rng.random(l.shape) < 0.3] = -np.inf
+    l[:, 0, 0, 0] = -np.inf  # a row with no keys at all
+    o[np.broadcast_to((l == -np.inf)[..., None], o.shape)] = np.nan  # never read
+    out = torch.empty((B, bl, Hq, D), dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty((B, Hq, bl), dtype=torch.float32, device="cuda")
+    nld.nld_split_kv_combine(torch.from_numpy(o).cuda(), torch.from_numpy(l).cuda(), out, lse)
+    ro, rl = orc.combine(np.nan_to_num(o, nan=0.0).reshape(S, -1, D), l.reshape(S, -1))
+    ro = ro.reshape(B, Hq, bl, D).transpose(0, 2, 1, 3)
+    rl = rl.reshape(B, Hq, bl)
+    got = out.float().cpu().numpy()
+    assert np.all(np.isfinite(got))
+    assert np.max(np.abs(got - ro)) <= 1e-2
+    gl = lse.cpu().numpy()
+    assert np.array_equal(np.isinf(gl), np.isinf(rl))
+    fin = np.isfinite(rl)
+    assert np.max(np.abs(gl[fin] - rl[fin])) <= 1e-4
+
+
+# ---------------------------------------------------------------------------
+# attention: small cases, every row
+# ---------------------------------------------------------------------------
+
+SMALL = [
+    # name, B, Hq, Hkv, D, P, bl, prefix lens
+    ("tinyshape", 1, 4, 1, 64, 256, 8, [256]),
+    ("d128_g4_bl16", 2, 8, 2, 128, 16, 16, [300, 77]),
+    ("d64_g2_bl5_ragged", 3, 4, 2, 64, 32, 5, [0, 13, 200]),
+    ("d128_g5_bl32", 1, 10, 2, 128, 16, 32, [500]),
+    ("d128_mha_bl1", 2, 4, 4, 128, 64, 1, [63, 64]),
+    ("d128_g8_bl20_p128", 2, 16, 2, 128, 128, 20, [129, 1000]),
+    ("d64_g1_bl32_p16", 1, 2, 2, 64, 16, 32, [31]),
+    ("prefix0_bl32", 2, 8, 2, 128, 16, 32, [0, 0]),
+]
+
+
+@pytest.mark.parametrize("spec", SMALL, ids=[s[0] for s in SMALL])
+@pytest.mark.parametrize("mode", [DIFF, VER], ids=["diffusion", "verify"])
+@pytest.mark.parametrize("splits", [0, 1, 3])
+def test_attention_small_all_rows(orc, spec, mode, splits):
+    name, B, Hq, Hkv, D, P, bl, prefix = spec
+    case = W.make_block_attn_case(name, B, Hq, Hkv, D, bl, P, prefix, seed=sum(prefix) + bl)
+    dc = DeviceCase(case)
+    out, lse = dc.run(mode, num_splits=splits)
+    ro, rl = oracle_full(orc, case, mode)
+    compare_attn(out, lse, ro, rl, f"{name} mode={mode} S={splits}")
+
+
+def test_attention_tail_slots_hold_nan(orc):
+    """Cache slots past the block inside the last page may be uninitialised;
+    NaN there must not reach the output."""
+    case = W.make_block_attn_case("nan_tail", 2, 8, 2, 128, 7, 16, [37, 100], seed=3)
+    kv = case.kv
+    k_bits, v_bits = kv.k_bits.copy(), kv.v_bits.copy()
+    nan = np.uint16(0x7FC0)
+    for b, L in enumerate(kv.prefix_lens):
+        N = int(L) + case.block_len
+        for t in range(N, ((N + 15) // 16) * 16):  # rest of the last page
+            page, slot = kv.page_table[b, t // kv.page_size], t % kv.page_size
+            k_bits[page, :, slot, :] = nan
+            v_bits[page, :, slot, :] = nan
+    case2 = W.BlockAttnCase(case.name, case.batch, case.num_q_heads, case.num_kv_heads, case.head_dim,
+                            case.block_len, case.scale, case.q_draft_bits, case.q_verify_bits,
+                            W.PagedKV(k_bits, v_bits, kv.page_table, kv.prefix_lens, kv.page_size,
+                                      kv.num_pages, kv.max_pages))
+    dc = DeviceCase(case2)
+    for mode in (DIFF, VER):
+        for splits in (1, 2):
+            out, lse = dc.run(mode, num_splits=splits)
+            ro, rl = oracle_full(orc, case2, mode)
+            compare_attn(out, lse, ro, rl, f"nan tail mode={mode} S={splits}")
+
+
+def test_attention_split_sweep(orc):
+    case = W.make_block_attn_case("sweep", 1, 8, 2, 128, 16, 16, [1000], seed=9)
+    dc = DeviceCase(case)
+    ro, rl = oracle_full(orc, case, VER)
+    for S in (1, 2, 3, 4, 8, 16, 32, 64, 128):
+        out, lse = dc.run(VER, num_splits=S)
+        compare_attn(out, lse, ro, rl, f"S={S}")
+
+
+# ---------------------------------------------------------------------------
+# attention: self-consistency on the GPU
+# ---------------------------------------------------------------------------
+
+def test_page_permutation_is_bit_identical():
+    case = W.make_block_attn_case("perm", 2, 8, 2, 128, 16, 16, [333, 90], seed=4)
+    kv = case.kv
+    perm = np.random.default_rng(1).permutation(kv.num_pages)
+    k2, v2 = np.empty_like(kv.k_bits), np.empty_like(kv.v_bits)
+    k2[perm], v2[perm] = kv.k_bits, kv.v_bits
+    t2 = np.where(kv.page_table >= 0, perm[np.maximum(kv.page_table, 0)], -1).astype(np.int32)
+    case2 = W.BlockAttnCase(case.name, case.batch, case.num_q_heads, case.num_kv_heads, case.head_dim,
+                            case.block_len, case.scale, case.q_draft_bits, case.q_verify_bits,
+                            W.PagedKV(k2, v2, t2, kv.prefix_lens, kv.page_size, kv.num_pages, kv.max_pages))
+    a, b = DeviceCase(case), DeviceCase(case2)
+    for mode in (DIFF, VER):
+        for S in (1, 4):
+            oa, la = a.run(mode, S)
+            ob, lb = b.run(mode, S)
+            assert torch.equal(oa, ob) and torch.equal(la, lb)
+
+
+def test_block_len_one_modes_agree():
+    case = W.make_block_attn_case("bl1", 3, 32, 8, 128, 16, 1, [5, 700, 4096], seed=5)
+    dc = DeviceCase(case)
+    q = dc.q[DIFF]
+    for S in (1, 0):
+        od, ld = dc.run(DIFF, S, q=q)
+        ov, lv = dc.run(VER, S, q=q)
+        assert torch.equal(od, ov) and torch.equal(ld, lv)
+
+
+def test_device_clamps_bad_prefix_and_page_ids():
+    """Out-of-range device values are clamped (no access leaves the buffers)
+    and flagged in the device error word."""
+    case = W.make_block_attn_case("bad", 2, 8, 2, 64, 16, 8, [40, 10], seed=6)
+    dc = DeviceCase(case)
+    nld.nld_device_error(clear=True)
+    dc.prefix = torch.tensor([10 ** 6, -5], dtype=torch.int32, device="cuda")
+    dc.run(VER, 2)
+    torch.cuda.synchronize()
+    assert nld.nld_device_error(clear=True) & nld.NLD_DEVERR_PREFIX_RANGE
+    dc = DeviceCase(case)
+    dc.table[0, 0] = 10 ** 6
+    dc.table[1, 0] = -3
+    dc.run(DIFF, 1)
+    torch.cuda.synchronize()
+    assert nld.nld_device_error(clear=True) & nld.NLD_DEVERR_PAGE_RANGE
+
+
+def test_workspace_too_small_launches_nothing():
+    case = W.make_block_attn_case("ws", 1, 8, 2, 128, 16, 16, [500], seed=7)
+    dc = DeviceCase(case)
+    p = dc.params(4)
+    need = nld.nld_block_attn_workspace_size(p, 16)
+    out = torch.zeros((1, 16, 8, 128), dtype=torch.bfloat16, device="cuda")
+    ws = torch.empty(need - 16, dtype=torch.uint8, device="cuda")
+    with pytest.raises(nld.NldError) as e:
+        nld.nld_block_attn(p, dc.q[VER], dc.k, dc.v, dc.table, dc.prefix, 16, VER, out, None, ws)
+    assert e.value.status == 3
+    torch.cuda.synchronize()
+    assert torch.count_nonzero(out) == 0
+
+
+# ---------------------------------------------------------------------------
+# attention: the named workloads at full size, sampled rows
+# ---------------------------------------------------------------------------
+
+FULL = ["tiny_b1_h4x1_d64_L256_bl8", "8b_b1_h32x8_d128_L4096_bl16", "long_b1_h32x8_d128_L32768_bl32",
+        "14b_b16_h40x8_d128_L8k-16k_bl32", "conc_b8_h32x8_d128_L512-8192_bl8", "conc_b128_h32x8_d128_L512-8192_bl8"]
+
+
+@pytest.mark.parametrize("name", FULL)
+def test_full_size_workload_sampled_rows(orc, name):
+    wl = W.make_workload(name, seed=0)
+    case = wl.attn
+    dc = DeviceCase(case)
+    for mode in (DIFF, VER):
+        if mode == DIFF and "diffusion" not in wl.steps:
+            continue
+        out, lse = dc.run(mode)  # automatic split count, as the bench runs it
+        rows = sample_rows(case, 48, seed=mode + 1)
+        qb = dc.q_bits(mode)
+        ro, rl = orc.block_attn_rows(qb, case.kv.k_bits, case.kv.v_bits, case.kv.page_table, case.kv.prefix_lens,
+                                     case.num_q_heads, case.num_kv_heads, case.block_len, mode, case.scale, rows)
+        o = out[rows[:, 0], rows[:, 1], rows[:, 2]]
+        l = lse[rows[:, 0], rows[:, 2], rows[:, 1]]
+        compare_attn(o, l, ro, rl, f"{name} mode={mode}")
+        assert torch.isfinite(out.float()).all()
+
+
+def test_long_context_split_sweep_sampled(orc):
+    wl = W.make_workload("long_b1_h32x8_d128_L32768_bl32", seed=1)
+    case = wl.attn
+    dc = DeviceCase(case)
+    rows = sample_rows(case, 24, seed=3)
+    ro, rl = orc.block_attn_rows(case.q_verify_bits, case.kv.k_bits, case.kv.v_bits, case.kv.page_table,
+                                 case.kv.prefix_lens, case.num_q_heads, case.num_kv_heads, case.block_len, VER,
+                                 case.scale, rows)
+    for S in (1, 2, 4, 8, 16, 32, 64):
+        out, lse = dc.run(VER, S)
+        compare_attn(out[rows[:, 0], rows[:, 1], rows[:, 2]], lse[rows[:, 0], rows[:, 2], rows[:, 1]], ro, rl,
+                     f"long S={S}")
