@@ -4,8 +4,10 @@
 // heads times the bl block tokens are packed into R = G*bl query rows, so each
 // K/V page is read from HBM once per (b, g) and feeds every row of the group.
 //
+// This is the mma.sync variant, used when more than 128 query rows are packed
+// (the tcgen05 kernel in block_attn_tc.cu covers up to 128).
 // Warp roles: warps 0 .. nwr*nwt-1 compute, the last warp streams K/V.
-//   - Producer: one thread issues 4-D TMA loads (16 tokens x 64 dims per box,
+//   - Producer (produce_kv): 4-D TMA loads (16 tokens x 64 dims per box,
 //     128-byte swizzle) of the pages of each 64-token tile into an nstage-deep
 //     ring of shared-memory stages, completing on a "full" mbarrier per stage;
 //     it refills a stage after the compute warps release its "empty" mbarrier.
@@ -20,21 +22,6 @@
 
 namespace nld {
 namespace {
-
-template <int D>
-struct TileGeom {
-  static constexpr int kColBlocks = D / 64;                 // 128-byte column blocks per row
-  static constexpr int kColBlockBytes = kTileTok * 128;     // one column block of a tile
-  static constexpr int kTileBytes = kColBlocks * kColBlockBytes;  // K (or V) tile
-  static constexpr int kStageBytes = 2 * kTileBytes;        // K + V
-};
-
-// Byte offset of (token r, 16-byte chunk c) in a tile written by TMA with the
-// 128-byte swizzle: within each 8-row x 128-byte atom, chunk c of row r sits
-// at chunk position c ^ (r % 8). Column blocks (64 dims each) are stacked.
-__device__ __forceinline__ uint32_t swz(int r, int c) {
-  return static_cast<uint32_t>((c >> 3) * (kTileTok * 128) + r * 128 + (((c & 7) ^ (r & 7)) << 4));
-}
 
 // Largest CTA per token split: nwt = 4 and 2 serve up to 2 and 4 row warps,
 // nwt = 1 up to kMaxRows / 16; plus the producer warp.
@@ -64,6 +51,21 @@ __global__ void __launch_bounds__(MaxWarps<NWT>::value * 32, 1)
   const int ncons = a.nwr * NWT;
 
   const int split = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < nstage; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], ncons);
+    }
+    fence_mbar_init();
+  }
+  if (warp == ncons && lane == 0) {
+    prefetch_tensormap(&tmk);
+    prefetch_tensormap(&tmv);
+  }
+  grid_dependency_wait();
+  grid_launch_dependents();
+  __syncthreads();
+
   const int lmax = a.max_pages * a.page_size - a.bl;
   int L = __ldg(a.prefix_lens + b);
   if (L < 0 || L > lmax) {
@@ -84,49 +86,8 @@ __global__ void __launch_bounds__(MaxWarps<NWT>::value * 32, 1)
   }
   const int ntiles = (t_end - t_begin + kTileTok - 1) / kTileTok;
 
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < nstage; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], ncons);
-    }
-    fence_mbar_init();
-  }
-  __syncthreads();
-
   if (warp == ncons) {
-    // ---------------- producer: stream this split's K/V pages ----------------
-    if (lane == 0) {
-      prefetch_tensormap(&tmk);
-      prefetch_tensormap(&tmv);
-      const int32_t* ptab = a.page_table + static_cast<size_t>(b) * a.max_pages;
-      for (int k = 0; k < ntiles; ++k) {
-        const int st = k % nstage;
-        if (k >= nstage && !mbar_wait(&empty[st], ((k / nstage) - 1) & 1, a.err)) break;
-        mbar_arrive_expect_tx(&full[st], Geo::kStageBytes);
-        uint8_t* kt = smem + st * Geo::kStageBytes;
-        uint8_t* vt = kt + Geo::kTileBytes;
-#pragma unroll
-        for (int grp = 0; grp < kTileTok / kGroupTok; ++grp) {
-          const int t = t_begin + k * kTileTok + grp * kGroupTok;
-          int page = a.num_pages;  // past the pool: TMA fills the box with zeros
-          int slot = 0;
-          if (t < t_end) {
-            page = __ldg(ptab + (t >> a.log2_page));
-            if (page < 0 || page >= a.num_pages) {
-              atomicOr(a.err, NLD_DEVERR_PAGE_RANGE);
-              page = min(max(page, 0), a.num_pages - 1);
-            }
-            slot = t & (a.page_size - 1);
-          }
-#pragma unroll
-          for (int cb = 0; cb < Geo::kColBlocks; ++cb) {
-            const int off = cb * Geo::kColBlockBytes + grp * kGroupTok * 128;
-            tma_load_4d(kt + off, &tmk, &full[st], cb * 64, slot, g, page);
-            tma_load_4d(vt + off, &tmv, &full[st], cb * 64, slot, g, page);
-          }
-        }
-      }
-    }
+    produce_kv<D>(a, &tmk, &tmv, smem, full, empty, nstage, g, b, t_begin, t_end, ntiles, lane);
     return;
   }
 
@@ -195,7 +156,7 @@ __global__ void __launch_bounds__(MaxWarps<NWT>::value * 32, 1)
         const int tok = wt * TW + jn * 8 + (lane & 7) + ((lane >> 4) << 3);
         const int chunk = kk * 2 + ((lane >> 3) & 1);
         uint32_t b0, b1, b2, b3;
-        ldsm_x4(kbase + swz(tok, chunk), b0, b1, b2, b3);
+        ldsm_x4(kbase + kv_swz(tok, chunk), b0, b1, b2, b3);
         mma_16816(s[jn], qa[kk], b0, b1);
         mma_16816(s[jn + 1], qa[kk], b2, b3);
       }
@@ -264,7 +225,7 @@ __global__ void __launch_bounds__(MaxWarps<NWT>::value * 32, 1)
         const int tok = tok_base + (lane & 7) + (((lane >> 3) & 1) << 3);
         const int chunk = dn + (lane >> 4);
         uint32_t b0, b1, b2, b3;
-        ldsm_x4_t(vbase + swz(tok, chunk), b0, b1, b2, b3);
+        ldsm_x4_t(vbase + kv_swz(tok, chunk), b0, b1, b2, b3);
         if (tail) {
           // b0/b2 hold tokens tok_base + qc + {0,1}; b1/b3 the same + 8.
           const int t0 = tok_base + qc, t1 = t0 + 8;
@@ -380,8 +341,7 @@ cudaError_t launch_t(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMa
     __atomic_store_n(&configured[dev], 1, __ATOMIC_RELEASE);
   }
   dim3 grid(a.num_splits, a.Hkv, a.B);
-  kern<<<grid, sh.threads, sh.smem, stream>>>(tmk, tmv, a);
-  return cudaGetLastError();
+  return launch_kernel(kern, grid, dim3(sh.threads), sh.smem, stream, tmk, tmv, a);
 }
 
 }  // namespace

@@ -1,0 +1,403 @@
+// Block attention over a paged bf16 KV cache on the 5th-generation tensor
+// cores (tcgen05, accumulators in tensor memory), for up to 128 packed query
+// rows (Sec. 2.2 mask; Sec. 3 Modes 2 and 3).
+//
+// One CTA serves one (KV split, KV head g, sequence b): its G = Hq/Hkv query
+// heads times the bl block tokens form R = G*bl <= 128 query rows, padded to
+// the 128-row MMA tile, so each K/V page leaves HBM once per (b, g).
+//
+// Warp roles (6 warps):
+//   warp 0    TMA producer: 64-token K/V tiles into a 4-stage ring (produce_kv).
+//   warp 1    allocates 256 TMEM columns; lane 0 issues every MMA:
+//               S_k = Q K_k^T   (M=128 rows, N=64 tokens, K=D; double-buffered in TMEM)
+//               O  += P_k V_k   (M=128 rows, N=D, K=64 tokens; V read MN-major)
+//             S_{k+1} is issued before O += P_k V_k so the tensor core computes
+//             the next scores while the softmax warps work on the current ones.
+//   warps 2-5 softmax: thread t owns query row 32*(warp%4)+lane (its TMEM lane).
+//             It loads its S row, applies the mask and the base-2 scale,
+//             keeps the running max and sum, writes P (bf16) to shared memory
+//             for the PV MMA, and at the end reads O from TMEM, divides by the
+//             sum and stores the row (or the split partial).
+// The running max is raised lazily: O is rescaled in TMEM only when a row's
+// max grows by more than 2^8 (P then stays below 256, exact enough in bf16);
+// the final division by the matching sum removes the reference max.
+#include "nld_internal.cuh"
+
+namespace nld {
+namespace {
+
+constexpr int kTcStages = 4;
+constexpr int kTcThreads = 192;
+constexpr uint32_t kTmemCols = 256;  // S0 | S1 (64 columns each) | O (D <= 128 columns)
+constexpr float kRescaleLog2 = 8.0f;
+
+template <int D>
+struct TcLayout {
+  using Geo = TileGeom<D>;
+  static constexpr int kQBytes = Geo::kColBlocks * 128 * 128;  // 128 rows x D bf16
+  static constexpr int kPBytes = 128 * kTileTok * 2;             // 128 rows x 64 tokens bf16
+  static constexpr int kQOff = kTcStages * Geo::kStageBytes;
+  static constexpr int kPOff = kQOff + kQBytes;
+  static constexpr int kBarOff = kPOff + 2 * kPBytes;
+  // kv_full[4], kv_empty[4], s_full[2], s_free[2], p_full[2], o_done[2], q_ready, drain, tmem slot
+  static constexpr int kNumBars = 2 * kTcStages + 8 + 2;
+  static constexpr int kBytes = kBarOff + kNumBars * 8 + 16;
+};
+
+template <int D>
+__global__ void __launch_bounds__(kTcThreads, 1)
+    block_attn_tc_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
+                         const AttnArgs a) {
+  using Geo = TileGeom<D>;
+  using Lay = TcLayout<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* q_s = smem + Lay::kQOff;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Lay::kBarOff);
+  uint64_t* kv_full = bars;
+  uint64_t* kv_empty = bars + kTcStages;
+  uint64_t* s_full = bars + 2 * kTcStages;
+  uint64_t* s_free = s_full + 2;
+  uint64_t* p_full = s_free + 2;
+  uint64_t* o_done = p_full + 2;
+  uint64_t* q_ready = o_done + 2;
+  uint64_t* drain = q_ready + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int split = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kTcStages; ++s) {
+      mbar_init(&kv_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
+    }
+    for (int j = 0; j < 2; ++j) {
+      mbar_init(&s_full[j], 1);
+      mbar_init(&s_free[j], 4);
+      mbar_init(&p_full[j], 4);
+      mbar_init(&o_done[j], 1);
+    }
+    mbar_init(q_ready, 4);
+    mbar_init(drain, 1);
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    prefetch_tensormap(&tmk);
+    prefetch_tensormap(&tmv);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tc_fence_before();
+  }
+  grid_dependency_wait();
+  grid_launch_dependents();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t tS0 = tmem, tS1 = tmem + kTileTok, tO = tmem + 2 * kTileTok;
+
+  const int lmax = a.max_pages * a.page_size - a.bl;
+  int L = __ldg(a.prefix_lens + b);
+  if (L < 0 || L > lmax) {
+    if (threadIdx.x == 0) atomicOr(a.err, NLD_DEVERR_PREFIX_RANGE);
+    L = min(max(L, 0), lmax);
+  }
+  const int N = L + a.bl;
+  const int t_begin = split * a.chunk;
+  const int t_end = min(t_begin + a.chunk, N);
+  const int ntiles = t_begin < t_end ? (t_end - t_begin + kTileTok - 1) / kTileTok : 0;
+
+  if (ntiles == 0) {
+    // This split lies past the sequence: its partials carry no keys.
+    for (int r = threadIdx.x; r < a.R; r += blockDim.x) {
+      const int i = r / a.G, h = g * a.G + (r - i * a.G);
+      a.lse_part[((static_cast<size_t>(split) * a.B + b) * a.Hq + h) * a.bl + i] = -INFINITY;
+    }
+  } else if (warp == 0) {
+    // ---------------- producer ----------------
+    const int issued = produce_kv<D>(a, &tmk, &tmv, smem, kv_full, kv_empty, kTcStages, g, b, t_begin, t_end,
+                                     ntiles, lane);
+    if (lane == 0 && issued < ntiles) {
+      // Stopped early on a wait timeout: let the copies already issued land
+      // before the CTA exits (bounded).
+      for (int k = max(0, issued - kTcStages); k < issued; ++k)
+        mbar_wait(&kv_full[k % kTcStages], (k / kTcStages) & 1, a.err);
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      bool ok = mbar_wait(q_ready, 0, a.err);
+      tc_fence_after();
+      const uint32_t q_addr = smem_u32(q_s);
+      const uint32_t idesc_s = umma_idesc_bf16(128, kTileTok, false);
+      const uint32_t idesc_o = umma_idesc_bf16(128, D, true);
+      auto issue_s = [&](int k) -> bool {
+        const int st = k % kTcStages;
+        if (!mbar_wait(&kv_full[st], (k / kTcStages) & 1, a.err)) return false;
+        if (k >= 2 && !mbar_wait(&s_free[k & 1], ((k - 2) >> 1) & 1, a.err)) return false;
+        tc_fence_after();
+        const uint32_t k_addr = smem_u32(smem + st * Geo::kStageBytes);
+        const uint32_t d = (k & 1) ? tS1 : tS0;
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t koff = (kk & 3) * 32;  // 16 elements along the 128-byte row
+          const int cb = kk >> 2;               // 64-dim column block
+          const uint64_t ad = sw128_desc(q_addr + cb * (128 * 128) + koff, 0, 1024);
+          const uint64_t bd = sw128_desc(k_addr + cb * Geo::kColBlockBytes + koff, 0, 1024);
+          umma_bf16(d, ad, bd, idesc_s, kk > 0 ? 1u : 0u);
+        }
+        umma_commit(&s_full[k & 1]);
+        return true;
+      };
+      if (ok) ok = issue_s(0);
+      for (int k = 0; ok && k < ntiles; ++k) {
+        if (k + 1 < ntiles && !issue_s(k + 1)) {
+          ok = false;
+          break;
+        }
+        if (!mbar_wait(&p_full[k & 1], (k >> 1) & 1, a.err)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const int st = k % kTcStages;
+        const uint32_t p_addr = smem_u32(smem + Lay::kPOff + (k & 1) * Lay::kPBytes);
+        const uint32_t v_addr = smem_u32(smem + st * Geo::kStageBytes + Geo::kTileBytes);
+#pragma unroll
+        for (int kt = 0; kt < kTileTok / 16; ++kt) {
+          // A = P rows (K-major, one 128-byte block of 64 tokens); B = V (MN-major:
+          // 64-dim atoms LBO apart, 8-token row groups SBO apart).
+          const uint64_t ad = sw128_desc(p_addr + kt * 32, 0, 1024);
+          const uint64_t bd = sw128_desc(v_addr + kt * 16 * 128, Geo::kColBlockBytes, 1024);
+          umma_bf16(tO, ad, bd, idesc_o, (k > 0 || kt > 0) ? 1u : 0u);
+        }
+        umma_commit(&o_done[k & 1]);
+        umma_commit(&kv_empty[st]);
+      }
+      if (!ok) {
+        // Let every MMA already issued finish before TMEM is released (bounded).
+        umma_commit(drain);
+        mbar_wait(drain, 0, a.err);
+      }
+    }
+    __syncwarp();
+  } else {
+    // ---------------- softmax warps ----------------
+    const int quad = warp & 3;
+    const int r = quad * 32 + lane;  // query row == TMEM lane
+    const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+    const bool warp_rows = quad * 32 < a.R;  // warp-uniform: the warp holds a real row
+    const bool row_ok = r < a.R;
+    const int row_i = r / a.G;
+    const int row_h = g * a.G + (r - row_i * a.G);
+    const int sm_tid = threadIdx.x - 64;  // 0..127 across the softmax warps
+
+    // Q row -> shared memory in the 128-byte-swizzled K-major layout; padding
+    // rows are zero. Padding rows of P are zeroed once for both buffers.
+    {
+      const uint4* qrow = reinterpret_cast<const uint4*>(
+          a.q + ((static_cast<size_t>(b) * a.bl + row_i) * a.Hq + row_h) * D);
+#pragma unroll
+      for (int c = 0; c < D / 8; ++c) {
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (row_ok) v = __ldg(qrow + c);
+        *reinterpret_cast<uint4*>(q_s + (c >> 3) * (128 * 128) + r * 128 + (((c & 7) ^ (r & 7)) << 4)) = v;
+      }
+      if (!row_ok) {
+#pragma unroll
+        for (int j = 0; j < 2; ++j)
+#pragma unroll
+          for (int c = 0; c < 8; ++c)
+            *reinterpret_cast<uint4*>(smem + Lay::kPOff + j * Lay::kPBytes + r * 128 + ((c ^ (r & 7)) << 4)) =
+                make_uint4(0, 0, 0, 0);
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(q_ready);
+    }
+
+    float m_run = -INFINITY, l_run = 0.f;
+    bool ok = true;
+    for (int k = 0; k < ntiles; ++k) {
+      const int buf = k & 1;
+      const int st = k % kTcStages;
+      const int tile_t0 = t_begin + k * kTileTok;
+      const int valid = t_end - tile_t0;
+      if (!mbar_wait(&s_full[buf], (k >> 1) & 1, a.err)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      float s[kTileTok];
+      if (warp_rows) {
+        const uint32_t ts = (buf ? tS1 : tS0) + lane_off;
+        tmem_ld32(ts, s);
+        tmem_ld32(ts + 32, s + 32);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_free[buf]);
+
+      float alpha = 1.f;
+      bool rescale = false;
+      if (warp_rows) {
+        const bool all_visible = (tile_t0 + kTileTok <= L) && (valid >= kTileTok);
+        float mx = -INFINITY;
+#pragma unroll
+        for (int j = 0; j < kTileTok; ++j) {
+          float v = s[j] * a.scale_log2;
+          if (!all_visible) {
+            const int t = tile_t0 + j;
+            const bool vis = j < valid && (t < L || a.mode == NLD_MODE_DIFFUSION || t - L <= row_i);
+            v = vis ? v : -INFINITY;
+          }
+          s[j] = v;
+          mx = fmaxf(mx, v);
+        }
+        if (m_run == -INFINITY) {
+          m_run = mx;  // nothing accumulated for this row yet
+        } else if (mx > m_run + kRescaleLog2) {
+          alpha = ex2(m_run - mx);
+          m_run = mx;
+          l_run *= alpha;
+          rescale = true;
+        }
+      }
+      if (__any_sync(0xffffffffu, rescale)) {
+        // O holds P_0..P_{k-1} V: wait for the last PV, then scale this warp's rows.
+        if (!mbar_wait(&o_done[(k - 1) & 1], ((k - 1) >> 1) & 1, a.err)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+#pragma unroll 1
+        for (int c = 0; c < D / 32; ++c) {
+          float o[32];
+          tmem_ld32(tO + lane_off + c * 32, o);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) o[j] *= alpha;
+          tmem_st32(tO + lane_off + c * 32, o);
+        }
+      }
+      // P buffer `buf` is free once the PV of tile k-2 has completed.
+      if (k >= 2 && !mbar_wait(&o_done[buf], ((k - 2) >> 1) & 1, a.err)) {
+        ok = false;
+        break;
+      }
+      if (warp_rows) {
+        const float mu = m_run == -INFINITY ? 0.f : m_run;
+        uint8_t* prow = smem + Lay::kPOff + buf * Lay::kPBytes + r * 128;
+#pragma unroll
+        for (int c = 0; c < kTileTok / 8; ++c) {
+          uint32_t w[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float p0 = ex2(s[c * 8 + 2 * e] - mu);
+            const float p1 = ex2(s[c * 8 + 2 * e + 1] - mu);
+            l_run += p0 + p1;
+            w[e] = pack_bf16(p0, p1);
+          }
+          *reinterpret_cast<uint4*>(prow + ((c ^ (r & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+      }
+      if (valid < kTileTok && (valid & (kGroupTok - 1))) {
+        // Cache slots past the sequence end inside its last page may hold
+        // stale or uninitialised data; P is 0 there but 0 * NaN = NaN, so
+        // zero those V rows before the PV MMA reads them.
+        if (!mbar_wait(&kv_full[st], (k / kTcStages) & 1, a.err)) {
+          ok = false;
+          break;
+        }
+        const int r0 = valid, r1 = (valid + kGroupTok - 1) & ~(kGroupTok - 1);
+        uint8_t* vt = smem + st * Geo::kStageBytes + Geo::kTileBytes;
+        for (int idx = sm_tid; idx < (r1 - r0) * (D / 8); idx += 128) {
+          const int row = r0 + idx / (D / 8), c = idx % (D / 8);
+          *reinterpret_cast<uint4*>(vt + kv_swz(row, c)) = make_uint4(0, 0, 0, 0);
+        }
+      }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_full[buf]);
+    }
+
+    // ---------------- epilogue ----------------
+    if (ok && mbar_wait(&o_done[(ntiles - 1) & 1], ((ntiles - 1) >> 1) & 1, a.err)) {
+      tc_fence_after();
+      if (warp_rows) {
+        const float l = l_run;
+        const float inv = l > 0.f ? 1.f / l : 0.f;
+        const float lse_v = l > 0.f ? (m_run + lg2(l)) * kLn2 : -INFINITY;
+        const bool split_out = a.o_part != nullptr;
+        const size_t orow = (static_cast<size_t>(b) * a.bl + row_i) * a.Hq + row_h;
+        const size_t prow = ((static_cast<size_t>(split) * a.B + b) * a.Hq + row_h) * a.bl + row_i;
+#pragma unroll 1
+        for (int c = 0; c < D / 32; ++c) {
+          float o[32];
+          tmem_ld32(tO + lane_off + c * 32, o);
+          if (!row_ok) continue;
+          if (!split_out) {
+            uint4* dst = reinterpret_cast<uint4*>(a.out + orow * D + c * 32);
+#pragma unroll
+            for (int q4 = 0; q4 < 4; ++q4) {
+              const int j = q4 * 8;
+              dst[q4] = make_uint4(pack_bf16(o[j] * inv, o[j + 1] * inv), pack_bf16(o[j + 2] * inv, o[j + 3] * inv),
+                                   pack_bf16(o[j + 4] * inv, o[j + 5] * inv), pack_bf16(o[j + 6] * inv, o[j + 7] * inv));
+            }
+          } else if (l > 0.f) {
+            float4* dst = reinterpret_cast<float4*>(a.o_part + prow * D + c * 32);
+#pragma unroll
+            for (int q4 = 0; q4 < 8; ++q4)
+              dst[q4] = make_float4(o[4 * q4] * inv, o[4 * q4 + 1] * inv, o[4 * q4 + 2] * inv, o[4 * q4 + 3] * inv);
+          }
+        }
+        if (row_ok) {
+          if (!split_out) {
+            if (a.lse != nullptr) a.lse[(static_cast<size_t>(b) * a.Hq + row_h) * a.bl + row_i] = lse_v;
+          } else {
+            a.lse_part[prow] = lse_v;
+          }
+        }
+      }
+    }
+    tc_fence_before();
+  }
+
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+template <int D>
+cudaError_t launch_tc_t(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, cudaStream_t stream) {
+  auto kern = block_attn_tc_kernel<D>;
+  const size_t smem = TcLayout<D>::kBytes + 1024;
+  static int configured[64] = {0};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (!__atomic_load_n(&configured[dev], __ATOMIC_ACQUIRE)) {
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    __atomic_store_n(&configured[dev], 1, __ATOMIC_RELEASE);
+  }
+  dim3 grid(a.num_splits, a.Hkv, a.B);
+  return launch_kernel(kern, grid, dim3(kTcThreads), smem, stream, tmk, tmv, a);
+}
+
+}  // namespace
+
+bool tc_supports(int R, int head_dim) { return R <= 128 && (head_dim == 64 || head_dim == 128); }
+
+cudaError_t launch_block_attn_tc(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, int head_dim,
+                                 cudaStream_t stream) {
+  if (head_dim == 128) return launch_tc_t<128>(a, tmk, tmv, stream);
+  return launch_tc_t<64>(a, tmk, tmv, stream);
+}
+
+}  // namespace nld

@@ -16,6 +16,8 @@ __global__ void __launch_bounds__(kCombineWarps * 32)
     combine_kernel(const float* __restrict__ o_part, const float* __restrict__ lse_part, int S, int B, int Hq,
                    int bl, __nv_bfloat16* __restrict__ out, float* __restrict__ lse) {
   constexpr int V = D / 32;  // dims per lane (2 or 4)
+  grid_dependency_wait();
+  grid_launch_dependents();
   const int lane = threadIdx.x & 31;
   const long row = static_cast<long>(blockIdx.x) * kCombineWarps + (threadIdx.x >> 5);
   const long R = static_cast<long>(B) * Hq * bl;
@@ -26,8 +28,16 @@ __global__ void __launch_bounds__(kCombineWarps * 32)
   const int h = static_cast<int>(bh % Hq);
   const int b = static_cast<int>(bh / Hq);
 
+  // Lane j holds lse of splits j, j+32, j+64, j+96 (S <= 128): all loads in flight at once.
+  constexpr int kMaxPerLane = kMaxSplits / 32;
+  float ls[kMaxPerLane];
   float m = -INFINITY;
-  for (int s = lane; s < S; s += 32) m = fmaxf(m, __ldg(lse_part + static_cast<long>(s) * R + row));
+#pragma unroll
+  for (int u = 0; u < kMaxPerLane; ++u) {
+    const int s = lane + 32 * u;
+    ls[u] = s < S ? __ldg(lse_part + static_cast<long>(s) * R + row) : -INFINITY;
+    m = fmaxf(m, ls[u]);
+  }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
 
@@ -37,20 +47,46 @@ __global__ void __launch_bounds__(kCombineWarps * 32)
   float csum = 0.f;
   if (m != -INFINITY) {
     const float m2 = m * kLog2e;
-#pragma unroll 4
-    for (int s = 0; s < S; ++s) {
-      const float ls = __ldg(lse_part + static_cast<long>(s) * R + row);
-      if (ls == -INFINITY) continue;  // no keys in this split: o_s is not read
-      const float c = ex2(ls * kLog2e - m2);
-      csum += c;
-      const float* op = o_part + (static_cast<long>(s) * R + row) * D + lane * V;
-      if constexpr (V == 4) {
-        const float4 x = __ldg(reinterpret_cast<const float4*>(op));
-        acc[0] += c * x.x; acc[1] += c * x.y; acc[2] += c * x.z; acc[3] += c * x.w;
-      } else {
-        const float2 x = __ldg(reinterpret_cast<const float2*>(op));
-        acc[0] += c * x.x; acc[1] += c * x.y;
+    float w[kMaxPerLane];  // weight of split lane + 32u; 0 for empty splits
+#pragma unroll
+    for (int u = 0; u < kMaxPerLane; ++u) {
+      w[u] = ls[u] == -INFINITY ? 0.f : ex2(ls[u] * kLog2e - m2);
+      csum += w[u];
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) csum += __shfl_xor_sync(0xffffffffu, csum, off);
+    // Accumulate 8 splits per round; the loads of a round are independent.
+    const float* base = o_part + static_cast<long>(row) * D + lane * V;
+    const long split_stride = R * static_cast<long>(D);
+    for (int s0 = 0; s0 < S; s0 += 8) {
+      float wv[8];
+      float x[8][V];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int s = s0 + u;
+        const int src = s & 31;
+        const int blk = s >> 5;  // warp-uniform
+        float wsel = blk == 0 ? w[0] : blk == 1 ? w[1] : blk == 2 ? w[2] : w[3];
+        wsel = __shfl_sync(0xffffffffu, wsel, src);
+        wv[u] = s < S ? wsel : 0.f;
+        if (wv[u] != 0.f) {  // warp-uniform: empty splits are never read
+          const float* op = base + s * split_stride;
+          if constexpr (V == 4) {
+            const float4 t = __ldg(reinterpret_cast<const float4*>(op));
+            x[u][0] = t.x; x[u][1] = t.y; x[u][2] = t.z; x[u][3] = t.w;
+          } else {
+            const float2 t = __ldg(reinterpret_cast<const float2*>(op));
+            x[u][0] = t.x; x[u][1] = t.y;
+          }
+        } else {
+#pragma unroll
+          for (int v = 0; v < V; ++v) x[u][v] = 0.f;
+        }
       }
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+#pragma unroll
+        for (int v = 0; v < V; ++v) acc[v] += wv[u] * x[u][v];
     }
   }
   const float inv = csum > 0.f ? 1.f / csum : 0.f;
@@ -69,10 +105,10 @@ cudaError_t launch_combine(const float* o_part, const float* lse_part, int S, in
   const long R = static_cast<long>(B) * Hq * bl;
   const unsigned blocks = static_cast<unsigned>((R + kCombineWarps - 1) / kCombineWarps);
   if (D == 128)
-    combine_kernel<128><<<blocks, kCombineWarps * 32, 0, stream>>>(o_part, lse_part, S, B, Hq, bl, out, lse);
-  else
-    combine_kernel<64><<<blocks, kCombineWarps * 32, 0, stream>>>(o_part, lse_part, S, B, Hq, bl, out, lse);
-  return cudaGetLastError();
+    return launch_kernel(combine_kernel<128>, dim3(blocks), dim3(kCombineWarps * 32), 0, stream, o_part, lse_part,
+                         S, B, Hq, bl, out, lse);
+  return launch_kernel(combine_kernel<64>, dim3(blocks), dim3(kCombineWarps * 32), 0, stream, o_part, lse_part, S,
+                       B, Hq, bl, out, lse);
 }
 
 }  // namespace nld

@@ -15,6 +15,8 @@ constexpr int kDecideWarps = 8;
 __global__ void __launch_bounds__(kDecideWarps * 32)
     accept_kernel(const int32_t* __restrict__ draft, const int32_t* __restrict__ verify, int B, int n,
                   int32_t* __restrict__ accepted) {
+  grid_dependency_wait();
+  grid_launch_dependents();
   const int lane = threadIdx.x & 31;
   const long b = static_cast<long>(blockIdx.x) * kDecideWarps + (threadIdx.x >> 5);
   if (b >= B) return;
@@ -26,6 +28,8 @@ __global__ void __launch_bounds__(kDecideWarps * 32)
 __global__ void __launch_bounds__(kDecideWarps * 32)
     unmask_kernel(const float* __restrict__ conf, int B, int n, int k, int32_t* __restrict__ positions,
                   int32_t* __restrict__ num_selected) {
+  grid_dependency_wait();
+  grid_launch_dependents();
   const int lane = threadIdx.x & 31;
   const long b = static_cast<long>(blockIdx.x) * kDecideWarps + (threadIdx.x >> 5);
   if (b >= B) return;
@@ -50,15 +54,13 @@ __global__ void __launch_bounds__(kDecideWarps * 32)
 cudaError_t launch_accept(const int32_t* draft, const int32_t* verify, int B, int n, int32_t* acc,
                           cudaStream_t stream) {
   const unsigned blocks = static_cast<unsigned>((B + kDecideWarps - 1) / kDecideWarps);
-  accept_kernel<<<blocks, kDecideWarps * 32, 0, stream>>>(draft, verify, B, n, acc);
-  return cudaGetLastError();
+  return launch_kernel(accept_kernel, dim3(blocks), dim3(kDecideWarps * 32), 0, stream, draft, verify, B, n, acc);
 }
 
 cudaError_t launch_unmask(const float* conf, int B, int n, int k, int32_t* pos, int32_t* nsel,
                           cudaStream_t stream) {
   const unsigned blocks = static_cast<unsigned>((B + kDecideWarps - 1) / kDecideWarps);
-  unmask_kernel<<<blocks, kDecideWarps * 32, 0, stream>>>(conf, B, n, k, pos, nsel);
-  return cudaGetLastError();
+  return launch_kernel(unmask_kernel, dim3(blocks), dim3(kDecideWarps * 32), 0, stream, conf, B, n, k, pos, nsel);
 }
 
 }  // namespace nld

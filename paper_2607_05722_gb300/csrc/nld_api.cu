@@ -3,6 +3,7 @@
 // memory or synchronises, except nld_device_error().
 #include <math.h>
 #include <stdio.h>
+#include <stdlib.h>
 
 #include <mutex>
 
@@ -138,6 +139,16 @@ nld_status_t encode_pool_map(CUtensorMap* map, const void* base, const nld_attn_
 
 }  // namespace
 
+namespace nld {
+bool pdl_enabled() {
+  static const bool on = [] {
+    const char* v = getenv("NLD_DISABLE_PDL");
+    return !(v != nullptr && v[0] == '1');
+  }();
+  return on;
+}
+}  // namespace nld
+
 extern "C" {
 
 const char* nld_status_string(nld_status_t s) {
@@ -226,7 +237,10 @@ nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_bloc
     a.o_part = static_cast<float*>(workspace);
     a.lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) + o_bytes);
   }
-  if (nld::launch_block_attn(a, tmk, tmv, params->head_dim, stream) != cudaSuccess) return NLD_ERR_CUDA;
+  const cudaError_t le = nld::tc_supports(a.R, params->head_dim)
+                            ? nld::launch_block_attn_tc(a, tmk, tmv, params->head_dim, stream)
+                            : nld::launch_block_attn(a, tmk, tmv, params->head_dim, stream);
+  if (le != cudaSuccess) return NLD_ERR_CUDA;
   if (plan.splits > 1 && run_combine) {
     if (nld::launch_combine(a.o_part, a.lse_part, plan.splits, a.B, a.Hq, block_len, params->head_dim, a.out, lse,
                             stream) != cudaSuccess)

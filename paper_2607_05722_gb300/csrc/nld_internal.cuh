@@ -7,6 +7,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "nld.h"
 
 namespace nld {
@@ -39,6 +41,10 @@ struct AttnArgs {
 // Launchers (defined next to their kernels). Return a CUDA error code.
 cudaError_t launch_block_attn(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv,
                               int head_dim, cudaStream_t stream);
+// tcgen05 kernel: query rows R <= 128 (one 128-row MMA tile).
+bool tc_supports(int R, int head_dim);
+cudaError_t launch_block_attn_tc(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv,
+                                 int head_dim, cudaStream_t stream);
 cudaError_t launch_combine(const float* o_part, const float* lse_part, int S, int B, int Hq, int bl,
                            int D, __nv_bfloat16* out, float* lse, cudaStream_t stream);
 cudaError_t launch_accept(const int32_t* draft, const int32_t* verify, int B, int n, int32_t* acc,
@@ -58,9 +64,39 @@ struct AttnShape {
 AttnShape attn_shape(int R, int head_dim);
 size_t max_smem_bytes(int head_dim);
 
+// Launch with programmatic stream serialization: the kernel may start while
+// its predecessor in the stream is still running; every kernel of this
+// library calls grid_dependency_wait() before it touches global memory, so
+// only launch latency and prologue (barrier setup, descriptor prefetch)
+// overlap the predecessor. Set NLD_DISABLE_PDL=1 to launch plainly.
+bool pdl_enabled();
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_kernel(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                          Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl_enabled() ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+}
+
 // ---------------------------------------------------------------------------
 // PTX wrappers
 // ---------------------------------------------------------------------------
+
+// Wait until the grids this one depends on have completed and their memory
+// is visible (no-op without a programmatic dependency).
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// Allow the next grid in the stream to be scheduled.
+__device__ __forceinline__ void grid_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -174,6 +210,163 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 
 __device__ __forceinline__ void named_bar_sync(int id, int threads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
+}
+
+// ---------------------------------------------------------------------------
+// tcgen05 (5th-generation tensor core) and tensor memory
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// Allocate `ncols` TMEM columns (a power of two >= 32); the base address is
+// written to shared memory. Executed by one whole warp.
+__device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot)),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+// Shared-memory matrix descriptor for a 128-byte-swizzled operand tile:
+// start address, leading-dimension and stride-dimension byte offsets (16-byte
+// units), descriptor version 1, swizzle mode 2 (128 B).
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr, uint32_t lbo_bytes, uint32_t sbo_bytes) {
+  uint64_t d = static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);
+  d |= static_cast<uint64_t>((lbo_bytes >> 4) & 0x3FFFu) << 16;
+  d |= static_cast<uint64_t>((sbo_bytes >> 4) & 0x3FFFu) << 32;
+  d |= static_cast<uint64_t>(1) << 46;
+  d |= static_cast<uint64_t>(2) << 61;
+  return d;
+}
+
+// Instruction descriptor of tcgen05.mma kind::f16 with bf16 A and B and an
+// fp32 accumulator: M x N tile, A K-major, B K-major or MN-major.
+__host__ __device__ constexpr uint32_t umma_idesc_bf16(int M, int N, bool b_mn_major) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
+         (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(M >> 4) << 24);
+}
+
+// D(tmem) (+)= A(smem) * B(smem), issued by one thread.
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive on an mbarrier once every tcgen05 operation this thread issued has completed.
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+
+// Warp-collective: each lane reads 32 consecutive fp32 columns of its TMEM
+// lane (lanes 32*(warp%4) .. +31), then waits for the load.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* out) {
+  uint32_t r[32];
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];\n\t"
+               "tcgen05.wait::ld.sync.aligned;"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+               : "r"(taddr)
+               : "memory");
+#pragma unroll
+  for (int j = 0; j < 32; ++j) out[j] = __uint_as_float(r[j]);
+}
+
+// Warp-collective: each lane writes 32 consecutive fp32 columns of its TMEM lane and waits.
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const float* in) {
+  uint32_t r[32];
+#pragma unroll
+  for (int j = 0; j < 32; ++j) r[j] = __float_as_uint(in[j]);
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};\n\t"
+               "tcgen05.wait::st.sync.aligned;" ::"r"(taddr),
+               "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+               : "memory");
+}
+
+// ---------------------------------------------------------------------------
+// K/V tile staging shared by the attention kernels
+// ---------------------------------------------------------------------------
+
+// A stage holds the K tile then the V tile of 64 tokens; each is D/64 column
+// blocks of 64 tokens x 128 bytes, written by TMA with the 128-byte swizzle
+// (chunk c of row r at chunk position c ^ (r % 8) within each 1024-byte atom).
+template <int D>
+struct TileGeom {
+  static constexpr int kColBlocks = D / 64;
+  static constexpr int kColBlockBytes = kTileTok * 128;
+  static constexpr int kTileBytes = kColBlocks * kColBlockBytes;
+  static constexpr int kStageBytes = 2 * kTileBytes;
+};
+
+// Byte offset of (token r, 16-byte chunk c) inside a K or V tile.
+__device__ __forceinline__ uint32_t kv_swz(int r, int c) {
+  return static_cast<uint32_t>((c >> 3) * (kTileTok * 128) + r * 128 + (((c & 7) ^ (r & 7)) << 4));
+}
+
+// Producer warp: streams the K/V tiles of tokens [t_begin, t_end) of
+// (sequence b, KV head g) into an nstage ring. Lane j holds the physical page
+// of 16-token group j of the current batch of 32 groups (8 tiles); the next
+// batch loads one batch ahead. Each tile's boxes are issued by separate
+// lanes. Returns the number of tiles issued.
+template <int D>
+__device__ __forceinline__ int produce_kv(const AttnArgs& a, const CUtensorMap* tmk, const CUtensorMap* tmv,
+                                          uint8_t* stages, uint64_t* full, uint64_t* empty, int nstage, int g,
+                                          int b, int t_begin, int t_end, int ntiles, int lane) {
+  using Geo = TileGeom<D>;
+  const int32_t* ptab = a.page_table + static_cast<size_t>(b) * a.max_pages;
+  auto group_page = [&](int gi) -> int {
+    const int t = t_begin + gi * kGroupTok;
+    if (t >= t_end) return a.num_pages;  // past the pool: TMA fills the box with zeros
+    int page = __ldg(ptab + (t >> a.log2_page));
+    if (page < 0 || page >= a.num_pages) {
+      atomicOr(a.err, NLD_DEVERR_PAGE_RANGE);
+      page = min(max(page, 0), a.num_pages - 1);
+    }
+    return page;
+  };
+  constexpr int kOpsPerGroup = 2 * Geo::kColBlocks;  // K and V boxes per 16-token group
+  constexpr int kOpsPerTile = (kTileTok / kGroupTok) * kOpsPerGroup;
+  static_assert(kOpsPerTile <= 32, "one TMA op per lane");
+  int page_cur = group_page(lane);
+  int page_next = ntiles > 8 ? group_page(32 + lane) : a.num_pages;
+  int issued = 0;
+  for (int k = 0; k < ntiles; ++k) {
+    const int st = k % nstage;
+    if (k >= nstage) {
+      int ok = 1;
+      if (lane == 0) ok = mbar_wait(&empty[st], ((k / nstage) - 1) & 1, a.err) ? 1 : 0;
+      if (!__shfl_sync(0xffffffffu, ok, 0)) break;
+    }
+    if (k > 0 && (k & 7) == 0) {
+      page_cur = page_next;
+      page_next = (k + 8) < ntiles ? group_page((k / 8 + 1) * 32 + lane) : a.num_pages;
+    }
+    if (lane == 0) mbar_arrive_expect_tx(&full[st], Geo::kStageBytes);
+    __syncwarp();
+    const int grp = lane / kOpsPerGroup;
+    const int page = __shfl_sync(0xffffffffu, page_cur, ((k & 7) * 4 + grp) & 31);
+    if (lane < kOpsPerTile) {
+      const int cb = (lane >> 1) % Geo::kColBlocks;
+      const bool is_v = lane & 1;
+      const int t = t_begin + k * kTileTok + grp * kGroupTok;
+      const int slot = page < a.num_pages ? (t & (a.page_size - 1)) : 0;
+      uint8_t* dst = stages + st * Geo::kStageBytes + (is_v ? Geo::kTileBytes : 0) + cb * Geo::kColBlockBytes +
+                     grp * kGroupTok * 128;
+      tma_load_4d(dst, is_v ? tmv : tmk, &full[st], cb * 64, slot, g, page);
+    }
+    issued = k + 1;
+  }
+  return issued;
 }
 
 }  // namespace nld

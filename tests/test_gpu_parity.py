@@ -86,7 +86,7 @@ def test_unmask_golden_cases():
 def test_unmask_ties_and_ineligible(orc):
     rng = np.random.default_rng(2)
     for n in (1, 2, 3, 8, 16, 31, 32):
-        for k in sorted({1, 2, max(1, n // 2), n}):
+        for k in sorted({k for k in (1, 2, max(1, n // 2), n) if k <= n}):
             conf = rng.integers(0, 3, size=(300, n)).astype(np.float32) / 2
             conf[rng.random((300, n)) < 0.2] = -np.inf
             conf[rng.random((300, n)) < 0.05] = np.nan
@@ -149,7 +149,9 @@ def test_combine_matches_oracle(orc, S, D):
     rl = rl.reshape(B, Hq, bl)
     got = out.float().cpu().numpy()
     assert np.all(np.isfinite(got))
-    assert np.max(np.abs(got - ro)) <= 1e-2
+    # bf16 round-to-nearest of the exact value (half an ulp, at most 2^-8 relative)
+    # plus fp32 accumulation error
+    assert np.all(np.abs(got - ro) <= 2.0 ** -8 * np.abs(ro) + 1e-5)
     gl = lse.cpu().numpy()
     assert np.array_equal(np.isinf(gl), np.isinf(rl))
     fin = np.isfinite(rl)
@@ -178,7 +180,8 @@ SMALL = [
 @pytest.mark.parametrize("splits", [0, 1, 3])
 def test_attention_small_all_rows(orc, spec, mode, splits):
     name, B, Hq, Hkv, D, P, bl, prefix = spec
-    case = W.make_block_attn_case(name, B, Hq, Hkv, D, bl, P, prefix, seed=sum(prefix) + bl)
+    case = W.make_block_attn_case(name, B, Hq, Hkv, D, block_len=bl, page_size=P, prefix_lens=prefix,
+                                  seed=sum(prefix) + bl)
     dc = DeviceCase(case)
     out, lse = dc.run(mode, num_splits=splits)
     ro, rl = oracle_full(orc, case, mode)
@@ -188,7 +191,7 @@ def test_attention_small_all_rows(orc, spec, mode, splits):
 def test_attention_tail_slots_hold_nan(orc):
     """Cache slots past the block inside the last page may be uninitialised;
     NaN there must not reach the output."""
-    case = W.make_block_attn_case("nan_tail", 2, 8, 2, 128, 7, 16, [37, 100], seed=3)
+    case = W.make_block_attn_case("nan_tail", 2, 8, 2, 128, block_len=7, page_size=16, prefix_lens=[37, 100], seed=3)
     kv = case.kv
     k_bits, v_bits = kv.k_bits.copy(), kv.v_bits.copy()
     nan = np.uint16(0x7FC0)
@@ -242,7 +245,7 @@ def test_page_permutation_is_bit_identical():
 
 
 def test_block_len_one_modes_agree():
-    case = W.make_block_attn_case("bl1", 3, 32, 8, 128, 16, 1, [5, 700, 4096], seed=5)
+    case = W.make_block_attn_case("bl1", 3, 32, 8, 128, block_len=1, page_size=16, prefix_lens=[5, 700, 4096], seed=5)
     dc = DeviceCase(case)
     q = dc.q[DIFF]
     for S in (1, 0):
@@ -254,7 +257,7 @@ def test_block_len_one_modes_agree():
 def test_device_clamps_bad_prefix_and_page_ids():
     """Out-of-range device values are clamped (no access leaves the buffers)
     and flagged in the device error word."""
-    case = W.make_block_attn_case("bad", 2, 8, 2, 64, 16, 8, [40, 10], seed=6)
+    case = W.make_block_attn_case("bad", 2, 8, 2, 64, block_len=8, page_size=16, prefix_lens=[40, 10], seed=6)
     dc = DeviceCase(case)
     nld.nld_device_error(clear=True)
     dc.prefix = torch.tensor([10 ** 6, -5], dtype=torch.int32, device="cuda")
