@@ -73,6 +73,8 @@ __global__ void __launch_bounds__(MaxWarps<NWT>::value * 32, 1)
     L = min(max(L, 0), lmax);
   }
   const int N = L + a.bl;
+  const float scl = a.scale_log2;
+  const bool diff_mode = a.mode == NLD_MODE_DIFFUSION;
   const int t_begin = split * a.chunk;
   const int t_end = min(t_begin + a.chunk, N);
 
@@ -87,7 +89,9 @@ __global__ void __launch_bounds__(MaxWarps<NWT>::value * 32, 1)
   const int ntiles = (t_end - t_begin + kTileTok - 1) / kTileTok;
 
   if (warp == ncons) {
-    produce_kv<D>(a, &tmk, &tmv, smem, full, empty, nstage, g, b, t_begin, t_end, ntiles, lane);
+    PagePrefetch first;
+    first.load(a, b, t_begin, 0, lane);
+    produce_kv<D>(a, &tmk, &tmv, smem, full, empty, nstage, g, b, t_begin, t_end, ntiles, lane, 3, first);
     return;
   }
 
@@ -163,23 +167,30 @@ __global__ void __launch_bounds__(MaxWarps<NWT>::value * 32, 1)
     }
 
     // ---- mask, scale (base 2), online softmax ----
-    const bool all_visible = (tile_t0 + kTileTok <= L) && (valid >= kTileTok);
+    // The mask only matters on a tile that reaches the block or the split
+    // end; there it is applied branch-free (a branch per element in these
+    // unrolled loops is several times slower than the arithmetic).
     float mx[2] = {-INFINITY, -INFINITY};
+    if ((tile_t0 + kTileTok <= L) && (valid >= kTileTok)) {
 #pragma unroll
-    for (int jn = 0; jn < NT; ++jn) {
+      for (int jn = 0; jn < NT; ++jn)
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int hf = e >> 1;
-        float v = s[jn][e] * a.scale_log2;
-        if (!all_visible) {
+        for (int e = 0; e < 4; ++e) {
+          s[jn][e] *= scl;
+          mx[e >> 1] = fmaxf(mx[e >> 1], s[jn][e]);
+        }
+    } else {
+#pragma unroll
+      for (int jn = 0; jn < NT; ++jn)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int hf = e >> 1;
           const int col = wt * TW + jn * 8 + qc + (e & 1);
           const int t = tile_t0 + col;
-          const bool vis = col < valid && (t < L || a.mode == NLD_MODE_DIFFUSION || t - L <= row_i[hf]);
-          v = vis ? v : -INFINITY;
+          const bool vis = (col < valid) & ((t < L) | diff_mode | (t - L <= row_i[hf]));
+          s[jn][e] = vis ? s[jn][e] * scl : -INFINITY;
+          mx[hf] = fmaxf(mx[hf], s[jn][e]);
         }
-        s[jn][e] = v;
-        mx[hf] = fmaxf(mx[hf], v);
-      }
     }
     float m_use[2];
 #pragma unroll

@@ -6,18 +6,21 @@
 // heads times the bl block tokens form R = G*bl <= 128 query rows, padded to
 // the 128-row MMA tile, so each K/V page leaves HBM once per (b, g).
 //
-// Warp roles (6 warps):
-//   warp 0    TMA producer: 64-token K/V tiles into a 4-stage ring (produce_kv).
-//   warp 1    allocates 256 TMEM columns; lane 0 issues every MMA:
+// Warp roles (7 warps):
+//   warps 0-1 TMA producers: the K (warp 0) and V (warp 1) boxes of 64-token
+//             tiles into a 4-stage ring (produce_kv); two issuing warps halve
+//             the issue time, which is per warp.
+//   warp 2    allocates 256 TMEM columns; lane 0 issues every MMA:
 //               S_k = Q K_k^T   (M=128 rows, N=64 tokens, K=D; double-buffered in TMEM)
 //               O  += P_k V_k   (M=128 rows, N=D, K=64 tokens; V read MN-major)
 //             S_{k+1} is issued before O += P_k V_k so the tensor core computes
 //             the next scores while the softmax warps work on the current ones.
-//   warps 2-5 softmax: thread t owns query row 32*(warp%4)+lane (its TMEM lane).
+//   warps 3-6 softmax: thread t owns query row 32*(warp%4)+lane (its TMEM lane).
 //             It loads its S row, applies the mask and the base-2 scale,
 //             keeps the running max and sum, writes P (bf16) to shared memory
 //             for the PV MMA, and at the end reads O from TMEM, divides by the
-//             sum and stores the row (or the split partial).
+//             sum and stages its rows in the freed K/V ring so that each row
+//             leaves as one coalesced store (bf16 output or fp32 split partial).
 // The running max is raised lazily: O is rescaled in TMEM only when a row's
 // max grows by more than 2^8 (P then stays below 256, exact enough in bf16);
 // the final division by the matching sum removes the reference max.
@@ -27,7 +30,9 @@ namespace nld {
 namespace {
 
 constexpr int kTcStages = 4;
-constexpr int kTcThreads = 192;
+constexpr int kTcThreads = 224;
+constexpr int kMmaWarp = 2;
+constexpr int kSoftmaxWarp0 = 3;
 constexpr uint32_t kTmemCols = 256;  // S0 | S1 (64 columns each) | O (D <= 128 columns)
 constexpr float kRescaleLog2 = 8.0f;
 
@@ -70,7 +75,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kTcStages; ++s) {
-      mbar_init(&kv_full[s], 1);
+      mbar_init(&kv_full[s], 2);  // K and V producer warps
       mbar_init(&kv_empty[s], 1);
     }
     for (int j = 0; j < 2; ++j) {
@@ -87,25 +92,32 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     prefetch_tensormap(&tmk);
     prefetch_tensormap(&tmv);
   }
-  if (warp == 1) {
+  if (warp == kMmaWarp) {
     tmem_alloc(tmem_slot, kTmemCols);
     tc_fence_before();
   }
   grid_dependency_wait();
   grid_launch_dependents();
+  const int t_begin = split * a.chunk;
+  // The producers' first page-id loads and the prefix-length load are
+  // independent, so they are in flight together.
+  PagePrefetch first;
+  first.raw = 0;
+  if (warp < 2) first.load(a, b, t_begin, 0, lane);
+  int L = __ldg(a.prefix_lens + b);
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const uint32_t tS0 = tmem, tS1 = tmem + kTileTok, tO = tmem + 2 * kTileTok;
 
   const int lmax = a.max_pages * a.page_size - a.bl;
-  int L = __ldg(a.prefix_lens + b);
   if (L < 0 || L > lmax) {
     if (threadIdx.x == 0) atomicOr(a.err, NLD_DEVERR_PREFIX_RANGE);
     L = min(max(L, 0), lmax);
   }
   const int N = L + a.bl;
-  const int t_begin = split * a.chunk;
+  const float scl = a.scale_log2;
+  const bool diff_mode = a.mode == NLD_MODE_DIFFUSION;
   const int t_end = min(t_begin + a.chunk, N);
   const int ntiles = t_begin < t_end ? (t_end - t_begin + kTileTok - 1) / kTileTok : 0;
 
@@ -115,17 +127,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       const int i = r / a.G, h = g * a.G + (r - i * a.G);
       a.lse_part[((static_cast<size_t>(split) * a.B + b) * a.Hq + h) * a.bl + i] = -INFINITY;
     }
-  } else if (warp == 0) {
-    // ---------------- producer ----------------
+  } else if (warp < 2) {
+    // ---------------- producers (warp 0: K, warp 1: V) ----------------
     const int issued = produce_kv<D>(a, &tmk, &tmv, smem, kv_full, kv_empty, kTcStages, g, b, t_begin, t_end,
-                                     ntiles, lane);
+                                     ntiles, lane, warp == 0 ? 1 : 2, first);
     if (lane == 0 && issued < ntiles) {
       // Stopped early on a wait timeout: let the copies already issued land
       // before the CTA exits (bounded).
       for (int k = max(0, issued - kTcStages); k < issued; ++k)
         mbar_wait(&kv_full[k % kTcStages], (k / kTcStages) & 1, a.err);
     }
-  } else if (warp == 1) {
+  } else if (warp == kMmaWarp) {
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
       bool ok = mbar_wait(q_ready, 0, a.err);
@@ -133,11 +145,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       const uint32_t q_addr = smem_u32(q_s);
       const uint32_t idesc_s = umma_idesc_bf16(128, kTileTok, false);
       const uint32_t idesc_o = umma_idesc_bf16(128, D, true);
-      auto issue_s = [&](int k) -> bool {
+      auto issue_s = [&](int k) {
         const int st = k % kTcStages;
-        if (!mbar_wait(&kv_full[st], (k / kTcStages) & 1, a.err)) return false;
-        if (k >= 2 && !mbar_wait(&s_free[k & 1], ((k - 2) >> 1) & 1, a.err)) return false;
-        tc_fence_after();
         const uint32_t k_addr = smem_u32(smem + st * Geo::kStageBytes);
         const uint32_t d = (k & 1) ? tS1 : tS0;
 #pragma unroll
@@ -149,19 +158,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           umma_bf16(d, ad, bd, idesc_s, kk > 0 ? 1u : 0u);
         }
         umma_commit(&s_full[k & 1]);
-        return true;
       };
-      if (ok) ok = issue_s(0);
-      for (int k = 0; ok && k < ntiles; ++k) {
-        if (k + 1 < ntiles && !issue_s(k + 1)) {
-          ok = false;
-          break;
-        }
-        if (!mbar_wait(&p_full[k & 1], (k >> 1) & 1, a.err)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
+      auto issue_pv = [&](int k) {
         const int st = k % kTcStages;
         const uint32_t p_addr = smem_u32(smem + Lay::kPOff + (k & 1) * Lay::kPBytes);
         const uint32_t v_addr = smem_u32(smem + st * Geo::kStageBytes + Geo::kTileBytes);
@@ -175,6 +173,34 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
         umma_commit(&o_done[k & 1]);
         umma_commit(&kv_empty[st]);
+      };
+      // Event-driven issue: S_k needs its K tile and a free S buffer (the
+      // softmax warps have read S_{k-2}); PV_k needs P_k. Whichever is ready
+      // goes first, so a late K/V tile never holds back a ready PV.
+      int next_s = 0, next_pv = 0;
+      const uint64_t t_start = global_timer_ns();
+      uint32_t spins = 0;
+      while (ok && next_pv < ntiles) {
+        bool progressed = false;
+        if (next_s < ntiles && next_s < next_pv + 2 &&
+            mbar_test(&kv_full[next_s % kTcStages], (next_s / kTcStages) & 1) &&
+            (next_s < 2 || mbar_test(&s_free[next_s & 1], ((next_s - 2) >> 1) & 1))) {
+          tc_fence_after();
+          issue_s(next_s++);
+          progressed = true;
+        }
+        if (next_pv < next_s && mbar_test(&p_full[next_pv & 1], (next_pv >> 1) & 1)) {
+          tc_fence_after();
+          issue_pv(next_pv++);
+          progressed = true;
+        }
+        if (!progressed) {
+          __nanosleep(20);  // this warp shares an SM sub-partition with a softmax warp
+          if ((++spins & 255u) == 0 && global_timer_ns() - t_start > kWaitLimitNs) {
+            atomicOr(a.err, NLD_DEVERR_WAIT_TIMEOUT);
+            ok = false;
+          }
+        }
       }
       if (!ok) {
         // Let every MMA already issued finish before TMEM is released (bounded).
@@ -192,7 +218,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const bool row_ok = r < a.R;
     const int row_i = r / a.G;
     const int row_h = g * a.G + (r - row_i * a.G);
-    const int sm_tid = threadIdx.x - 64;  // 0..127 across the softmax warps
+    const int sm_tid = threadIdx.x - 32 * kSoftmaxWarp0;  // 0..127 across the softmax warps
 
     // Q row -> shared memory in the 128-byte-swizzled K-major layout; padding
     // rows are zero. Padding rows of P are zeroed once for both buffers.
@@ -243,18 +269,24 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       float alpha = 1.f;
       bool rescale = false;
       if (warp_rows) {
-        const bool all_visible = (tile_t0 + kTileTok <= L) && (valid >= kTileTok);
+        // Scale to base 2 and take the row max. The mask only matters on a
+        // tile that reaches the block or the split end; it is applied there
+        // branch-free (a branch per element in this unrolled loop costs ~8x).
         float mx = -INFINITY;
+        if ((tile_t0 + kTileTok <= L) && (valid >= kTileTok)) {
 #pragma unroll
-        for (int j = 0; j < kTileTok; ++j) {
-          float v = s[j] * a.scale_log2;
-          if (!all_visible) {
-            const int t = tile_t0 + j;
-            const bool vis = j < valid && (t < L || a.mode == NLD_MODE_DIFFUSION || t - L <= row_i);
-            v = vis ? v : -INFINITY;
+          for (int j = 0; j < kTileTok; ++j) {
+            s[j] *= scl;
+            mx = fmaxf(mx, s[j]);
           }
-          s[j] = v;
-          mx = fmaxf(mx, v);
+        } else {
+#pragma unroll
+          for (int j = 0; j < kTileTok; ++j) {
+            const int t = tile_t0 + j;
+            const bool vis = (j < valid) & ((t < L) | diff_mode | (t - L <= row_i));
+            s[j] = vis ? s[j] * scl : -INFINITY;
+            mx = fmaxf(mx, s[j]);
+          }
         }
         if (m_run == -INFINITY) {
           m_run = mx;  // nothing accumulated for this row yet
@@ -324,6 +356,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
 
     // ---------------- epilogue ----------------
+    // Every PV has completed once o_done of the last tile fires, so the K/V
+    // ring is free: each warp stages its 32 rows there (padded pitch, no bank
+    // conflicts), then writes each row with one coalesced warp-wide store.
     if (ok && mbar_wait(&o_done[(ntiles - 1) & 1], ((ntiles - 1) >> 1) & 1, a.err)) {
       tc_fence_after();
       if (warp_rows) {
@@ -331,33 +366,52 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const float inv = l > 0.f ? 1.f / l : 0.f;
         const float lse_v = l > 0.f ? (m_run + lg2(l)) * kLn2 : -INFINITY;
         const bool split_out = a.o_part != nullptr;
-        const size_t orow = (static_cast<size_t>(b) * a.bl + row_i) * a.Hq + row_h;
-        const size_t prow = ((static_cast<size_t>(split) * a.B + b) * a.Hq + row_h) * a.bl + row_i;
+        const int row_bytes = split_out ? D * 4 : D * 2;
+        const int pitch = row_bytes + 16;
+        uint8_t* stage = smem + quad * 32 * pitch;  // quad * 32 * (512 + 16) < ring size
+        uint8_t* my = stage + lane * pitch;
 #pragma unroll 1
         for (int c = 0; c < D / 32; ++c) {
           float o[32];
           tmem_ld32(tO + lane_off + c * 32, o);
-          if (!row_ok) continue;
-          if (!split_out) {
-            uint4* dst = reinterpret_cast<uint4*>(a.out + orow * D + c * 32);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) o[j] *= inv;
+          if (split_out) {
+#pragma unroll
+            for (int q4 = 0; q4 < 8; ++q4)
+              *reinterpret_cast<float4*>(my + c * 128 + q4 * 16) =
+                  make_float4(o[4 * q4], o[4 * q4 + 1], o[4 * q4 + 2], o[4 * q4 + 3]);
+          } else {
 #pragma unroll
             for (int q4 = 0; q4 < 4; ++q4) {
               const int j = q4 * 8;
-              dst[q4] = make_uint4(pack_bf16(o[j] * inv, o[j + 1] * inv), pack_bf16(o[j + 2] * inv, o[j + 3] * inv),
-                                   pack_bf16(o[j + 4] * inv, o[j + 5] * inv), pack_bf16(o[j + 6] * inv, o[j + 7] * inv));
+              *reinterpret_cast<uint4*>(my + c * 64 + q4 * 16) =
+                  make_uint4(pack_bf16(o[j], o[j + 1]), pack_bf16(o[j + 2], o[j + 3]), pack_bf16(o[j + 4], o[j + 5]),
+                             pack_bf16(o[j + 6], o[j + 7]));
             }
-          } else if (l > 0.f) {
-            float4* dst = reinterpret_cast<float4*>(a.o_part + prow * D + c * 32);
-#pragma unroll
-            for (int q4 = 0; q4 < 8; ++q4)
-              dst[q4] = make_float4(o[4 * q4] * inv, o[4 * q4 + 1] * inv, o[4 * q4 + 2] * inv, o[4 * q4 + 3] * inv);
           }
+        }
+        // Global row of each lane's query row: output row (unsplit) or partial row.
+        const size_t my_row = split_out
+                                  ? ((static_cast<size_t>(split) * a.B + b) * a.Hq + row_h) * a.bl + row_i
+                                  : (static_cast<size_t>(b) * a.bl + row_i) * a.Hq + row_h;
+        const bool my_write = row_ok && (!split_out || l > 0.f);
+        __syncwarp();
+        const int chunks = row_bytes / 16;  // 8..32 lanes move one row
+        uint8_t* gbase = split_out ? reinterpret_cast<uint8_t*>(a.o_part) : reinterpret_cast<uint8_t*>(a.out);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const size_t row = __shfl_sync(0xffffffffu, my_row, j);
+          const bool w = __shfl_sync(0xffffffffu, my_write, j);
+          if (w && lane < chunks)
+            *reinterpret_cast<uint4*>(gbase + row * row_bytes + lane * 16) =
+                *reinterpret_cast<const uint4*>(stage + j * pitch + lane * 16);
         }
         if (row_ok) {
           if (!split_out) {
             if (a.lse != nullptr) a.lse[(static_cast<size_t>(b) * a.Hq + row_h) * a.bl + row_i] = lse_v;
           } else {
-            a.lse_part[prow] = lse_v;
+            a.lse_part[((static_cast<size_t>(split) * a.B + b) * a.Hq + row_h) * a.bl + row_i] = lse_v;
           }
         }
       }
@@ -366,7 +420,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   }
 
   __syncthreads();
-  if (warp == 1) {
+  if (warp == kMmaWarp) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }

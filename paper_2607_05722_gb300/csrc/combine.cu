@@ -55,14 +55,16 @@ __global__ void __launch_bounds__(kCombineWarps * 32)
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) csum += __shfl_xor_sync(0xffffffffu, csum, off);
-    // Accumulate 8 splits per round; the loads of a round are independent.
+    // Accumulate kRound splits per round; the loads of a round are
+    // independent, so a row with up to kRound splits costs one L2 latency.
     const float* base = o_part + static_cast<long>(row) * D + lane * V;
     const long split_stride = R * static_cast<long>(D);
-    for (int s0 = 0; s0 < S; s0 += 8) {
-      float wv[8];
-      float x[8][V];
+    constexpr int kRound = 32;
+    for (int s0 = 0; s0 < S; s0 += kRound) {
+      float wv[kRound];
+      float x[kRound][V];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
+      for (int u = 0; u < kRound; ++u) {
         const int s = s0 + u;
         const int src = s & 31;
         const int blk = s >> 5;  // warp-uniform
@@ -84,7 +86,7 @@ __global__ void __launch_bounds__(kCombineWarps * 32)
         }
       }
 #pragma unroll
-      for (int u = 0; u < 8; ++u)
+      for (int u = 0; u < kRound; ++u)
 #pragma unroll
         for (int v = 0; v < V; ++v) acc[v] += wv[u] * x[u][v];
     }

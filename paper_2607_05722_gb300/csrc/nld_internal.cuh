@@ -132,6 +132,19 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// Non-blocking test of an mbarrier phase.
+__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
 __device__ __forceinline__ uint64_t global_timer_ns() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
@@ -313,32 +326,50 @@ __device__ __forceinline__ uint32_t kv_swz(int r, int c) {
   return static_cast<uint32_t>((c >> 3) * (kTileTok * 128) + r * 128 + (((c & 7) ^ (r & 7)) << 4));
 }
 
-// Producer warp: streams the K/V tiles of tokens [t_begin, t_end) of
-// (sequence b, KV head g) into an nstage ring. Lane j holds the physical page
-// of 16-token group j of the current batch of 32 groups (8 tiles); the next
-// batch loads one batch ahead. Each tile's boxes are issued by separate
-// lanes. Returns the number of tiles issued.
+// Page id of each 16-token group of a split, loaded ahead: lane j of the
+// producer warp holds group j of a batch of 32 groups (8 tiles). The load
+// does not depend on the prefix length (the index is clamped into the table
+// row), so it can be issued before the length is known; validate() then
+// marks groups past the split end as out of the pool (TMA zero fill) and
+// clamps corrupt ids into range, flagging them.
+struct PagePrefetch {
+  int raw;
+  __device__ __forceinline__ void load(const AttnArgs& a, int b, int t_begin, int batch, int lane) {
+    const int t = t_begin + (batch * 32 + lane) * kGroupTok;
+    const int lp = min(t >> a.log2_page, a.max_pages - 1);
+    raw = __ldg(a.page_table + static_cast<size_t>(b) * a.max_pages + lp);
+  }
+  __device__ __forceinline__ int validate(const AttnArgs& a, int t_begin, int t_end, int batch, int lane) const {
+    const int t = t_begin + (batch * 32 + lane) * kGroupTok;
+    if (t >= t_end) return a.num_pages;
+    if (raw < 0 || raw >= a.num_pages) {
+      atomicOr(a.err, NLD_DEVERR_PAGE_RANGE);
+      return min(max(raw, 0), a.num_pages - 1);
+    }
+    return raw;
+  }
+};
+
+// Producer warp: streams the K tiles (kinds & 1), the V tiles (kinds & 2) or
+// both of tokens [t_begin, t_end) of (sequence b, KV head g) into an nstage
+// ring. `first` holds the page ids of the first 32 groups, already loaded.
+// The boxes of a tile are issued by separate lanes; a warp's expect_tx covers
+// only the bytes it issues, so `full` expects one arrival per producing warp.
+// Returns the number of tiles issued.
 template <int D>
 __device__ __forceinline__ int produce_kv(const AttnArgs& a, const CUtensorMap* tmk, const CUtensorMap* tmv,
                                           uint8_t* stages, uint64_t* full, uint64_t* empty, int nstage, int g,
-                                          int b, int t_begin, int t_end, int ntiles, int lane) {
+                                          int b, int t_begin, int t_end, int ntiles, int lane, int kinds,
+                                          const PagePrefetch& first) {
   using Geo = TileGeom<D>;
-  const int32_t* ptab = a.page_table + static_cast<size_t>(b) * a.max_pages;
-  auto group_page = [&](int gi) -> int {
-    const int t = t_begin + gi * kGroupTok;
-    if (t >= t_end) return a.num_pages;  // past the pool: TMA fills the box with zeros
-    int page = __ldg(ptab + (t >> a.log2_page));
-    if (page < 0 || page >= a.num_pages) {
-      atomicOr(a.err, NLD_DEVERR_PAGE_RANGE);
-      page = min(max(page, 0), a.num_pages - 1);
-    }
-    return page;
-  };
-  constexpr int kOpsPerGroup = 2 * Geo::kColBlocks;  // K and V boxes per 16-token group
-  constexpr int kOpsPerTile = (kTileTok / kGroupTok) * kOpsPerGroup;
-  static_assert(kOpsPerTile <= 32, "one TMA op per lane");
-  int page_cur = group_page(lane);
-  int page_next = ntiles > 8 ? group_page(32 + lane) : a.num_pages;
+  const int nkinds = (kinds & 1) + ((kinds >> 1) & 1);
+  const int ops_per_group = nkinds * Geo::kColBlocks;
+  const int ops_per_tile = (kTileTok / kGroupTok) * ops_per_group;  // <= 32
+  const uint32_t bytes = nkinds * Geo::kTileBytes;
+  int page_cur = first.validate(a, t_begin, t_end, 0, lane);
+  PagePrefetch nxt;
+  nxt.raw = 0;
+  if (ntiles > 8) nxt.load(a, b, t_begin, 1, lane);
   int issued = 0;
   for (int k = 0; k < ntiles; ++k) {
     const int st = k % nstage;
@@ -348,16 +379,18 @@ __device__ __forceinline__ int produce_kv(const AttnArgs& a, const CUtensorMap* 
       if (!__shfl_sync(0xffffffffu, ok, 0)) break;
     }
     if (k > 0 && (k & 7) == 0) {
-      page_cur = page_next;
-      page_next = (k + 8) < ntiles ? group_page((k / 8 + 1) * 32 + lane) : a.num_pages;
+      const int batch = k >> 3;
+      page_cur = nxt.validate(a, t_begin, t_end, batch, lane);
+      if ((k + 8) < ntiles) nxt.load(a, b, t_begin, batch + 1, lane);
     }
-    if (lane == 0) mbar_arrive_expect_tx(&full[st], Geo::kStageBytes);
+    if (lane == 0) mbar_arrive_expect_tx(&full[st], bytes);
     __syncwarp();
-    const int grp = lane / kOpsPerGroup;
+    const int grp = lane / ops_per_group;
     const int page = __shfl_sync(0xffffffffu, page_cur, ((k & 7) * 4 + grp) & 31);
-    if (lane < kOpsPerTile) {
-      const int cb = (lane >> 1) % Geo::kColBlocks;
-      const bool is_v = lane & 1;
+    if (lane < ops_per_tile) {
+      const int r = lane - grp * ops_per_group;
+      const int cb = r % Geo::kColBlocks;
+      const bool is_v = (kinds == 2) || (kinds == 3 && r >= Geo::kColBlocks);
       const int t = t_begin + k * kTileTok + grp * kGroupTok;
       const int slot = page < a.num_pages ? (t & (a.page_size - 1)) : 0;
       uint8_t* dst = stages + st * Geo::kStageBytes + (is_v ? Geo::kTileBytes : 0) + cb * Geo::kColBlockBytes +
