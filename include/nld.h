@@ -150,6 +150,30 @@ nld_status_t nld_block_attn_partials(const nld_attn_params_t *params, const void
                                      cudaStream_t stream);
 
 /*
+ * nld_block_attn for callers that cannot allocate device memory (the paper
+ * has no counterpart: this is a deployment convenience of this library).
+ * Plugins running inside another runtime's enqueue step, code bound to a
+ * fixed memory budget, or callers holding only raw input/output pointers may
+ * have no way to provide a workspace. This entry point takes the same
+ * arguments as nld_block_attn minus the workspace and keeps the split
+ * partials in a 16 MiB array compiled into the library (held by every GPU
+ * that loads it until exit). It allocates and frees nothing.
+ *   - Returns NLD_ERR_WORKSPACE, launching nothing, when the split plan
+ *     needs more than 16 MiB of partials (nld_block_attn_workspace_size()
+ *     > 16 MiB); ask for fewer splits (params->num_splits) or use
+ *     nld_block_attn with your own workspace.
+ *   - The first call made with a device current looks up the array's device
+ *     address on that device; make it before any stream capture.
+ *   - All calls on a device share the array. Calls whose kernels may overlap
+ *     on the GPU (unordered streams) race on it; order them on one stream.
+ */
+nld_status_t nld_block_attn_static_scratch(const nld_attn_params_t *params, const void *q_block,
+                                           const void *k_pages, const void *v_pages,
+                                           const int32_t *page_table, const int32_t *prefix_lens,
+                                           int block_len, nld_mode_t mode, void *out, float *lse,
+                                           cudaStream_t stream);
+
+/*
  * Merge split-KV partials (each a softmax-normalised partial output and its
  * log-sum-exp over one key range) into the full result:
  *   m = max_s lse_s, c_s = exp(lse_s - m),

@@ -62,6 +62,8 @@ def lib(path: Optional[str] = None):
     L.nld_block_attn.restype = I
     L.nld_block_attn_partials.argtypes = [PP, V, V, V, V, V, I, I, V, V, V, Sz, V]
     L.nld_block_attn_partials.restype = I
+    L.nld_block_attn_static_scratch.argtypes = [PP, V, V, V, V, V, I, I, V, V, V]
+    L.nld_block_attn_static_scratch.restype = I
     L.nld_split_kv_combine.argtypes = [V, V, I, I, I, I, I, V, V, V]
     L.nld_split_kv_combine.restype = I
     L.nld_accept.argtypes = [V, V, I, I, V, V]
@@ -181,6 +183,25 @@ def nld_block_attn_partials(params: AttnParams, q_block, k_pages, v_pages, page_
     """The attention kernel alone; with several splits only the workspace partials are written."""
     nld_block_attn(params, q_block, k_pages, v_pages, page_table, prefix_lens, block_len, mode, out, lse,
                    workspace, stream, _entry="nld_block_attn_partials")
+
+
+def nld_block_attn_static_scratch(params: AttnParams, q_block, k_pages, v_pages, page_table, prefix_lens,
+                                  block_len: int, mode: int, out, lse=None, stream=None):
+    """nld_block_attn without a workspace: the split partials live in a fixed
+    16 MiB device array inside the library (for callers that cannot allocate)."""
+    B, Hq, Hkv, D, P = params.batch, params.num_q_heads, params.num_kv_heads, params.head_dim, params.page_size
+    _expect(q_block, torch.bfloat16, (B, block_len, Hq, D), "q_block")
+    _expect(k_pages, torch.bfloat16, (params.num_pages, Hkv, P, D), "k_pages")
+    _expect(v_pages, torch.bfloat16, (params.num_pages, Hkv, P, D), "v_pages")
+    _expect(page_table, torch.int32, (B, params.max_pages_per_seq), "page_table")
+    _expect(prefix_lens, torch.int32, (B,), "prefix_lens")
+    _expect(out, torch.bfloat16, (B, block_len, Hq, D), "out")
+    if lse is not None:
+        _expect(lse, torch.float32, (B, Hq, block_len), "lse")
+    st = lib().nld_block_attn_static_scratch(ctypes.byref(params), _ptr(q_block), _ptr(k_pages), _ptr(v_pages),
+                                             _ptr(page_table), _ptr(prefix_lens), int(block_len), int(mode),
+                                             _ptr(out), _ptr(lse), _stream(stream))
+    _check(st, "nld_block_attn_static_scratch")
 
 
 def nld_split_kv_combine(o_part, lse_part, out, lse=None, stream=None):
