@@ -58,6 +58,8 @@ def parse_args():
     ap.add_argument("--pools", type=int, default=32, help="rotating KV pools (cold-L2 rotation)")
     ap.add_argument("--splits", type=int, default=0, help="KV splits (0 = automatic)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-prefix-ready", action="store_true",
+                    help="do not let attention stream prefix KV before its dependency wait")
     ap.add_argument("--seed", type=int, default=0)
     return ap.parse_args()
 
@@ -196,7 +198,11 @@ def run_ours(args, world, rank, local):
     table = torch.from_numpy(kv.page_table).to(dev)
     prefix = torch.from_numpy(kv.prefix_lens).to(dev)
     q_d, q_v = dev_bf16(c.q_draft_bits), dev_bf16(c.q_verify_bits)
-    params = nld.make_params(B, Hq, Hkv, D, c.page_size, kv.num_pages, kv.max_pages, args.splits, 0.0)
+    # The page table, prefix lengths and prefix KV are not written by the
+    # kernels of the step, so each attention pass may start streaming its
+    # prefix before waiting on the previous kernel (NLD_ATTN_PREFIX_READY).
+    params = nld.make_params(B, Hq, Hkv, D, c.page_size, kv.num_pages, kv.max_pages, args.splits, 0.0,
+                             0 if args.no_prefix_ready else nld.NLD_ATTN_PREFIX_READY)
     splits = nld.nld_block_attn_num_splits(params, bl)
     ws = torch.empty(max(nld.nld_block_attn_workspace_size(params, bl), 16), dtype=torch.uint8, device=dev)
     out_d = torch.empty((B, bl, Hq, D), dtype=torch.bfloat16, device=dev)
@@ -334,7 +340,8 @@ def run_ours(args, world, rank, local):
     attn_iso_ms = float(np.mean([x.elapsed_time(y) for x, y in evs]))
 
     # ---- end to end through the API with host buffers ----
-    e2e = run_e2e(args, torch, nld, dev, stream, wl, params, splits, kv_bytes, world)
+    e2e_params = nld.make_params(B, Hq, Hkv, D, c.page_size, kv.num_pages, kv.max_pages, args.splits, 0.0, 0)
+    e2e = run_e2e(args, torch, nld, dev, stream, wl, e2e_params, splits, kv_bytes, world)
 
     if world > 1:
         dist.barrier()
@@ -364,7 +371,7 @@ def run_ours(args, world, rank, local):
             "workload": WORKLOAD,
             "batch_per_gpu": B, "q_heads": Hq, "kv_heads": Hkv, "head_dim": D, "prefix": int(kv.prefix_lens[0]),
             "block_len": bl, "page_size": c.page_size, "page_order": "random permutation",
-            "kv_splits": splits, "unmask_k": k_unmask,
+            "kv_splits": splits, "unmask_k": k_unmask, "prefix_ready_flag": not args.no_prefix_ready,
             "step": "diffusion attention + unmask + verify attention + accept (one attention layer)",
             "l2": f"cold: each pass reads its own KV pool from a rotation of {npool} pools "
                   f"({npool * kv_bytes / 2**20:.0f} MiB > 3x L2 {l2 / 2**20:.0f} MiB)",

@@ -71,6 +71,7 @@ typedef enum {
  *   num_splits        KV splits per (sequence, KV head); 0 = choose from the
  *                     SM count. Values above 128 are rejected.
  *   softmax_scale     score scale; 0 = 1/sqrt(head_dim)
+ *   flags             0, or NLD_ATTN_PREFIX_READY
  */
 typedef struct {
     int batch;
@@ -82,7 +83,20 @@ typedef struct {
     int max_pages_per_seq;
     int num_splits;
     float softmax_scale;
+    unsigned int flags;
 } nld_attn_params_t;
+
+/*
+ * NLD_ATTN_PREFIX_READY: the caller guarantees that page_table, prefix_lens
+ * and the cached prefix K/V (slots below L_b) are not written by kernels
+ * that were enqueued earlier on the same stream and may still be running.
+ * The attention kernels are launched with programmatic stream serialization;
+ * with this flag they start streaming the prefix K/V before waiting for
+ * those earlier kernels, overlapping the load ramp with them. The block's
+ * own K/V slots, q_block and the outputs are still accessed only after the
+ * wait. Without the flag nothing is read before the wait.
+ */
+#define NLD_ATTN_PREFIX_READY 0x1u
 
 /*
  * Number of KV splits nld_block_attn will use for these parameters (>= 1),

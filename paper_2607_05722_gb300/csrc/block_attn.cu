@@ -62,8 +62,8 @@ __global__ void __launch_bounds__(MaxWarps<NWT>::value * 32, 1)
     prefetch_tensormap(&tmk);
     prefetch_tensormap(&tmv);
   }
+  grid_launch_dependents();  // dependents launch early; they wait on this grid themselves
   grid_dependency_wait();
-  grid_launch_dependents();
   __syncthreads();
 
   const int lmax = a.max_pages * a.page_size - a.bl;
@@ -91,7 +91,7 @@ __global__ void __launch_bounds__(MaxWarps<NWT>::value * 32, 1)
   if (warp == ncons) {
     PagePrefetch first;
     first.load(a, b, t_begin, 0, lane);
-    produce_kv<D>(a, &tmk, &tmv, smem, full, empty, nstage, g, b, t_begin, t_end, ntiles, lane, 3, first);
+    produce_kv<D>(a, &tmk, &tmv, smem, full, empty, nstage, g, b, t_begin, t_end, ntiles, lane, 0, 1, first, 0);
     return;
   }
 

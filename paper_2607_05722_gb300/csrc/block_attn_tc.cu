@@ -6,16 +6,19 @@
 // heads times the bl block tokens form R = G*bl <= 128 query rows, padded to
 // the 128-row MMA tile, so each K/V page leaves HBM once per (b, g).
 //
-// Warp roles (7 warps):
-//   warps 0-1 TMA producers: the K (warp 0) and V (warp 1) boxes of 64-token
-//             tiles into a 4-stage ring (produce_kv); two issuing warps halve
-//             the issue time, which is per warp.
-//   warp 2    allocates 256 TMEM columns; lane 0 issues every MMA:
+// Warp roles (9 warps):
+//   warps 0-2, 8  TMA producers: the boxes of each 64-token K/V tile (16 tokens
+//             x 64 dims each) dealt four ways into a 4-stage ring (produce_kv);
+//             TMA issue cost is per warp, so four issuing warps land a tile
+//             sooner.
+//   warp 3    allocates 256 TMEM columns; lane 0 issues every MMA (it shares
+//             an SM sub-partition with the softmax warp of rows 96-127, which
+//             are padding for the shapes with fewer packed rows):
 //               S_k = Q K_k^T   (M=128 rows, N=64 tokens, K=D; double-buffered in TMEM)
 //               O  += P_k V_k   (M=128 rows, N=D, K=64 tokens; V read MN-major)
 //             S_{k+1} is issued before O += P_k V_k so the tensor core computes
 //             the next scores while the softmax warps work on the current ones.
-//   warps 3-6 softmax: thread t owns query row 32*(warp%4)+lane (its TMEM lane).
+//   warps 4-7 softmax: thread t owns query row 32*(warp%4)+lane (its TMEM lane).
 //             It loads its S row, applies the mask and the base-2 scale,
 //             keeps the running max and sum, writes P (bf16) to shared memory
 //             for the PV MMA, and at the end reads O from TMEM, divides by the
@@ -30,9 +33,12 @@ namespace nld {
 namespace {
 
 constexpr int kTcStages = 4;
-constexpr int kTcThreads = 224;
-constexpr int kMmaWarp = 2;
-constexpr int kSoftmaxWarp0 = 3;
+constexpr int kProducers = 4;
+constexpr int kMmaWarp = 3;
+constexpr int kSoftmaxWarp0 = 4;
+constexpr int kTcThreads = 32 * 9;
+// producer index of a warp, or -1
+__device__ __forceinline__ int producer_index(int warp) { return warp < 3 ? warp : (warp == 8 ? 3 : -1); }
 constexpr uint32_t kTmemCols = 256;  // S0 | S1 (64 columns each) | O (D <= 128 columns)
 constexpr float kRescaleLog2 = 8.0f;
 
@@ -75,7 +81,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kTcStages; ++s) {
-      mbar_init(&kv_full[s], 2);  // K and V producer warps
+      mbar_init(&kv_full[s], kProducers);  // one expect_tx arrival per producer warp
       mbar_init(&kv_empty[s], 1);
     }
     for (int j = 0; j < 2; ++j) {
@@ -96,14 +102,19 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     tmem_alloc(tmem_slot, kTmemCols);
     tc_fence_before();
   }
-  grid_dependency_wait();
-  grid_launch_dependents();
+  // Without NLD_ATTN_PREFIX_READY nothing global is read before the
+  // dependency wait. With it, the page table, the prefix lengths and
+  // prefix-only K/V tiles are read first, and only the block slots, Q and the
+  // outputs wait (producers: in produce_kv; softmax warps: before Q).
+  const bool early = a.prefix_ready != 0;
+  grid_launch_dependents();  // dependents launch early; they wait on this grid themselves
+  if (!early) grid_dependency_wait();
   const int t_begin = split * a.chunk;
   // The producers' first page-id loads and the prefix-length load are
   // independent, so they are in flight together.
   PagePrefetch first;
   first.raw = 0;
-  if (warp < 2) first.load(a, b, t_begin, 0, lane);
+  if (producer_index(warp) >= 0) first.load(a, b, t_begin, 0, lane);
   int L = __ldg(a.prefix_lens + b);
   __syncthreads();
   tc_fence_after();
@@ -123,14 +134,22 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
   if (ntiles == 0) {
     // This split lies past the sequence: its partials carry no keys.
+    if (early) grid_dependency_wait();
     for (int r = threadIdx.x; r < a.R; r += blockDim.x) {
       const int i = r / a.G, h = g * a.G + (r - i * a.G);
       a.lse_part[((static_cast<size_t>(split) * a.B + b) * a.Hq + h) * a.bl + i] = -INFINITY;
     }
-  } else if (warp < 2) {
-    // ---------------- producers (warp 0: K, warp 1: V) ----------------
+  } else if (producer_index(warp) >= 0) {
+    // ---------------- producers ----------------
+    int early_tiles = 0;  // leading tiles made of prefix tokens only
+    if (early) {
+      while (early_tiles < kTcStages && early_tiles < ntiles &&
+             min(t_begin + (early_tiles + 1) * kTileTok, t_end) <= L)
+        ++early_tiles;
+      if (early_tiles == 0) grid_dependency_wait();
+    }
     const int issued = produce_kv<D>(a, &tmk, &tmv, smem, kv_full, kv_empty, kTcStages, g, b, t_begin, t_end,
-                                     ntiles, lane, warp == 0 ? 1 : 2, first);
+                                     ntiles, lane, producer_index(warp), kProducers, first, early_tiles);
     if (lane == 0 && issued < ntiles) {
       // Stopped early on a wait timeout: let the copies already issued land
       // before the CTA exits (bounded).
@@ -222,6 +241,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
     // Q row -> shared memory in the 128-byte-swizzled K-major layout; padding
     // rows are zero. Padding rows of P are zeroed once for both buffers.
+    if (early) grid_dependency_wait();
     {
       const uint4* qrow = reinterpret_cast<const uint4*>(
           a.q + ((static_cast<size_t>(b) * a.bl + row_i) * a.Hq + row_h) * D);
@@ -399,13 +419,23 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         __syncwarp();
         const int chunks = row_bytes / 16;  // 8..32 lanes move one row
         uint8_t* gbase = split_out ? reinterpret_cast<uint8_t*>(a.o_part) : reinterpret_cast<uint8_t*>(a.out);
+        // Eight rows per batch: all shared-memory reads of a batch are issued
+        // before its global stores (through generic pointers the compiler
+        // cannot reorder a read after an earlier store on its own).
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const size_t row = __shfl_sync(0xffffffffu, my_row, j);
-          const bool w = __shfl_sync(0xffffffffu, my_write, j);
-          if (w && lane < chunks)
-            *reinterpret_cast<uint4*>(gbase + row * row_bytes + lane * 16) =
-                *reinterpret_cast<const uint4*>(stage + j * pitch + lane * 16);
+        for (int j0 = 0; j0 < 32; j0 += 8) {
+          uint4 v[8];
+          size_t row[8];
+          bool w[8];
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            row[u] = __shfl_sync(0xffffffffu, my_row, j0 + u);
+            w[u] = __shfl_sync(0xffffffffu, my_write, j0 + u) && lane < chunks;
+            v[u] = *reinterpret_cast<const uint4*>(stage + (j0 + u) * pitch + lane * 16);
+          }
+#pragma unroll
+          for (int u = 0; u < 8; ++u)
+            if (w[u]) *reinterpret_cast<uint4*>(gbase + row[u] * row_bytes + lane * 16) = v[u];
         }
         if (row_ok) {
           if (!split_out) {

@@ -16,8 +16,8 @@ __global__ void __launch_bounds__(kCombineWarps * 32)
     combine_kernel(const float* __restrict__ o_part, const float* __restrict__ lse_part, int S, int B, int Hq,
                    int bl, __nv_bfloat16* __restrict__ out, float* __restrict__ lse) {
   constexpr int V = D / 32;  // dims per lane (2 or 4)
+  grid_launch_dependents();  // dependents launch early; they wait on this grid themselves
   grid_dependency_wait();
-  grid_launch_dependents();
   const int lane = threadIdx.x & 31;
   const long row = static_cast<long>(blockIdx.x) * kCombineWarps + (threadIdx.x >> 5);
   const long R = static_cast<long>(B) * Hq * bl;
@@ -28,16 +28,41 @@ __global__ void __launch_bounds__(kCombineWarps * 32)
   const int h = static_cast<int>(bh % Hq);
   const int b = static_cast<int>(bh / Hq);
 
-  // Lane j holds lse of splits j, j+32, j+64, j+96 (S <= 128): all loads in flight at once.
+  // One memory round trip per 32 splits: each lane loads its share of the
+  // partial rows at the same time as the lse values (lane j holds lse of
+  // splits j, j+32, ...). Partials of splits without keys (lse = -inf) were
+  // never written; their loads are discarded by a select, not multiplied.
   constexpr int kMaxPerLane = kMaxSplits / 32;
+  constexpr int kRound = 32;
+  const long split_stride = R * static_cast<long>(D);
+  const float* base = o_part + static_cast<long>(row) * D + lane * V;
   float ls[kMaxPerLane];
-  float m = -INFINITY;
 #pragma unroll
   for (int u = 0; u < kMaxPerLane; ++u) {
     const int s = lane + 32 * u;
     ls[u] = s < S ? __ldg(lse_part + static_cast<long>(s) * R + row) : -INFINITY;
-    m = fmaxf(m, ls[u]);
   }
+  float x[kRound][V];
+  auto load_round = [&](int s0) {
+#pragma unroll
+    for (int u = 0; u < kRound; ++u) {
+      const int s = s0 + u;
+      if (s < S) {
+        const float* op = base + s * split_stride;
+        if constexpr (V == 4) {
+          const float4 t = __ldg(reinterpret_cast<const float4*>(op));
+          x[u][0] = t.x; x[u][1] = t.y; x[u][2] = t.z; x[u][3] = t.w;
+        } else {
+          const float2 t = __ldg(reinterpret_cast<const float2*>(op));
+          x[u][0] = t.x; x[u][1] = t.y;
+        }
+      }
+    }
+  };
+  load_round(0);
+  float m = -INFINITY;
+#pragma unroll
+  for (int u = 0; u < kMaxPerLane; ++u) m = fmaxf(m, ls[u]);
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
 
@@ -55,40 +80,18 @@ __global__ void __launch_bounds__(kCombineWarps * 32)
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) csum += __shfl_xor_sync(0xffffffffu, csum, off);
-    // Accumulate kRound splits per round; the loads of a round are
-    // independent, so a row with up to kRound splits costs one L2 latency.
-    const float* base = o_part + static_cast<long>(row) * D + lane * V;
-    const long split_stride = R * static_cast<long>(D);
-    constexpr int kRound = 32;
     for (int s0 = 0; s0 < S; s0 += kRound) {
-      float wv[kRound];
-      float x[kRound][V];
+      if (s0 > 0) load_round(s0);
+      const int blk = s0 >> 5;  // warp-uniform
+      const float wsrc = blk == 0 ? w[0] : blk == 1 ? w[1] : blk == 2 ? w[2] : w[3];
 #pragma unroll
       for (int u = 0; u < kRound; ++u) {
-        const int s = s0 + u;
-        const int src = s & 31;
-        const int blk = s >> 5;  // warp-uniform
-        float wsel = blk == 0 ? w[0] : blk == 1 ? w[1] : blk == 2 ? w[2] : w[3];
-        wsel = __shfl_sync(0xffffffffu, wsel, src);
-        wv[u] = s < S ? wsel : 0.f;
-        if (wv[u] != 0.f) {  // warp-uniform: empty splits are never read
-          const float* op = base + s * split_stride;
-          if constexpr (V == 4) {
-            const float4 t = __ldg(reinterpret_cast<const float4*>(op));
-            x[u][0] = t.x; x[u][1] = t.y; x[u][2] = t.z; x[u][3] = t.w;
-          } else {
-            const float2 t = __ldg(reinterpret_cast<const float2*>(op));
-            x[u][0] = t.x; x[u][1] = t.y;
-          }
-        } else {
+        const float wu = __shfl_sync(0xffffffffu, wsrc, u);
+        if (s0 + u < S && wu > 0.f) {
 #pragma unroll
-          for (int v = 0; v < V; ++v) x[u][v] = 0.f;
+          for (int v = 0; v < V; ++v) acc[v] += wu * x[u][v];
         }
       }
-#pragma unroll
-      for (int u = 0; u < kRound; ++u)
-#pragma unroll
-        for (int v = 0; v < V; ++v) acc[v] += wv[u] * x[u][v];
     }
   }
   const float inv = csum > 0.f ? 1.f / csum : 0.f;

@@ -15,8 +15,8 @@ constexpr int kDecideWarps = 8;
 __global__ void __launch_bounds__(kDecideWarps * 32)
     accept_kernel(const int32_t* __restrict__ draft, const int32_t* __restrict__ verify, int B, int n,
                   int32_t* __restrict__ accepted) {
+  grid_launch_dependents();  // dependents launch early; they wait on this grid themselves
   grid_dependency_wait();
-  grid_launch_dependents();
   const int lane = threadIdx.x & 31;
   const long b = static_cast<long>(blockIdx.x) * kDecideWarps + (threadIdx.x >> 5);
   if (b >= B) return;
@@ -28,8 +28,8 @@ __global__ void __launch_bounds__(kDecideWarps * 32)
 __global__ void __launch_bounds__(kDecideWarps * 32)
     unmask_kernel(const float* __restrict__ conf, int B, int n, int k, int32_t* __restrict__ positions,
                   int32_t* __restrict__ num_selected) {
+  grid_launch_dependents();  // dependents launch early; they wait on this grid themselves
   grid_dependency_wait();
-  grid_launch_dependents();
   const int lane = threadIdx.x & 31;
   const long b = static_cast<long>(blockIdx.x) * kDecideWarps + (threadIdx.x >> 5);
   if (b >= B) return;

@@ -49,6 +49,7 @@ nld_status_t check_params(const nld_attn_params_t* p, int block_len) {
       p->max_pages_per_seq < 1 || p->num_splits < 0 || p->softmax_scale < 0.f || !isfinite(p->softmax_scale))
     return NLD_ERR_INVALID_ARG;
   if (p->num_q_heads % p->num_kv_heads != 0) return NLD_ERR_INVALID_ARG;
+  if (p->flags & ~NLD_ATTN_PREFIX_READY) return NLD_ERR_INVALID_ARG;
   if (block_len < 1 || block_len > nld::kMaxBlock) return NLD_ERR_INVALID_ARG;
   if (p->num_splits > nld::kMaxSplits) return NLD_ERR_INVALID_ARG;
   if (!is_pow2(p->page_size) || p->page_size < 16 || p->page_size > 256) return NLD_ERR_INVALID_ARG;
@@ -233,6 +234,7 @@ nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_bloc
   a.chunk = plan.chunk;
   a.mode = static_cast<int>(mode);
   a.scale_log2 = scale * nld::kLog2e;
+  a.prefix_ready = (params->flags & NLD_ATTN_PREFIX_READY) ? 1 : 0;
   if (plan.splits > 1) {
     a.o_part = static_cast<float*>(workspace);
     a.lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) + o_bytes);

@@ -36,6 +36,7 @@ struct AttnArgs {
   int num_splits, chunk;       // splits and tokens per split (multiple of 16)
   int mode, nstage, nwr;       // mask mode, pipeline depth, 16-row warp groups
   float scale_log2;            // softmax scale * log2(e)
+  int prefix_ready;            // NLD_ATTN_PREFIX_READY: prefix K/V may be read before the dependency wait
 };
 
 // Launchers (defined next to their kernels). Return a CUDA error code.
@@ -65,10 +66,13 @@ AttnShape attn_shape(int R, int head_dim);
 size_t max_smem_bytes(int head_dim);
 
 // Launch with programmatic stream serialization: the kernel may start while
-// its predecessor in the stream is still running; every kernel of this
-// library calls grid_dependency_wait() before it touches global memory, so
-// only launch latency and prologue (barrier setup, descriptor prefetch)
-// overlap the predecessor. Set NLD_DISABLE_PDL=1 to launch plainly.
+// its predecessor in the stream is still running. Every kernel of this
+// library releases its dependents at its start (they can only launch once
+// all of this grid's CTAs are resident, so none of them can be starved) and
+// calls grid_dependency_wait() before it touches data an earlier kernel may
+// produce, so launch latency and prologue (barrier setup, descriptor
+// prefetch, and with NLD_ATTN_PREFIX_READY the prefix K/V stream) overlap
+// the predecessor. Set NLD_DISABLE_PDL=1 to launch plainly.
 bool pdl_enabled();
 
 template <typename... KArgs, typename... Args>
@@ -350,22 +354,24 @@ struct PagePrefetch {
   }
 };
 
-// Producer warp: streams the K tiles (kinds & 1), the V tiles (kinds & 2) or
-// both of tokens [t_begin, t_end) of (sequence b, KV head g) into an nstage
-// ring. `first` holds the page ids of the first 32 groups, already loaded.
-// The boxes of a tile are issued by separate lanes; a warp's expect_tx covers
-// only the bytes it issues, so `full` expects one arrival per producing warp.
-// Returns the number of tiles issued.
+// Producer warp `pw` of `nprod`: streams its share of the TMA boxes of the
+// K/V tiles of tokens [t_begin, t_end) of (sequence b, KV head g) into an
+// nstage ring. A tile has 4 groups x D/64 column blocks x {K, V} boxes
+// (16 tokens x 64 dims each); they are dealt to the producer warps in equal
+// shares and, within a warp, one box per lane. TMA issue cost is per warp, so
+// more producer warps land a tile sooner. A warp's expect_tx covers only its
+// own boxes, so `full` expects one arrival per producer warp. `first` holds
+// the page ids of the first 32 groups, already loaded. Returns tiles issued.
 template <int D>
 __device__ __forceinline__ int produce_kv(const AttnArgs& a, const CUtensorMap* tmk, const CUtensorMap* tmv,
                                           uint8_t* stages, uint64_t* full, uint64_t* empty, int nstage, int g,
-                                          int b, int t_begin, int t_end, int ntiles, int lane, int kinds,
-                                          const PagePrefetch& first) {
+                                          int b, int t_begin, int t_end, int ntiles, int lane, int pw, int nprod,
+                                          const PagePrefetch& first, int early_tiles) {
   using Geo = TileGeom<D>;
-  const int nkinds = (kinds & 1) + ((kinds >> 1) & 1);
-  const int ops_per_group = nkinds * Geo::kColBlocks;
-  const int ops_per_tile = (kTileTok / kGroupTok) * ops_per_group;  // <= 32
-  const uint32_t bytes = nkinds * Geo::kTileBytes;
+  constexpr int kGroups = kTileTok / kGroupTok;
+  constexpr int kOpsPerTile = kGroups * 2 * Geo::kColBlocks;  // 16 (D=128) or 8 (D=64)
+  const int my_ops = kOpsPerTile / nprod;                     // nprod divides kOpsPerTile
+  const uint32_t bytes = static_cast<uint32_t>(my_ops) * kGroupTok * 128;
   int page_cur = first.validate(a, t_begin, t_end, 0, lane);
   PagePrefetch nxt;
   nxt.raw = 0;
@@ -373,6 +379,9 @@ __device__ __forceinline__ int produce_kv(const AttnArgs& a, const CUtensorMap* 
   int issued = 0;
   for (int k = 0; k < ntiles; ++k) {
     const int st = k % nstage;
+    // The first `early_tiles` tiles hold prefix tokens only and may be issued
+    // before the dependency wait (NLD_ATTN_PREFIX_READY); the rest wait.
+    if (k == early_tiles && early_tiles > 0) grid_dependency_wait();
     if (k >= nstage) {
       int ok = 1;
       if (lane == 0) ok = mbar_wait(&empty[st], ((k / nstage) - 1) & 1, a.err) ? 1 : 0;
@@ -385,12 +394,15 @@ __device__ __forceinline__ int produce_kv(const AttnArgs& a, const CUtensorMap* 
     }
     if (lane == 0) mbar_arrive_expect_tx(&full[st], bytes);
     __syncwarp();
-    const int grp = lane / ops_per_group;
-    const int page = __shfl_sync(0xffffffffu, page_cur, ((k & 7) * 4 + grp) & 31);
-    if (lane < ops_per_tile) {
-      const int r = lane - grp * ops_per_group;
-      const int cb = r % Geo::kColBlocks;
-      const bool is_v = (kinds == 2) || (kinds == 3 && r >= Geo::kColBlocks);
+    // op -> (group, kind, column block): group fastest, so a warp's boxes
+    // spread over the tile's pages.
+    const int op = pw * my_ops + (lane < my_ops ? lane : 0);
+    const int grp = op % kGroups;
+    const int kind_cb = op / kGroups;  // 0 .. 2*kColBlocks-1
+    const bool is_v = kind_cb >= Geo::kColBlocks;
+    const int cb = kind_cb % Geo::kColBlocks;
+    const int page = __shfl_sync(0xffffffffu, page_cur, ((k & 7) * kGroups + grp) & 31);
+    if (lane < my_ops) {
       const int t = t_begin + k * kTileTok + grp * kGroupTok;
       const int slot = page < a.num_pages ? (t & (a.page_size - 1)) : 0;
       uint8_t* dst = stages + st * Geo::kStageBytes + (is_v ? Geo::kTileBytes : 0) + cb * Geo::kColBlockBytes +

@@ -23,6 +23,7 @@ NLD_MODE_VERIFY = 1
 NLD_DEVERR_PREFIX_RANGE = 0x1
 NLD_DEVERR_PAGE_RANGE = 0x2
 NLD_DEVERR_WAIT_TIMEOUT = 0x4
+NLD_ATTN_PREFIX_READY = 0x1
 
 HEADER = os.path.join(_build.INCLUDE, "nld.h")
 
@@ -37,7 +38,7 @@ class AttnParams(ctypes.Structure):
     _fields_ = [("batch", ctypes.c_int), ("num_q_heads", ctypes.c_int), ("num_kv_heads", ctypes.c_int),
                 ("head_dim", ctypes.c_int), ("page_size", ctypes.c_int), ("num_pages", ctypes.c_int),
                 ("max_pages_per_seq", ctypes.c_int), ("num_splits", ctypes.c_int),
-                ("softmax_scale", ctypes.c_float)]
+                ("softmax_scale", ctypes.c_float), ("flags", ctypes.c_uint)]
 
 
 _lib = None
@@ -117,16 +118,16 @@ def _expect(t: torch.Tensor, dtype, shape, name):
 
 
 def make_params(batch, num_q_heads, num_kv_heads, head_dim, page_size, num_pages, max_pages_per_seq,
-                num_splits=0, softmax_scale=0.0) -> AttnParams:
+                num_splits=0, softmax_scale=0.0, flags=0) -> AttnParams:
     return AttnParams(batch, num_q_heads, num_kv_heads, head_dim, page_size, num_pages, max_pages_per_seq,
-                      num_splits, softmax_scale)
+                      num_splits, softmax_scale, flags)
 
 
 def params_for(q_block: torch.Tensor, k_pages: torch.Tensor, page_table: torch.Tensor, num_splits=0,
-               softmax_scale=0.0) -> AttnParams:
+               softmax_scale=0.0, flags=0) -> AttnParams:
     B, bl, Hq, D = q_block.shape
     num_pages, Hkv, P, _ = k_pages.shape
-    return make_params(B, Hq, Hkv, D, P, num_pages, page_table.shape[1], num_splits, softmax_scale)
+    return make_params(B, Hq, Hkv, D, P, num_pages, page_table.shape[1], num_splits, softmax_scale, flags)
 
 
 def nld_block_attn_num_splits(params: AttnParams, block_len: int) -> int:

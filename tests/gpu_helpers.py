@@ -34,14 +34,14 @@ class DeviceCase:
     def q_bits(self, mode):
         return self.case.q_draft_bits if mode == W.MODE_DIFFUSION else self.case.q_verify_bits
 
-    def params(self, num_splits=0):
+    def params(self, num_splits=0, flags=0):
         c = self.case
         return nld.make_params(c.batch, c.num_q_heads, c.num_kv_heads, c.head_dim, c.page_size,
-                               c.kv.num_pages, c.kv.max_pages, num_splits, 0.0)
+                               c.kv.num_pages, c.kv.max_pages, num_splits, 0.0, flags)
 
-    def run(self, mode, num_splits=0, q=None):
+    def run(self, mode, num_splits=0, q=None, flags=0):
         c = self.case
-        p = self.params(num_splits)
+        p = self.params(num_splits, flags)
         q = self.q[mode] if q is None else q
         out = torch.empty((c.batch, c.block_len, c.num_q_heads, c.head_dim), dtype=torch.bfloat16, device=q.device)
         lse = torch.empty((c.batch, c.num_q_heads, c.block_len), dtype=torch.float32, device=q.device)

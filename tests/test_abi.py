@@ -64,6 +64,7 @@ def test_split_plan_and_workspace_size(L):
     (dict(), 33, 1),                        # block_len > 32
     (dict(num_q_heads=48, num_kv_heads=8), 32, 2),  # 6 * 32 = 192 packed rows > 160
     (dict(batch=0), 16, 1),
+    (dict(flags=2), 16, 1),                 # unknown flag bit
 ])
 def test_block_attn_rejects_bad_shapes(L, kw, bl, code):
     p = params(**kw)

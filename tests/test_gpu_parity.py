@@ -188,6 +188,23 @@ def test_attention_small_all_rows(orc, spec, mode, splits):
     compare_attn(out, lse, ro, rl, f"{name} mode={mode} S={splits}")
 
 
+@pytest.mark.parametrize("spec", SMALL, ids=[s[0] for s in SMALL])
+def test_prefix_ready_flag_same_result(orc, spec):
+    """NLD_ATTN_PREFIX_READY only moves prefix loads before the dependency
+    wait: results are bit-identical to the unflagged call and match the oracle."""
+    name, B, Hq, Hkv, D, P, bl, prefix = spec
+    case = W.make_block_attn_case(name, B, Hq, Hkv, D, block_len=bl, page_size=P, prefix_lens=prefix,
+                                  seed=sum(prefix) + 2 * bl)
+    dc = DeviceCase(case)
+    for mode in (DIFF, VER):
+        for splits in (0, 1, 3):
+            o0, l0 = dc.run(mode, splits)
+            o1, l1 = dc.run(mode, splits, flags=nld.NLD_ATTN_PREFIX_READY)
+            assert torch.equal(o0, o1) and torch.equal(l0, l1)
+            ro, rl = oracle_full(orc, case, mode)
+            compare_attn(o1, l1, ro, rl, f"{name} flag mode={mode} S={splits}")
+
+
 def test_attention_tail_slots_hold_nan(orc):
     """Cache slots past the block inside the last page may be uninitialised;
     NaN there must not reach the output."""
@@ -302,7 +319,8 @@ def test_full_size_workload_sampled_rows(orc, name):
     for mode in (DIFF, VER):
         if mode == DIFF and "diffusion" not in wl.steps:
             continue
-        out, lse = dc.run(mode)  # automatic split count, as the bench runs it
+        # automatic split count and the prefix-ready flag, as the bench runs it
+        out, lse = dc.run(mode, flags=nld.NLD_ATTN_PREFIX_READY)
         rows = sample_rows(case, 48, seed=mode + 1)
         qb = dc.q_bits(mode)
         ro, rl = orc.block_attn_rows(qb, case.kv.k_bits, case.kv.v_bits, case.kv.page_table, case.kv.prefix_lens,
