@@ -371,7 +371,7 @@ def run_ours(args, world, rank, local):
             "workload": WORKLOAD,
             "batch_per_gpu": B, "q_heads": Hq, "kv_heads": Hkv, "head_dim": D, "prefix": int(kv.prefix_lens[0]),
             "block_len": bl, "page_size": c.page_size, "page_order": "random permutation",
-            "kv_splits": splits, "unmask_k": k_unmask, "prefix_ready_flag": not args.no_prefix_ready,
+            "kv_partials": splits, "unmask_k": k_unmask, "prefix_ready_flag": not args.no_prefix_ready,
             "step": "diffusion attention + unmask + verify attention + accept (one attention layer)",
             "l2": f"cold: each pass reads its own KV pool from a rotation of {npool} pools "
                   f"({npool * kv_bytes / 2**20:.0f} MiB > 3x L2 {l2 / 2**20:.0f} MiB)",

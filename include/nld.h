@@ -68,8 +68,9 @@ typedef enum {
  *   page_size         P, tokens per page: a power of two in [16, 256]
  *   num_pages         pages in the pool (first dim of k_pages / v_pages)
  *   max_pages_per_seq second dim of page_table
- *   num_splits        KV splits per (sequence, KV head); 0 = choose from the
- *                     SM count. Values above 128 are rejected.
+ *   num_splits        pieces the KV range of each (sequence, KV head) is cut
+ *                     into; 0 = choose from the SM count. Values above 128
+ *                     are rejected.
  *   softmax_scale     score scale; 0 = 1/sqrt(head_dim)
  *   flags             0, or NLD_ATTN_PREFIX_READY
  */
@@ -99,9 +100,13 @@ typedef struct {
 #define NLD_ATTN_PREFIX_READY 0x1u
 
 /*
- * Number of KV splits nld_block_attn will use for these parameters (>= 1),
- * or -1 if the parameters are invalid. With num_splits = 0 it queries the
- * current device's SM count.
+ * Number of split partials per output row that nld_block_attn leaves in the
+ * workspace and merges with the split combine (1: the call writes the final
+ * output directly and needs no workspace), or -1 if the parameters are
+ * invalid. The KV range of each (sequence, KV head) is cut into
+ * params->num_splits pieces (0: chosen from the current device's SM count);
+ * pieces that run as one thread-block cluster merge on chip into a single
+ * partial, so this count can be smaller than the number of pieces.
  */
 int nld_block_attn_num_splits(const nld_attn_params_t *params, int block_len);
 

@@ -24,6 +24,11 @@
 //             for the PV MMA, and at the end reads O from TMEM, divides by the
 //             sum and stages its rows in the freed K/V ring so that each row
 //             leaves as one coalesced store (bf16 output or fp32 split partial).
+// When the KV range of a (sequence, KV head) is split over a thread-block
+// cluster, the CTAs stage their normalised rows in shared memory and merge
+// them through distributed shared memory (a cluster barrier, then each CTA
+// combines a slice of rows from all peers): the final output, or one partial
+// per cluster, leaves the kernel instead of one partial per split.
 // The running max is raised lazily: O is rescaled in TMEM only when a row's
 // max grows by more than 2^8 (P then stays below 256, exact enough in bf16);
 // the final division by the matching sum removes the reference max.
@@ -41,6 +46,12 @@ constexpr int kTcThreads = 32 * 9;
 __device__ __forceinline__ int producer_index(int warp) { return warp < 3 ? warp : (warp == 8 ? 3 : -1); }
 constexpr uint32_t kTmemCols = 256;  // S0 | S1 (64 columns each) | O (D <= 128 columns)
 constexpr float kRescaleLog2 = 8.0f;
+
+// Cluster merge staging in the freed K/V ring: 128 rows of D fp32 (padded
+// pitch), then 128 log2-sum-exp values.
+constexpr int kMergePitchRows = 128;
+template <int D>
+__host__ __device__ constexpr int merge_pitch() { return D * 4 + 16; }
 
 template <int D>
 struct TcLayout {
@@ -135,9 +146,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   if (ntiles == 0) {
     // This split lies past the sequence: its partials carry no keys.
     if (early) grid_dependency_wait();
-    for (int r = threadIdx.x; r < a.R; r += blockDim.x) {
-      const int i = r / a.G, h = g * a.G + (r - i * a.G);
-      a.lse_part[((static_cast<size_t>(split) * a.B + b) * a.Hq + h) * a.bl + i] = -INFINITY;
+    if (a.csize > 1) {
+      float* lse_stage = reinterpret_cast<float*>(smem + kMergePitchRows * merge_pitch<D>());
+      for (int r = threadIdx.x; r < 128; r += blockDim.x) lse_stage[r] = -INFINITY;
+    } else {
+      for (int r = threadIdx.x; r < a.R; r += blockDim.x) {
+        const int i = r / a.G, h = g * a.G + (r - i * a.G);
+        a.lse_part[((static_cast<size_t>(split) * a.B + b) * a.Hq + h) * a.bl + i] = -INFINITY;
+      }
     }
   } else if (producer_index(warp) >= 0) {
     // ---------------- producers ----------------
@@ -379,7 +395,30 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // Every PV has completed once o_done of the last tile fires, so the K/V
     // ring is free: each warp stages its 32 rows there (padded pitch, no bank
     // conflicts), then writes each row with one coalesced warp-wide store.
-    if (ok && mbar_wait(&o_done[(ntiles - 1) & 1], ((ntiles - 1) >> 1) & 1, a.err)) {
+    const bool o_ready = ok && mbar_wait(&o_done[(ntiles - 1) & 1], ((ntiles - 1) >> 1) & 1, a.err);
+    if (a.csize > 1) {
+      // Cluster: stage this CTA's normalised rows and their log2-sum-exp in
+      // the freed ring for the merge across the cluster (rows without keys,
+      // or after a timeout, carry lse = -inf and are skipped by the merge).
+      if (o_ready) tc_fence_after();
+      float* lse_stage = reinterpret_cast<float*>(smem + kMergePitchRows * merge_pitch<D>());
+      const float l = l_run;
+      const bool has = o_ready && row_ok && l > 0.f;
+      lse_stage[r] = has ? m_run + lg2(l) : -INFINITY;
+      if (warp_rows && o_ready) {
+        const float inv = l > 0.f ? 1.f / l : 0.f;
+        uint8_t* my = smem + r * merge_pitch<D>();
+#pragma unroll 1
+        for (int c = 0; c < D / 32; ++c) {
+          float o[32];
+          tmem_ld32(tO + lane_off + c * 32, o);
+#pragma unroll
+          for (int q4 = 0; q4 < 8; ++q4)
+            *reinterpret_cast<float4*>(my + c * 128 + q4 * 16) =
+                make_float4(o[4 * q4] * inv, o[4 * q4 + 1] * inv, o[4 * q4 + 2] * inv, o[4 * q4 + 3] * inv);
+        }
+      }
+    } else if (o_ready) {
       tc_fence_after();
       if (warp_rows) {
         const float l = l_run;
@@ -449,6 +488,99 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     tc_fence_before();
   }
 
+  if (a.csize > 1) {
+    // Merge across the cluster (the splits of this sequence and KV head):
+    // CTA `rank` combines rows [rank*Rc, (rank+1)*Rc) from every peer's
+    // staged rows through distributed shared memory, by the same rule as the
+    // split combine, and writes the final output (one cluster per sequence
+    // and KV head) or this cluster's partial.
+    cluster_sync();
+    if (warp >= kSoftmaxWarp0 && warp < kSoftmaxWarp0 + 4) {
+      const uint32_t rank = cluster_ctarank();
+      const int Rc = (a.R + a.csize - 1) / a.csize;
+      const int r0 = static_cast<int>(rank) * Rc;
+      const int nrows = max(0, min(a.R, r0 + Rc) - r0);
+      const uint32_t stage_u32 = smem_u32(smem);
+      const uint32_t lse_u32 = stage_u32 + kMergePitchRows * merge_pitch<D>();
+      // this CTA's merge weights, local: [row][peer] and the merged lse per row
+      float* wts = reinterpret_cast<float*>(smem + kMergePitchRows * merge_pitch<D>() + 512);
+      float* lse_out = wts + 128 * 8;
+      const int tid = threadIdx.x - 32 * kSoftmaxWarp0;
+      // 1) per-row weights: one thread per row, the peers' lse loads in flight together
+      if (tid < nrows) {
+        const int r = r0 + tid;
+        float lp[8];
+        float m = -INFINITY;
+#pragma unroll
+        for (int p = 0; p < 8; ++p) lp[p] = p < a.csize ? ld_dsmem_f32(dsmem_addr(lse_u32 + r * 4, p)) : -INFINITY;
+#pragma unroll
+        for (int p = 0; p < 8; ++p) m = fmaxf(m, lp[p]);
+        float w[8];
+        float wsum = 0.f;
+#pragma unroll
+        for (int p = 0; p < 8; ++p) {
+          w[p] = (m != -INFINITY && lp[p] != -INFINITY) ? ex2(lp[p] - m) : 0.f;
+          wsum += w[p];
+        }
+        const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
+#pragma unroll
+        for (int p = 0; p < 8; ++p) wts[tid * 8 + p] = w[p] * inv;
+        lse_out[tid] = wsum > 0.f ? (m + lg2(wsum)) * kLn2 : -INFINITY;
+      }
+      named_bar_sync(1, 128);
+      // 2) rows: two (row, 4-dim) items per thread per round, every peer load in flight
+      const bool final_out = a.num_partials == 1;
+      const int pidx = split / a.csize;
+      const int items = nrows * (D / 4);
+      for (int base = tid; base < items; base += 256) {
+        float4 acc[2];
+        int ridx[2], d4[2];
+        bool live[2];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const int idx = base + u * 128;
+          live[u] = idx < items;
+          ridx[u] = live[u] ? idx / (D / 4) : 0;
+          d4[u] = idx % (D / 4);
+          acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+        float4 o[2][8];
+#pragma unroll
+        for (int u = 0; u < 2; ++u)
+#pragma unroll
+          for (int p = 0; p < 8; ++p)
+            if (live[u] && p < a.csize && wts[ridx[u] * 8 + p] > 0.f)  // rows without keys are never read
+              o[u][p] = ld_dsmem_f4(dsmem_addr(stage_u32 + (r0 + ridx[u]) * merge_pitch<D>() + d4[u] * 16, p));
+            else
+              o[u][p] = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+#pragma unroll
+          for (int p = 0; p < 8; ++p) {
+            const float w = p < a.csize ? wts[ridx[u] * 8 + p] : 0.f;
+            acc[u].x += w * o[u][p].x; acc[u].y += w * o[u][p].y;
+            acc[u].z += w * o[u][p].z; acc[u].w += w * o[u][p].w;
+          }
+          if (!live[u]) continue;
+          const int r = r0 + ridx[u];
+          const int i = r / a.G, h = g * a.G + (r - i * a.G);
+          const float lse_v = lse_out[ridx[u]];
+          if (final_out) {
+            __nv_bfloat16* orow = a.out + ((static_cast<size_t>(b) * a.bl + i) * a.Hq + h) * D;
+            *reinterpret_cast<uint2*>(orow + d4[u] * 4) =
+                make_uint2(pack_bf16(acc[u].x, acc[u].y), pack_bf16(acc[u].z, acc[u].w));
+            if (d4[u] == 0 && a.lse != nullptr) a.lse[(static_cast<size_t>(b) * a.Hq + h) * a.bl + i] = lse_v;
+          } else {
+            const size_t prow = ((static_cast<size_t>(pidx) * a.B + b) * a.Hq + h) * a.bl + i;
+            if (lse_v != -INFINITY) *reinterpret_cast<float4*>(a.o_part + prow * D + d4[u] * 4) = acc[u];
+            if (d4[u] == 0) a.lse_part[prow] = lse_v;
+          }
+        }
+      }
+    }
+    cluster_sync();  // peers keep their shared memory until every merge has read it
+  }
+
   __syncthreads();
   if (warp == kMmaWarp) {
     tc_fence_after();
@@ -457,26 +589,65 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 }
 
 template <int D>
-cudaError_t launch_tc_t(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, cudaStream_t stream) {
-  auto kern = block_attn_tc_kernel<D>;
-  const size_t smem = TcLayout<D>::kBytes + 1024;
+cudaError_t configure_tc(int dev) {
   static int configured[64] = {0};
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   if (!__atomic_load_n(&configured[dev], __ATOMIC_ACQUIRE)) {
-    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    cudaError_t e = cudaFuncSetAttribute(block_attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(TcLayout<D>::kBytes + 1024));
     if (e != cudaSuccess) return e;
     __atomic_store_n(&configured[dev], 1, __ATOMIC_RELEASE);
   }
+  return cudaSuccess;
+}
+
+template <int D>
+cudaError_t launch_tc_t(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, cudaStream_t stream) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if ((e = configure_tc<D>(dev)) != cudaSuccess) return e;
   dim3 grid(a.num_splits, a.Hkv, a.B);
-  return launch_kernel(kern, grid, dim3(kTcThreads), smem, stream, tmk, tmv, a);
+  return launch_kernel_cluster(block_attn_tc_kernel<D>, grid, dim3(kTcThreads), TcLayout<D>::kBytes + 1024, stream,
+                               a.csize, tmk, tmv, a);
+}
+
+template <int D>
+int max_active_clusters_t(int csize) {
+  static int cache[64][4];  // [device][log2 csize - 1] + 1 (0 = not queried)
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  const int slot = csize == 2 ? 0 : csize == 4 ? 1 : csize == 8 ? 2 : 3;
+  int v = __atomic_load_n(&cache[dev][slot], __ATOMIC_ACQUIRE);
+  if (v) return v - 1;
+  if (configure_tc<D>(dev) != cudaSuccess) return 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(csize, 1, 1);
+  cfg.blockDim = dim3(kTcThreads);
+  cfg.dynamicSmemBytes = TcLayout<D>::kBytes + 1024;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = csize;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, block_attn_tc_kernel<D>, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    n = 0;
+  }
+  __atomic_store_n(&cache[dev][slot], n + 1, __ATOMIC_RELEASE);
+  return n;
 }
 
 }  // namespace
 
 bool tc_supports(int R, int head_dim) { return R <= 128 && (head_dim == 64 || head_dim == 128); }
+
+int tc_max_active_clusters(int csize, int head_dim) {
+  return head_dim == 128 ? max_active_clusters_t<128>(csize) : max_active_clusters_t<64>(csize);
+}
 
 cudaError_t launch_block_attn_tc(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, int head_dim,
                                  cudaStream_t stream) {

@@ -66,30 +66,60 @@ nld_status_t check_params(const nld_attn_params_t* p, int block_len) {
 // possible sequence, max_pages_per_seq * page_size tokens. Splits past a
 // shorter sequence's end do no work. With num_splits = 0 the count is
 // chosen so that (splits x sequences x KV heads) covers the SMs once.
+// On the tcgen05 kernel the splits of a (sequence, KV head) can run as one
+// thread-block cluster that merges its results on chip and writes the final
+// output, so no workspace and no combine launch are needed. An automatic plan
+// takes floor(SMs / units) splits (one wave) and, when that is 2..8, rounds
+// it down to 2, 4 or 8 and uses one cluster per unit if those clusters are
+// resident at once. An explicit split count of 2, 4 or 8 uses one cluster; a
+// larger count divisible by 8, 4 or 2 uses clusters of that size, leaving
+// one partial per cluster for the combine.
 struct SplitPlan {
-  int splits;
-  int chunk;
+  int splits;    // CTAs along the KV range per (sequence, KV head)
+  int chunk;     // tokens per split
+  int csize;     // cluster size (1 = none)
+  int partials;  // splits / csize
 };
 
 nld_status_t plan_splits(const nld_attn_params_t* p, int block_len, SplitPlan* out) {
   const long long max_tokens = static_cast<long long>(p->max_pages_per_seq) * p->page_size;
+  const long long units = static_cast<long long>(p->batch) * p->num_kv_heads;
+  const bool tc = nld::tc_supports((p->num_q_heads / p->num_kv_heads) * block_len, p->head_dim);
+  const bool automatic = p->num_splits == 0;
   int want = p->num_splits;
-  if (want == 0) {
+  int csize = 1;
+  if (automatic) {
     int sms = 0;
     nld_status_t st = device_state(nullptr, &sms);
     if (st != NLD_OK) return st;
-    const long long units = static_cast<long long>(p->batch) * p->num_kv_heads;
-    long long s = (sms + units - 1) / units;
+    long long s = sms / units;
     const long long by_tiles = (max_tokens + nld::kTileTok - 1) / nld::kTileTok;  // >= one tile per split
     if (s > by_tiles) s = by_tiles;
     if (s > nld::kMaxSplits) s = nld::kMaxSplits;
-    want = static_cast<int>(s < 1 ? 1 : s);
+    if (s < 1) s = 1;
+    want = static_cast<int>(s);
+    if (tc && want >= 2 && want <= 8) {
+      const int cs = want >= 8 ? 8 : want >= 4 ? 4 : 2;
+      if (units <= nld::tc_max_active_clusters(cs, p->head_dim)) {
+        want = cs;
+        csize = cs;
+      }
+    }
+  } else if (tc && want >= 2) {
+    for (int cs = 8; cs >= 2; cs >>= 1)
+      if (want % cs == 0) {
+        csize = cs;
+        break;
+      }
   }
   long long chunk = (max_tokens + want - 1) / want;
   chunk = (chunk + nld::kGroupTok - 1) / nld::kGroupTok * nld::kGroupTok;
+  long long splits = (max_tokens + chunk - 1) / chunk;
+  splits = (splits + csize - 1) / csize * csize;  // trailing empty splits complete a cluster
   out->chunk = static_cast<int>(chunk);
-  out->splits = static_cast<int>((max_tokens + chunk - 1) / chunk);
-  (void)block_len;
+  out->splits = static_cast<int>(splits);
+  out->csize = csize;
+  out->partials = static_cast<int>(splits / csize);
   return NLD_OK;
 }
 
@@ -167,15 +197,16 @@ int nld_block_attn_num_splits(const nld_attn_params_t* params, int block_len) {
   if (check_params(params, block_len) != NLD_OK) return -1;
   SplitPlan plan;
   if (plan_splits(params, block_len, &plan) != NLD_OK) return -1;
-  return plan.splits;
+  return plan.partials;
 }
 
 size_t nld_block_attn_workspace_size(const nld_attn_params_t* params, int block_len) {
   if (check_params(params, block_len) != NLD_OK) return static_cast<size_t>(-1);
   SplitPlan plan;
   if (plan_splits(params, block_len, &plan) != NLD_OK) return static_cast<size_t>(-1);
-  if (plan.splits == 1) return 0;
-  return align256(partial_o_bytes(params, block_len, plan.splits)) + partial_lse_bytes(params, block_len, plan.splits);
+  if (plan.partials == 1) return 0;
+  return align256(partial_o_bytes(params, block_len, plan.partials)) +
+         partial_lse_bytes(params, block_len, plan.partials);
 }
 
 }  // extern "C"
@@ -197,9 +228,9 @@ nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_bloc
   st = plan_splits(params, block_len, &plan);
   if (st != NLD_OK) return st;
   size_t o_bytes = 0;
-  if (plan.splits > 1) {
-    o_bytes = align256(partial_o_bytes(params, block_len, plan.splits));
-    const size_t need = o_bytes + partial_lse_bytes(params, block_len, plan.splits);
+  if (plan.partials > 1) {
+    o_bytes = align256(partial_o_bytes(params, block_len, plan.partials));
+    const size_t need = o_bytes + partial_lse_bytes(params, block_len, plan.partials);
     if (workspace == nullptr || workspace_bytes < need) return NLD_ERR_WORKSPACE;
     if (!aligned(workspace, 16)) return NLD_ERR_INVALID_ARG;
   }
@@ -232,10 +263,12 @@ nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_bloc
   a.max_pages = params->max_pages_per_seq;
   a.num_splits = plan.splits;
   a.chunk = plan.chunk;
+  a.csize = plan.csize;
+  a.num_partials = plan.partials;
   a.mode = static_cast<int>(mode);
   a.scale_log2 = scale * nld::kLog2e;
   a.prefix_ready = (params->flags & NLD_ATTN_PREFIX_READY) ? 1 : 0;
-  if (plan.splits > 1) {
+  if (plan.partials > 1) {
     a.o_part = static_cast<float*>(workspace);
     a.lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) + o_bytes);
   }
@@ -243,8 +276,8 @@ nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_bloc
                             ? nld::launch_block_attn_tc(a, tmk, tmv, params->head_dim, stream)
                             : nld::launch_block_attn(a, tmk, tmv, params->head_dim, stream);
   if (le != cudaSuccess) return NLD_ERR_CUDA;
-  if (plan.splits > 1 && run_combine) {
-    if (nld::launch_combine(a.o_part, a.lse_part, plan.splits, a.B, a.Hq, block_len, params->head_dim, a.out, lse,
+  if (plan.partials > 1 && run_combine) {
+    if (nld::launch_combine(a.o_part, a.lse_part, plan.partials, a.B, a.Hq, block_len, params->head_dim, a.out, lse,
                             stream) != cudaSuccess)
       return NLD_ERR_CUDA;
   }

@@ -37,7 +37,7 @@ def test_status_strings(L):
 
 def params(**kw):
     base = dict(batch=1, num_q_heads=32, num_kv_heads=8, head_dim=128, page_size=16, num_pages=300,
-                max_pages_per_seq=257, num_splits=4, softmax_scale=0.0)
+                max_pages_per_seq=257, num_splits=3, softmax_scale=0.0)
     base.update(kw)
     return nld.make_params(**base)
 
@@ -50,7 +50,15 @@ def test_split_plan_and_workspace_size(L):
     o = S * B * Hq * bl * D * 4
     assert nld.nld_block_attn_workspace_size(p, 16) == ((o + 255) // 256) * 256 + S * B * Hq * bl * 4
     assert nld.nld_block_attn_workspace_size(params(num_splits=1), 16) == 0
-    assert nld.nld_block_attn_num_splits(params(num_splits=64, max_pages_per_seq=4), 8) == 4  # chunk >= 16
+    # 16 pieces run as two clusters of 8 (tcgen05 kernel, 64 packed rows): 2 partials
+    assert nld.nld_block_attn_num_splits(params(num_splits=16), 16) == 2
+    assert nld.nld_block_attn_workspace_size(params(num_splits=16), 16) == \
+        ((2 * Hq * bl * D * 4 + 255) // 256) * 256 + 2 * Hq * bl * 4
+    # 4 pieces (chunk >= 16 tokens of 64) merge in one cluster: final output, no workspace
+    assert nld.nld_block_attn_num_splits(params(num_splits=64, max_pages_per_seq=4), 8) == 1
+    assert nld.nld_block_attn_workspace_size(params(num_splits=8), 16) == 0
+    # 160 packed rows use the mma.sync kernel: no clusters, one partial per piece
+    assert nld.nld_block_attn_num_splits(params(num_q_heads=40, num_splits=8), 32) == 8
 
 
 @pytest.mark.parametrize("kw,bl,code", [

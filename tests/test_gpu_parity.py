@@ -292,7 +292,7 @@ def test_device_clamps_bad_prefix_and_page_ids():
 def test_workspace_too_small_launches_nothing():
     case = W.make_block_attn_case("ws", 1, 8, 2, 128, 16, 16, [500], seed=7)
     dc = DeviceCase(case)
-    p = dc.params(4)
+    p = dc.params(3)  # 3 pieces: no cluster, three partials in the workspace
     need = nld.nld_block_attn_workspace_size(p, 16)
     out = torch.zeros((1, 16, 8, 128), dtype=torch.bfloat16, device="cuda")
     ws = torch.empty(need - 16, dtype=torch.uint8, device="cuda")

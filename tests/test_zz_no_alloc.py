@@ -73,10 +73,11 @@ def test_static_scratch_matches_workspace_entry_twice(name):
 
 
 def test_static_scratch_rejects_oversized_plan():
-    # 64 splits of the 32768-token prefix need 64*32*32*128*4 bytes > 16 MiB
+    # 127 pieces (no cluster divides 127, so 127 partials) of the 32768-token
+    # prefix need 127*32*32*128*4 bytes > 16 MiB
     wl = W.make_workload("long_b1_h32x8_d128_L32768_bl32", seed=0, prefix_override=[32768])
     dc = DeviceCase(wl.attn)
-    params = dc.params(64)
+    params = dc.params(127)
     assert nld.nld_block_attn_workspace_size(params, 32) > STATIC_SCRATCH_BYTES
     out = torch.zeros((1, 32, 32, 128), dtype=torch.bfloat16, device="cuda")
     lse = torch.zeros((1, 32, 32), dtype=torch.float32, device="cuda")
