@@ -46,7 +46,7 @@ PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_HBM_GBS = 6800.0
 TRAFFIC_NOTE = os.path.join(ROOT, "profiles", "block_attn_8b_b1_L4096_bl16.md")
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2607_05722_gb300", "csrc", f)
-                  for f in ("block_attn.cu", "nld_internal.cuh")]
+                  for f in ("block_attn_tc.cu", "nld_internal.cuh")]
 
 
 def parse_args():
@@ -58,6 +58,7 @@ def parse_args():
     ap.add_argument("--pools", type=int, default=32, help="rotating KV pools (cold-L2 rotation)")
     ap.add_argument("--splits", type=int, default=0, help="KV splits (0 = automatic)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--headline-only", action="store_true", help="skip the other named workloads")
     ap.add_argument("--no-prefix-ready", action="store_true",
                     help="do not let attention stream prefix KV before its dependency wait")
     ap.add_argument("--seed", type=int, default=0)
@@ -383,7 +384,7 @@ def run_ours(args, world, rank, local):
         "e2e": e2e,
         "gpu_launches": launches_per_step * args.steps,
         "roofline": {
-            "kernel": "block_attn_mma_kernel (attention, split partials)",
+            "kernel": "block_attn_tc_kernel (attention; split partials when the plan has several)",
             "bound": "hbm",
             "achieved": round(attn_gbs, 1),
             "peak": peak,
@@ -398,6 +399,8 @@ def run_ours(args, world, rank, local):
             "combine_avg_launch_us": round(comb_ms * 1e3, 3),
         },
     }
+    if not args.headline_only:
+        line["workloads"] = run_workloads(torch, nld, dev, stream, peak, l2)
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, budget_s=12.0)
     print(json.dumps(line), flush=True)
@@ -469,6 +472,98 @@ def run_e2e(args, torch, nld, dev, stream, wl, params, splits, kv_bytes, world):
     return {"value": round(2 * kv_bytes * world / (ms * 1e-3) / 1e9, 2), "unit": "GB/s",
             "ms_per_step": ms, "steps": nsteps, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "note": "every input copied from pinned host memory and outputs read back each step, in a CUDA graph"}
+
+
+# ---------------------------------------------------------------------------
+# the other named workloads (each with its own step sequence)
+# ---------------------------------------------------------------------------
+
+def time_graph(torch, stream, body, nsteps, reps):
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(stream):
+        body(0)  # eager once (per-device setup outside the capture)
+        torch.cuda.synchronize()
+        with torch.cuda.graph(g, stream=stream):
+            for i in range(nsteps):
+                body(i)
+        g.replay()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            g.replay()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / (reps * nsteps)
+
+
+def run_workloads(torch, nld, dev, stream, peak, l2):
+    """Each named workload's step (SURVEY-style sequences: passes, then the
+    decisions), inputs drawn on the device, pools rotated past L2 where the
+    KV is smaller than three times L2."""
+    res = {}
+    for name in W.WORKLOADS:
+        if name == WORKLOAD:
+            continue
+        w = W.make_device_workload(name, seed=0, device=dev)
+        B, bl, Hq, Hkv, D = w["batch"], w["bl"], w["hq"], w["hkv"], w["d"]
+        kvb = w["kv_bytes_per_pass"]
+        npool = int(min(64, max(1, np.ceil(3 * l2 / kvb))))
+        pools = [(w["k"], w["v"])] + [(w["k"].clone(), w["v"].clone()) for _ in range(npool - 1)]
+        params = nld.make_params(B, Hq, Hkv, D, w["page"], w["num_pages"], w["max_pages"], 0, 0.0,
+                                 nld.NLD_ATTN_PREFIX_READY)
+        parts = nld.nld_block_attn_num_splits(params, bl)
+        ws = torch.empty(max(nld.nld_block_attn_workspace_size(params, bl), 16), dtype=torch.uint8, device=dev)
+        out = torch.empty((B, bl, Hq, D), dtype=torch.bfloat16, device=dev)
+        lse = torch.empty((B, Hq, bl), dtype=torch.float32, device=dev)
+        acc = torch.empty((B,), dtype=torch.int32, device=dev)
+        kk = max(w["unmask_k"])
+        pos = torch.empty((B, kk), dtype=torch.int32, device=dev)
+        nsel = torch.empty((B,), dtype=torch.int32, device=dev)
+        seq = w["steps"]
+        npass = sum(1 for s_ in seq if s_ in ("diffusion", "verify"))
+        counter = {"p": 0}
+
+        def step(i, seq=seq, pools=pools, params=params):
+            for s_ in seq:
+                if s_ in ("diffusion", "verify"):
+                    kp, vp = pools[counter["p"] % len(pools)]
+                    counter["p"] += 1
+                    mode = nld.NLD_MODE_DIFFUSION if s_ == "diffusion" else nld.NLD_MODE_VERIFY
+                    q = w["q_draft"] if s_ == "diffusion" else w["q_verify"]
+                    nld.nld_block_attn(params, q, kp, vp, w["page_table"], w["prefix_lens"], bl, mode, out, lse, ws)
+                elif s_ == "accept":
+                    nld.nld_accept(w["draft_ids"], w["verify_ids"], acc)
+                elif s_ == "unmask":
+                    nld.nld_unmask(w["conf"][0], kk, pos, nsel)
+
+        nsteps = max(1, min(64, 512 // max(1, len(seq))))
+        ms = time_graph(torch, stream, step, nsteps, reps=8)
+        gbs = npass * kvb / (ms * 1e-3) / 1e9
+        entry = {"step": " + ".join(seq), "ms_per_step": round(ms, 5), "kv_gbs": round(gbs, 1),
+                 "pct_of_hbm_peak": round(100 * gbs / peak, 2), "steps_per_s": round(1e3 / ms, 1),
+                 "kv_bytes_per_pass": kvb, "kv_partials": parts,
+                 "l2": ("cold: %d rotating pools" % npool) if npool * kvb >= 3 * l2 else
+                       "warm: KV fits in L2 (%d pools, launch-bound shape)" % npool}
+        if name.startswith("long"):
+            sweep = {}
+            for S in (1, 2, 4, 8, 16, 32, 64):
+                pS = nld.make_params(B, Hq, Hkv, D, w["page"], w["num_pages"], w["max_pages"], S, 0.0,
+                                     nld.NLD_ATTN_PREFIX_READY)
+                wsS = torch.empty(max(nld.nld_block_attn_workspace_size(pS, bl), 16), dtype=torch.uint8, device=dev)
+
+                def one(i, pS=pS, wsS=wsS):
+                    kp, vp = pools[i % len(pools)]
+                    nld.nld_block_attn(pS, w["q_verify"], kp, vp, w["page_table"], w["prefix_lens"], bl,
+                                       nld.NLD_MODE_VERIFY, out, lse, wsS)
+                msS = time_graph(torch, stream, one, 16, reps=8)
+                sweep[str(S)] = {"us_per_pass": round(msS * 1e3, 2), "kv_gbs": round(kvb / (msS * 1e-3) / 1e9, 1),
+                                 "kv_partials": nld.nld_block_attn_num_splits(pS, bl)}
+            entry["verify_pass_split_sweep"] = sweep
+        res[name] = entry
+        del pools, w
+        torch.cuda.empty_cache()
+    return res
 
 
 # ---------------------------------------------------------------------------

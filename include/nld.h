@@ -135,7 +135,7 @@ size_t nld_block_attn_workspace_size(const nld_attn_params_t *params, int block_
  *   page_table  int32 [B, max_pages_per_seq]; entries for logical pages
  *               0 .. ceil((L_b + block_len) / P) - 1 must be valid page ids
  *   prefix_lens int32 [B], L_b >= 0 and L_b + block_len <= max_pages_per_seq * P
- *   block_len   1 .. 32, with (Hq / Hkv) * block_len <= 160
+ *   block_len   1 .. 32, with (Hq / Hkv) * block_len <= 256
  *   mode        NLD_MODE_DIFFUSION or NLD_MODE_VERIFY
  *   out         bf16 [B, block_len, Hq, D]
  *   lse         fp32 [B, Hq, block_len] (natural log), or NULL

@@ -37,41 +37,60 @@
 namespace nld {
 namespace {
 
-constexpr int kTcStages = 4;
 constexpr int kProducers = 4;
 constexpr int kMmaWarp = 3;
 constexpr int kSoftmaxWarp0 = 4;
-constexpr int kTcThreads = 32 * 9;
-// producer index of a warp, or -1
-__device__ __forceinline__ int producer_index(int warp) { return warp < 3 ? warp : (warp == 8 ? 3 : -1); }
-constexpr uint32_t kTmemCols = 256;  // S0 | S1 (64 columns each) | O (D <= 128 columns)
+
+// MT 128-row M tiles per CTA (MT = 2 for 129..256 packed rows): each K/V tile
+// feeds MT score and MT PV products; 4*MT softmax warps; the ring shrinks to
+// 3 stages so that two Q tiles and four P buffers fit in shared memory.
+template <int MT>
+struct TcCfg {
+  static constexpr int kStages = MT == 1 ? 4 : 3;
+  static constexpr int kWarps = 5 + 4 * MT;  // 4 producers, 1 MMA, 4*MT softmax
+  static constexpr int kThreads = 32 * kWarps;
+  static constexpr uint32_t kTmemCols = MT == 1 ? 256 : 512;  // MT x (S0 | S1), then MT x O
+};
+
+// producer index of a warp, or -1: warps 0-2 and the last warp
+template <int MT>
+__device__ __forceinline__ int producer_index(int warp) {
+  return warp < 3 ? warp : (warp == TcCfg<MT>::kWarps - 1 ? 3 : -1);
+}
 constexpr float kRescaleLog2 = 8.0f;
 
-// Cluster merge staging in the freed K/V ring: 128 rows of D fp32 (padded
-// pitch), then 128 log2-sum-exp values.
-constexpr int kMergePitchRows = 128;
+// Epilogue staging in the freed K/V ring and Q tiles: 128*MT rows of D fp32
+// (padded pitch), then 128*MT log2-sum-exp values, then the cluster merge
+// weights [rows][8] and merged lse per row.
 template <int D>
 __host__ __device__ constexpr int merge_pitch() { return D * 4 + 16; }
 
-template <int D>
+template <int D, int MT>
 struct TcLayout {
   using Geo = TileGeom<D>;
-  static constexpr int kQBytes = Geo::kColBlocks * 128 * 128;  // 128 rows x D bf16
-  static constexpr int kPBytes = 128 * kTileTok * 2;             // 128 rows x 64 tokens bf16
-  static constexpr int kQOff = kTcStages * Geo::kStageBytes;
-  static constexpr int kPOff = kQOff + kQBytes;
-  static constexpr int kBarOff = kPOff + 2 * kPBytes;
-  // kv_full[4], kv_empty[4], s_full[2], s_free[2], p_full[2], o_done[2], q_ready, drain, tmem slot
-  static constexpr int kNumBars = 2 * kTcStages + 8 + 2;
+  static constexpr int kStages = TcCfg<MT>::kStages;
+  static constexpr int kQBytes = Geo::kColBlocks * 128 * 128;  // one 128-row Q tile, bf16
+  static constexpr int kPBytes = 128 * kTileTok * 2;             // one 128-row x 64-token P buffer, bf16
+  static constexpr int kQOff = kStages * Geo::kStageBytes;
+  static constexpr int kPOff = kQOff + MT * kQBytes;
+  static constexpr int kBarOff = kPOff + MT * 2 * kPBytes;
+  // kv_full[st], kv_empty[st], s_full[2], s_free[2], p_full[2], o_done[2], q_ready, drain, tmem slot
+  static constexpr int kNumBars = 2 * kStages + 8 + 2;
   static constexpr int kBytes = kBarOff + kNumBars * 8 + 16;
+  static constexpr int kMergeRows = 128 * MT;
+  static constexpr int kLseOff = kMergeRows * merge_pitch<D>();
+  static constexpr int kWtsOff = kLseOff + kMergeRows * 4;
+  static constexpr int kLseOutOff = kWtsOff + kMergeRows * 8 * 4;
+  static_assert(kLseOutOff + kMergeRows * 4 <= kPOff, "epilogue staging overlaps the live buffers");
 };
 
-template <int D>
-__global__ void __launch_bounds__(kTcThreads, 1)
+template <int D, int MT>
+__global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
     block_attn_tc_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
                          const AttnArgs a) {
   using Geo = TileGeom<D>;
-  using Lay = TcLayout<D>;
+  using Lay = TcLayout<D, MT>;
+  constexpr int kTcStages = Lay::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* q_s = smem + Lay::kQOff;
@@ -97,11 +116,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     for (int j = 0; j < 2; ++j) {
       mbar_init(&s_full[j], 1);
-      mbar_init(&s_free[j], 4);
-      mbar_init(&p_full[j], 4);
+      mbar_init(&s_free[j], 4 * MT);
+      mbar_init(&p_full[j], 4 * MT);
       mbar_init(&o_done[j], 1);
     }
-    mbar_init(q_ready, 4);
+    mbar_init(q_ready, 4 * MT);
     mbar_init(drain, 1);
     fence_mbar_init();
   }
@@ -110,7 +129,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     prefetch_tensormap(&tmv);
   }
   if (warp == kMmaWarp) {
-    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_alloc(tmem_slot, TcCfg<MT>::kTmemCols);
     tc_fence_before();
   }
   // Without NLD_ATTN_PREFIX_READY nothing global is read before the
@@ -125,12 +144,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   // independent, so they are in flight together.
   PagePrefetch first;
   first.raw = 0;
-  if (producer_index(warp) >= 0) first.load(a, b, t_begin, 0, lane);
+  if (producer_index<MT>(warp) >= 0) first.load(a, b, t_begin, 0, lane);
   int L = __ldg(a.prefix_lens + b);
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t tS0 = tmem, tS1 = tmem + kTileTok, tO = tmem + 2 * kTileTok;
+  // TMEM columns: S of M tile mt, buffer j at (2*mt + j)*64; O of tile mt after all S buffers.
+  auto tS = [&](int mt, int j) -> uint32_t { return tmem + static_cast<uint32_t>((2 * mt + j) * kTileTok); };
+  auto tO = [&](int mt) -> uint32_t { return tmem + static_cast<uint32_t>(2 * MT * kTileTok + mt * D); };
 
   const int lmax = a.max_pages * a.page_size - a.bl;
   if (L < 0 || L > lmax) {
@@ -147,15 +168,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // This split lies past the sequence: its partials carry no keys.
     if (early) grid_dependency_wait();
     if (a.csize > 1) {
-      float* lse_stage = reinterpret_cast<float*>(smem + kMergePitchRows * merge_pitch<D>());
-      for (int r = threadIdx.x; r < 128; r += blockDim.x) lse_stage[r] = -INFINITY;
+      float* lse_stage = reinterpret_cast<float*>(smem + Lay::kLseOff);
+      for (int r = threadIdx.x; r < Lay::kMergeRows; r += blockDim.x) lse_stage[r] = -INFINITY;
     } else {
       for (int r = threadIdx.x; r < a.R; r += blockDim.x) {
         const int i = r / a.G, h = g * a.G + (r - i * a.G);
         a.lse_part[((static_cast<size_t>(split) * a.B + b) * a.Hq + h) * a.bl + i] = -INFINITY;
       }
     }
-  } else if (producer_index(warp) >= 0) {
+  } else if (producer_index<MT>(warp) >= 0) {
     // ---------------- producers ----------------
     int early_tiles = 0;  // leading tiles made of prefix tokens only
     if (early) {
@@ -165,7 +186,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       if (early_tiles == 0) grid_dependency_wait();
     }
     const int issued = produce_kv<D>(a, &tmk, &tmv, smem, kv_full, kv_empty, kTcStages, g, b, t_begin, t_end,
-                                     ntiles, lane, producer_index(warp), kProducers, first, early_tiles);
+                                     ntiles, lane, producer_index<MT>(warp), kProducers, first, early_tiles);
     if (lane == 0 && issued < ntiles) {
       // Stopped early on a wait timeout: let the copies already issued land
       // before the CTA exits (bounded).
@@ -183,28 +204,34 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       auto issue_s = [&](int k) {
         const int st = k % kTcStages;
         const uint32_t k_addr = smem_u32(smem + st * Geo::kStageBytes);
-        const uint32_t d = (k & 1) ? tS1 : tS0;
 #pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t koff = (kk & 3) * 32;  // 16 elements along the 128-byte row
-          const int cb = kk >> 2;               // 64-dim column block
-          const uint64_t ad = sw128_desc(q_addr + cb * (128 * 128) + koff, 0, 1024);
-          const uint64_t bd = sw128_desc(k_addr + cb * Geo::kColBlockBytes + koff, 0, 1024);
-          umma_bf16(d, ad, bd, idesc_s, kk > 0 ? 1u : 0u);
+        for (int mt = 0; mt < MT; ++mt) {
+          const uint32_t d = tS(mt, k & 1);
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t koff = (kk & 3) * 32;  // 16 elements along the 128-byte row
+            const int cb = kk >> 2;               // 64-dim column block
+            const uint64_t ad = sw128_desc(q_addr + mt * Lay::kQBytes + cb * (128 * 128) + koff, 0, 1024);
+            const uint64_t bd = sw128_desc(k_addr + cb * Geo::kColBlockBytes + koff, 0, 1024);
+            umma_bf16(d, ad, bd, idesc_s, kk > 0 ? 1u : 0u);
+          }
         }
         umma_commit(&s_full[k & 1]);
       };
       auto issue_pv = [&](int k) {
         const int st = k % kTcStages;
-        const uint32_t p_addr = smem_u32(smem + Lay::kPOff + (k & 1) * Lay::kPBytes);
         const uint32_t v_addr = smem_u32(smem + st * Geo::kStageBytes + Geo::kTileBytes);
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt) {
+        const uint32_t p_addr = smem_u32(smem + Lay::kPOff + (mt * 2 + (k & 1)) * Lay::kPBytes);
 #pragma unroll
         for (int kt = 0; kt < kTileTok / 16; ++kt) {
           // A = P rows (K-major, one 128-byte block of 64 tokens); B = V (MN-major:
           // 64-dim atoms LBO apart, 8-token row groups SBO apart).
           const uint64_t ad = sw128_desc(p_addr + kt * 32, 0, 1024);
           const uint64_t bd = sw128_desc(v_addr + kt * 16 * 128, Geo::kColBlockBytes, 1024);
-          umma_bf16(tO, ad, bd, idesc_o, (k > 0 || kt > 0) ? 1u : 0u);
+          umma_bf16(tO(mt), ad, bd, idesc_o, (k > 0 || kt > 0) ? 1u : 0u);
+        }
         }
         umma_commit(&o_done[k & 1]);
         umma_commit(&kv_empty[st]);
@@ -246,14 +273,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     __syncwarp();
   } else {
     // ---------------- softmax warps ----------------
-    const int quad = warp & 3;
-    const int r = quad * 32 + lane;  // query row == TMEM lane
+    const int quad = warp & 3;                      // TMEM lanes 32*quad .. +31
+    const int mt = (warp - kSoftmaxWarp0) >> 2;     // M tile of this warp
+    const int r_loc = quad * 32 + lane;             // row within the M tile == TMEM lane
+    const int r = mt * 128 + r_loc;                 // packed query row
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
-    const bool warp_rows = quad * 32 < a.R;  // warp-uniform: the warp holds a real row
+    const bool warp_rows = mt * 128 + quad * 32 < a.R;  // warp-uniform: the warp holds a real row
     const bool row_ok = r < a.R;
     const int row_i = r / a.G;
     const int row_h = g * a.G + (r - row_i * a.G);
-    const int sm_tid = threadIdx.x - 32 * kSoftmaxWarp0;  // 0..127 across the softmax warps
+    const int sm_tid = threadIdx.x - 32 * kSoftmaxWarp0;  // 0 .. 128*MT-1 across the softmax warps
+    uint8_t* q_tile = q_s + mt * Lay::kQBytes;
+    auto p_buf = [&](int j) -> uint8_t* { return smem + Lay::kPOff + (mt * 2 + j) * Lay::kPBytes; };
 
     // Q row -> shared memory in the 128-byte-swizzled K-major layout; padding
     // rows are zero. Padding rows of P are zeroed once for both buffers.
@@ -265,15 +296,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       for (int c = 0; c < D / 8; ++c) {
         uint4 v = make_uint4(0, 0, 0, 0);
         if (row_ok) v = __ldg(qrow + c);
-        *reinterpret_cast<uint4*>(q_s + (c >> 3) * (128 * 128) + r * 128 + (((c & 7) ^ (r & 7)) << 4)) = v;
+        *reinterpret_cast<uint4*>(q_tile + (c >> 3) * (128 * 128) + r_loc * 128 + (((c & 7) ^ (r & 7)) << 4)) = v;
       }
       if (!row_ok) {
 #pragma unroll
         for (int j = 0; j < 2; ++j)
 #pragma unroll
           for (int c = 0; c < 8; ++c)
-            *reinterpret_cast<uint4*>(smem + Lay::kPOff + j * Lay::kPBytes + r * 128 + ((c ^ (r & 7)) << 4)) =
-                make_uint4(0, 0, 0, 0);
+            *reinterpret_cast<uint4*>(p_buf(j) + r_loc * 128 + ((c ^ (r & 7)) << 4)) = make_uint4(0, 0, 0, 0);
       }
       fence_proxy_async_smem();
       __syncwarp();
@@ -294,7 +324,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       tc_fence_after();
       float s[kTileTok];
       if (warp_rows) {
-        const uint32_t ts = (buf ? tS1 : tS0) + lane_off;
+        const uint32_t ts = tS(mt, buf) + lane_off;
         tmem_ld32(ts, s);
         tmem_ld32(ts + 32, s + 32);
       }
@@ -343,10 +373,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 #pragma unroll 1
         for (int c = 0; c < D / 32; ++c) {
           float o[32];
-          tmem_ld32(tO + lane_off + c * 32, o);
+          tmem_ld32(tO(mt) + lane_off + c * 32, o);
 #pragma unroll
           for (int j = 0; j < 32; ++j) o[j] *= alpha;
-          tmem_st32(tO + lane_off + c * 32, o);
+          tmem_st32(tO(mt) + lane_off + c * 32, o);
         }
       }
       // P buffer `buf` is free once the PV of tile k-2 has completed.
@@ -356,7 +386,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       }
       if (warp_rows) {
         const float mu = m_run == -INFINITY ? 0.f : m_run;
-        uint8_t* prow = smem + Lay::kPOff + buf * Lay::kPBytes + r * 128;
+        uint8_t* prow = p_buf(buf) + r_loc * 128;
 #pragma unroll
         for (int c = 0; c < kTileTok / 8; ++c) {
           uint32_t w[4];
@@ -380,7 +410,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
         const int r0 = valid, r1 = (valid + kGroupTok - 1) & ~(kGroupTok - 1);
         uint8_t* vt = smem + st * Geo::kStageBytes + Geo::kTileBytes;
-        for (int idx = sm_tid; idx < (r1 - r0) * (D / 8); idx += 128) {
+        for (int idx = sm_tid; idx < (r1 - r0) * (D / 8); idx += 128 * MT) {
           const int row = r0 + idx / (D / 8), c = idx % (D / 8);
           *reinterpret_cast<uint4*>(vt + kv_swz(row, c)) = make_uint4(0, 0, 0, 0);
         }
@@ -401,7 +431,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       // the freed ring for the merge across the cluster (rows without keys,
       // or after a timeout, carry lse = -inf and are skipped by the merge).
       if (o_ready) tc_fence_after();
-      float* lse_stage = reinterpret_cast<float*>(smem + kMergePitchRows * merge_pitch<D>());
+      float* lse_stage = reinterpret_cast<float*>(smem + Lay::kLseOff);
       const float l = l_run;
       const bool has = o_ready && row_ok && l > 0.f;
       lse_stage[r] = has ? m_run + lg2(l) : -INFINITY;
@@ -411,7 +441,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 #pragma unroll 1
         for (int c = 0; c < D / 32; ++c) {
           float o[32];
-          tmem_ld32(tO + lane_off + c * 32, o);
+          tmem_ld32(tO(mt) + lane_off + c * 32, o);
 #pragma unroll
           for (int q4 = 0; q4 < 8; ++q4)
             *reinterpret_cast<float4*>(my + c * 128 + q4 * 16) =
@@ -427,12 +457,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const bool split_out = a.o_part != nullptr;
         const int row_bytes = split_out ? D * 4 : D * 2;
         const int pitch = row_bytes + 16;
-        uint8_t* stage = smem + quad * 32 * pitch;  // quad * 32 * (512 + 16) < ring size
+        uint8_t* stage = smem + (mt * 128 + quad * 32) * pitch;  // inside the freed ring and Q tiles
         uint8_t* my = stage + lane * pitch;
 #pragma unroll 1
         for (int c = 0; c < D / 32; ++c) {
           float o[32];
-          tmem_ld32(tO + lane_off + c * 32, o);
+          tmem_ld32(tO(mt) + lane_off + c * 32, o);
 #pragma unroll
           for (int j = 0; j < 32; ++j) o[j] *= inv;
           if (split_out) {
@@ -495,16 +525,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // split combine, and writes the final output (one cluster per sequence
     // and KV head) or this cluster's partial.
     cluster_sync();
-    if (warp >= kSoftmaxWarp0 && warp < kSoftmaxWarp0 + 4) {
+    if (warp >= kSoftmaxWarp0 && warp < kSoftmaxWarp0 + 4 * MT) {
       const uint32_t rank = cluster_ctarank();
       const int Rc = (a.R + a.csize - 1) / a.csize;
       const int r0 = static_cast<int>(rank) * Rc;
       const int nrows = max(0, min(a.R, r0 + Rc) - r0);
       const uint32_t stage_u32 = smem_u32(smem);
-      const uint32_t lse_u32 = stage_u32 + kMergePitchRows * merge_pitch<D>();
+      const uint32_t lse_u32 = stage_u32 + Lay::kLseOff;
       // this CTA's merge weights, local: [row][peer] and the merged lse per row
-      float* wts = reinterpret_cast<float*>(smem + kMergePitchRows * merge_pitch<D>() + 512);
-      float* lse_out = wts + 128 * 8;
+      float* wts = reinterpret_cast<float*>(smem + Lay::kWtsOff);
+      float* lse_out = reinterpret_cast<float*>(smem + Lay::kLseOutOff);
       const int tid = threadIdx.x - 32 * kSoftmaxWarp0;
       // 1) per-row weights: one thread per row, the peers' lse loads in flight together
       if (tid < nrows) {
@@ -527,18 +557,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         for (int p = 0; p < 8; ++p) wts[tid * 8 + p] = w[p] * inv;
         lse_out[tid] = wsum > 0.f ? (m + lg2(wsum)) * kLn2 : -INFINITY;
       }
-      named_bar_sync(1, 128);
+      named_bar_sync(1, 128 * MT);
       // 2) rows: two (row, 4-dim) items per thread per round, every peer load in flight
       const bool final_out = a.num_partials == 1;
       const int pidx = split / a.csize;
       const int items = nrows * (D / 4);
-      for (int base = tid; base < items; base += 256) {
+      for (int base = tid; base < items; base += 2 * 128 * MT) {
         float4 acc[2];
         int ridx[2], d4[2];
         bool live[2];
 #pragma unroll
         for (int u = 0; u < 2; ++u) {
-          const int idx = base + u * 128;
+          const int idx = base + u * 128 * MT;
           live[u] = idx < items;
           ridx[u] = live[u] ? idx / (D / 4) : 0;
           d4[u] = idx % (D / 4);
@@ -584,47 +614,47 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __syncthreads();
   if (warp == kMmaWarp) {
     tc_fence_after();
-    tmem_dealloc(tmem, kTmemCols);
+    tmem_dealloc(tmem, TcCfg<MT>::kTmemCols);
   }
 }
 
-template <int D>
+template <int D, int MT>
 cudaError_t configure_tc(int dev) {
   static int configured[64] = {0};
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   if (!__atomic_load_n(&configured[dev], __ATOMIC_ACQUIRE)) {
-    cudaError_t e = cudaFuncSetAttribute(block_attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(TcLayout<D>::kBytes + 1024));
+    cudaError_t e = cudaFuncSetAttribute(block_attn_tc_kernel<D, MT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(TcLayout<D, MT>::kBytes + 1024));
     if (e != cudaSuccess) return e;
     __atomic_store_n(&configured[dev], 1, __ATOMIC_RELEASE);
   }
   return cudaSuccess;
 }
 
-template <int D>
+template <int D, int MT>
 cudaError_t launch_tc_t(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, cudaStream_t stream) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  if ((e = configure_tc<D>(dev)) != cudaSuccess) return e;
+  if ((e = configure_tc<D, MT>(dev)) != cudaSuccess) return e;
   dim3 grid(a.num_splits, a.Hkv, a.B);
-  return launch_kernel_cluster(block_attn_tc_kernel<D>, grid, dim3(kTcThreads), TcLayout<D>::kBytes + 1024, stream,
-                               a.csize, tmk, tmv, a);
+  return launch_kernel_cluster(block_attn_tc_kernel<D, MT>, grid, dim3(TcCfg<MT>::kThreads),
+                               TcLayout<D, MT>::kBytes + 1024, stream, a.csize, tmk, tmv, a);
 }
 
-template <int D>
+template <int D, int MT>
 int max_active_clusters_t(int csize) {
-  static int cache[64][4];  // [device][log2 csize - 1] + 1 (0 = not queried)
+  static int cache[64][4];  // [device][cluster size 2/4/8] + 1 (0 = not queried)
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
   const int slot = csize == 2 ? 0 : csize == 4 ? 1 : csize == 8 ? 2 : 3;
   int v = __atomic_load_n(&cache[dev][slot], __ATOMIC_ACQUIRE);
   if (v) return v - 1;
-  if (configure_tc<D>(dev) != cudaSuccess) return 0;
+  if (configure_tc<D, MT>(dev) != cudaSuccess) return 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(csize, 1, 1);
-  cfg.blockDim = dim3(kTcThreads);
-  cfg.dynamicSmemBytes = TcLayout<D>::kBytes + 1024;
+  cfg.blockDim = dim3(TcCfg<MT>::kThreads);
+  cfg.dynamicSmemBytes = TcLayout<D, MT>::kBytes + 1024;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = csize;
@@ -633,7 +663,7 @@ int max_active_clusters_t(int csize) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, block_attn_tc_kernel<D>, &cfg) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveClusters(&n, block_attn_tc_kernel<D, MT>, &cfg) != cudaSuccess) {
     cudaGetLastError();
     n = 0;
   }
@@ -643,16 +673,17 @@ int max_active_clusters_t(int csize) {
 
 }  // namespace
 
-bool tc_supports(int R, int head_dim) { return R <= 128 && (head_dim == 64 || head_dim == 128); }
+bool tc_supports(int R, int head_dim) { return R <= 256 && (head_dim == 64 || head_dim == 128); }
 
-int tc_max_active_clusters(int csize, int head_dim) {
-  return head_dim == 128 ? max_active_clusters_t<128>(csize) : max_active_clusters_t<64>(csize);
+int tc_max_active_clusters(int csize, int head_dim, int rows) {
+  if (rows > 128) return head_dim == 128 ? max_active_clusters_t<128, 2>(csize) : max_active_clusters_t<64, 2>(csize);
+  return head_dim == 128 ? max_active_clusters_t<128, 1>(csize) : max_active_clusters_t<64, 1>(csize);
 }
 
 cudaError_t launch_block_attn_tc(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, int head_dim,
                                  cudaStream_t stream) {
-  if (head_dim == 128) return launch_tc_t<128>(a, tmk, tmv, stream);
-  return launch_tc_t<64>(a, tmk, tmv, stream);
+  if (a.R > 128) return head_dim == 128 ? launch_tc_t<128, 2>(a, tmk, tmv, stream) : launch_tc_t<64, 2>(a, tmk, tmv, stream);
+  return head_dim == 128 ? launch_tc_t<128, 1>(a, tmk, tmv, stream) : launch_tc_t<64, 1>(a, tmk, tmv, stream);
 }
 
 }  // namespace nld

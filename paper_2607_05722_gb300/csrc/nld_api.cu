@@ -100,7 +100,7 @@ nld_status_t plan_splits(const nld_attn_params_t* p, int block_len, SplitPlan* o
     want = static_cast<int>(s);
     if (tc && want >= 2 && want <= 8) {
       const int cs = want >= 8 ? 8 : want >= 4 ? 4 : 2;
-      if (units <= nld::tc_max_active_clusters(cs, p->head_dim)) {
+      if (units <= nld::tc_max_active_clusters(cs, p->head_dim, (p->num_q_heads / p->num_kv_heads) * block_len)) {
         want = cs;
         csize = cs;
       }
@@ -272,10 +272,7 @@ nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_bloc
     a.o_part = static_cast<float*>(workspace);
     a.lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) + o_bytes);
   }
-  const cudaError_t le = nld::tc_supports(a.R, params->head_dim)
-                            ? nld::launch_block_attn_tc(a, tmk, tmv, params->head_dim, stream)
-                            : nld::launch_block_attn(a, tmk, tmv, params->head_dim, stream);
-  if (le != cudaSuccess) return NLD_ERR_CUDA;
+  if (nld::launch_block_attn_tc(a, tmk, tmv, params->head_dim, stream) != cudaSuccess) return NLD_ERR_CUDA;
   if (plan.partials > 1 && run_combine) {
     if (nld::launch_combine(a.o_part, a.lse_part, plan.partials, a.B, a.Hq, block_len, params->head_dim, a.out, lse,
                             stream) != cudaSuccess)

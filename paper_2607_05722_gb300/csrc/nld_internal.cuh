@@ -1,5 +1,5 @@
 // Internal declarations of libnld: kernel argument blocks, launch helpers and
-// thin inline-PTX wrappers (mbarrier, TMA, ldmatrix, mma) used by the kernels.
+// thin inline-PTX wrappers (mbarrier, TMA, clusters, tcgen05) used by the kernels.
 #pragma once
 
 #include <cuda.h>
@@ -16,7 +16,7 @@ namespace nld {
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kMaxSplits = 128;
-constexpr int kMaxRows = 160;   // (Hq / Hkv) * block_len handled by one CTA
+constexpr int kMaxRows = 256;   // (Hq / Hkv) * block_len handled by one CTA (two 128-row M tiles)
 constexpr int kMaxBlock = 32;   // block_len and the decision width n
 constexpr int kTileTok = 64;    // KV tokens per pipeline stage
 constexpr int kGroupTok = 16;   // KV tokens per TMA box (never crosses a page: P % 16 == 0)
@@ -34,7 +34,7 @@ struct AttnArgs {
   int B, Hq, Hkv, G, bl, R;    // R = G * bl query rows per CTA
   int page_size, log2_page, num_pages, max_pages;
   int num_splits, chunk;       // splits and tokens per split (multiple of 16)
-  int mode, nstage, nwr;       // mask mode, pipeline depth, 16-row warp groups
+  int mode;                    // NLD_MODE_DIFFUSION or NLD_MODE_VERIFY
   float scale_log2;            // softmax scale * log2(e)
   int prefix_ready;            // NLD_ATTN_PREFIX_READY: prefix K/V may be read before the dependency wait
   int csize;                   // thread-block cluster size along the splits (1 = no cluster)
@@ -42,9 +42,7 @@ struct AttnArgs {
 };
 
 // Launchers (defined next to their kernels). Return a CUDA error code.
-cudaError_t launch_block_attn(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv,
-                              int head_dim, cudaStream_t stream);
-// tcgen05 kernel: query rows R <= 128 (one 128-row MMA tile).
+// tcgen05 kernel: query rows R <= 256 (one or two 128-row MMA tiles).
 bool tc_supports(int R, int head_dim);
 cudaError_t launch_block_attn_tc(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv,
                                  int head_dim, cudaStream_t stream);
@@ -54,18 +52,6 @@ cudaError_t launch_accept(const int32_t* draft, const int32_t* verify, int B, in
                           cudaStream_t stream);
 cudaError_t launch_unmask(const float* conf, int B, int n, int k, int32_t* pos, int32_t* nsel,
                           cudaStream_t stream);
-
-// Pipeline shape the attention launcher picks for R query rows (shared with
-// the host-side checks so both agree).
-struct AttnShape {
-  int nwr;      // warps along rows (16 rows each)
-  int nwt;      // warps along KV tokens of a tile
-  int nstage;   // pipeline stages
-  int threads;  // consumers + one producer warp
-  size_t smem;  // dynamic shared memory bytes
-};
-AttnShape attn_shape(int R, int head_dim);
-size_t max_smem_bytes(int head_dim);
 
 // Launch with programmatic stream serialization: the kernel may start while
 // its predecessor in the stream is still running. Every kernel of this
@@ -112,7 +98,7 @@ cudaError_t launch_kernel(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t 
 
 // Resident clusters of `csize` CTAs of the tcgen05 attention kernel on the
 // current device (cached), for the split plan.
-int tc_max_active_clusters(int csize, int head_dim);
+int tc_max_active_clusters(int csize, int head_dim, int rows);
 
 // ---------------------------------------------------------------------------
 // PTX wrappers
@@ -205,28 +191,6 @@ __device__ __forceinline__ void tma_load_4d(void* dst, const CUtensorMap* map, u
 
 __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
-}
-
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-
-__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
-                                          uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-
-// D += A * B for one m16n8k16 bf16 tile with fp32 accumulators.
-__device__ __forceinline__ void mma_16816(float* d, const uint32_t* a, uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
-      "{%0, %1, %2, %3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
 // Hardware base-2 exponential (MUFU.EX2): ex2(-inf) = +0.

@@ -235,3 +235,43 @@ def make_workload(name: str, seed: int = 0, batch: Optional[int] = None,
     conf = [make_confidences(rng, B, cfg["bl"], cfg["conf"]) for _ in range(nconf)]
     return Workload(attn, draft, verify, conf, list(cfg["k"]), cfg["vocab"], cfg["p"],
                     list(cfg["steps"]), name)
+
+
+# ---------------------------------------------------------------------------
+# Device-side draws for timing the large workloads (up to ~2.2 GB of KV):
+# the same shapes and distributions, drawn with a seeded torch generator on
+# the GPU instead of numpy on the host. Parity tests use the numpy path.
+# ---------------------------------------------------------------------------
+
+def make_device_workload(name: str, seed: int, device, batch: Optional[int] = None):
+    """A named workload with Q/K/V drawn on `device` (bf16 from N(0,1) fp32),
+    prefix lengths, page table, ids and confidences drawn on the host.
+    Returns a dict of device tensors plus the host-side metadata."""
+    import torch
+
+    cfg = WORKLOADS[name]
+    B = cfg["batch"] if batch is None else batch
+    rng = np.random.Generator(np.random.PCG64(seed))
+    prefix = np.asarray(cfg["prefix"](rng, B), dtype=np.int32)
+    table, num_pages, max_pages = make_page_table(rng, prefix, cfg["bl"], cfg["page"], cfg["shuffle"])
+    draft, verify = make_accept_ids(rng, B, cfg["bl"], cfg["vocab"], cfg["p"])
+    nconf = max(1, cfg["denoise_steps"])
+    conf = [make_confidences(rng, B, cfg["bl"], cfg["conf"]) for _ in range(nconf)]
+    gen = torch.Generator(device=device)
+    gen.manual_seed(seed)
+
+    def normal(shape):
+        return torch.randn(shape, generator=gen, device=device, dtype=torch.float32).to(torch.bfloat16)
+
+    kshape = (num_pages, cfg["hkv"], cfg["page"], cfg["d"])
+    qshape = (B, cfg["bl"], cfg["hq"], cfg["d"])
+    return {
+        "name": name, "batch": B, "hq": cfg["hq"], "hkv": cfg["hkv"], "d": cfg["d"], "bl": cfg["bl"],
+        "page": cfg["page"], "num_pages": num_pages, "max_pages": max_pages, "unmask_k": list(cfg["k"]),
+        "denoise_steps": cfg["denoise_steps"], "steps": list(cfg["steps"]),
+        "k": normal(kshape), "v": normal(kshape), "q_draft": normal(qshape), "q_verify": normal(qshape),
+        "page_table": torch.from_numpy(table).to(device), "prefix_lens": torch.from_numpy(prefix).to(device),
+        "draft_ids": torch.from_numpy(draft).to(device), "verify_ids": torch.from_numpy(verify).to(device),
+        "conf": [torch.from_numpy(c).to(device) for c in conf],
+        "kv_bytes_per_pass": int(np.sum(prefix.astype(np.int64) + cfg["bl"])) * cfg["hkv"] * cfg["d"] * 4,
+    }

@@ -57,8 +57,8 @@ def test_split_plan_and_workspace_size(L):
     # 4 pieces (chunk >= 16 tokens of 64) merge in one cluster: final output, no workspace
     assert nld.nld_block_attn_num_splits(params(num_splits=64, max_pages_per_seq=4), 8) == 1
     assert nld.nld_block_attn_workspace_size(params(num_splits=8), 16) == 0
-    # 160 packed rows use the mma.sync kernel: no clusters, one partial per piece
-    assert nld.nld_block_attn_num_splits(params(num_q_heads=40, num_splits=8), 32) == 8
+    # 160 packed rows use two M tiles of the tcgen05 kernel: 8 pieces merge in one cluster
+    assert nld.nld_block_attn_num_splits(params(num_q_heads=40, num_splits=8), 32) == 1
 
 
 @pytest.mark.parametrize("kw,bl,code", [
@@ -70,7 +70,7 @@ def test_split_plan_and_workspace_size(L):
     (dict(num_splits=129), 16, 1),          # too many splits
     (dict(), 0, 1),                         # block_len 0
     (dict(), 33, 1),                        # block_len > 32
-    (dict(num_q_heads=48, num_kv_heads=8), 32, 2),  # 6 * 32 = 192 packed rows > 160
+    (dict(num_q_heads=72, num_kv_heads=8), 32, 2),  # 9 * 32 = 288 packed rows > 256
     (dict(batch=0), 16, 1),
     (dict(flags=2), 16, 1),                 # unknown flag bit
 ])

@@ -172,6 +172,8 @@ SMALL = [
     ("d128_g8_bl20_p128", 2, 16, 2, 128, 128, 20, [129, 1000]),
     ("d64_g1_bl32_p16", 1, 2, 2, 64, 16, 32, [31]),
     ("prefix0_bl32", 2, 8, 2, 128, 16, 32, [0, 0]),
+    ("d128_g8_bl32_256rows", 2, 16, 2, 128, 16, 32, [700, 33]),
+    ("d64_g6_bl30_180rows", 1, 6, 1, 64, 32, 30, [150]),
 ]
 
 
