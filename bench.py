@@ -59,6 +59,9 @@ def parse_args():
     ap.add_argument("--splits", type=int, default=0, help="KV splits (0 = automatic)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--headline-only", action="store_true", help="skip the other named workloads")
+    ap.add_argument("--only-workload", default=None,
+                    help="time only this named workload (device-drawn inputs), e.g. for a profiler")
+    ap.add_argument("--workload-batch", type=int, default=None, help="batch override for --only-workload")
     ap.add_argument("--no-prefix-ready", action="store_true",
                     help="do not let attention stream prefix KV before its dependency wait")
     ap.add_argument("--seed", type=int, default=0)
@@ -165,6 +168,24 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------
+
+def run_only_workload(args, local):
+    """Time one named workload's step (for profilers); prints one JSON line."""
+    import torch
+
+    from paper_2607_05722_gb300 import build as nld_build
+    from paper_2607_05722_gb300 import nld
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    nld_build.build()
+    nld.lib()
+    peak, _ = hbm_peak()
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    stream = torch.cuda.Stream(device=dev)
+    res = run_workloads(torch, nld, dev, stream, peak, l2, only=args.only_workload, batch=args.workload_batch)
+    print(json.dumps({"workload": args.only_workload, "batch": args.workload_batch, **res[args.only_workload]}))
+
 
 def run_ours(args, world, rank, local):
     import torch
@@ -497,15 +518,15 @@ def time_graph(torch, stream, body, nsteps, reps):
     return e0.elapsed_time(e1) / (reps * nsteps)
 
 
-def run_workloads(torch, nld, dev, stream, peak, l2):
+def run_workloads(torch, nld, dev, stream, peak, l2, only=None, batch=None):
     """Each named workload's step (SURVEY-style sequences: passes, then the
     decisions), inputs drawn on the device, pools rotated past L2 where the
     KV is smaller than three times L2."""
     res = {}
     for name in W.WORKLOADS:
-        if name == WORKLOAD:
+        if (only is None and name == WORKLOAD) or (only is not None and name != only):
             continue
-        w = W.make_device_workload(name, seed=0, device=dev)
+        w = W.make_device_workload(name, seed=0, device=dev, batch=batch)
         B, bl, Hq, Hkv, D = w["batch"], w["bl"], w["hq"], w["hkv"], w["d"]
         kvb = w["kv_bytes_per_pass"]
         npool = int(min(64, max(1, np.ceil(3 * l2 / kvb))))
@@ -545,7 +566,7 @@ def run_workloads(torch, nld, dev, stream, peak, l2):
                  "kv_bytes_per_pass": kvb, "kv_partials": parts,
                  "l2": ("cold: %d rotating pools" % npool) if npool * kvb >= 3 * l2 else
                        "warm: KV fits in L2 (%d pools, launch-bound shape)" % npool}
-        if name.startswith("long"):
+        if name.startswith("long") and only is None:
             sweep = {}
             for S in (1, 2, 4, 8, 16, 32, 64):
                 pS = nld.make_params(B, Hq, Hkv, D, w["page"], w["num_pages"], w["max_pages"], S, 0.0,
@@ -657,6 +678,9 @@ def main():
         print(f"--gpus {args.gpus} but WORLD_SIZE {world}", file=sys.stderr)
     if args.impl == "reference":
         run_reference(args, world, rank)
+        return
+    if args.only_workload is not None:
+        run_only_workload(args, local)
         return
     run_ours(args, world, rank, local)
 

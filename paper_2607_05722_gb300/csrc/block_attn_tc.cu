@@ -237,8 +237,10 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
         umma_commit(&kv_empty[st]);
       };
       // Event-driven issue: S_k needs its K tile and a free S buffer (the
-      // softmax warps have read S_{k-2}); PV_k needs P_k. Whichever is ready
-      // goes first, so a late K/V tile never holds back a ready PV.
+      // softmax warps have read S_{k-2} into registers); PV_k needs P_k.
+      // Whichever is ready goes first, so a late K/V tile never holds back a
+      // ready PV. (Letting S_{k+2} run ahead of PV_k measured slower: it
+      // queues in front of the PV on the tensor core.)
       int next_s = 0, next_pv = 0;
       const uint64_t t_start = global_timer_ns();
       uint32_t spins = 0;

@@ -74,6 +74,8 @@ nld_status_t check_params(const nld_attn_params_t* p, int block_len) {
 // resident at once. An explicit split count of 2, 4 or 8 uses one cluster; a
 // larger count divisible by 8, 4 or 2 uses clusters of that size, leaving
 // one partial per cluster for the combine.
+constexpr long long kMaxAutoChunk = 2048;  // tokens per piece in an automatic plan (1 MiB of K+V at D=128)
+
 struct SplitPlan {
   int splits;    // CTAs along the KV range per (sequence, KV head)
   int chunk;     // tokens per split
@@ -92,7 +94,16 @@ nld_status_t plan_splits(const nld_attn_params_t* p, int block_len, SplitPlan* o
     int sms = 0;
     nld_status_t st = device_state(nullptr, &sms);
     if (st != NLD_OK) return st;
+    // Fill the SMs once; when the (sequence, KV head) units fit in one wave,
+    // also cut long ranges into pieces of at most kMaxAutoChunk tokens: with
+    // ragged lengths (not known on the host) the longest sequence would
+    // otherwise set the time; pieces past a shorter sequence's end exit at
+    // once. With more units than SMs the hardware scheduler balances them.
     long long s = sms / units;
+    if (units < sms) {  // a single wave: the longest range would set the time
+      const long long by_chunk = (max_tokens + kMaxAutoChunk - 1) / kMaxAutoChunk;
+      if (s < by_chunk) s = by_chunk;
+    }
     const long long by_tiles = (max_tokens + nld::kTileTok - 1) / nld::kTileTok;  // >= one tile per split
     if (s > by_tiles) s = by_tiles;
     if (s > nld::kMaxSplits) s = nld::kMaxSplits;
