@@ -1,29 +1,32 @@
 // Block attention over a paged bf16 KV cache on the 5th-generation tensor
-// cores (tcgen05, accumulators in tensor memory), for up to 128 packed query
+// cores (tcgen05, accumulators in tensor memory), for up to 256 packed query
 // rows (Sec. 2.2 mask; Sec. 3 Modes 2 and 3).
 //
 // One CTA serves one (KV split, KV head g, sequence b): its G = Hq/Hkv query
-// heads times the bl block tokens form R = G*bl <= 128 query rows, padded to
-// the 128-row MMA tile, so each K/V page leaves HBM once per (b, g).
+// heads times the bl block tokens form R = G*bl <= 256 query rows in one or
+// two 128-row MMA tiles, so each K/V page leaves HBM once per (b, g).
 //
 // Warp roles (9 warps):
 //   warps 0-2, 8  TMA producers: the boxes of each 64-token K/V tile (16 tokens
 //             x 64 dims each) dealt four ways into a 4-stage ring (produce_kv);
 //             TMA issue cost is per warp, so four issuing warps land a tile
 //             sooner.
-//   warp 3    allocates 256 TMEM columns; lane 0 issues every MMA (it shares
-//             an SM sub-partition with the softmax warp of rows 96-127, which
-//             are padding for the shapes with fewer packed rows):
+//   warp 3    allocates the TMEM columns; lane 0 issues every MMA:
 //               S_k = Q K_k^T   (M=128 rows, N=64 tokens, K=D; double-buffered in TMEM)
 //               O  += P_k V_k   (M=128 rows, N=D, K=64 tokens; V read MN-major)
 //             S_{k+1} is issued before O += P_k V_k so the tensor core computes
 //             the next scores while the softmax warps work on the current ones.
-//   warps 4-7 softmax: thread t owns query row 32*(warp%4)+lane (its TMEM lane).
-//             It loads its S row, applies the mask and the base-2 scale,
+//   warps 4-7 softmax: thread t owns TMEM lane 32*(warp%4)+lane, one query
+//             row. It loads its S row, applies the mask and the base-2 scale,
 //             keeps the running max and sum, writes P (bf16) to shared memory
 //             for the PV MMA, and at the end reads O from TMEM, divides by the
-//             sum and stages its rows in the freed K/V ring so that each row
-//             leaves as one coalesced store (bf16 output or fp32 split partial).
+//             sum and stages its row in the freed K/V ring, from where one
+//             bulk copy per row writes it (bf16 output or fp32 split partial).
+//             With at most 64 (32) packed rows, Q is replicated into the idle
+//             lane quadrants (REP = 2 or 4): each copy of a row takes a 64/REP-
+//             token slice of every tile with its own running max and sum, so
+//             every softmax warp works and each does 1/REP of the exponentials;
+//             the slices are merged once, before the epilogue.
 // When the KV range of a (sequence, KV head) is split over a thread-block
 // cluster, the CTAs stage their normalised rows in shared memory and merge
 // them through distributed shared memory (a cluster barrier, then each CTA
@@ -84,10 +87,12 @@ struct TcLayout {
   static_assert(kLseOutOff + kMergeRows * 4 <= kPOff, "epilogue staging overlaps the live buffers");
 };
 
-template <int D, int MT>
+template <int D, int MT, int REP>
 __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
     block_attn_tc_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
                          const AttnArgs a) {
+  static_assert(REP == 1 || REP == 2 || REP == 4, "replication of 1, 2 or 4");
+  static_assert(MT == 1 || REP == 1, "replication only with one M tile");
   using Geo = TileGeom<D>;
   using Lay = TcLayout<D, MT>;
   constexpr int kTcStages = Lay::kStages;
@@ -275,43 +280,69 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
     __syncwarp();
   } else {
     // ---------------- softmax warps ----------------
-    const int quad = warp & 3;                      // TMEM lanes 32*quad .. +31
+    // Warp `quad` reads TMEM lanes 32*quad..+31. With REP > 1 those lanes hold
+    // a copy of row block rq = quad % kRowQuads and the warp takes the token
+    // slice cp = quad / kRowQuads (columns c0 .. c0+kCols-1) of every tile.
+    constexpr int kRowQuads = 4 / REP;
+    constexpr int kCols = kTileTok / REP;           // S columns per thread and tile
+    const int quad = warp & 3;
     const int mt = (warp - kSoftmaxWarp0) >> 2;     // M tile of this warp
-    const int r_loc = quad * 32 + lane;             // row within the M tile == TMEM lane
-    const int r = mt * 128 + r_loc;                 // packed query row
+    const int rq = quad % kRowQuads;                // row block
+    const int cp = quad / kRowQuads;                // token slice
+    const int c0 = cp * kCols;
+    const int r_loc = quad * 32 + lane;             // TMEM lane == row of the Q and P tiles
+    const int r = mt * 128 + rq * 32 + lane;        // packed query row
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
-    const bool warp_rows = mt * 128 + quad * 32 < a.R;  // warp-uniform: the warp holds a real row
+    const bool warp_rows = mt * 128 + rq * 32 < a.R;  // warp-uniform: the warp holds a real row
     const bool row_ok = r < a.R;
     const int row_i = r / a.G;
     const int row_h = g * a.G + (r - row_i * a.G);
     const int sm_tid = threadIdx.x - 32 * kSoftmaxWarp0;  // 0 .. 128*MT-1 across the softmax warps
+    const int swz = r_loc & 7;                      // 128-byte swizzle phase of this tile row
     uint8_t* q_tile = q_s + mt * Lay::kQBytes;
     auto p_buf = [&](int j) -> uint8_t* { return smem + Lay::kPOff + (mt * 2 + j) * Lay::kPBytes; };
 
-    // Q row -> shared memory in the 128-byte-swizzled K-major layout; padding
-    // rows are zero. Padding rows of P are zeroed once for both buffers.
+    // Q row -> shared memory in the 128-byte-swizzled K-major layout (padding
+    // rows zero); slice 0 loads it once and writes every copy. The columns of
+    // P a thread never writes (other slices' tokens, or all of a padding row)
+    // are zeroed once in both buffers.
     if (early) grid_dependency_wait();
     {
-      const uint4* qrow = reinterpret_cast<const uint4*>(
-          a.q + ((static_cast<size_t>(b) * a.bl + row_i) * a.Hq + row_h) * D);
+      if (cp == 0) {
+        const uint4* qrow = reinterpret_cast<const uint4*>(
+            a.q + ((static_cast<size_t>(b) * a.bl + row_i) * a.Hq + row_h) * D);
+        uint4 v[D / 8];
 #pragma unroll
-      for (int c = 0; c < D / 8; ++c) {
-        uint4 v = make_uint4(0, 0, 0, 0);
-        if (row_ok) v = __ldg(qrow + c);
-        *reinterpret_cast<uint4*>(q_tile + (c >> 3) * (128 * 128) + r_loc * 128 + (((c & 7) ^ (r & 7)) << 4)) = v;
+        for (int c = 0; c < D / 8; ++c) v[c] = row_ok ? __ldg(qrow + c) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+        for (int q = 0; q < REP; ++q) {
+          const int rl = r_loc + q * kRowQuads * 32;  // TMEM lane of copy q (same swizzle phase)
+#pragma unroll
+          for (int c = 0; c < D / 8; ++c)
+            *reinterpret_cast<uint4*>(q_tile + (c >> 3) * (128 * 128) + rl * 128 + (((c & 7) ^ swz) << 4)) = v[c];
+        }
       }
-      if (!row_ok) {
 #pragma unroll
-        for (int j = 0; j < 2; ++j)
+      for (int j = 0; j < 2; ++j)
 #pragma unroll
-          for (int c = 0; c < 8; ++c)
-            *reinterpret_cast<uint4*>(p_buf(j) + r_loc * 128 + ((c ^ (r & 7)) << 4)) = make_uint4(0, 0, 0, 0);
-      }
+        for (int c = 0; c < 8; ++c)
+          if (!row_ok || c < c0 / 8 || c >= (c0 + kCols) / 8)
+            *reinterpret_cast<uint4*>(p_buf(j) + r_loc * 128 + ((c ^ swz) << 4)) = make_uint4(0, 0, 0, 0);
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(q_ready);
     }
 
+    // The keys this row may see inside [t_begin, t_end) are exactly t < lim
+    // (Sec. 2.2: the whole prefix; in the draft pass every block slot, in the
+    // verify pass the block slots up to the row's own), so the mask is one
+    // compare per element on every tile, with no separate code path.
+    const int lim = diff_mode ? t_end : min(t_end, L + row_i + 1);
+    // A wait that gives up does so for the whole warp, so that no lane skips
+    // a warp-collective TMEM instruction the others execute.
+    auto warp_wait = [&](uint64_t* bar, uint32_t parity) {
+      return __all_sync(0xffffffffu, mbar_wait(bar, parity, a.err));
+    };
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
     for (int k = 0; k < ntiles; ++k) {
@@ -319,16 +350,21 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
       const int st = k % kTcStages;
       const int tile_t0 = t_begin + k * kTileTok;
       const int valid = t_end - tile_t0;
-      if (!mbar_wait(&s_full[buf], (k >> 1) & 1, a.err)) {
+      if (!warp_wait(&s_full[buf], (k >> 1) & 1)) {
         ok = false;
         break;
       }
       tc_fence_after();
-      float s[kTileTok];
+      float s[kCols];
       if (warp_rows) {
-        const uint32_t ts = tS(mt, buf) + lane_off;
-        tmem_ld32(ts, s);
-        tmem_ld32(ts + 32, s + 32);
+        const uint32_t ts = tS(mt, buf) + lane_off + static_cast<uint32_t>(c0);
+        if constexpr (kCols == 64) {
+          tmem_ld64(ts, s);
+        } else if constexpr (kCols == 32) {
+          tmem_ld32(ts, s);
+        } else {
+          tmem_ld16(ts, s);
+        }
       }
       tc_fence_before();
       __syncwarp();
@@ -337,24 +373,13 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
       float alpha = 1.f;
       bool rescale = false;
       if (warp_rows) {
-        // Scale to base 2 and take the row max. The mask only matters on a
-        // tile that reaches the block or the split end; it is applied there
-        // branch-free (a branch per element in this unrolled loop costs ~8x).
+        // Mask, base-2 scale and row max, branch-free.
+        const int nv = lim - (tile_t0 + c0);
         float mx = -INFINITY;
-        if ((tile_t0 + kTileTok <= L) && (valid >= kTileTok)) {
 #pragma unroll
-          for (int j = 0; j < kTileTok; ++j) {
-            s[j] *= scl;
-            mx = fmaxf(mx, s[j]);
-          }
-        } else {
-#pragma unroll
-          for (int j = 0; j < kTileTok; ++j) {
-            const int t = tile_t0 + j;
-            const bool vis = (j < valid) & ((t < L) | diff_mode | (t - L <= row_i));
-            s[j] = vis ? s[j] * scl : -INFINITY;
-            mx = fmaxf(mx, s[j]);
-          }
+        for (int j = 0; j < kCols; ++j) {
+          s[j] = j < nv ? s[j] * scl : -INFINITY;
+          mx = fmaxf(mx, s[j]);
         }
         if (m_run == -INFINITY) {
           m_run = mx;  // nothing accumulated for this row yet
@@ -367,7 +392,7 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
       }
       if (__any_sync(0xffffffffu, rescale)) {
         // O holds P_0..P_{k-1} V: wait for the last PV, then scale this warp's rows.
-        if (!mbar_wait(&o_done[(k - 1) & 1], ((k - 1) >> 1) & 1, a.err)) {
+        if (!warp_wait(&o_done[(k - 1) & 1], ((k - 1) >> 1) & 1)) {
           ok = false;
           break;
         }
@@ -382,7 +407,7 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
         }
       }
       // P buffer `buf` is free once the PV of tile k-2 has completed.
-      if (k >= 2 && !mbar_wait(&o_done[buf], ((k - 2) >> 1) & 1, a.err)) {
+      if (k >= 2 && !warp_wait(&o_done[buf], ((k - 2) >> 1) & 1)) {
         ok = false;
         break;
       }
@@ -390,7 +415,7 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
         const float mu = m_run == -INFINITY ? 0.f : m_run;
         uint8_t* prow = p_buf(buf) + r_loc * 128;
 #pragma unroll
-        for (int c = 0; c < kTileTok / 8; ++c) {
+        for (int c = 0; c < kCols / 8; ++c) {
           uint32_t w[4];
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
@@ -399,14 +424,15 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
             l_run += p0 + p1;
             w[e] = pack_bf16(p0, p1);
           }
-          *reinterpret_cast<uint4*>(prow + ((c ^ (r & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+          const int chunk = c0 / 8 + c;
+          *reinterpret_cast<uint4*>(prow + ((chunk ^ swz) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
         }
       }
       if (valid < kTileTok && (valid & (kGroupTok - 1))) {
         // Cache slots past the sequence end inside its last page may hold
         // stale or uninitialised data; P is 0 there but 0 * NaN = NaN, so
         // zero those V rows before the PV MMA reads them.
-        if (!mbar_wait(&kv_full[st], (k / kTcStages) & 1, a.err)) {
+        if (!warp_wait(&kv_full[st], (k / kTcStages) & 1)) {
           ok = false;
           break;
         }
@@ -425,9 +451,87 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
 
     // ---------------- epilogue ----------------
     // Every PV has completed once o_done of the last tile fires, so the K/V
-    // ring is free: each warp stages its 32 rows there (padded pitch, no bank
-    // conflicts), then writes each row with one coalesced warp-wide store.
-    const bool o_ready = ok && mbar_wait(&o_done[(ntiles - 1) & 1], ((ntiles - 1) >> 1) & 1, a.err);
+    // ring is free for staging.
+    // Warp-uniform, like every condition around the warp-collective TMEM
+    // loads and stores below.
+    const bool o_ready =
+        __all_sync(0xffffffffu, ok && mbar_wait(&o_done[(ntiles - 1) & 1], ((ntiles - 1) >> 1) & 1, a.err));
+    // Weights of the token slices of each row, by the split-combine rule
+    // (Sec. 3 Mode 2, here on one SM): slices cp > 0 leave their max, sum and
+    // unscaled O row in the freed ring (rows 32*kRowQuads.. of it); slice 0
+    // weighs them against its own and adds them in as it stages its output.
+    float w_self = 1.f;
+    float w_rep[REP > 1 ? REP - 1 : 1];
+    w_rep[0] = 0.f;
+    if constexpr (REP > 1) {
+      float* part_ml = reinterpret_cast<float*>(smem + Lay::kWtsOff);  // [TMEM lane][max, sum]
+      if (o_ready) tc_fence_after();
+      if (cp > 0) {
+        part_ml[2 * r_loc] = o_ready ? m_run : -INFINITY;  // a slice cut short by a timeout is dropped
+        part_ml[2 * r_loc + 1] = l_run;
+        if (warp_rows && o_ready) {
+          uint8_t* xrow = smem + r_loc * merge_pitch<D>();
+#pragma unroll 1
+          for (int c = 0; c < D / 32; ++c) {
+            float o[32];
+            tmem_ld32(tO(mt) + lane_off + c * 32, o);
+#pragma unroll
+            for (int q4 = 0; q4 < 8; ++q4)
+              *reinterpret_cast<float4*>(xrow + c * 128 + q4 * 16) =
+                  make_float4(o[4 * q4], o[4 * q4 + 1], o[4 * q4 + 2], o[4 * q4 + 3]);
+          }
+        }
+      }
+      named_bar_sync(2, 128);  // the four softmax warps
+      if (cp == 0) {
+        float m = m_run, mp[REP - 1], lp[REP - 1];
+#pragma unroll
+        for (int q = 0; q < REP - 1; ++q) {
+          const int lq = ((q + 1) * kRowQuads + rq) * 32 + lane;
+          mp[q] = part_ml[2 * lq];
+          lp[q] = part_ml[2 * lq + 1];
+          m = fmaxf(m, mp[q]);
+        }
+        // A row that saw no key in any slice (possible in the verify pass)
+        // keeps m = -inf, sum 0 and weight 0 everywhere.
+        w_self = m_run == -INFINITY ? 0.f : ex2(m_run - m);
+        float l = w_self * l_run;
+#pragma unroll
+        for (int q = 0; q < REP - 1; ++q) {
+          w_rep[q] = mp[q] == -INFINITY ? 0.f : ex2(mp[q] - m);
+          l += w_rep[q] * lp[q];
+        }
+        if (m != -INFINITY) {
+          m_run = m;
+          l_run = l;
+        }
+      }
+    }
+    // Unnormalised O of this thread's row, columns 64c..64c+63: its own TMEM
+    // lane plus, with REP > 1, the other slices of the row. Warp-collective.
+    auto load_o = [&](int c, float* o) {
+      tmem_ld64(tO(mt) + lane_off + c * 64, o);
+      if constexpr (REP > 1) {
+#pragma unroll
+        for (int j = 0; j < 64; ++j) o[j] *= w_self;
+#pragma unroll
+        for (int q = 0; q < REP - 1; ++q) {
+          if (w_rep[q] == 0.f) continue;  // a slice without keys never wrote its row
+          const uint8_t* xrow = smem + ((q + 1) * kRowQuads * 32 + rq * 32 + lane) * merge_pitch<D>() + c * 256;
+#pragma unroll
+          for (int q4 = 0; q4 < 16; ++q4) {
+            const float4 x = *reinterpret_cast<const float4*>(xrow + q4 * 16);
+            o[4 * q4] += w_rep[q] * x.x;
+            o[4 * q4 + 1] += w_rep[q] * x.y;
+            o[4 * q4 + 2] += w_rep[q] * x.z;
+            o[4 * q4 + 3] += w_rep[q] * x.w;
+          }
+        }
+      }
+    };
+    // One thread per output row from here on (slice 0 of each row).
+    const bool out_warp = warp_rows && cp == 0;
+    const bool out_row = row_ok && cp == 0;
     if (a.csize > 1) {
       // Cluster: stage this CTA's normalised rows and their log2-sum-exp in
       // the freed ring for the merge across the cluster (rows without keys,
@@ -435,78 +539,61 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
       if (o_ready) tc_fence_after();
       float* lse_stage = reinterpret_cast<float*>(smem + Lay::kLseOff);
       const float l = l_run;
-      const bool has = o_ready && row_ok && l > 0.f;
-      lse_stage[r] = has ? m_run + lg2(l) : -INFINITY;
-      if (warp_rows && o_ready) {
+      const bool has = o_ready && out_row && l > 0.f;
+      if (cp == 0) lse_stage[r] = has ? m_run + lg2(l) : -INFINITY;
+      if (out_warp && o_ready) {
         const float inv = l > 0.f ? 1.f / l : 0.f;
         uint8_t* my = smem + r * merge_pitch<D>();
 #pragma unroll 1
-        for (int c = 0; c < D / 32; ++c) {
-          float o[32];
-          tmem_ld32(tO(mt) + lane_off + c * 32, o);
+        for (int c = 0; c < D / 64; ++c) {
+          float o[64];
+          load_o(c, o);
 #pragma unroll
-          for (int q4 = 0; q4 < 8; ++q4)
-            *reinterpret_cast<float4*>(my + c * 128 + q4 * 16) =
+          for (int q4 = 0; q4 < 16; ++q4)
+            *reinterpret_cast<float4*>(my + c * 256 + q4 * 16) =
                 make_float4(o[4 * q4] * inv, o[4 * q4 + 1] * inv, o[4 * q4 + 2] * inv, o[4 * q4 + 3] * inv);
         }
       }
     } else if (o_ready) {
+      // Each thread stages its row (padded pitch, no bank conflicts) and
+      // hands it to the TMA engine as one bulk copy.
       tc_fence_after();
-      if (warp_rows) {
+      if (out_warp) {
         const float l = l_run;
         const float inv = l > 0.f ? 1.f / l : 0.f;
         const float lse_v = l > 0.f ? (m_run + lg2(l)) * kLn2 : -INFINITY;
         const bool split_out = a.o_part != nullptr;
         const int row_bytes = split_out ? D * 4 : D * 2;
-        const int pitch = row_bytes + 16;
-        uint8_t* stage = smem + (mt * 128 + quad * 32) * pitch;  // inside the freed ring and Q tiles
-        uint8_t* my = stage + lane * pitch;
+        uint8_t* my = smem + (mt * 128 + r_loc) * (row_bytes + 16);
 #pragma unroll 1
-        for (int c = 0; c < D / 32; ++c) {
-          float o[32];
-          tmem_ld32(tO(mt) + lane_off + c * 32, o);
+        for (int c = 0; c < D / 64; ++c) {
+          float o[64];
+          load_o(c, o);
 #pragma unroll
-          for (int j = 0; j < 32; ++j) o[j] *= inv;
+          for (int j = 0; j < 64; ++j) o[j] *= inv;
           if (split_out) {
 #pragma unroll
-            for (int q4 = 0; q4 < 8; ++q4)
-              *reinterpret_cast<float4*>(my + c * 128 + q4 * 16) =
+            for (int q4 = 0; q4 < 16; ++q4)
+              *reinterpret_cast<float4*>(my + c * 256 + q4 * 16) =
                   make_float4(o[4 * q4], o[4 * q4 + 1], o[4 * q4 + 2], o[4 * q4 + 3]);
           } else {
 #pragma unroll
-            for (int q4 = 0; q4 < 4; ++q4) {
+            for (int q4 = 0; q4 < 8; ++q4) {
               const int j = q4 * 8;
-              *reinterpret_cast<uint4*>(my + c * 64 + q4 * 16) =
+              *reinterpret_cast<uint4*>(my + c * 128 + q4 * 16) =
                   make_uint4(pack_bf16(o[j], o[j + 1]), pack_bf16(o[j + 2], o[j + 3]), pack_bf16(o[j + 4], o[j + 5]),
                              pack_bf16(o[j + 6], o[j + 7]));
             }
           }
         }
-        // Global row of each lane's query row: output row (unsplit) or partial row.
-        const size_t my_row = split_out
-                                  ? ((static_cast<size_t>(split) * a.B + b) * a.Hq + row_h) * a.bl + row_i
-                                  : (static_cast<size_t>(b) * a.bl + row_i) * a.Hq + row_h;
-        const bool my_write = row_ok && (!split_out || l > 0.f);
-        __syncwarp();
-        const int chunks = row_bytes / 16;  // 8..32 lanes move one row
-        uint8_t* gbase = split_out ? reinterpret_cast<uint8_t*>(a.o_part) : reinterpret_cast<uint8_t*>(a.out);
-        // Eight rows per batch: all shared-memory reads of a batch are issued
-        // before its global stores (through generic pointers the compiler
-        // cannot reorder a read after an earlier store on its own).
-#pragma unroll
-        for (int j0 = 0; j0 < 32; j0 += 8) {
-          uint4 v[8];
-          size_t row[8];
-          bool w[8];
-#pragma unroll
-          for (int u = 0; u < 8; ++u) {
-            row[u] = __shfl_sync(0xffffffffu, my_row, j0 + u);
-            w[u] = __shfl_sync(0xffffffffu, my_write, j0 + u) && lane < chunks;
-            v[u] = *reinterpret_cast<const uint4*>(stage + (j0 + u) * pitch + lane * 16);
-          }
-#pragma unroll
-          for (int u = 0; u < 8; ++u)
-            if (w[u]) *reinterpret_cast<uint4*>(gbase + row[u] * row_bytes + lane * 16) = v[u];
+        // Output row (unsplit) or partial row; partial rows without keys are
+        // not written (their lse is -inf and the combine skips them).
+        if (row_ok && (!split_out || l > 0.f)) {
+          const size_t grow = split_out ? ((static_cast<size_t>(split) * a.B + b) * a.Hq + row_h) * a.bl + row_i
+                                        : (static_cast<size_t>(b) * a.bl + row_i) * a.Hq + row_h;
+          uint8_t* gbase = split_out ? reinterpret_cast<uint8_t*>(a.o_part) : reinterpret_cast<uint8_t*>(a.out);
+          fence_proxy_async_smem();  // this thread's staged row, visible to the TMA engine
+          bulk_store(gbase + grow * row_bytes, my, static_cast<uint32_t>(row_bytes));
         }
         if (row_ok) {
           if (!split_out) {
@@ -515,6 +602,7 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
             a.lse_part[((static_cast<size_t>(split) * a.B + b) * a.Hq + row_h) * a.bl + row_i] = lse_v;
           }
         }
+        bulk_store_wait_read();  // the staged row stays in place until the copy has read it
       }
     }
     tc_fence_before();
@@ -620,12 +708,12 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
   }
 }
 
-template <int D, int MT>
+template <int D, int MT, int REP>
 cudaError_t configure_tc(int dev) {
   static int configured[64] = {0};
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   if (!__atomic_load_n(&configured[dev], __ATOMIC_ACQUIRE)) {
-    cudaError_t e = cudaFuncSetAttribute(block_attn_tc_kernel<D, MT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(block_attn_tc_kernel<D, MT, REP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(TcLayout<D, MT>::kBytes + 1024));
     if (e != cudaSuccess) return e;
     __atomic_store_n(&configured[dev], 1, __ATOMIC_RELEASE);
@@ -633,18 +721,18 @@ cudaError_t configure_tc(int dev) {
   return cudaSuccess;
 }
 
-template <int D, int MT>
+template <int D, int MT, int REP>
 cudaError_t launch_tc_t(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, cudaStream_t stream) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  if ((e = configure_tc<D, MT>(dev)) != cudaSuccess) return e;
+  if ((e = configure_tc<D, MT, REP>(dev)) != cudaSuccess) return e;
   dim3 grid(a.num_splits, a.Hkv, a.B);
-  return launch_kernel_cluster(block_attn_tc_kernel<D, MT>, grid, dim3(TcCfg<MT>::kThreads),
+  return launch_kernel_cluster(block_attn_tc_kernel<D, MT, REP>, grid, dim3(TcCfg<MT>::kThreads),
                                TcLayout<D, MT>::kBytes + 1024, stream, a.csize, tmk, tmv, a);
 }
 
-template <int D, int MT>
+template <int D, int MT, int REP>
 int max_active_clusters_t(int csize) {
   static int cache[64][4];  // [device][cluster size 2/4/8] + 1 (0 = not queried)
   int dev = 0;
@@ -652,7 +740,7 @@ int max_active_clusters_t(int csize) {
   const int slot = csize == 2 ? 0 : csize == 4 ? 1 : csize == 8 ? 2 : 3;
   int v = __atomic_load_n(&cache[dev][slot], __ATOMIC_ACQUIRE);
   if (v) return v - 1;
-  if (configure_tc<D, MT>(dev) != cudaSuccess) return 0;
+  if (configure_tc<D, MT, REP>(dev) != cudaSuccess) return 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(csize, 1, 1);
   cfg.blockDim = dim3(TcCfg<MT>::kThreads);
@@ -665,7 +753,7 @@ int max_active_clusters_t(int csize) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, block_attn_tc_kernel<D, MT>, &cfg) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveClusters(&n, block_attn_tc_kernel<D, MT, REP>, &cfg) != cudaSuccess) {
     cudaGetLastError();
     n = 0;
   }
@@ -673,19 +761,41 @@ int max_active_clusters_t(int csize) {
   return n;
 }
 
+// Copies of each Q row in the 128 TMEM lanes of one M tile: 4 for up to 32
+// packed rows, 2 for up to 64, else 1 (and 1 with two M tiles).
+int tc_replication(int rows) { return rows <= 32 ? 4 : rows <= 64 ? 2 : 1; }
+
+template <int D>
+int max_active_clusters_d(int csize, int rows) {
+  if (rows > 128) return max_active_clusters_t<D, 2, 1>(csize);
+  switch (tc_replication(rows)) {
+    case 4: return max_active_clusters_t<D, 1, 4>(csize);
+    case 2: return max_active_clusters_t<D, 1, 2>(csize);
+    default: return max_active_clusters_t<D, 1, 1>(csize);
+  }
+}
+
+template <int D>
+cudaError_t launch_tc_d(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, cudaStream_t stream) {
+  if (a.R > 128) return launch_tc_t<D, 2, 1>(a, tmk, tmv, stream);
+  switch (tc_replication(a.R)) {
+    case 4: return launch_tc_t<D, 1, 4>(a, tmk, tmv, stream);
+    case 2: return launch_tc_t<D, 1, 2>(a, tmk, tmv, stream);
+    default: return launch_tc_t<D, 1, 1>(a, tmk, tmv, stream);
+  }
+}
+
 }  // namespace
 
 bool tc_supports(int R, int head_dim) { return R <= 256 && (head_dim == 64 || head_dim == 128); }
 
 int tc_max_active_clusters(int csize, int head_dim, int rows) {
-  if (rows > 128) return head_dim == 128 ? max_active_clusters_t<128, 2>(csize) : max_active_clusters_t<64, 2>(csize);
-  return head_dim == 128 ? max_active_clusters_t<128, 1>(csize) : max_active_clusters_t<64, 1>(csize);
+  return head_dim == 128 ? max_active_clusters_d<128>(csize, rows) : max_active_clusters_d<64>(csize, rows);
 }
 
 cudaError_t launch_block_attn_tc(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, int head_dim,
                                  cudaStream_t stream) {
-  if (a.R > 128) return head_dim == 128 ? launch_tc_t<128, 2>(a, tmk, tmv, stream) : launch_tc_t<64, 2>(a, tmk, tmv, stream);
-  return head_dim == 128 ? launch_tc_t<128, 1>(a, tmk, tmv, stream) : launch_tc_t<64, 1>(a, tmk, tmv, stream);
+  return head_dim == 128 ? launch_tc_d<128>(a, tmk, tmv, stream) : launch_tc_d<64>(a, tmk, tmv, stream);
 }
 
 }  // namespace nld
