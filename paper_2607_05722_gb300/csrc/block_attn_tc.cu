@@ -44,21 +44,33 @@ constexpr int kProducers = 4;
 constexpr int kMmaWarp = 3;
 constexpr int kSoftmaxWarp0 = 4;
 
-// MT 128-row M tiles per CTA (MT = 2 for 129..256 packed rows): each K/V tile
-// feeds MT score and MT PV products; 4*MT softmax warps; the ring shrinks to
-// 3 stages so that two Q tiles and four P buffers fit in shared memory.
-template <int MT>
+// MT 128-row M tiles per CTA (MT = 2 for 129..256 packed rows); 4*MT
+// softmax warps; TPS 64-token K/V tiles per score product. TPS = 2 (one M
+// tile, a split short enough to sit in the ring whole): N = 128 products,
+// which the tensor core runs at full rate (N = 64 at about half), half as
+// many steps in the chain S -> softmax -> PV, and four P buffers so that the
+// softmax of one pair never waits for the PV products of the last. A long
+// split streams with TPS = 1, where a stage frees after each tile and more
+// of the ring stays in flight. With two M tiles the ring shrinks to 3
+// stages, so that two Q tiles and 2x2 P buffers fit.
+template <int MT, int TPS>
 struct TcCfg {
+  static_assert(TPS == 1 || (TPS == 2 && MT == 1), "paired score products with one M tile");
   static constexpr int kStages = MT == 1 ? 4 : 3;
-  static constexpr int kWarps = 5 + 4 * MT;  // 4 producers, 1 MMA, 4*MT softmax
+  static constexpr int kTPS = TPS;               // K/V tiles per score product
+  static constexpr int kSTok = kTPS * kTileTok;  // tokens (N) of a score product
+  static constexpr int kPBufs = 2 * kTPS;        // P buffers per M tile
+  static constexpr int kWarps = 5 + 4 * MT;      // 4 producers, 1 MMA, 4*MT softmax
   static constexpr int kThreads = 32 * kWarps;
-  static constexpr uint32_t kTmemCols = MT == 1 ? 256 : 512;  // MT x (S0 | S1), then MT x O
+  static constexpr uint32_t kTmemCols = 512;     // MT x (S0 | S1), then MT x O
+  static_assert(kStages % kTPS == 0, "a score product never wraps around the ring");
+  static_assert(2 * MT * kSTok + MT * 128 <= 512, "TMEM columns");
 };
 
 // producer index of a warp, or -1: warps 0-2 and the last warp
 template <int MT>
 __device__ __forceinline__ int producer_index(int warp) {
-  return warp < 3 ? warp : (warp == TcCfg<MT>::kWarps - 1 ? 3 : -1);
+  return warp < 3 ? warp : (warp == TcCfg<MT, 1>::kWarps - 1 ? 3 : -1);
 }
 constexpr float kRescaleLog2 = 8.0f;
 
@@ -68,18 +80,24 @@ constexpr float kRescaleLog2 = 8.0f;
 template <int D>
 __host__ __device__ constexpr int merge_pitch() { return D * 4 + 16; }
 
-template <int D, int MT>
+// K/V ring: the K tiles column-block-major ([column block][stage], so that
+// the K tiles of consecutive stages form one operand of 128 rows), then the
+// V tiles stage-major ([stage][column block]).
+template <int D, int MT, int TPS>
 struct TcLayout {
   using Geo = TileGeom<D>;
-  static constexpr int kStages = TcCfg<MT>::kStages;
+  static constexpr int kStages = TcCfg<MT, TPS>::kStages;
+  static constexpr int kPBufs = TcCfg<MT, TPS>::kPBufs;
+  static constexpr int kVOff = kStages * Geo::kTileBytes;       // V tiles after the K tiles
   static constexpr int kQBytes = Geo::kColBlocks * 128 * 128;  // one 128-row Q tile, bf16
   static constexpr int kPBytes = 128 * kTileTok * 2;             // one 128-row x 64-token P buffer, bf16
   static constexpr int kQOff = kStages * Geo::kStageBytes;
   static constexpr int kPOff = kQOff + MT * kQBytes;
-  static constexpr int kBarOff = kPOff + MT * 2 * kPBytes;
-  // kv_full[st], kv_empty[st], s_full[2], s_free[2], p_full[2], o_done[2], q_ready, drain, tmem slot
-  static constexpr int kNumBars = 2 * kStages + 8 + 2;
+  static constexpr int kBarOff = kPOff + MT * kPBufs * kPBytes;
+  // kv_full[st], kv_empty[st], s_full[2], s_free[2], p_full[P], o_done[P], q_ready, drain, tmem slot
+  static constexpr int kNumBars = 2 * kStages + 4 + 2 * kPBufs + 2;
   static constexpr int kBytes = kBarOff + kNumBars * 8 + 16;
+  static_assert(kBytes + 1024 <= 232448, "shared memory per CTA");
   static constexpr int kMergeRows = 128 * MT;
   static constexpr int kLseOff = kMergeRows * merge_pitch<D>();
   static constexpr int kWtsOff = kLseOff + kMergeRows * 4;
@@ -87,14 +105,15 @@ struct TcLayout {
   static_assert(kLseOutOff + kMergeRows * 4 <= kPOff, "epilogue staging overlaps the live buffers");
 };
 
-template <int D, int MT, int REP>
-__global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
+template <int D, int MT, int REP, int TPS>
+__global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     block_attn_tc_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
                          const AttnArgs a) {
   static_assert(REP == 1 || REP == 2 || REP == 4, "replication of 1, 2 or 4");
   static_assert(MT == 1 || REP == 1, "replication only with one M tile");
   using Geo = TileGeom<D>;
-  using Lay = TcLayout<D, MT>;
+  using Cfg = TcCfg<MT, TPS>;
+  using Lay = TcLayout<D, MT, TPS>;
   constexpr int kTcStages = Lay::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -105,8 +124,8 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
   uint64_t* s_full = bars + 2 * kTcStages;
   uint64_t* s_free = s_full + 2;
   uint64_t* p_full = s_free + 2;
-  uint64_t* o_done = p_full + 2;
-  uint64_t* q_ready = o_done + 2;
+  uint64_t* o_done = p_full + Cfg::kPBufs;
+  uint64_t* q_ready = o_done + Cfg::kPBufs;
   uint64_t* drain = q_ready + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
 
@@ -122,6 +141,8 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
     for (int j = 0; j < 2; ++j) {
       mbar_init(&s_full[j], 1);
       mbar_init(&s_free[j], 4 * MT);
+    }
+    for (int j = 0; j < Cfg::kPBufs; ++j) {
       mbar_init(&p_full[j], 4 * MT);
       mbar_init(&o_done[j], 1);
     }
@@ -134,7 +155,7 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
     prefetch_tensormap(&tmv);
   }
   if (warp == kMmaWarp) {
-    tmem_alloc(tmem_slot, TcCfg<MT>::kTmemCols);
+    tmem_alloc(tmem_slot, Cfg::kTmemCols);
     tc_fence_before();
   }
   // Without NLD_ATTN_PREFIX_READY nothing global is read before the
@@ -154,9 +175,12 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  // TMEM columns: S of M tile mt, buffer j at (2*mt + j)*64; O of tile mt after all S buffers.
-  auto tS = [&](int mt, int j) -> uint32_t { return tmem + static_cast<uint32_t>((2 * mt + j) * kTileTok); };
-  auto tO = [&](int mt) -> uint32_t { return tmem + static_cast<uint32_t>(2 * MT * kTileTok + mt * D); };
+  // TMEM columns: S of M tile mt, buffer j at (2*mt + j)*kSTok; O of tile mt after all S buffers.
+  constexpr int kTPS = Cfg::kTPS;
+  constexpr int kSTok = Cfg::kSTok;
+  constexpr int kPBufs = Cfg::kPBufs;
+  auto tS = [&](int mt, int j) -> uint32_t { return tmem + static_cast<uint32_t>((2 * mt + j) * kSTok); };
+  auto tO = [&](int mt) -> uint32_t { return tmem + static_cast<uint32_t>(2 * MT * kSTok + mt * D); };
 
   const int lmax = a.max_pages * a.page_size - a.bl;
   if (L < 0 || L > lmax) {
@@ -204,31 +228,35 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
       bool ok = mbar_wait(q_ready, 0, a.err);
       tc_fence_after();
       const uint32_t q_addr = smem_u32(q_s);
-      const uint32_t idesc_s = umma_idesc_bf16(128, kTileTok, false);
+      const uint32_t idesc_s = umma_idesc_bf16(128, kSTok, false);
       const uint32_t idesc_o = umma_idesc_bf16(128, D, true);
-      auto issue_s = [&](int k) {
-        const int st = k % kTcStages;
-        const uint32_t k_addr = smem_u32(smem + st * Geo::kStageBytes);
+      // Score product j: tiles kTPS*j .. kTPS*j+kTPS-1, whose K tiles sit in
+      // consecutive stages (one operand of kSTok rows per column block). If
+      // the last product has a single tile, its second half reads a stage
+      // no tile of this CTA still needs; those columns are never used.
+      auto issue_s = [&](int j) {
+        const int st = (j * kTPS) % kTcStages;
+        const uint32_t k_addr = smem_u32(smem) + static_cast<uint32_t>(st * Geo::kColBlockBytes);
 #pragma unroll
         for (int mt = 0; mt < MT; ++mt) {
-          const uint32_t d = tS(mt, k & 1);
+          const uint32_t d = tS(mt, j & 1);
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk) {
             const uint32_t koff = (kk & 3) * 32;  // 16 elements along the 128-byte row
             const int cb = kk >> 2;               // 64-dim column block
             const uint64_t ad = sw128_desc(q_addr + mt * Lay::kQBytes + cb * (128 * 128) + koff, 0, 1024);
-            const uint64_t bd = sw128_desc(k_addr + cb * Geo::kColBlockBytes + koff, 0, 1024);
+            const uint64_t bd = sw128_desc(k_addr + cb * kTcStages * Geo::kColBlockBytes + koff, 0, 1024);
             umma_bf16(d, ad, bd, idesc_s, kk > 0 ? 1u : 0u);
           }
         }
-        umma_commit(&s_full[k & 1]);
+        umma_commit(&s_full[j & 1]);
       };
       auto issue_pv = [&](int k) {
         const int st = k % kTcStages;
-        const uint32_t v_addr = smem_u32(smem + st * Geo::kStageBytes + Geo::kTileBytes);
+        const uint32_t v_addr = smem_u32(smem + Lay::kVOff + st * Geo::kTileBytes);
 #pragma unroll
         for (int mt = 0; mt < MT; ++mt) {
-        const uint32_t p_addr = smem_u32(smem + Lay::kPOff + (mt * 2 + (k & 1)) * Lay::kPBytes);
+        const uint32_t p_addr = smem_u32(smem + Lay::kPOff + (mt * kPBufs + k % kPBufs) * Lay::kPBytes);
 #pragma unroll
         for (int kt = 0; kt < kTileTok / 16; ++kt) {
           // A = P rows (K-major, one 128-byte block of 64 tokens); B = V (MN-major:
@@ -238,27 +266,31 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
           umma_bf16(tO(mt), ad, bd, idesc_o, (k > 0 || kt > 0) ? 1u : 0u);
         }
         }
-        umma_commit(&o_done[k & 1]);
+        umma_commit(&o_done[k % kPBufs]);
         umma_commit(&kv_empty[st]);
       };
-      // Event-driven issue: S_k needs its K tile and a free S buffer (the
-      // softmax warps have read S_{k-2} into registers); PV_k needs P_k.
-      // Whichever is ready goes first, so a late K/V tile never holds back a
-      // ready PV. (Letting S_{k+2} run ahead of PV_k measured slower: it
-      // queues in front of the PV on the tensor core.)
+      // Event-driven issue: score product j needs its K tiles and a free S
+      // buffer (the softmax warps have read product j-2), and waits until
+      // the PV products of product j-2 are issued; PV_k needs P_k. Whichever
+      // is ready goes first, so a late K/V tile never holds back a ready PV.
+      // (Letting scores run further ahead measured slower: they queue in
+      // front of the PV products on the tensor core.)
+      const int nprod = (ntiles + kTPS - 1) / kTPS;
       int next_s = 0, next_pv = 0;
       const uint64_t t_start = global_timer_ns();
       uint32_t spins = 0;
       while (ok && next_pv < ntiles) {
         bool progressed = false;
-        if (next_s < ntiles && next_s < next_pv + 2 &&
-            mbar_test(&kv_full[next_s % kTcStages], (next_s / kTcStages) & 1) &&
+        const int t0 = next_s * kTPS;  // first tile of the next score product
+        if (next_s < nprod && t0 - kTPS <= next_pv &&
+            mbar_test(&kv_full[t0 % kTcStages], (t0 / kTcStages) & 1) &&
+            (kTPS == 1 || t0 + 1 >= ntiles || mbar_test(&kv_full[(t0 + 1) % kTcStages], ((t0 + 1) / kTcStages) & 1)) &&
             (next_s < 2 || mbar_test(&s_free[next_s & 1], ((next_s - 2) >> 1) & 1))) {
           tc_fence_after();
           issue_s(next_s++);
           progressed = true;
         }
-        if (next_pv < next_s && mbar_test(&p_full[next_pv & 1], (next_pv >> 1) & 1)) {
+        if (next_pv < next_s * kTPS && mbar_test(&p_full[next_pv % kPBufs], (next_pv / kPBufs) & 1)) {
           tc_fence_after();
           issue_pv(next_pv++);
           progressed = true;
@@ -300,12 +332,12 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
     const int sm_tid = threadIdx.x - 32 * kSoftmaxWarp0;  // 0 .. 128*MT-1 across the softmax warps
     const int swz = r_loc & 7;                      // 128-byte swizzle phase of this tile row
     uint8_t* q_tile = q_s + mt * Lay::kQBytes;
-    auto p_buf = [&](int j) -> uint8_t* { return smem + Lay::kPOff + (mt * 2 + j) * Lay::kPBytes; };
+    auto p_buf = [&](int j) -> uint8_t* { return smem + Lay::kPOff + (mt * kPBufs + j) * Lay::kPBytes; };
 
     // Q row -> shared memory in the 128-byte-swizzled K-major layout (padding
     // rows zero); slice 0 loads it once and writes every copy. The columns of
     // P a thread never writes (other slices' tokens, or all of a padding row)
-    // are zeroed once in both buffers.
+    // are zeroed once in every buffer.
     if (early) grid_dependency_wait();
     {
       if (cp == 0) {
@@ -323,7 +355,7 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
         }
       }
 #pragma unroll
-      for (int j = 0; j < 2; ++j)
+      for (int j = 0; j < kPBufs; ++j)
 #pragma unroll
         for (int c = 0; c < 8; ++c)
           if (!row_ok || c < c0 / 8 || c >= (c0 + kCols) / 8)
@@ -346,18 +378,19 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
     for (int k = 0; k < ntiles; ++k) {
-      const int buf = k & 1;
+      const int j = k / kTPS, half = k % kTPS;  // score product and its 64-token half
+      const int buf = k % kPBufs;               // P buffer
       const int st = k % kTcStages;
       const int tile_t0 = t_begin + k * kTileTok;
       const int valid = t_end - tile_t0;
-      if (!warp_wait(&s_full[buf], (k >> 1) & 1)) {
+      if (half == 0 && !warp_wait(&s_full[j & 1], (j >> 1) & 1)) {
         ok = false;
         break;
       }
       tc_fence_after();
       float s[kCols];
       if (warp_rows) {
-        const uint32_t ts = tS(mt, buf) + lane_off + static_cast<uint32_t>(c0);
+        const uint32_t ts = tS(mt, j & 1) + lane_off + static_cast<uint32_t>(half * kTileTok + c0);
         if constexpr (kCols == 64) {
           tmem_ld64(ts, s);
         } else if constexpr (kCols == 32) {
@@ -368,7 +401,7 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&s_free[buf]);
+      if (lane == 0 && (half == kTPS - 1 || k == ntiles - 1)) mbar_arrive(&s_free[j & 1]);
 
       float alpha = 1.f;
       bool rescale = false;
@@ -392,7 +425,7 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
       }
       if (__any_sync(0xffffffffu, rescale)) {
         // O holds P_0..P_{k-1} V: wait for the last PV, then scale this warp's rows.
-        if (!warp_wait(&o_done[(k - 1) & 1], ((k - 1) >> 1) & 1)) {
+        if (!warp_wait(&o_done[(k - 1) % kPBufs], ((k - 1) / kPBufs) & 1)) {
           ok = false;
           break;
         }
@@ -406,8 +439,8 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
           tmem_st32(tO(mt) + lane_off + c * 32, o);
         }
       }
-      // P buffer `buf` is free once the PV of tile k-2 has completed.
-      if (k >= 2 && !warp_wait(&o_done[buf], ((k - 2) >> 1) & 1)) {
+      // P buffer `buf` is free once the PV of tile k-kPBufs has completed.
+      if (k >= kPBufs && !warp_wait(&o_done[buf], ((k / kPBufs) - 1) & 1)) {
         ok = false;
         break;
       }
@@ -437,7 +470,7 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
           break;
         }
         const int r0 = valid, r1 = (valid + kGroupTok - 1) & ~(kGroupTok - 1);
-        uint8_t* vt = smem + st * Geo::kStageBytes + Geo::kTileBytes;
+        uint8_t* vt = smem + Lay::kVOff + st * Geo::kTileBytes;
         for (int idx = sm_tid; idx < (r1 - r0) * (D / 8); idx += 128 * MT) {
           const int row = r0 + idx / (D / 8), c = idx % (D / 8);
           *reinterpret_cast<uint4*>(vt + kv_swz(row, c)) = make_uint4(0, 0, 0, 0);
@@ -455,7 +488,7 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
     // Warp-uniform, like every condition around the warp-collective TMEM
     // loads and stores below.
     const bool o_ready =
-        __all_sync(0xffffffffu, ok && mbar_wait(&o_done[(ntiles - 1) & 1], ((ntiles - 1) >> 1) & 1, a.err));
+        __all_sync(0xffffffffu, ok && mbar_wait(&o_done[(ntiles - 1) % kPBufs], ((ntiles - 1) / kPBufs) & 1, a.err));
     // Weights of the token slices of each row, by the split-combine rule
     // (Sec. 3 Mode 2, here on one SM): slices cp > 0 leave their max, sum and
     // unscaled O row in the freed ring (rows 32*kRowQuads.. of it); slice 0
@@ -704,34 +737,37 @@ __global__ void __launch_bounds__(TcCfg<MT>::kThreads, 1)
   __syncthreads();
   if (warp == kMmaWarp) {
     tc_fence_after();
-    tmem_dealloc(tmem, TcCfg<MT>::kTmemCols);
+    tmem_dealloc(tmem, Cfg::kTmemCols);
   }
 }
 
-template <int D, int MT, int REP>
+template <int D, int MT, int REP, int TPS>
 cudaError_t configure_tc(int dev) {
   static int configured[64] = {0};
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   if (!__atomic_load_n(&configured[dev], __ATOMIC_ACQUIRE)) {
-    cudaError_t e = cudaFuncSetAttribute(block_attn_tc_kernel<D, MT, REP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(TcLayout<D, MT>::kBytes + 1024));
+    cudaError_t e = cudaFuncSetAttribute(block_attn_tc_kernel<D, MT, REP, TPS>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(TcLayout<D, MT, TPS>::kBytes + 1024));
     if (e != cudaSuccess) return e;
     __atomic_store_n(&configured[dev], 1, __ATOMIC_RELEASE);
   }
   return cudaSuccess;
 }
 
-template <int D, int MT, int REP>
+template <int D, int MT, int REP, int TPS>
 cudaError_t launch_tc_t(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, cudaStream_t stream) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  if ((e = configure_tc<D, MT, REP>(dev)) != cudaSuccess) return e;
+  if ((e = configure_tc<D, MT, REP, TPS>(dev)) != cudaSuccess) return e;
   dim3 grid(a.num_splits, a.Hkv, a.B);
-  return launch_kernel_cluster(block_attn_tc_kernel<D, MT, REP>, grid, dim3(TcCfg<MT>::kThreads),
-                               TcLayout<D, MT>::kBytes + 1024, stream, a.csize, tmk, tmv, a);
+  return launch_kernel_cluster(block_attn_tc_kernel<D, MT, REP, TPS>, grid, dim3(TcCfg<MT, TPS>::kThreads),
+                               TcLayout<D, MT, TPS>::kBytes + 1024, stream, a.csize, tmk, tmv, a);
 }
 
+// With one CTA per SM either way, cluster residency is the same for both
+// score-product widths; the query uses TPS = 1.
 template <int D, int MT, int REP>
 int max_active_clusters_t(int csize) {
   static int cache[64][4];  // [device][cluster size 2/4/8] + 1 (0 = not queried)
@@ -740,11 +776,11 @@ int max_active_clusters_t(int csize) {
   const int slot = csize == 2 ? 0 : csize == 4 ? 1 : csize == 8 ? 2 : 3;
   int v = __atomic_load_n(&cache[dev][slot], __ATOMIC_ACQUIRE);
   if (v) return v - 1;
-  if (configure_tc<D, MT, REP>(dev) != cudaSuccess) return 0;
+  if (configure_tc<D, MT, REP, 1>(dev) != cudaSuccess) return 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(csize, 1, 1);
-  cfg.blockDim = dim3(TcCfg<MT>::kThreads);
-  cfg.dynamicSmemBytes = TcLayout<D, MT>::kBytes + 1024;
+  cfg.blockDim = dim3(TcCfg<MT, 1>::kThreads);
+  cfg.dynamicSmemBytes = TcLayout<D, MT, 1>::kBytes + 1024;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = csize;
@@ -753,7 +789,7 @@ int max_active_clusters_t(int csize) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, block_attn_tc_kernel<D, MT, REP>, &cfg) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveClusters(&n, block_attn_tc_kernel<D, MT, REP, 1>, &cfg) != cudaSuccess) {
     cudaGetLastError();
     n = 0;
   }
@@ -775,14 +811,22 @@ int max_active_clusters_d(int csize, int rows) {
   }
 }
 
+template <int D, int TPS>
+cudaError_t launch_tc_rep(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, cudaStream_t stream) {
+  switch (tc_replication(a.R)) {
+    case 4: return launch_tc_t<D, 1, 4, TPS>(a, tmk, tmv, stream);
+    case 2: return launch_tc_t<D, 1, 2, TPS>(a, tmk, tmv, stream);
+    default: return launch_tc_t<D, 1, 1, TPS>(a, tmk, tmv, stream);
+  }
+}
+
+// Paired score products when a split fits in the ring whole (it is then
+// latency-bound: fewer, wider steps help); single tiles when it streams.
 template <int D>
 cudaError_t launch_tc_d(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, cudaStream_t stream) {
-  if (a.R > 128) return launch_tc_t<D, 2, 1>(a, tmk, tmv, stream);
-  switch (tc_replication(a.R)) {
-    case 4: return launch_tc_t<D, 1, 4>(a, tmk, tmv, stream);
-    case 2: return launch_tc_t<D, 1, 2>(a, tmk, tmv, stream);
-    default: return launch_tc_t<D, 1, 1>(a, tmk, tmv, stream);
-  }
+  if (a.R > 128) return launch_tc_t<D, 2, 1, 1>(a, tmk, tmv, stream);
+  if (a.chunk <= TcCfg<1, 2>::kStages * kTileTok) return launch_tc_rep<D, 2>(a, tmk, tmv, stream);
+  return launch_tc_rep<D, 1>(a, tmk, tmv, stream);
 }
 
 }  // namespace

@@ -416,7 +416,9 @@ struct PagePrefetch {
 
 // Producer warp `pw` of `nprod`: streams its share of the TMA boxes of the
 // K/V tiles of tokens [t_begin, t_end) of (sequence b, KV head g) into an
-// nstage ring. A tile has 4 groups x D/64 column blocks x {K, V} boxes
+// nstage ring: K tiles at [column block][stage], so that the K of
+// consecutive stages is contiguous per column block, then V tiles at
+// [stage][column block]. A tile has 4 groups x D/64 column blocks x {K, V} boxes
 // (16 tokens x 64 dims each); they are dealt to the producer warps in equal
 // shares and, within a warp, one box per lane. TMA issue cost is per warp, so
 // more producer warps land a tile sooner. A warp's expect_tx covers only its
@@ -465,7 +467,8 @@ __device__ __forceinline__ int produce_kv(const AttnArgs& a, const CUtensorMap* 
     if (lane < my_ops) {
       const int t = t_begin + k * kTileTok + grp * kGroupTok;
       const int slot = page < a.num_pages ? (t & (a.page_size - 1)) : 0;
-      uint8_t* dst = stages + st * Geo::kStageBytes + (is_v ? Geo::kTileBytes : 0) + cb * Geo::kColBlockBytes +
+      uint8_t* dst = (is_v ? stages + (nstage + st) * Geo::kTileBytes + cb * Geo::kColBlockBytes
+                           : stages + (cb * nstage + st) * Geo::kColBlockBytes) +
                      grp * kGroupTok * 128;
       tma_load_4d(dst, is_v ? tmv : tmk, &full[st], cb * 64, slot, g, page);
     }

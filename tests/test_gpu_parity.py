@@ -174,6 +174,9 @@ SMALL = [
     ("prefix0_bl32", 2, 8, 2, 128, 16, 32, [0, 0]),
     ("d128_g8_bl32_256rows", 2, 16, 2, 128, 16, 32, [700, 33]),
     ("d64_g6_bl30_180rows", 1, 6, 1, 64, 32, 30, [150]),
+    # 96 packed rows: one M tile without row copies, several tiles per split
+    ("d128_g3_bl32_96rows", 2, 6, 2, 128, 16, 32, [450, 190]),
+    ("d64_g4_bl24_96rows", 1, 8, 2, 64, 32, 24, [230]),
 ]
 
 
