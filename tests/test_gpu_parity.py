@@ -177,6 +177,10 @@ SMALL = [
     # 96 packed rows: one M tile without row copies, several tiles per split
     ("d128_g3_bl32_96rows", 2, 6, 2, 128, 16, 32, [450, 190]),
     ("d64_g4_bl24_96rows", 1, 8, 2, 64, 32, 24, [230]),
+    # two M tiles: the rows past 128 copied 2 or 4 times, or not at all
+    ("d128_g6_bl30_180rows", 1, 6, 1, 128, 32, 30, [260]),
+    ("d64_g5_bl32_160rows", 2, 10, 2, 64, 16, 32, [300, 45]),
+    ("d64_g8_bl32_256rows", 1, 16, 2, 64, 16, 32, [100]),
 ]
 
 
@@ -208,6 +212,32 @@ def test_prefix_ready_flag_same_result(orc, spec):
             assert torch.equal(o0, o1) and torch.equal(l0, l1)
             ro, rl = oracle_full(orc, case, mode)
             compare_attn(o1, l1, ro, rl, f"{name} flag mode={mode} S={splits}")
+
+
+@pytest.mark.parametrize("spec", [SMALL[1], SMALL[3], SMALL[10]], ids=[SMALL[1][0], SMALL[3][0], SMALL[10][0]])
+@pytest.mark.parametrize("splits", [3, 19])
+def test_partials_entry_point_then_combine(orc, spec, splits):
+    """nld_block_attn_partials + nld_split_kv_combine run the same kernels as
+    nld_block_attn: bit-identical result, within tolerance of the oracle."""
+    name, B, Hq, Hkv, D, P, bl, prefix = spec
+    case = W.make_block_attn_case(name, B, Hq, Hkv, D, block_len=bl, page_size=P, prefix_lens=prefix,
+                                  seed=sum(prefix) + 5 * bl)
+    dc = DeviceCase(case)
+    p = dc.params(splits)
+    if nld.nld_block_attn_num_splits(p, bl) < 2:
+        pytest.skip("plan merges on chip: no partials")
+    for mode in (DIFF, VER):
+        ref_out, ref_lse = dc.run(mode, splits)
+        ws = torch.empty(nld.nld_block_attn_workspace_size(p, bl), dtype=torch.uint8, device="cuda")
+        out = torch.full_like(ref_out, float("nan"))
+        lse = torch.full_like(ref_lse, float("nan"))
+        nld.nld_block_attn_partials(p, dc.q[mode], dc.k, dc.v, dc.table, dc.prefix, bl, mode, out, lse, ws)
+        assert torch.isnan(out).all(), "the partials call leaves out untouched"
+        o_part, lse_part = nld.workspace_views(p, bl, ws)
+        nld.nld_split_kv_combine(o_part, lse_part, out, lse)
+        assert torch.equal(out, ref_out) and torch.equal(lse, ref_lse)
+        ro, rl = oracle_full(orc, case, mode)
+        compare_attn(out, lse, ro, rl, f"{name} partials mode={mode} S={splits}")
 
 
 def test_attention_tail_slots_hold_nan(orc):
