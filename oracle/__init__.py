@@ -1,4 +1,5 @@
-"""fp64 CPU oracle for paged block attention, split combine, accept and unmask.
+"""fp64 CPU oracle for paged block attention, split combine, accept, top-k,
+threshold and greedy unmasking.
 
 TEST INFRASTRUCTURE ONLY: the tests, ``__graft_entry__.smoke()`` and the CPU
 baseline of ``bench.py`` use it. The product path never imports it. It shares
@@ -67,6 +68,10 @@ class Oracle:
         lib.nldo_accept.restype = None
         lib.nldo_unmask.argtypes = [P, I, I, I, P, P]
         lib.nldo_unmask.restype = None
+        lib.nldo_unmask_threshold.argtypes = [P, I, I, ctypes.c_float, P, P]
+        lib.nldo_unmask_threshold.restype = None
+        lib.nldo_greedy_accept.argtypes = [P, P, P, I, I, P, P]
+        lib.nldo_greedy_accept.restype = None
         lib.nldo_max_threads.argtypes = []
         lib.nldo_max_threads.restype = I
         self.lib = lib
@@ -150,6 +155,28 @@ class Oracle:
         pos = np.zeros((B, k), dtype=np.int32)
         nsel = np.zeros((B,), dtype=np.int32)
         self.lib.nldo_unmask(self._p(c), B, n, int(k), self._p(pos), self._p(nsel))
+        return pos, nsel
+
+    def unmask_threshold(self, conf, threshold):
+        """(positions [B, n] ascending then -1, num_selected [B]) of one
+        threshold-unmasking step with the top-1 fallback."""
+        c = np.ascontiguousarray(conf, dtype=np.float32)
+        B, n = c.shape
+        pos = np.zeros((B, n), dtype=np.int32)
+        nsel = np.zeros((B,), dtype=np.int32)
+        self.lib.nldo_unmask_threshold(self._p(c), B, n, float(np.float32(threshold)), self._p(pos), self._p(nsel))
+        return pos, nsel
+
+    def greedy_accept(self, pred, target, conf):
+        """(positions [B, n] ascending then -1, num_selected [B]) of one greedy
+        parallel acceptance iteration."""
+        p = np.ascontiguousarray(pred, dtype=np.int32)
+        t = np.ascontiguousarray(target, dtype=np.int32)
+        c = np.ascontiguousarray(conf, dtype=np.float32)
+        B, n = c.shape
+        pos = np.zeros((B, n), dtype=np.int32)
+        nsel = np.zeros((B,), dtype=np.int32)
+        self.lib.nldo_greedy_accept(self._p(p), self._p(t), self._p(c), B, n, self._p(pos), self._p(nsel))
         return pos, nsel
 
 

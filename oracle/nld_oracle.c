@@ -28,6 +28,10 @@
  *    commits the highest-confidence position): the k eligible positions with
  *    the largest confidence, ordered by (confidence descending, position
  *    ascending). -inf and NaN mark ineligible positions.
+ *  - Threshold unmasking with a top-1 fallback (Sec. 2, confidence-based
+ *    sampling) and greedy parallel acceptance against a serial target
+ *    (Sec. 5, diffusion SOL construction): the positions one denoising step
+ *    commits, in ascending order.
  *
  * Build: gcc -O2 -fopenmp -ffp-contract=off -shared -fPIC (see build.py).
  */
@@ -308,4 +312,75 @@ void nldo_unmask(const float *conf, int B, int n, int k, int32_t *positions, int
         if (num_selected) num_selected[b] = sel;
     }
     free(idx);
+}
+
+static int eligible(float c)
+{
+    return !isnan(c) && !(isinf(c) && c < 0);
+}
+
+/* Position of the highest eligible confidence (lower index on ties), or -1. */
+static int top1(const float *c, int n)
+{
+    int best = -1;
+    for (int i = 0; i < n; ++i)
+        if (eligible(c[i]) && (best < 0 || ranks_before(c[i], i, c[best], best))) best = i;
+    return best;
+}
+
+/*
+ * Threshold unmasking (Sec. 2, confidence-based sampling: one denoising step
+ * commits every masked position whose confidence exceeds the threshold),
+ * with a top-1 fallback so that every step commits at least one position
+ * while any is masked (the single highest-confidence position, as in the
+ * fallback of Sec. 5 greedy acceptance). "Exceeds" is read as strictly
+ * greater, compared in fp32. positions [B, n]: the committed positions in
+ * ascending order, then -1; num_selected [B] (nullable). Eligible (still
+ * masked): not NaN and not -inf.
+ */
+void nldo_unmask_threshold(const float *conf, int B, int n, float threshold, int32_t *positions,
+                           int32_t *num_selected)
+{
+    for (int b = 0; b < B; ++b) {
+        const float *c = conf + (long)b * n;
+        int32_t *pos = positions + (long)b * n;
+        int count = 0;
+        for (int i = 0; i < n; ++i)
+            if (eligible(c[i]) && c[i] > threshold) pos[count++] = i;
+        if (count == 0) {
+            const int best = top1(c, n);
+            if (best >= 0) pos[count++] = best;
+        }
+        for (int r = count; r < n; ++r) pos[r] = -1;
+        if (num_selected) num_selected[b] = count;
+    }
+}
+
+/*
+ * Greedy parallel acceptance (Sec. 5, diffusion SOL construction): one
+ * iteration commits every masked position j whose argmax prediction equals
+ * the serial target, {j : x_j = [M] and pred_j = target_j}; if there is none,
+ * it commits the single highest-confidence masked position. pred, target
+ * [B, n] int32; conf [B, n] fp32 marks the masked positions (eligible as
+ * above) and ranks them for the fallback. Output as for
+ * nldo_unmask_threshold.
+ */
+void nldo_greedy_accept(const int32_t *pred, const int32_t *target, const float *conf, int B, int n,
+                        int32_t *positions, int32_t *num_selected)
+{
+    for (int b = 0; b < B; ++b) {
+        const float *c = conf + (long)b * n;
+        const int32_t *p = pred + (long)b * n;
+        const int32_t *t = target + (long)b * n;
+        int32_t *pos = positions + (long)b * n;
+        int count = 0;
+        for (int j = 0; j < n; ++j)
+            if (eligible(c[j]) && p[j] == t[j]) pos[count++] = j;
+        if (count == 0) {
+            const int fallback = top1(c, n);
+            if (fallback >= 0) pos[count++] = fallback;
+        }
+        for (int r = count; r < n; ++r) pos[r] = -1;
+        if (num_selected) num_selected[b] = count;
+    }
 }

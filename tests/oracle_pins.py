@@ -411,9 +411,138 @@ def pin_unmask_lexsort(orc):
     assert all(sorted(row) == list(range(32)) for row in p.tolist()), "k = n is a permutation"
 
 
+def _nums(text, dtype):
+    return np.array([[float(x) for x in text.split()]], dtype=dtype)
+
+
+def pin_threshold_golden(orc):
+    for c, thr, pos, nsel in read_golden("unmask_threshold_cases.txt"):
+        p, s = orc.unmask_threshold(_nums(c, np.float32), np.float32(float(thr)))
+        assert p[0].tolist() == [int(x) for x in pos.split()], f"threshold {c} | {thr}: {p[0]}"
+        assert int(s[0]) == int(nsel)
+
+
+def brute_threshold(conf, thr):
+    B, n = conf.shape
+    pos = np.full((B, n), -1, dtype=np.int32)
+    nsel = np.zeros(B, dtype=np.int32)
+    for b in range(B):
+        c = [float(x) for x in conf[b]]
+        elig = [i for i in range(n) if not (math.isnan(c[i]) or c[i] == -math.inf)]
+        chosen = [i for i in elig if c[i] > float(thr)]
+        if not chosen and elig:
+            chosen = [sorted(elig, key=lambda i: (-c[i], i))[0]]
+        pos[b, :len(chosen)] = chosen
+        nsel[b] = len(chosen)
+    return pos, nsel
+
+
+def _tied_confidences(rng, B, n):
+    conf = rng.integers(0, 5, size=(B, n)).astype(np.float32) / 4
+    conf[rng.random((B, n)) < 0.2] = -np.inf
+    conf[rng.random((B, n)) < 0.05] = np.nan
+    return conf
+
+
+def pin_threshold_brute(orc):
+    rng = np.random.default_rng(21)
+    for n in (1, 2, 8, 16, 32):
+        conf = _tied_confidences(rng, 60, n)
+        for thr in (-1.0, 0.0, 0.25, 0.5, 0.75, 1.0, 2.0):
+            p, s = orc.unmask_threshold(conf, thr)
+            bp, bs = brute_threshold(conf, thr)
+            assert np.array_equal(p, bp) and np.array_equal(s, bs), f"n={n} thr={thr}"
+
+
+def pin_threshold_limits(orc):
+    """A threshold of -inf commits every masked position (numpy's flatnonzero);
+    +inf always falls back to the single top-1 position of the pinned top-k rule."""
+    rng = np.random.default_rng(22)
+    conf = _tied_confidences(rng, 100, 32)
+    p, s = orc.unmask_threshold(conf, -np.inf)
+    for b in range(conf.shape[0]):
+        idx = np.flatnonzero(~np.isnan(conf[b]) & (conf[b] != -np.inf))
+        assert p[b][:s[b]].tolist() == idx.tolist() and np.all(p[b][s[b]:] == -1)
+    p, s = orc.unmask_threshold(conf, np.inf)
+    top, ts = orc.unmask(conf, 1)
+    assert np.array_equal(s, ts) and np.array_equal(p[:, 0], top[:, 0])
+    assert np.all(p[:, 1:] == -1)
+
+
+def pin_greedy_golden(orc):
+    for pr, tg, c, pos, nsel in read_golden("greedy_accept_cases.txt"):
+        p, s = orc.greedy_accept(_nums(pr, np.int32), _nums(tg, np.int32), _nums(c, np.float32))
+        assert p[0].tolist() == [int(x) for x in pos.split()], f"greedy {pr} | {tg} | {c}: {p[0]}"
+        assert int(s[0]) == int(nsel)
+
+
+def brute_greedy(pred, target, conf):
+    B, n = conf.shape
+    pos = np.full((B, n), -1, dtype=np.int32)
+    nsel = np.zeros(B, dtype=np.int32)
+    for b in range(B):
+        c = [float(x) for x in conf[b]]
+        masked = [j for j in range(n) if not (math.isnan(c[j]) or c[j] == -math.inf)]
+        chosen = [j for j in masked if int(pred[b, j]) == int(target[b, j])]
+        if not chosen and masked:
+            chosen = [max(masked, key=lambda j: (c[j], -j))]
+        pos[b, :len(chosen)] = chosen
+        nsel[b] = len(chosen)
+    return pos, nsel
+
+
+def pin_greedy_brute(orc):
+    rng = np.random.default_rng(23)
+    for n in (1, 2, 8, 16, 32):
+        conf = _tied_confidences(rng, 60, n)
+        for p_match in (0.0, 0.1, 0.5, 1.0):
+            target = rng.integers(0, 100, size=(60, n)).astype(np.int32)
+            pred = np.where(rng.random((60, n)) < p_match, target, target + 1).astype(np.int32)
+            p, s = orc.greedy_accept(pred, target, conf)
+            bp, bs = brute_greedy(pred, target, conf)
+            assert np.array_equal(p, bp) and np.array_equal(s, bs), f"n={n} p={p_match}"
+
+
+def pin_greedy_chain(orc):
+    """Iterating greedy acceptance unmasks a block in K <= n iterations, at least
+    one position each (TPF = n / K, Sec. 5). When no prediction ever matches,
+    every iteration commits one position and the order is the serial
+    denoising order: the pinned top-k ranking of the confidences. When every
+    prediction matches, one iteration commits the whole block."""
+    rng = np.random.default_rng(24)
+    B, n = 40, 32
+    base = rng.random((B, n), dtype=np.float32)
+    target = rng.integers(0, 1000, size=(B, n)).astype(np.int32)
+    order, _ = orc.unmask(base, n)
+    never = target + 1
+    conf = base.copy()
+    seq = []
+    for _ in range(n):
+        p, s = orc.greedy_accept(never, target, conf)
+        assert np.all(s == 1)
+        seq.append(p[:, 0].copy())
+        conf[np.arange(B), p[:, 0]] = -np.inf
+    assert np.array_equal(np.stack(seq, axis=1), order)
+    p, s = orc.greedy_accept(target, target, base)
+    assert np.all(s == n) and np.all(p == np.arange(n))
+    for p_match in (0.3, 0.7):
+        conf = base.copy()
+        iters = np.zeros(B, dtype=np.int64)
+        for _ in range(n):
+            pred = np.where(rng.random((B, n)) < p_match, target, target + 1).astype(np.int32)
+            p, s = orc.greedy_accept(pred, target, conf)
+            live = ~np.all(conf == -np.inf, axis=1)
+            assert np.all(s[live] >= 1) and np.all(s[~live] == 0)
+            iters += live
+            for b in range(B):
+                conf[b, p[b, :s[b]]] = -np.inf
+        assert np.all(conf == -np.inf) and np.all((iters >= 1) & (iters <= n))
+
+
 ATTENTION_PINS = [pin_decode_bl1, pin_diffusion_full_attention, pin_verify_causal_tail, pin_lse_logsumexp,
                   pin_softmax_rows, pin_page_permutation, pin_block_permutation, pin_closed_forms,
                   pin_golden_uniform, pin_split_combine]
 DECISION_PINS = [pin_accept_golden, pin_accept_brute, pin_accept_statistics, pin_unmask_golden,
-                 pin_unmask_brute, pin_unmask_lexsort]
+                 pin_unmask_brute, pin_unmask_lexsort, pin_threshold_golden, pin_threshold_brute,
+                 pin_threshold_limits, pin_greedy_golden, pin_greedy_brute, pin_greedy_chain]
 ALL_PINS = ATTENTION_PINS + DECISION_PINS

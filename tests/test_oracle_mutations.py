@@ -45,6 +45,25 @@ MUTANTS = {
     # unmask: -inf treated as eligible
     "unmask_neginf_eligible": ("if (!isnan(c[i]) && !(isinf(c[i]) && c[i] < 0)) idx[m++] = i;",
                                "if (!isnan(c[i])) idx[m++] = i;"),
+    # threshold: "exceeds" taken as >=
+    "threshold_ge": ("if (eligible(c[i]) && c[i] > threshold) pos[count++] = i;",
+                     "if (eligible(c[i]) && c[i] >= threshold) pos[count++] = i;"),
+    # threshold: no top-1 fallback
+    "threshold_no_fallback": ("            if (best >= 0) pos[count++] = best;\n", ""),
+    # fallback picks the lowest confidence
+    "top1_lowest": ("if (eligible(c[i]) && (best < 0 || ranks_before(c[i], i, c[best], best))) best = i;",
+                    "if (eligible(c[i]) && (best < 0 || ranks_before(c[best], best, c[i], i))) best = i;"),
+    # fallback breaks ties towards the higher position
+    "top1_tie_high": ("if (eligible(c[i]) && (best < 0 || ranks_before(c[i], i, c[best], best))) best = i;",
+                      "if (eligible(c[i]) && (best < 0 || c[i] >= c[best])) best = i;"),
+    # greedy commits matches at positions already unmasked
+    "greedy_ignores_mask": ("if (eligible(c[j]) && p[j] == t[j]) pos[count++] = j;",
+                            "if (p[j] == t[j]) pos[count++] = j;"),
+    # greedy commits the mismatches
+    "greedy_mismatch": ("if (eligible(c[j]) && p[j] == t[j]) pos[count++] = j;",
+                        "if (eligible(c[j]) && p[j] != t[j]) pos[count++] = j;"),
+    # nan confidence taken as still masked
+    "eligible_nan": ("return !isnan(c) && !(isinf(c) && c < 0);", "return !(isinf(c) && c < 0);"),
     # unmask: ascending order
     "unmask_ascending": ("if (ca > cb) return 1;\n    if (ca < cb) return 0;",
                          "if (ca < cb) return 1;\n    if (ca > cb) return 0;"),
