@@ -422,6 +422,7 @@ def run_ours(args, world, rank, local):
     }
     if not args.headline_only:
         line["workloads"] = run_workloads(torch, nld, dev, stream, peak, l2)
+        line["decisions"] = run_decisions(torch, nld, dev, stream)
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, budget_s=12.0)
     print(json.dumps(line), flush=True)
@@ -516,6 +517,34 @@ def time_graph(torch, stream, body, nsteps, reps):
         e1.record(stream)
     torch.cuda.synchronize()
     return e0.elapsed_time(e1) / (reps * nsteps)
+
+
+def run_decisions(torch, nld, dev, stream):
+    """Each token-decision kernel alone (latency-bound: a few hundred bytes per
+    sequence), as a CUDA graph of back-to-back calls: us per call at B = 1 and
+    B = 128 sequences of n = 32 positions."""
+    res = {}
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(7)
+    for B in (1, 128):
+        n = 32
+        conf = torch.rand((B, n), generator=gen, device=dev)
+        ids_a = torch.randint(0, 131072, (B, n), generator=gen, device=dev, dtype=torch.int32)
+        ids_b = torch.where(torch.rand((B, n), generator=gen, device=dev) < 0.7, ids_a, ids_a + 1)
+        pos_k = torch.empty((B, 8), dtype=torch.int32, device=dev)
+        pos_n = torch.empty((B, n), dtype=torch.int32, device=dev)
+        nsel = torch.empty((B,), dtype=torch.int32, device=dev)
+        acc = torch.empty((B,), dtype=torch.int32, device=dev)
+        calls = {
+            "accept": lambda i: nld.nld_accept(ids_a, ids_b, acc),
+            "unmask_top8": lambda i: nld.nld_unmask(conf, 8, pos_k, nsel),
+            "unmask_threshold_0.9": lambda i: nld.nld_unmask_threshold(conf, 0.9, pos_n, nsel),
+            "greedy_accept": lambda i: nld.nld_greedy_accept(ids_a, ids_b, conf, pos_n, nsel),
+        }
+        res[f"b{B}_n{n}_us_per_call"] = {k: round(time_graph(torch, stream, f, 256, 10) * 1e3, 3)
+                                          for k, f in calls.items()}
+    res["timing"] = "CUDA graph of 256 back-to-back calls (PDL), events around 10 replays"
+    return res
 
 
 def run_workloads(torch, nld, dev, stream, peak, l2, only=None, batch=None):

@@ -236,6 +236,40 @@ nld_status_t nld_accept(const int32_t *draft_ids, const int32_t *verify_ids, int
 nld_status_t nld_unmask(const float *confidences, int batch, int n, int k, int32_t *positions,
                         int32_t *num_selected, cudaStream_t stream);
 
+/*
+ * Threshold unmasking with a top-1 fallback (Sec. 2, confidence-based
+ * sampling: a denoising step commits every masked position whose
+ * confidence exceeds the threshold). Commits every eligible position whose
+ * confidence is strictly greater than `threshold` (fp32 comparison); if none
+ * is, commits the single highest-confidence eligible position (the lower
+ * position on ties; +0 and -0 tie), so that a step commits at least one
+ * position while any remains masked. -inf and NaN mark positions already
+ * committed (not eligible).
+ *
+ *   confidences  fp32 [B, n], 1 <= n <= 32
+ *   positions    int32 [B, n]: the committed positions in ascending order,
+ *                then -1
+ *   num_selected int32 [B] (may be NULL): committed count (0 only when no
+ *                position is eligible)
+ */
+nld_status_t nld_unmask_threshold(const float *confidences, int batch, int n, float threshold,
+                                  int32_t *positions, int32_t *num_selected, cudaStream_t stream);
+
+/*
+ * Greedy parallel acceptance against a serial target (Sec. 5, diffusion SOL
+ * construction): one iteration commits every masked position j whose argmax
+ * prediction equals the target, pred_ids[b][j] == target_ids[b][j]; if none
+ * does, the single highest-confidence masked position (lower position on
+ * ties). A position is masked when its confidence is neither -inf nor NaN;
+ * the confidences also rank the fallback.
+ *
+ *   pred_ids, target_ids int32 [B, n]; confidences fp32 [B, n], 1 <= n <= 32
+ *   positions, num_selected as for nld_unmask_threshold
+ */
+nld_status_t nld_greedy_accept(const int32_t *pred_ids, const int32_t *target_ids,
+                               const float *confidences, int batch, int n, int32_t *positions,
+                               int32_t *num_selected, cudaStream_t stream);
+
 /* A static, human-readable name for a status code. */
 const char *nld_status_string(nld_status_t status);
 

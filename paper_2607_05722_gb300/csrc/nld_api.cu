@@ -345,6 +345,29 @@ nld_status_t nld_unmask(const float* confidences, int batch, int n, int k, int32
              : NLD_ERR_CUDA;
 }
 
+nld_status_t nld_unmask_threshold(const float* confidences, int batch, int n, float threshold, int32_t* positions,
+                                  int32_t* num_selected, cudaStream_t stream) {
+  if (batch < 1 || n < 1 || n > nld::kMaxBlock) return NLD_ERR_INVALID_ARG;
+  if (!aligned(confidences, 4) || !aligned(positions, 4)) return NLD_ERR_INVALID_ARG;
+  if (num_selected != nullptr && !aligned(num_selected, 4)) return NLD_ERR_INVALID_ARG;
+  return nld::launch_unmask_threshold(confidences, batch, n, threshold, positions, num_selected, stream) ==
+                 cudaSuccess
+             ? NLD_OK
+             : NLD_ERR_CUDA;
+}
+
+nld_status_t nld_greedy_accept(const int32_t* pred_ids, const int32_t* target_ids, const float* confidences,
+                               int batch, int n, int32_t* positions, int32_t* num_selected, cudaStream_t stream) {
+  if (batch < 1 || n < 1 || n > nld::kMaxBlock) return NLD_ERR_INVALID_ARG;
+  if (!aligned(pred_ids, 4) || !aligned(target_ids, 4) || !aligned(confidences, 4) || !aligned(positions, 4))
+    return NLD_ERR_INVALID_ARG;
+  if (num_selected != nullptr && !aligned(num_selected, 4)) return NLD_ERR_INVALID_ARG;
+  return nld::launch_greedy_accept(pred_ids, target_ids, confidences, batch, n, positions, num_selected, stream) ==
+                 cudaSuccess
+             ? NLD_OK
+             : NLD_ERR_CUDA;
+}
+
 nld_status_t nld_device_error(uint32_t* bits, int clear) {
   if (bits == nullptr) return NLD_ERR_INVALID_ARG;
   unsigned int* err = nullptr;

@@ -52,6 +52,10 @@ cudaError_t launch_accept(const int32_t* draft, const int32_t* verify, int B, in
                           cudaStream_t stream);
 cudaError_t launch_unmask(const float* conf, int B, int n, int k, int32_t* pos, int32_t* nsel,
                           cudaStream_t stream);
+cudaError_t launch_unmask_threshold(const float* conf, int B, int n, float threshold, int32_t* pos, int32_t* nsel,
+                                    cudaStream_t stream);
+cudaError_t launch_greedy_accept(const int32_t* pred, const int32_t* target, const float* conf, int B, int n,
+                                 int32_t* pos, int32_t* nsel, cudaStream_t stream);
 
 // Launch with programmatic stream serialization: the kernel may start while
 // its predecessor in the stream is still running. Every kernel of this

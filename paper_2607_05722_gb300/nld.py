@@ -70,6 +70,10 @@ def lib(path: Optional[str] = None):
     L.nld_accept.argtypes = [V, V, I, I, V, V]
     L.nld_accept.restype = I
     L.nld_unmask.argtypes = [V, I, I, I, V, V, V]
+    L.nld_unmask_threshold.argtypes = [V, I, I, ctypes.c_float, V, V, V]
+    L.nld_unmask_threshold.restype = I
+    L.nld_greedy_accept.argtypes = [V, V, V, I, I, V, V, V]
+    L.nld_greedy_accept.restype = I
     L.nld_unmask.restype = I
     L.nld_status_string.argtypes = [I]
     L.nld_status_string.restype = ctypes.c_char_p
@@ -238,6 +242,32 @@ def nld_unmask(confidences, k: int, positions, num_selected=None, stream=None):
     _check(lib().nld_unmask(_ptr(confidences), B, n, int(k), _ptr(positions), _ptr(num_selected),
                             _stream(stream)), "nld_unmask")
 
+
+
+def nld_unmask_threshold(confidences, threshold: float, positions, num_selected=None, stream=None):
+    """Commit every masked position with confidence > threshold, else the top-1
+    (positions ascending, then -1)."""
+    B, n = confidences.shape
+    _expect(confidences, torch.float32, (B, n), "confidences")
+    _expect(positions, torch.int32, (B, n), "positions")
+    if num_selected is not None:
+        _expect(num_selected, torch.int32, (B,), "num_selected")
+    _check(lib().nld_unmask_threshold(_ptr(confidences), B, n, float(threshold), _ptr(positions),
+                                      _ptr(num_selected), _stream(stream)), "nld_unmask_threshold")
+
+
+def nld_greedy_accept(pred_ids, target_ids, confidences, positions, num_selected=None, stream=None):
+    """Commit every masked position whose prediction equals the target, else the
+    top-1 (positions ascending, then -1)."""
+    B, n = confidences.shape
+    _expect(pred_ids, torch.int32, (B, n), "pred_ids")
+    _expect(target_ids, torch.int32, (B, n), "target_ids")
+    _expect(confidences, torch.float32, (B, n), "confidences")
+    _expect(positions, torch.int32, (B, n), "positions")
+    if num_selected is not None:
+        _expect(num_selected, torch.int32, (B,), "num_selected")
+    _check(lib().nld_greedy_accept(_ptr(pred_ids), _ptr(target_ids), _ptr(confidences), B, n, _ptr(positions),
+                                   _ptr(num_selected), _stream(stream)), "nld_greedy_accept")
 
 def nld_device_error(clear: bool = False) -> int:
     bits = ctypes.c_uint32(0)

@@ -103,6 +103,14 @@ def test_decisions_reject_bad_sizes(L):
     assert L.nld_unmask(FAKE, 1, 8, 9, FAKE, None, None) == 1
     assert L.nld_unmask(FAKE, 1, 8, 0, FAKE, None, None) == 1
     assert L.nld_unmask(FAKE, 1, 40, 4, FAKE, None, None) == 1
+    assert L.nld_unmask_threshold(FAKE, 1, 33, 0.5, FAKE, None, None) == 1
+    assert L.nld_unmask_threshold(FAKE, 0, 8, 0.5, FAKE, None, None) == 1
+    assert L.nld_unmask_threshold(FAKE, 1, 0, 0.5, FAKE, None, None) == 1
+    assert L.nld_unmask_threshold(None, 1, 8, 0.5, FAKE, None, None) == 1
+    assert L.nld_greedy_accept(FAKE, FAKE, FAKE, 1, 33, FAKE, None, None) == 1
+    assert L.nld_greedy_accept(FAKE, FAKE, FAKE, 0, 8, FAKE, None, None) == 1
+    assert L.nld_greedy_accept(FAKE, None, FAKE, 1, 8, FAKE, None, None) == 1
+    assert L.nld_greedy_accept(FAKE, FAKE, FAKE, 1, 8, FAKE, ctypes.c_void_p(0x10002), None) == 1
     assert L.nld_split_kv_combine(FAKE, FAKE, 0, 1, 4, 8, 128, FAKE, None, None) == 1
     assert L.nld_split_kv_combine(FAKE, FAKE, 2, 1, 4, 8, 80, FAKE, None, None) == 2
 

@@ -51,6 +51,95 @@ def gpu_unmask(conf, k):
     return pos.cpu().numpy(), nsel.cpu().numpy()
 
 
+def gpu_unmask_threshold(conf, thr):
+    ct = torch.from_numpy(np.ascontiguousarray(conf, dtype=np.float32)).cuda()
+    pos = torch.full(conf.shape, -7, dtype=torch.int32, device="cuda")
+    nsel = torch.full((conf.shape[0],), -7, dtype=torch.int32, device="cuda")
+    nld.nld_unmask_threshold(ct, float(np.float32(thr)), pos, nsel)
+    return pos.cpu().numpy(), nsel.cpu().numpy()
+
+
+def gpu_greedy(pred, target, conf):
+    pt = torch.from_numpy(np.ascontiguousarray(pred, dtype=np.int32)).cuda()
+    tt = torch.from_numpy(np.ascontiguousarray(target, dtype=np.int32)).cuda()
+    ct = torch.from_numpy(np.ascontiguousarray(conf, dtype=np.float32)).cuda()
+    pos = torch.full(conf.shape, -7, dtype=torch.int32, device="cuda")
+    nsel = torch.full((conf.shape[0],), -7, dtype=torch.int32, device="cuda")
+    nld.nld_greedy_accept(pt, tt, ct, pos, nsel)
+    return pos.cpu().numpy(), nsel.cpu().numpy()
+
+
+def tied_confidences(rng, B, n):
+    conf = rng.integers(0, 5, size=(B, n)).astype(np.float32) / 4
+    conf[rng.random((B, n)) < 0.2] = -np.inf
+    conf[rng.random((B, n)) < 0.05] = np.nan
+    z = rng.random((B, n)) < 0.05
+    conf[z] = np.where(rng.random(z.sum()) < 0.5, 0.0, -0.0)
+    return conf
+
+
+def test_unmask_threshold_golden_cases():
+    for c, thr, pos, nsel in oracle_pins.read_golden("unmask_threshold_cases.txt"):
+        conf = np.array([[float(x) for x in c.split()]], dtype=np.float32)
+        p, s = gpu_unmask_threshold(conf, float(thr))
+        assert p[0].tolist() == [int(x) for x in pos.split()] and int(s[0]) == int(nsel), f"{c} | {thr}"
+
+
+@pytest.mark.parametrize("n", [1, 5, 8, 16, 31, 32])
+def test_unmask_threshold_matches_oracle(orc, n):
+    rng = np.random.default_rng(300 + n)
+    conf = tied_confidences(rng, 257, n)
+    for thr in (-np.inf, -1.0, 0.0, 0.25, 0.5, 0.75, 1.0, np.inf, np.nan):
+        p, s = gpu_unmask_threshold(conf, thr)
+        po, so = orc.unmask_threshold(conf, thr)
+        assert np.array_equal(p, po) and np.array_equal(s, so), f"n={n} thr={thr}"
+    conf = rng.random((5000, n), dtype=np.float32)  # many CTAs, no ties
+    p, s = gpu_unmask_threshold(conf, 0.9)
+    po, so = orc.unmask_threshold(conf, 0.9)
+    assert np.array_equal(p, po) and np.array_equal(s, so)
+
+
+def test_greedy_accept_golden_cases():
+    for pr, tg, c, pos, nsel in oracle_pins.read_golden("greedy_accept_cases.txt"):
+        row = lambda t, dt: np.array([[float(x) for x in t.split()]], dtype=dt)
+        p, s = gpu_greedy(row(pr, np.int32), row(tg, np.int32), row(c, np.float32))
+        assert p[0].tolist() == [int(x) for x in pos.split()] and int(s[0]) == int(nsel), f"{pr} | {tg} | {c}"
+
+
+@pytest.mark.parametrize("n", [1, 7, 8, 16, 32])
+def test_greedy_accept_matches_oracle(orc, n):
+    rng = np.random.default_rng(400 + n)
+    for p_match in (0.0, 0.1, 0.5, 1.0):
+        conf = tied_confidences(rng, 257, n)
+        target = rng.integers(0, 131072, size=(257, n)).astype(np.int32)
+        pred = np.where(rng.random((257, n)) < p_match, target, rng.integers(0, 131072, size=(257, n))).astype(np.int32)
+        p, s = gpu_greedy(pred, target, conf)
+        po, so = orc.greedy_accept(pred, target, conf)
+        assert np.array_equal(p, po) and np.array_equal(s, so), f"n={n} p={p_match}"
+
+
+def test_greedy_accept_chain(orc):
+    """Iterated greedy acceptance until a 32-position block is unmasked (Sec. 5):
+    each side chains its own commits; they agree at every iteration."""
+    rng = np.random.default_rng(41)
+    B, n = 64, 32
+    target = rng.integers(0, 131072, size=(B, n)).astype(np.int32)
+    conf_g = rng.random((B, n), dtype=np.float32)
+    conf_o = conf_g.copy()
+    for it in range(n):
+        fresh = rng.random((B, n), dtype=np.float32)
+        pred = np.where(rng.random((B, n)) < 0.4, target, target + 1).astype(np.int32)
+        cg = np.where(conf_g == -np.inf, -np.inf, fresh).astype(np.float32)
+        co = np.where(conf_o == -np.inf, -np.inf, fresh).astype(np.float32)
+        pg, sg = gpu_greedy(pred, target, cg)
+        po, so = orc.greedy_accept(pred, target, co)
+        assert np.array_equal(pg, po) and np.array_equal(sg, so), f"iteration {it}"
+        for b in range(B):
+            conf_g[b, pg[b, :sg[b]]] = -np.inf
+            conf_o[b, po[b, :so[b]]] = -np.inf
+    assert np.all(conf_g == -np.inf), "the block is fully unmasked within n iterations"
+
+
 def test_accept_golden_cases():
     for d, v, acc in oracle_pins.read_golden("accept_cases.txt"):
         d = np.array([[int(x) for x in d.split()]], dtype=np.int32)
