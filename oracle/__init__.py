@@ -1,5 +1,5 @@
 """fp64 CPU oracle for paged block attention, split combine, accept, top-k,
-threshold and greedy unmasking.
+threshold and greedy unmasking, and logits -> (argmax, confidence).
 
 TEST INFRASTRUCTURE ONLY: the tests, ``__graft_entry__.smoke()`` and the CPU
 baseline of ``bench.py`` use it. The product path never imports it. It shares
@@ -72,6 +72,8 @@ class Oracle:
         lib.nldo_unmask_threshold.restype = None
         lib.nldo_greedy_accept.argtypes = [P, P, P, I, I, P, P]
         lib.nldo_greedy_accept.restype = None
+        lib.nldo_logits_argmax.argtypes = [P, Lg, I, Lg, P, P]
+        lib.nldo_logits_argmax.restype = None
         lib.nldo_max_threads.argtypes = []
         lib.nldo_max_threads.restype = I
         self.lib = lib
@@ -166,6 +168,17 @@ class Oracle:
         nsel = np.zeros((B,), dtype=np.int32)
         self.lib.nldo_unmask_threshold(self._p(c), B, n, float(np.float32(threshold)), self._p(pos), self._p(nsel))
         return pos, nsel
+
+    def logits_argmax(self, logits_bits, vocab=None):
+        """(ids [rows] int32, conf [rows] fp64) of bf16 logits [rows, ld] (bit
+        patterns as uint16); the first `vocab` columns are used (default: all)."""
+        lb = np.ascontiguousarray(logits_bits, dtype=np.uint16)
+        rows, ld = lb.shape
+        vocab = ld if vocab is None else int(vocab)
+        ids = np.zeros((rows,), dtype=np.int32)
+        conf = np.zeros((rows,), dtype=np.float64)
+        self.lib.nldo_logits_argmax(self._p(lb), rows, vocab, ld, self._p(ids), self._p(conf))
+        return ids, conf
 
     def greedy_accept(self, pred, target, conf):
         """(positions [B, n] ascending then -1, num_selected [B]) of one greedy

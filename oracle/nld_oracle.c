@@ -32,6 +32,8 @@
  *    sampling) and greedy parallel acceptance against a serial target
  *    (Sec. 5, diffusion SOL construction): the positions one denoising step
  *    commits, in ascending order.
+ *  - Logits -> (argmax id, max softmax probability) per position, the
+ *    inputs of the two decisions (Sec. 2; Sec. 5).
  *
  * Build: gcc -O2 -fopenmp -ffp-contract=off -shared -fPIC (see build.py).
  */
@@ -382,5 +384,34 @@ void nldo_greedy_accept(const int32_t *pred, const int32_t *target, const float 
         }
         for (int r = count; r < n; ++r) pos[r] = -1;
         if (num_selected) num_selected[b] = count;
+    }
+}
+
+/*
+ * Logits -> (argmax id, confidence) per position, the confidence being the
+ * highest peak probability of the position's output distribution (Sec. 5,
+ * serial denoising; Sec. 2, confidence-based sampling):
+ *   m = max_v l_v over the non-NaN logits, id = the lowest v with l_v = m,
+ *   conf = max_v softmax(l)_v = exp(m - lse) = 1 / sum_v exp(l_v - m).
+ * logits bf16 bits [rows, ld] (the first `vocab` of each row are used).
+ * A NaN logit never wins the argmax and makes the confidence NaN (the sum
+ * takes it); a row with no logit above -inf gets id 0 and confidence 0.
+ */
+void nldo_logits_argmax(const uint16_t *logits, long rows, int vocab, long ld, int32_t *ids, double *conf)
+{
+    #pragma omp parallel for schedule(dynamic, 1)
+    for (long r = 0; r < rows; ++r) {
+        const uint16_t *row = logits + r * ld;
+        double m = -INFINITY;
+        int id = 0;
+        for (int v = 0; v < vocab; ++v) {
+            const double l = bf16_to_f64(row[v]);
+            if (l > m) { m = l; id = v; }
+        }
+        ids[r] = id;
+        if (m == -INFINITY) { conf[r] = 0.0; continue; }
+        double sum = 0.0;
+        for (int v = 0; v < vocab; ++v) sum += exp(bf16_to_f64(row[v]) - m);
+        conf[r] = 1.0 / sum;
     }
 }

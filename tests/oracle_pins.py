@@ -539,10 +539,84 @@ def pin_greedy_chain(orc):
         assert np.all(conf == -np.inf) and np.all((iters >= 1) & (iters <= n))
 
 
+# --------------------------------------------------------------------------
+# logits -> (argmax, confidence) pins
+# --------------------------------------------------------------------------
+
+def _bf16_rows(x):
+    return W.f32_to_bf16_bits(np.asarray(x, dtype=np.float32))
+
+
+def pin_logits_golden(orc):
+    for lg, idx, cf in read_golden("logits_argmax_cases.txt"):
+        x = np.array([[float(v) for v in lg.split()]], dtype=np.float32)
+        ids, conf = orc.logits_argmax(_bf16_rows(x))
+        assert int(ids[0]) == int(idx), f"argmax of {lg}: {ids[0]}"
+        want = float(cf)
+        if math.isnan(want):
+            assert math.isnan(conf[0]), f"confidence of {lg}: {conf[0]}"
+        else:
+            assert abs(conf[0] - want) <= 1e-15 * max(1.0, want), f"confidence of {lg}: {conf[0]} vs {want}"
+
+
+def pin_logits_scipy(orc):
+    """Against scipy.special.softmax (max probability) and numpy's argmax (first
+    index of the max) on the same bf16 values, up to the full vocabulary."""
+    rng = np.random.default_rng(31)
+    for rows, V in ((64, 1), (64, 7), (32, 1000), (4, 131072)):
+        bits = W.f32_to_bf16_bits((rng.standard_normal((rows, V)) * 3.0).astype(np.float32))
+        vals = W.bf16_bits_to_f32(bits).astype(np.float64)
+        ids, conf = orc.logits_argmax(bits)
+        assert np.array_equal(ids, np.argmax(vals, axis=1))
+        ref = scipy.special.softmax(vals, axis=1).max(axis=1)
+        assert np.allclose(conf, ref, rtol=1e-12, atol=0), f"V={V}"
+
+
+def pin_logits_closed_forms(orc):
+    """One logit c above V-1 zeros: conf = 1 / (1 + (V-1) e^-c), id its index.
+    Equal logits: conf = 1/V, id 0. Ties between maxima: the lowest index."""
+    for V, c, at in ((2, 1.0, 1), (100, 4.0, 57), (131072, 16.0, 131071), (5, -3.0, 2)):
+        x = np.zeros((1, V), dtype=np.float32)
+        x[0, at] = c
+        ids, conf = orc.logits_argmax(_bf16_rows(x))
+        bound = V * 2.0 ** -52  # a plain fp64 sum of V terms
+        if c > 0:
+            assert int(ids[0]) == at
+            assert abs(conf[0] - 1.0 / (1.0 + (V - 1) * math.exp(-c))) <= bound
+        else:
+            assert int(ids[0]) == (1 if at == 0 else 0)
+            assert abs(conf[0] - 1.0 / (V - 1 + math.exp(c))) <= bound
+    for V in (1, 3, 1024):
+        ids, conf = orc.logits_argmax(_bf16_rows(np.full((1, V), 0.5, np.float32)))
+        assert int(ids[0]) == 0 and abs(conf[0] - 1.0 / V) < 1e-15
+    rng = np.random.default_rng(32)
+    x = rng.integers(-4, 4, size=(200, 50)).astype(np.float32)  # many tied maxima
+    ids, _ = orc.logits_argmax(_bf16_rows(x))
+    assert all(int(ids[r]) == x[r].tolist().index(max(x[r].tolist())) for r in range(200))
+
+
+def pin_logits_brute(orc):
+    rng = np.random.default_rng(33)
+    x = rng.standard_normal((40, 33)).astype(np.float32) * 4
+    x[rng.random(x.shape) < 0.1] = -np.inf
+    x[5, :] = -np.inf
+    bits = _bf16_rows(x)
+    vals = W.bf16_bits_to_f32(bits).astype(np.float64).tolist()
+    ids, conf = orc.logits_argmax(bits)
+    for r, row in enumerate(vals):
+        m = max(row)
+        if m == -math.inf:
+            assert int(ids[r]) == 0 and conf[r] == 0.0
+            continue
+        assert int(ids[r]) == row.index(m)
+        assert abs(conf[r] - 1.0 / sum(math.exp(v - m) for v in row)) < 1e-14
+
+
 ATTENTION_PINS = [pin_decode_bl1, pin_diffusion_full_attention, pin_verify_causal_tail, pin_lse_logsumexp,
                   pin_softmax_rows, pin_page_permutation, pin_block_permutation, pin_closed_forms,
                   pin_golden_uniform, pin_split_combine]
 DECISION_PINS = [pin_accept_golden, pin_accept_brute, pin_accept_statistics, pin_unmask_golden,
                  pin_unmask_brute, pin_unmask_lexsort, pin_threshold_golden, pin_threshold_brute,
                  pin_threshold_limits, pin_greedy_golden, pin_greedy_brute, pin_greedy_chain]
-ALL_PINS = ATTENTION_PINS + DECISION_PINS
+LOGITS_PINS = [pin_logits_golden, pin_logits_scipy, pin_logits_closed_forms, pin_logits_brute]
+ALL_PINS = ATTENTION_PINS + DECISION_PINS + LOGITS_PINS

@@ -64,6 +64,17 @@ MUTANTS = {
                         "if (eligible(c[j]) && p[j] != t[j]) pos[count++] = j;"),
     # nan confidence taken as still masked
     "eligible_nan": ("return !isnan(c) && !(isinf(c) && c < 0);", "return !(isinf(c) && c < 0);"),
+    # logits: ties go to the last maximum
+    "logits_argmax_last": ("if (l > m) { m = l; id = v; }", "if (l >= m) { m = l; id = v; }"),
+    # logits: confidence without the max shift
+    "logits_no_shift": ("for (int v = 0; v < vocab; ++v) sum += exp(bf16_to_f64(row[v]) - m);",
+                        "for (int v = 0; v < vocab; ++v) sum += exp(bf16_to_f64(row[v]));"),
+    # logits: the sum leaves out the maximum's own term
+    "logits_sum_skips_max": ("for (int v = 0; v < vocab; ++v) sum += exp(bf16_to_f64(row[v]) - m);",
+                             "for (int v = 0; v < vocab; ++v) if (v != id) sum += exp(bf16_to_f64(row[v]) - m);"),
+    # logits: a row of -inf reads as certain
+    "logits_empty_certain": ("if (m == -INFINITY) { conf[r] = 0.0; continue; }",
+                             "if (m == -INFINITY) { conf[r] = 1.0; continue; }"),
     # unmask: ascending order
     "unmask_ascending": ("if (ca > cb) return 1;\n    if (ca < cb) return 0;",
                          "if (ca < cb) return 1;\n    if (ca > cb) return 0;"),
