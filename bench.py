@@ -423,6 +423,7 @@ def run_ours(args, world, rank, local):
     if not args.headline_only:
         line["workloads"] = run_workloads(torch, nld, dev, stream, peak, l2)
         line["decisions"] = run_decisions(torch, nld, dev, stream)
+        line["logits_argmax"] = run_logits(torch, nld, dev, stream, peak, l2)
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, budget_s=12.0)
     print(json.dumps(line), flush=True)
@@ -517,6 +518,31 @@ def time_graph(torch, stream, body, nsteps, reps):
         e1.record(stream)
     torch.cuda.synchronize()
     return e0.elapsed_time(e1) / (reps * nsteps)
+
+
+def run_logits(torch, nld, dev, stream, peak, l2):
+    """nld_logits_argmax over a 131072-token vocabulary for the positions of
+    one step: 16 (8B shape, one diffusion block), 512 (14B shape, 16 x 32) and
+    1024 (128 sequences x 8 verify positions). Logits bytes read / time, cold:
+    each call reads its own buffer from a rotation past 3x L2."""
+    V = 131072
+    res = {}
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(11)
+    for rows in (16, 512, 1024):
+        nbytes = rows * V * 2
+        nbuf = int(max(1, np.ceil(3 * l2 / nbytes)))
+        bufs = [(torch.randn((rows, V), generator=gen, device=dev) * 3).to(torch.bfloat16) for _ in range(nbuf)]
+        ids = torch.empty((rows,), dtype=torch.int32, device=dev)
+        conf = torch.empty((rows,), dtype=torch.float32, device=dev)
+        ncall = max(nbuf, 8)
+        us = time_graph(torch, stream, lambda i: nld.nld_logits_argmax(bufs[i % nbuf], ids, conf), ncall, 10) * 1e3
+        gbs = nbytes / (us * 1e-6) / 1e9
+        res[f"rows{rows}_v{V}"] = {"us_per_call": round(us, 3), "logits_gbs": round(gbs, 1),
+                                   "pct_of_hbm_peak": round(100 * gbs / peak, 2), "buffers": nbuf}
+        del bufs
+    res["timing"] = "CUDA graph of back-to-back calls over rotating buffers, events around 10 replays"
+    return res
 
 
 def run_decisions(torch, nld, dev, stream):

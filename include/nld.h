@@ -270,6 +270,24 @@ nld_status_t nld_greedy_accept(const int32_t *pred_ids, const int32_t *target_id
                                const float *confidences, int batch, int n, int32_t *positions,
                                int32_t *num_selected, cudaStream_t stream);
 
+/*
+ * Logits -> (argmax id, confidence) per position, the inputs of the token
+ * decisions above (the confidence of Sec. 2 confidence-based sampling; Sec. 5
+ * serial denoising commits the position with the highest peak probability):
+ *   m = max_v logits[r][v],  ids[r] = the lowest v with logits[r][v] = m,
+ *   conf[r] = max_v softmax(logits[r])_v = 1 / sum_v exp(logits[r][v] - m).
+ * A NaN logit never wins the argmax and makes conf NaN; a row with nothing
+ * above -inf gets id 0 and conf 0. fp32 arithmetic (relative error of conf
+ * within a few 1e-6 at vocab 131072).
+ *
+ *   logits  bf16 [rows, ld], the first `vocab` entries of each row used;
+ *           ld >= vocab and a multiple of 8, base 16-byte aligned
+ *   ids     int32 [rows]
+ *   conf    fp32 [rows]
+ */
+nld_status_t nld_logits_argmax(const void *logits, int rows, int vocab, int ld, int32_t *ids,
+                               float *conf, cudaStream_t stream);
+
 /* A static, human-readable name for a status code. */
 const char *nld_status_string(nld_status_t status);
 

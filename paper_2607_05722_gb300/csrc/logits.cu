@@ -1,0 +1,234 @@
+// Logits -> (argmax id, confidence) per position: the inputs of the token
+// decisions (Sec. 2 confidence-based sampling; Sec. 5 serial denoising
+// commits the position with the highest peak probability).
+//   m = max_v l_v, id = the lowest v with l_v = m,
+//   conf = max_v softmax(l)_v = 1 / sum_v exp(l_v - m).
+// A row is cut into `split` pieces, one CTA each (a thread-block cluster when
+// split > 1). In a CTA one producer warp streams the piece through a ring of
+// 16 KB stages with bulk copies (TMA engine) and eight warps fold each 8-logit
+// vector into a running (max, sum of exp(l - max), argmax): the vector max
+// comes first, so the rare rescale happens once per vector, then one exp per
+// logit. The partial states merge by the log-sum-exp rule (ties: the lower
+// index) across the warps, the CTA and, through distributed shared memory,
+// the cluster. NaN logits never win the argmax and make the sum NaN; a row
+// with nothing above -inf gets id 0 and confidence 0.
+#include "nld_internal.cuh"
+
+namespace nld {
+namespace {
+
+constexpr int kLgConsumerWarps = 8;
+constexpr int kLgThreads = 32 * (kLgConsumerWarps + 1);  // + the producer warp
+constexpr int kLgStages = 4;
+constexpr int kLgStageVecs = 1024;                       // 16-byte vectors (8 logits): 16 KB a stage
+constexpr int kLgRingBytes = kLgStages * kLgStageVecs * 16;
+constexpr int kLgSmemBytes = kLgRingBytes + 2 * kLgStages * 8 + 4 * 8 * 3 + 16 + 128;  // + alignment slack
+
+// Merge (m2, s2, i2) into (m, s, i): the max, the sums rescaled to it, and
+// the argmax (the lower index when the maxima are equal). A state whose max
+// is still -inf has sum 0, or NaN if it met a NaN logit; it enters the merge
+// as sum * 0, which keeps the NaN.
+__device__ __forceinline__ void lg_merge(float& m, float& s, int& i, float m2, float s2, int i2) {
+  const float mm = fmaxf(m, m2);
+  i = m > m2 ? i : (m2 > m ? i2 : min(i, i2));
+  const float a = m == -INFINITY ? s * 0.f : s * ex2((m - mm) * kLog2e);
+  const float b = m2 == -INFINITY ? s2 * 0.f : s2 * ex2((m2 - mm) * kLog2e);
+  m = mm;
+  s = a + b;
+}
+
+// Fold x[0..n) (logits e0 .. e0+n-1, in index order) into (m, s, i).
+template <int N>
+__device__ __forceinline__ void lg_fold(const float (&x)[N], int e0, float& m, float& s, int& i) {
+  float vm = x[0];
+#pragma unroll
+  for (int j = 1; j < N; ++j) vm = fmaxf(vm, x[j]);
+  if (vm > m) {  // a new running max (NaN never is)
+    s = m == -INFINITY ? s * 0.f : s * ex2((m - vm) * kLog2e);
+    m = vm;
+    int first = N - 1;
+#pragma unroll
+    for (int j = N - 1; j >= 0; --j)
+      if (x[j] == vm) first = j;
+    i = e0 + first;
+  }
+  if (m != -INFINITY) {
+#pragma unroll
+    for (int j = 0; j < N; ++j) s += ex2((x[j] - m) * kLog2e);  // a NaN logit makes s NaN
+  } else {
+#pragma unroll
+    for (int j = 0; j < N; ++j)
+      if (isnan(x[j])) s = NAN;  // nothing finite yet: the NaN must still reach the sum
+  }
+}
+
+__global__ void __launch_bounds__(kLgThreads)
+    logits_argmax_kernel(const __nv_bfloat16* __restrict__ logits, int vocab, long ld, int split,
+                         int32_t* __restrict__ ids, float* __restrict__ conf, unsigned int* err) {
+  extern __shared__ uint8_t lg_smem_raw[];
+  uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(lg_smem_raw) + 127) & ~uintptr_t(127));
+  uint64_t* full = reinterpret_cast<uint64_t*>(ring + kLgRingBytes);
+  uint64_t* empty = full + kLgStages;
+  float* red = reinterpret_cast<float*>(empty + kLgStages);  // [consumer warp][m, s, i]
+  float* part = red + 3 * kLgConsumerWarps;                   // this CTA's merged state, for the cluster
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int piece = static_cast<int>(blockIdx.x % split);
+  const long row = static_cast<long>(blockIdx.x / split);
+  const int nvec = vocab >> 3, tail = vocab & 7;
+  const int per = (nvec + split - 1) / split;
+  const int v0 = min(nvec, piece * per), v1 = min(nvec, v0 + per);
+  const int nst = (v1 - v0 + kLgStageVecs - 1) / kLgStageVecs;
+
+  if (threadIdx.x == 0) {
+    for (int st = 0; st < kLgStages; ++st) {
+      mbar_init(&full[st], 1);
+      mbar_init(&empty[st], kLgConsumerWarps);
+    }
+    fence_mbar_init();
+  }
+  __syncthreads();
+  grid_launch_dependents();  // dependents launch early; they wait on this grid themselves
+  grid_dependency_wait();    // the logits come from the previous kernel
+  const uint8_t* grow = reinterpret_cast<const uint8_t*>(logits + row * ld);
+
+  float m = -INFINITY, s = 0.f;
+  int idx = 0;
+  if (warp == kLgConsumerWarps) {
+    // ---- producer: one lane issues the stages of this piece ----
+    if (lane == 0) {
+      int issued = 0;
+      bool ok = true;
+      for (int k = 0; k < nst; ++k) {
+        const int st = k % kLgStages;
+        if (k >= kLgStages && !mbar_wait(&empty[st], ((k / kLgStages) - 1) & 1, err)) {
+          ok = false;
+          break;
+        }
+        const uint32_t bytes = static_cast<uint32_t>(min(kLgStageVecs, v1 - v0 - k * kLgStageVecs)) * 16u;
+        mbar_arrive_expect_tx(&full[st], bytes);
+        bulk_load(ring + st * kLgStageVecs * 16, grow + static_cast<long>(v0 + k * kLgStageVecs) * 16, bytes,
+                  &full[st]);
+        issued = k + 1;
+      }
+      if (!ok) {
+        // Gave up on a timeout: let the copies in flight land before exit (bounded).
+        for (int k = max(0, issued - kLgStages); k < issued; ++k)
+          mbar_wait(&full[k % kLgStages], (k / kLgStages) & 1, err);
+      }
+    }
+  } else {
+    // ---- consumers: thread t folds vectors t, t+256, ... of each stage ----
+    const int t = threadIdx.x;
+    for (int k = 0; k < nst; ++k) {
+      const int st = k % kLgStages;
+      if (!__all_sync(0xffffffffu, mbar_wait(&full[st], (k / kLgStages) & 1, err))) break;
+      const int nv = min(kLgStageVecs, v1 - v0 - k * kLgStageVecs);
+      const uint4* sv = reinterpret_cast<const uint4*>(ring + st * kLgStageVecs * 16);
+      const int ebase = (v0 + k * kLgStageVecs) * 8;
+      for (int j = t; j < nv; j += 32 * kLgConsumerWarps) {
+        const uint4 w = sv[j];
+        float x[8];
+        unpack_bf16(w.x, x[0], x[1]);
+        unpack_bf16(w.y, x[2], x[3]);
+        unpack_bf16(w.z, x[4], x[5]);
+        unpack_bf16(w.w, x[6], x[7]);
+        lg_fold(x, ebase + j * 8, m, s, idx);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[st]);
+    }
+    if (piece == split - 1 && t < tail) {  // the last vocab % 8 logits, after every vector
+      const uint16_t bits = reinterpret_cast<const uint16_t*>(grow)[nvec * 8 + t];
+      const float x[1] = {__uint_as_float(static_cast<uint32_t>(bits) << 16)};
+      lg_fold(x, nvec * 8 + t, m, s, idx);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+      const float s2 = __shfl_xor_sync(0xffffffffu, s, off);
+      const int i2 = __shfl_xor_sync(0xffffffffu, idx, off);
+      lg_merge(m, s, idx, m2, s2, i2);
+    }
+    if (lane == 0) {
+      red[3 * warp] = m;
+      red[3 * warp + 1] = s;
+      red[3 * warp + 2] = __int_as_float(idx);
+    }
+  }
+  __syncthreads();
+  if (warp == 0) {
+    m = lane < kLgConsumerWarps ? red[3 * lane] : -INFINITY;
+    s = lane < kLgConsumerWarps ? red[3 * lane + 1] : 0.f;
+    idx = lane < kLgConsumerWarps ? __float_as_int(red[3 * lane + 2]) : 0;
+#pragma unroll
+    for (int off = 4; off > 0; off >>= 1) {
+      const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+      const float s2 = __shfl_xor_sync(0xffffffffu, s, off);
+      const int i2 = __shfl_xor_sync(0xffffffffu, idx, off);
+      lg_merge(m, s, idx, m2, s2, i2);
+    }
+    if (lane == 0) {
+      if (split == 1) {
+        ids[row] = idx;
+        conf[row] = m == -INFINITY ? 0.f : 1.f / s;
+      } else {
+        part[0] = m;
+        part[1] = s;
+        part[2] = __int_as_float(idx);
+      }
+    }
+  }
+  if (split > 1) {
+    // Merge the pieces of the row: rank 0 reads every CTA's state through
+    // distributed shared memory; the second barrier keeps the peers' shared
+    // memory alive until it has.
+    cluster_sync();
+    if (cluster_ctarank() == 0 && warp == 0) {
+      const uint32_t pa = smem_u32(part);
+      m = -INFINITY;
+      s = 0.f;
+      idx = 0;
+      if (lane < split) {
+        m = ld_dsmem_f32(dsmem_addr(pa, lane));
+        s = ld_dsmem_f32(dsmem_addr(pa + 4, lane));
+        idx = __float_as_int(ld_dsmem_f32(dsmem_addr(pa + 8, lane)));
+      }
+#pragma unroll
+      for (int off = 4; off > 0; off >>= 1) {
+        const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+        const float s2 = __shfl_xor_sync(0xffffffffu, s, off);
+        const int i2 = __shfl_xor_sync(0xffffffffu, idx, off);
+        lg_merge(m, s, idx, m2, s2, i2);
+      }
+      if (lane == 0) {
+        ids[row] = idx;
+        conf[row] = m == -INFINITY ? 0.f : 1.f / s;
+      }
+    }
+    cluster_sync();
+  }
+}
+
+}  // namespace
+
+int logits_split_vectors() { return kLgStageVecs; }
+
+cudaError_t launch_logits_argmax(const __nv_bfloat16* logits, int rows, int vocab, long ld, int split, int32_t* ids,
+                                 float* conf, unsigned int* err, cudaStream_t stream) {
+  static int configured[64] = {0};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (!__atomic_load_n(&configured[dev], __ATOMIC_ACQUIRE)) {
+    e = cudaFuncSetAttribute(logits_argmax_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kLgSmemBytes);
+    if (e != cudaSuccess) return e;
+    __atomic_store_n(&configured[dev], 1, __ATOMIC_RELEASE);
+  }
+  const dim3 grid(static_cast<unsigned>(static_cast<long>(rows) * split));
+  return launch_kernel_cluster(logits_argmax_kernel, grid, dim3(kLgThreads), kLgSmemBytes, stream, split, logits,
+                               vocab, ld, split, ids, conf, err);
+}
+
+}  // namespace nld

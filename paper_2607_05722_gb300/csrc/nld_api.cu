@@ -368,6 +368,29 @@ nld_status_t nld_greedy_accept(const int32_t* pred_ids, const int32_t* target_id
              : NLD_ERR_CUDA;
 }
 
+nld_status_t nld_logits_argmax(const void* logits, int rows, int vocab, int ld, int32_t* ids, float* conf,
+                               cudaStream_t stream) {
+  if (rows < 1 || vocab < 1 || ld < vocab || ld % 8 != 0) return NLD_ERR_INVALID_ARG;
+  if (!aligned(logits, 16) || !aligned(ids, 4) || !aligned(conf, 4)) return NLD_ERR_INVALID_ARG;
+  unsigned int* err = nullptr;
+  int sms = 0;
+  nld_status_t st = device_state(&err, &sms);
+  if (st != NLD_OK) return st;
+  // Pieces per row: fill the SMs once when there are fewer rows than SMs, at
+  // least one ring stage of vectors a piece, at most one cluster of 8.
+  int split = 1;
+  if (rows < sms) {
+    const int by_sms = sms / rows;
+    const int by_len = (vocab / 8) / nld::logits_split_vectors();
+    const int want = by_sms < by_len ? by_sms : by_len;
+    while (split * 2 <= want && split * 2 <= 8) split *= 2;
+  }
+  return nld::launch_logits_argmax(static_cast<const __nv_bfloat16*>(logits), rows, vocab, ld, split, ids, conf, err,
+                                   stream) == cudaSuccess
+             ? NLD_OK
+             : NLD_ERR_CUDA;
+}
+
 nld_status_t nld_device_error(uint32_t* bits, int clear) {
   if (bits == nullptr) return NLD_ERR_INVALID_ARG;
   unsigned int* err = nullptr;

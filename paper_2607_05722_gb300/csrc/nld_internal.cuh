@@ -56,6 +56,10 @@ cudaError_t launch_unmask_threshold(const float* conf, int B, int n, float thres
                                     cudaStream_t stream);
 cudaError_t launch_greedy_accept(const int32_t* pred, const int32_t* target, const float* conf, int B, int n,
                                  int32_t* pos, int32_t* nsel, cudaStream_t stream);
+// Logits -> (argmax, confidence): `split` CTAs per row (a cluster when > 1).
+cudaError_t launch_logits_argmax(const __nv_bfloat16* logits, int rows, int vocab, long ld, int split, int32_t* ids,
+                                 float* conf, unsigned int* err, cudaStream_t stream);
+int logits_split_vectors();  // 16-byte vectors a CTA streams per ring stage
 
 // Launch with programmatic stream serialization: the kernel may start while
 // its predecessor in the stream is still running. Every kernel of this
@@ -211,6 +215,12 @@ __device__ __forceinline__ float lg2(float x) {
   return y;
 }
 
+// Two bf16 values (low half first) widened exactly to fp32.
+__device__ __forceinline__ void unpack_bf16(uint32_t w, float& lo, float& hi) {
+  lo = __uint_as_float(w << 16);
+  hi = __uint_as_float(w & 0xFFFF0000u);
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
@@ -261,6 +271,16 @@ __device__ __forceinline__ float4 ld_dsmem_f4(uint32_t addr) {
 // ---------------------------------------------------------------------------
 // tcgen05 (5th-generation tensor core) and tensor memory
 // ---------------------------------------------------------------------------
+
+// Bulk copy (TMA engine) of `bytes` from global to this CTA's shared memory,
+// completing on an mbarrier (expect_tx set by the caller); both addresses
+// 16-byte aligned, bytes a multiple of 16.
+__device__ __forceinline__ void bulk_load(void* sdst, const void* gsrc, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_u32(sdst)),
+               "l"(gsrc), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
+}
 
 // Bulk copy (TMA engine) of `bytes` from this CTA's shared memory to global
 // memory; both addresses 16-byte aligned, bytes a multiple of 16. The issuing

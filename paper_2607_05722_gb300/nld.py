@@ -74,6 +74,8 @@ def lib(path: Optional[str] = None):
     L.nld_unmask_threshold.restype = I
     L.nld_greedy_accept.argtypes = [V, V, V, I, I, V, V, V]
     L.nld_greedy_accept.restype = I
+    L.nld_logits_argmax.argtypes = [V, I, I, I, V, V, V]
+    L.nld_logits_argmax.restype = I
     L.nld_unmask.restype = I
     L.nld_status_string.argtypes = [I]
     L.nld_status_string.restype = ctypes.c_char_p
@@ -268,6 +270,19 @@ def nld_greedy_accept(pred_ids, target_ids, confidences, positions, num_selected
         _expect(num_selected, torch.int32, (B,), "num_selected")
     _check(lib().nld_greedy_accept(_ptr(pred_ids), _ptr(target_ids), _ptr(confidences), B, n, _ptr(positions),
                                    _ptr(num_selected), _stream(stream)), "nld_greedy_accept")
+
+
+def nld_logits_argmax(logits, ids, conf, vocab=None, stream=None):
+    """Per row of bf16 logits [rows, ld]: the argmax over the first `vocab`
+    entries (lowest index on ties) and the max softmax probability."""
+    if logits.dtype != torch.bfloat16 or logits.dim() != 2 or not logits.is_cuda or logits.stride(1) != 1:
+        raise ValueError("logits: a CUDA bf16 [rows, ld] tensor with unit column stride")
+    rows, ld = logits.shape[0], logits.stride(0)
+    vocab = logits.shape[1] if vocab is None else int(vocab)
+    _expect(ids, torch.int32, (rows,), "ids")
+    _expect(conf, torch.float32, (rows,), "conf")
+    _check(lib().nld_logits_argmax(_ptr(logits), rows, vocab, ld, _ptr(ids), _ptr(conf), _stream(stream)),
+           "nld_logits_argmax")
 
 def nld_device_error(clear: bool = False) -> int:
     bits = ctypes.c_uint32(0)

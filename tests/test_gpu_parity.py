@@ -6,6 +6,8 @@ Small cases run the oracle on every row; the full-size workloads run in the
 launch configuration the bench times (automatic split count) and compare a
 sample of rows the oracle computes one by one.
 """
+import math
+
 import numpy as np
 import pytest
 import torch
@@ -138,6 +140,73 @@ def test_greedy_accept_chain(orc):
             conf_g[b, pg[b, :sg[b]]] = -np.inf
             conf_o[b, po[b, :so[b]]] = -np.inf
     assert np.all(conf_g == -np.inf), "the block is fully unmasked within n iterations"
+
+
+# ---------------------------------------------------------------------------
+# logits -> (argmax id, confidence)
+# ---------------------------------------------------------------------------
+
+# conf relative tolerance: one ex2.approx per logit (relative error ~2^-21)
+# plus fp32 sums of at most 512 positive terms per thread before an fp32
+# tree merge (<= 512 * 2^-24 = 3.1e-5 relative).
+LOGITS_RTOL = 4e-5
+
+
+def gpu_logits(bits, vocab=None):
+    rows, ld = bits.shape
+    t = torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).cuda()
+    ids = torch.full((rows,), -7, dtype=torch.int32, device="cuda")
+    conf = torch.full((rows,), -7.0, dtype=torch.float32, device="cuda")
+    nld.nld_logits_argmax(t, ids, conf, vocab=vocab)
+    return ids.cpu().numpy(), conf.cpu().numpy().astype(np.float64)
+
+
+def check_logits(got, ref, what):
+    (gi, gc), (ri, rc) = got, ref
+    assert np.array_equal(gi, ri), f"{what}: argmax differs at {np.flatnonzero(gi != ri)[:5]}"
+    nan = np.isnan(rc)
+    assert np.array_equal(np.isnan(gc), nan), f"{what}: NaN pattern"
+    err = np.abs(gc[~nan] - rc[~nan])
+    assert np.all(err <= LOGITS_RTOL * np.abs(rc[~nan])), f"{what}: conf rel err {np.max(err / np.maximum(rc[~nan], 1e-30)):.2e}"
+
+
+def test_logits_golden_cases():
+    for lg, idx, cf in oracle_pins.read_golden("logits_argmax_cases.txt"):
+        x = np.array([[float(v) for v in lg.split()]], dtype=np.float32)
+        V = x.shape[1]
+        bits = np.zeros((1, (V + 7) // 8 * 8), dtype=np.uint16)
+        bits[0, :V] = W.f32_to_bf16_bits(x)[0]
+        gi, gc = gpu_logits(bits, vocab=V)
+        assert int(gi[0]) == int(idx), lg
+        want = float(cf)
+        assert (math.isnan(gc[0]) and math.isnan(want)) or abs(gc[0] - want) <= LOGITS_RTOL * max(want, 1e-30), lg
+
+
+@pytest.mark.parametrize("rows,vocab,ld", [(1, 1, 8), (3, 7, 8), (5, 8, 8), (7, 9, 16), (16, 131072, 131072),
+                                           (16, 131077, 131080), (2, 50000, 50008), (300, 32000, 32000),
+                                           (1024, 4096, 4096), (152, 131072, 131072)])
+def test_logits_matches_oracle(orc, rows, vocab, ld):
+    rng = np.random.default_rng(rows * 7 + vocab)
+    x = (rng.standard_normal((rows, ld)) * 3.0).astype(np.float32)
+    x[:, vocab:] = 1e4  # padding past vocab must never be read
+    if rows >= 3:
+        x[0, :vocab] = -np.inf                                   # nothing above -inf
+        x[1, rng.integers(0, vocab)] = np.nan                    # a NaN logit
+        x[2, :vocab] = np.round(x[2, :vocab])                    # many ties
+    x[rng.random(x.shape) < 0.01] = -np.inf
+    bits = W.f32_to_bf16_bits(x)
+    check_logits(gpu_logits(bits, vocab), orc.logits_argmax(bits, vocab), f"rows={rows} V={vocab} ld={ld}")
+
+
+def test_logits_peaked_rows(orc):
+    """Peaked rows (a confident prediction): the confidence near 1 is kept to
+    the same relative bound."""
+    rng = np.random.default_rng(77)
+    x = (rng.standard_normal((64, 131072)) * 1.0).astype(np.float32)
+    hot = rng.integers(0, 131072, size=64)
+    x[np.arange(64), hot] = np.linspace(2, 30, 64)
+    bits = W.f32_to_bf16_bits(x)
+    check_logits(gpu_logits(bits), orc.logits_argmax(bits), "peaked")
 
 
 def test_accept_golden_cases():
