@@ -1,5 +1,6 @@
 """fp64 CPU oracle for paged block attention, split combine, accept, top-k,
-threshold and greedy unmasking, and logits -> (argmax, confidence).
+threshold and greedy unmasking, logits -> (argmax, confidence), and the block
+KV commit into the paged cache.
 
 TEST INFRASTRUCTURE ONLY: the tests, ``__graft_entry__.smoke()`` and the CPU
 baseline of ``bench.py`` use it. The product path never imports it. It shares
@@ -74,6 +75,8 @@ class Oracle:
         lib.nldo_greedy_accept.restype = None
         lib.nldo_logits_argmax.argtypes = [P, Lg, I, Lg, P, P]
         lib.nldo_logits_argmax.restype = None
+        lib.nldo_kv_commit.argtypes = [P, P, P, P, P, I, P, P, I, I, I, I, I, I, I]
+        lib.nldo_kv_commit.restype = None
         lib.nldo_max_threads.argtypes = []
         lib.nldo_max_threads.restype = I
         self.lib = lib
@@ -179,6 +182,22 @@ class Oracle:
         conf = np.zeros((rows,), dtype=np.float64)
         self.lib.nldo_logits_argmax(self._p(lb), rows, vocab, ld, self._p(ids), self._p(conf))
         return ids, conf
+
+    def kv_commit(self, k_new_bits, v_new_bits, counts, page_table, prefix_lens, k_bits, v_bits, advance):
+        """Commit rows of a [B, bl, Hkv, D] K/V block into copies of the page
+        pools; returns (k_pages, v_pages, prefix_lens) after the commit."""
+        kn = np.ascontiguousarray(k_new_bits, dtype=np.uint16)
+        vn = np.ascontiguousarray(v_new_bits, dtype=np.uint16)
+        B, bl, Hkv, D = kn.shape
+        kp = np.array(k_bits, dtype=np.uint16, copy=True, order="C")
+        vp = np.array(v_bits, dtype=np.uint16, copy=True, order="C")
+        P = kp.shape[2]
+        table = np.ascontiguousarray(page_table, dtype=np.int32)
+        pl = np.array(prefix_lens, dtype=np.int32, copy=True)
+        cnt = None if counts is None else np.ascontiguousarray(counts, dtype=np.int32)
+        self.lib.nldo_kv_commit(self._p(kn), self._p(vn), self._p(cnt), self._p(table), self._p(pl), int(bool(advance)),
+                                self._p(kp), self._p(vp), B, Hkv, D, P, kp.shape[0], table.shape[1], bl)
+        return kp, vp, pl
 
     def greedy_accept(self, pred, target, conf):
         """(positions [B, n] ascending then -1, num_selected [B]) of one greedy

@@ -34,6 +34,8 @@
  *    commits, in ascending order.
  *  - Logits -> (argmax id, max softmax probability) per position, the
  *    inputs of the two decisions (Sec. 2; Sec. 5).
+ *  - Block KV commit into the paged slots after the prefix, with the prefix
+ *    advanced by the committed rows (Sec. 3 Mode 3; Sec. 2 block refresh).
  *
  * Build: gcc -O2 -fopenmp -ffp-contract=off -shared -fPIC (see build.py).
  */
@@ -413,5 +415,44 @@ void nldo_logits_argmax(const uint16_t *logits, long rows, int vocab, long ld, i
         double sum = 0.0;
         for (int v = 0; v < vocab; ++v) sum += exp(bf16_to_f64(row[v]) - m);
         conf[r] = 1.0 / sum;
+    }
+}
+
+/*
+ * Block KV commit into the paged cache (Sec. 3 Mode 3: the accepted prefix is
+ * committed to the verified prefix and the verifier's cache is rebuilt at the
+ * rejection point; Sec. 2: a completed block's KV cache is refreshed). Row j
+ * of the block (j < count_b; count_b = counts[b], or bl when counts is NULL)
+ * is written to logical slot L_b + j, i.e. physical page
+ * page_table[b][(L_b + j) / P], slot (L_b + j) mod P, for every KV head.
+ * With `advance`, L_b becomes L_b + count_b afterwards (slots past it are
+ * left as they are: they are simply no longer part of the prefix).
+ * k_new, v_new bf16 bits [B, bl, Hkv, D]; pools [num_pages, Hkv, P, D].
+ * A slot past the page table, or a page id outside the pool, is not written.
+ */
+void nldo_kv_commit(const uint16_t *k_new, const uint16_t *v_new, const int32_t *counts,
+                    const int32_t *page_table, int32_t *prefix_lens, int advance,
+                    uint16_t *k_pages, uint16_t *v_pages, int B, int Hkv, int D, int P,
+                    int num_pages, int max_pages, int bl)
+{
+    for (int b = 0; b < B; ++b) {
+        const long L = prefix_lens[b];
+        const int count = counts ? counts[b] : bl;
+        for (int j = 0; j < count; ++j) {
+            const long t = L + j;
+            if (t < 0 || t >= (long)max_pages * P) continue;
+            const long page = page_table[(long)b * max_pages + t / P];
+            if (page < 0 || page >= num_pages) continue;
+            const long slot = t % P;
+            for (int g = 0; g < Hkv; ++g) {
+                const long src = (((long)b * bl + j) * Hkv + g) * D;
+                const long dst = ((page * Hkv + g) * P + slot) * D;
+                for (int d = 0; d < D; ++d) {
+                    k_pages[dst + d] = k_new[src + d];
+                    v_pages[dst + d] = v_new[src + d];
+                }
+            }
+        }
+        if (advance) prefix_lens[b] = (int32_t)(L + count);
     }
 }

@@ -612,6 +612,101 @@ def pin_logits_brute(orc):
         assert abs(conf[r] - 1.0 / sum(math.exp(v - m) for v in row)) < 1e-14
 
 
+# --------------------------------------------------------------------------
+# block KV commit pins
+# --------------------------------------------------------------------------
+
+def _commit_inputs(rng, case):
+    kv = case.kv
+    shape = (case.batch, case.block_len, case.num_kv_heads, case.head_dim)
+    k_new = W.f32_to_bf16_bits(rng.standard_normal(shape).astype(np.float32))
+    v_new = W.f32_to_bf16_bits(rng.standard_normal(shape).astype(np.float32))
+    return kv, k_new, v_new
+
+
+def pin_commit_gather(orc):
+    """Committed rows read back through the page table with numpy indexing
+    equal the new rows; every other slot keeps its bits; the prefix advances
+    by the committed count (or stays, without advance)."""
+    rng = np.random.default_rng(51)
+    for seed, prefix in ((1, (7, 12)), (2, (0, 3)), (3, (16, 1))):
+        case = small_case(seed, prefix=prefix)
+        kv, k_new, v_new = _commit_inputs(rng, case)
+        P, bl = kv.page_size, case.block_len
+        for counts, advance in ((None, True), (rng.integers(0, bl + 1, case.batch).astype(np.int32), True),
+                                (np.array([0, bl], np.int32), False)):
+            kp, vp, pl = orc.kv_commit(k_new, v_new, counts, kv.page_table, kv.prefix_lens, kv.k_bits, kv.v_bits,
+                                       advance)
+            cnt = np.full(case.batch, bl, np.int32) if counts is None else counts
+            written = np.zeros(kv.k_bits.shape[:3], dtype=bool)  # [page, head, slot]
+            for b in range(case.batch):
+                L = int(kv.prefix_lens[b])
+                t = L + np.arange(cnt[b])
+                pages, slots = kv.page_table[b, t // P], t % P
+                assert np.array_equal(kp[pages, :, slots, :], k_new[b, :cnt[b]])
+                assert np.array_equal(vp[pages, :, slots, :], v_new[b, :cnt[b]])
+                written[pages, :, slots] = True
+            assert np.array_equal(kp[~written], kv.k_bits[~written]) and np.array_equal(vp[~written], kv.v_bits[~written])
+            assert np.array_equal(pl, kv.prefix_lens + cnt if advance else kv.prefix_lens)
+
+
+def pin_commit_then_attention(orc):
+    """A block staged by the commit (all bl rows, no advance) is what the
+    attention reads as the block's own keys: the result equals fp64 SDPA over
+    the prefix K/V followed by the new block K/V (both passes)."""
+    rng = np.random.default_rng(52)
+    case = small_case(9, prefix=(6, 13))
+    kv, k_new, v_new = _commit_inputs(rng, case)
+    kp, vp, _ = orc.kv_commit(k_new, v_new, None, kv.page_table, kv.prefix_lens, kv.k_bits, kv.v_bits, False)
+    G = case.num_q_heads // case.num_kv_heads
+    for mode, qbits in ((DIFF, case.q_draft_bits), (VER, case.q_verify_bits)):
+        out, _ = orc.block_attn(qbits, kp, vp, kv.page_table, kv.prefix_lens, case.num_q_heads,
+                                case.num_kv_heads, case.block_len, mode, case.scale)
+        for b in range(case.batch):
+            L = int(kv.prefix_lens[b])
+            k_pre, v_pre = gather_contiguous(case, b)  # the original pools: the prefix part is untouched
+            kb = np.transpose(W.bf16_bits_to_f32(k_new[b]).astype(np.float64), (1, 0, 2))
+            vb = np.transpose(W.bf16_bits_to_f32(v_new[b]).astype(np.float64), (1, 0, 2))
+            k = np.concatenate([k_pre[:, :L], kb], axis=1)
+            v = np.concatenate([v_pre[:, :L], vb], axis=1)
+            q = np.transpose(q_f64(qbits[b]), (1, 0, 2))
+            if mode == DIFF:
+                ref = sdpa(q, repeat_heads(k, G), repeat_heads(v, G), case.scale)
+            else:
+                qfull = np.concatenate([rng.standard_normal((case.num_q_heads, L, case.head_dim)), q], axis=1)
+                ref = sdpa(qfull, repeat_heads(k, G), repeat_heads(v, G), case.scale, causal=True)[:, L:, :]
+            assert_close(np.transpose(out[b], (1, 0, 2)), ref, 1e-12, f"commit + attention mode={mode}")
+
+
+def pin_commit_rollback_chain(orc):
+    """Linear self-speculation steps: commit the accepted rows (accepted_len
+    from the pinned accept rule) and advance; the next step's block lands
+    right after them, over the rejected rows (the cache rebuilt at the
+    rejection point, Sec. 3 Mode 3)."""
+    rng = np.random.default_rng(53)
+    case = small_case(11, B=3, prefix=(4, 9, 0))
+    kv = case.kv
+    P, bl = kv.page_size, case.block_len
+    kp, vp, pl = kv.k_bits.copy(), kv.v_bits.copy(), kv.prefix_lens.copy()
+    history = [[] for _ in range(case.batch)]  # committed rows in order, per sequence
+    for step in range(3):
+        _, k_new, v_new = _commit_inputs(rng, case)
+        d, v = W.make_accept_ids(rng, case.batch, bl, 50, 0.6)
+        acc = orc.accept(d, v)
+        room = (kv.page_table.shape[1] * P - pl).astype(np.int32)
+        acc = np.minimum(acc, room).astype(np.int32)
+        kp, vp, pl_new = orc.kv_commit(k_new, v_new, acc, kv.page_table, pl, kp, vp, True)
+        assert np.array_equal(pl_new, pl + acc)
+        for b in range(case.batch):
+            history[b] += [k_new[b, j] for j in range(acc[b])]
+        pl = pl_new
+    for b in range(case.batch):
+        L0 = int(kv.prefix_lens[b])
+        t = L0 + np.arange(len(history[b]))
+        got = kp[kv.page_table[b, t // P], :, t % P, :]
+        assert np.array_equal(got, np.array(history[b]).reshape(got.shape))
+
+
 ATTENTION_PINS = [pin_decode_bl1, pin_diffusion_full_attention, pin_verify_causal_tail, pin_lse_logsumexp,
                   pin_softmax_rows, pin_page_permutation, pin_block_permutation, pin_closed_forms,
                   pin_golden_uniform, pin_split_combine]
@@ -619,4 +714,5 @@ DECISION_PINS = [pin_accept_golden, pin_accept_brute, pin_accept_statistics, pin
                  pin_unmask_brute, pin_unmask_lexsort, pin_threshold_golden, pin_threshold_brute,
                  pin_threshold_limits, pin_greedy_golden, pin_greedy_brute, pin_greedy_chain]
 LOGITS_PINS = [pin_logits_golden, pin_logits_scipy, pin_logits_closed_forms, pin_logits_brute]
-ALL_PINS = ATTENTION_PINS + DECISION_PINS + LOGITS_PINS
+COMMIT_PINS = [pin_commit_gather, pin_commit_then_attention, pin_commit_rollback_chain]
+ALL_PINS = ATTENTION_PINS + DECISION_PINS + LOGITS_PINS + COMMIT_PINS

@@ -75,6 +75,17 @@ MUTANTS = {
     # logits: a row of -inf reads as certain
     "logits_empty_certain": ("if (m == -INFINITY) { conf[r] = 0.0; continue; }",
                              "if (m == -INFINITY) { conf[r] = 1.0; continue; }"),
+    # commit: slot from the page index
+    "commit_slot": ("const long slot = t % P;", "const long slot = (t / P) % P;"),
+    # commit: the prefix advances by the whole block
+    "commit_advance_bl": ("if (advance) prefix_lens[b] = (int32_t)(L + count);",
+                          "if (advance) prefix_lens[b] = (int32_t)(L + bl);"),
+    # commit: the bonus position's row committed as well
+    "commit_plus_bonus": ("const int count = counts ? counts[b] : bl;",
+                          "const int count = counts ? (counts[b] < bl ? counts[b] + 1 : bl) : bl;"),
+    # commit: pool written as [page, slot, head] instead of [page, head, slot]
+    "commit_layout": ("const long dst = ((page * Hkv + g) * P + slot) * D;",
+                      "const long dst = ((page * P + slot) * Hkv + g) * D;"),
     # unmask: ascending order
     "unmask_ascending": ("if (ca > cb) return 1;\n    if (ca < cb) return 0;",
                          "if (ca < cb) return 1;\n    if (ca > cb) return 0;"),
