@@ -424,6 +424,7 @@ def run_ours(args, world, rank, local):
         line["workloads"] = run_workloads(torch, nld, dev, stream, peak, l2)
         line["decisions"] = run_decisions(torch, nld, dev, stream)
         line["logits_argmax"] = run_logits(torch, nld, dev, stream, peak, l2)
+        line["kv_commit"] = run_kv_commit(torch, nld, dev, stream)
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, budget_s=12.0)
     print(json.dumps(line), flush=True)
@@ -518,6 +519,35 @@ def time_graph(torch, stream, body, nsteps, reps):
         e1.record(stream)
     torch.cuda.synchronize()
     return e0.elapsed_time(e1) / (reps * nsteps)
+
+
+def run_kv_commit(torch, nld, dev, stream):
+    """nld_kv_commit of one verify step's accepted rows (counts from the accept
+    rule's typical length, advance) at the 8B shape (B=1, bl=16) and for 128
+    sequences (bl=8): us per call; bytes moved = 2 x (read + write) of the
+    committed K/V rows."""
+    res = {}
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(13)
+    for B, bl in ((1, 16), (128, 8)):
+        Hkv, D, P = 8, 128, 16
+        L = 4096
+        pages = (L + bl + P - 1) // P
+        num_pages = B * pages
+        kp = torch.zeros((num_pages, Hkv, P, D), dtype=torch.bfloat16, device=dev)
+        vp = torch.zeros_like(kp)
+        table = torch.arange(num_pages, dtype=torch.int32, device=dev).view(B, pages)
+        prefix = torch.full((B,), L, dtype=torch.int32, device=dev)
+        k_new = torch.randn((B, bl, Hkv, D), generator=gen, device=dev).to(torch.bfloat16)
+        v_new = torch.randn_like(k_new)
+        counts = torch.full((B,), bl, dtype=torch.int32, device=dev)
+        p = nld.make_params(B, 4 * Hkv, Hkv, D, P, num_pages, pages, 0, 0.0, 0)
+        us = time_graph(torch, stream, lambda i: nld.nld_kv_commit(p, k_new, v_new, counts, table, prefix, bl, False,
+                                                                   kp, vp), 64, 10) * 1e3
+        moved = 2 * 2 * B * bl * Hkv * D * 2
+        res[f"b{B}_bl{bl}"] = {"us_per_call": round(us, 3), "gbs_moved": round(moved / (us * 1e-6) / 1e9, 1)}
+    res["timing"] = "CUDA graph of 64 back-to-back calls (no advance, so every call writes the same slots)"
+    return res
 
 
 def run_logits(torch, nld, dev, stream, peak, l2):

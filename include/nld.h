@@ -288,6 +288,43 @@ nld_status_t nld_greedy_accept(const int32_t *pred_ids, const int32_t *target_id
 nld_status_t nld_logits_argmax(const void *logits, int rows, int vocab, int ld, int32_t *ids,
                                float *conf, cudaStream_t stream);
 
+/*
+ * Block KV commit into the paged cache (Sec. 3 Mode 3: the accepted drafts
+ * are committed to the verified prefix and the verifier's cache is rebuilt
+ * at the rejection point; Sec. 2: a completed diffusion block's KV cache is
+ * refreshed). Row j < count_b of the new block K/V is written to logical
+ * slot L_b + j, i.e. page page_table[b][(L_b + j) / P], slot (L_b + j) % P,
+ * for every KV head; with advance != 0, prefix_lens[b] then grows by
+ * count_b. Slots past the committed rows are left untouched (they are no
+ * longer part of the prefix: that is the rollback).
+ *
+ * Uses:
+ *   - before an attention pass, stage the block's own K/V in slots
+ *     [L_b, L_b + bl): counts = NULL, advance = 0;
+ *   - after verification, commit the accepted drafts (the verify pass's K/V
+ *     of those positions): counts = accepted_len from nld_accept, advance = 1
+ *     (the bonus token's K/V comes from the next forward pass);
+ *   - when a diffusion block completes, commit its refreshed K/V:
+ *     counts = NULL, advance = 1.
+ *
+ *   params      shapes as for nld_block_attn (batch, num_kv_heads, head_dim,
+ *               page_size, num_pages, max_pages_per_seq)
+ *   k_new, v_new bf16 [B, block_len, Hkv, D]
+ *   counts      int32 [B] on the device, 0 .. block_len, or NULL (= block_len)
+ *   page_table  int32 [B, max_pages_per_seq], covering the written slots
+ *   prefix_lens int32 [B] on the device (read; updated when advance != 0)
+ *   k_pages, v_pages bf16 [num_pages, Hkv, P, D], written
+ *
+ * Device-side range errors (a count outside 0..block_len, a slot past the
+ * page table, a page id outside the pool) are flagged in nld_device_error
+ * and the row is skipped. The call writes the cache and prefix_lens: an
+ * attention call enqueued after it must not pass NLD_ATTN_PREFIX_READY.
+ */
+nld_status_t nld_kv_commit(const nld_attn_params_t *params, const void *k_new, const void *v_new,
+                           const int32_t *counts, const int32_t *page_table, int32_t *prefix_lens,
+                           int block_len, int advance, void *k_pages, void *v_pages,
+                           cudaStream_t stream);
+
 /* A static, human-readable name for a status code. */
 const char *nld_status_string(nld_status_t status);
 

@@ -391,6 +391,26 @@ nld_status_t nld_logits_argmax(const void* logits, int rows, int vocab, int ld, 
              : NLD_ERR_CUDA;
 }
 
+nld_status_t nld_kv_commit(const nld_attn_params_t* params, const void* k_new, const void* v_new,
+                           const int32_t* counts, const int32_t* page_table, int32_t* prefix_lens, int block_len,
+                           int advance, void* k_pages, void* v_pages, cudaStream_t stream) {
+  nld_status_t st = check_params(params, block_len);
+  if (st != NLD_OK) return st;
+  if (!aligned(k_new, 16) || !aligned(v_new, 16) || !aligned(k_pages, 16) || !aligned(v_pages, 16) ||
+      !aligned(page_table, 4) || !aligned(prefix_lens, 4))
+    return NLD_ERR_INVALID_ARG;
+  if (counts != nullptr && !aligned(counts, 4)) return NLD_ERR_INVALID_ARG;
+  unsigned int* err = nullptr;
+  if ((st = device_state(&err, nullptr)) != NLD_OK) return st;
+  return nld::launch_kv_commit(static_cast<const __nv_bfloat16*>(k_new), static_cast<const __nv_bfloat16*>(v_new),
+                               counts, page_table, prefix_lens, static_cast<__nv_bfloat16*>(k_pages),
+                               static_cast<__nv_bfloat16*>(v_pages), params->batch, params->num_kv_heads,
+                               params->head_dim, params->page_size, params->num_pages, params->max_pages_per_seq,
+                               block_len, advance != 0, err, stream) == cudaSuccess
+             ? NLD_OK
+             : NLD_ERR_CUDA;
+}
+
 nld_status_t nld_device_error(uint32_t* bits, int clear) {
   if (bits == nullptr) return NLD_ERR_INVALID_ARG;
   unsigned int* err = nullptr;

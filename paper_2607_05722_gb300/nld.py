@@ -76,6 +76,8 @@ def lib(path: Optional[str] = None):
     L.nld_greedy_accept.restype = I
     L.nld_logits_argmax.argtypes = [V, I, I, I, V, V, V]
     L.nld_logits_argmax.restype = I
+    L.nld_kv_commit.argtypes = [PP, V, V, V, V, V, I, I, V, V, V]
+    L.nld_kv_commit.restype = I
     L.nld_unmask.restype = I
     L.nld_status_string.argtypes = [I]
     L.nld_status_string.restype = ctypes.c_char_p
@@ -283,6 +285,24 @@ def nld_logits_argmax(logits, ids, conf, vocab=None, stream=None):
     _expect(conf, torch.float32, (rows,), "conf")
     _check(lib().nld_logits_argmax(_ptr(logits), rows, vocab, ld, _ptr(ids), _ptr(conf), _stream(stream)),
            "nld_logits_argmax")
+
+
+def nld_kv_commit(params: AttnParams, k_new, v_new, counts, page_table, prefix_lens, block_len: int, advance: bool,
+                  k_pages, v_pages, stream=None):
+    """Write rows j < counts[b] (all block_len rows when counts is None) of the
+    block K/V [B, bl, Hkv, D] to slots prefix_lens[b] + j; advance the prefix."""
+    B, Hkv, D, P = params.batch, params.num_kv_heads, params.head_dim, params.page_size
+    _expect(k_new, torch.bfloat16, (B, block_len, Hkv, D), "k_new")
+    _expect(v_new, torch.bfloat16, (B, block_len, Hkv, D), "v_new")
+    if counts is not None:
+        _expect(counts, torch.int32, (B,), "counts")
+    _expect(page_table, torch.int32, (B, params.max_pages_per_seq), "page_table")
+    _expect(prefix_lens, torch.int32, (B,), "prefix_lens")
+    _expect(k_pages, torch.bfloat16, (params.num_pages, Hkv, P, D), "k_pages")
+    _expect(v_pages, torch.bfloat16, (params.num_pages, Hkv, P, D), "v_pages")
+    _check(lib().nld_kv_commit(ctypes.byref(params), _ptr(k_new), _ptr(v_new), _ptr(counts), _ptr(page_table),
+                               _ptr(prefix_lens), int(block_len), int(bool(advance)), _ptr(k_pages), _ptr(v_pages),
+                               _stream(stream)), "nld_kv_commit")
 
 def nld_device_error(clear: bool = False) -> int:
     bits = ctypes.c_uint32(0)

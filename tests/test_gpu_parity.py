@@ -143,6 +143,123 @@ def test_greedy_accept_chain(orc):
 
 
 # ---------------------------------------------------------------------------
+# block KV commit
+# ---------------------------------------------------------------------------
+
+def bits_dev(bits):
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).cuda()
+
+
+def dev_bits(t):
+    return t.cpu().view(torch.int16).numpy().view(np.uint16)
+
+
+def commit_case(seed, B=3, Hq=8, Hkv=2, D=128, P=16, bl=12, prefix=(40, 3, 100)):
+    rng = np.random.default_rng(seed)
+    case = W.make_block_attn_case("commit", B, Hq, Hkv, D, block_len=bl, page_size=P, prefix_lens=list(prefix),
+                                  seed=seed)
+    shape = (B, bl, Hkv, D)
+    k_new = W.f32_to_bf16_bits(rng.standard_normal(shape).astype(np.float32))
+    v_new = W.f32_to_bf16_bits(rng.standard_normal(shape).astype(np.float32))
+    return rng, case, k_new, v_new
+
+
+def gpu_commit(case, k_new, v_new, counts, advance, k_bits=None, v_bits=None, prefix=None, table=None):
+    kv = case.kv
+    p = nld.make_params(case.batch, case.num_q_heads, case.num_kv_heads, case.head_dim, case.page_size,
+                        kv.num_pages, kv.max_pages, 0, 0.0, 0)
+    kp = bits_dev(kv.k_bits if k_bits is None else k_bits)
+    vp = bits_dev(kv.v_bits if v_bits is None else v_bits)
+    pl = torch.from_numpy(np.array(kv.prefix_lens if prefix is None else prefix, np.int32)).cuda()
+    cnt = None if counts is None else torch.from_numpy(np.asarray(counts, np.int32)).cuda()
+    tab = torch.from_numpy(np.ascontiguousarray(kv.page_table if table is None else table, np.int32)).cuda()
+    nld.nld_kv_commit(p, bits_dev(k_new), bits_dev(v_new), cnt, tab, pl,
+                      case.block_len, advance, kp, vp)
+    return dev_bits(kp), dev_bits(vp), pl.cpu().numpy()
+
+
+@pytest.mark.parametrize("D,P", [(128, 16), (64, 32), (128, 256)])
+def test_kv_commit_matches_oracle(orc, D, P):
+    rng, case, k_new, v_new = commit_case(D + P, D=D, P=P)
+    kv = case.kv
+    for counts, advance in ((None, False), (None, True), (rng.integers(0, case.block_len + 1, case.batch), True),
+                            (np.array([0, case.block_len, 5]), False)):
+        g = gpu_commit(case, k_new, v_new, counts, advance)
+        o = orc.kv_commit(k_new, v_new, counts, kv.page_table, kv.prefix_lens, kv.k_bits, kv.v_bits, advance)
+        for x, y, what in zip(g, o, ("k_pages", "v_pages", "prefix_lens")):
+            assert np.array_equal(x, y), f"{what} counts={counts} advance={advance}"
+
+
+def test_kv_commit_staged_block_attention(orc):
+    """The block's K/V staged by nld_kv_commit is what nld_block_attn reads:
+    bit-identical to attention over pools staged on the host by the oracle,
+    and within tolerance of the oracle's attention."""
+    _, case, k_new, v_new = commit_case(5)
+    kv = case.kv
+    kp, vp, _ = gpu_commit(case, k_new, v_new, None, False)
+    okp, ovp, _ = orc.kv_commit(k_new, v_new, None, kv.page_table, kv.prefix_lens, kv.k_bits, kv.v_bits, False)
+    assert np.array_equal(kp, okp) and np.array_equal(vp, ovp)
+    p = nld.make_params(case.batch, case.num_q_heads, case.num_kv_heads, case.head_dim, case.page_size,
+                        kv.num_pages, kv.max_pages, 0, 0.0, 0)
+    for mode, qb in ((DIFF, case.q_draft_bits), (VER, case.q_verify_bits)):
+        out = torch.empty((case.batch, case.block_len, case.num_q_heads, case.head_dim), dtype=torch.bfloat16,
+                          device="cuda")
+        lse = torch.empty((case.batch, case.num_q_heads, case.block_len), dtype=torch.float32, device="cuda")
+        ws = torch.empty(max(16, nld.nld_block_attn_workspace_size(p, case.block_len)), dtype=torch.uint8,
+                         device="cuda")
+        nld.nld_block_attn(p, bits_dev(qb), bits_dev(kp), bits_dev(vp), torch.from_numpy(kv.page_table).cuda(),
+                           torch.from_numpy(kv.prefix_lens).cuda(), case.block_len, mode, out, lse, ws)
+        ro, rl = orc.block_attn(qb, okp, ovp, kv.page_table, kv.prefix_lens, case.num_q_heads, case.num_kv_heads,
+                                case.block_len, mode, case.scale)
+        compare_attn(out, lse, ro, rl, f"staged block mode={mode}")
+
+
+def test_kv_commit_verify_chain(orc):
+    """Three verify steps: accept on the GPU, commit the accepted rows and
+    advance; pools and prefix lengths equal the oracle's chain."""
+    rng, case, _, _ = commit_case(6, prefix=(0, 17, 33))
+    kv = case.kv
+    gk, gv, gl = kv.k_bits.copy(), kv.v_bits.copy(), kv.prefix_lens.copy()
+    ok, ov, ol = kv.k_bits.copy(), kv.v_bits.copy(), kv.prefix_lens.copy()
+    cap = kv.max_pages * case.page_size
+    for _ in range(3):
+        shape = (case.batch, case.block_len, case.num_kv_heads, case.head_dim)
+        k_new = W.f32_to_bf16_bits(rng.standard_normal(shape).astype(np.float32))
+        v_new = W.f32_to_bf16_bits(rng.standard_normal(shape).astype(np.float32))
+        d, v = W.make_accept_ids(rng, case.batch, case.block_len, 131072, 0.7)
+        acc = np.minimum(gpu_accept(d, v), cap - gl).astype(np.int32)
+        assert np.array_equal(acc, np.minimum(orc.accept(d, v), cap - ol))
+        gk, gv, gl = gpu_commit(case, k_new, v_new, acc, True, gk, gv, gl)
+        ok, ov, ol = orc.kv_commit(k_new, v_new, acc, kv.page_table, ol, ok, ov, True)
+        assert np.array_equal(gk, ok) and np.array_equal(gv, ov) and np.array_equal(gl, ol)
+
+
+def test_kv_commit_range_flags(orc):
+    """Counts past the block, a slot past the page table and a page id outside
+    the pool are flagged on the device; those rows are not written."""
+    _, case, k_new, v_new = commit_case(7)
+    kv = case.kv
+    err = nld.nld_device_error(clear=True)
+    kp, vp, pl = gpu_commit(case, k_new, v_new, np.array([case.block_len + 3, 0, 0]), False)
+    err = nld.nld_device_error(clear=True)
+    assert err & nld.NLD_DEVERR_PREFIX_RANGE
+    okp, _, _ = orc.kv_commit(k_new, v_new, np.array([case.block_len, 0, 0]), kv.page_table, kv.prefix_lens,
+                              kv.k_bits, kv.v_bits, False)
+    assert np.array_equal(kp, okp), "an oversized count is clamped to the block"
+    far = kv.prefix_lens.copy()
+    far[1] = kv.max_pages * case.page_size  # every row of sequence 1 past the table
+    kp, _, _ = gpu_commit(case, k_new, v_new, np.array([0, 4, 0]), False, prefix=far)
+    assert nld.nld_device_error(clear=True) & nld.NLD_DEVERR_PREFIX_RANGE
+    assert np.array_equal(kp, kv.k_bits), "nothing written"
+    bad = kv.page_table.copy()
+    L2 = int(kv.prefix_lens[2])
+    bad[2, L2 // case.page_size] = kv.num_pages + 5  # the page of sequence 2's first block slot
+    kp, _, _ = gpu_commit(case, k_new, v_new, np.array([0, 0, 1]), False, table=bad)
+    assert nld.nld_device_error(clear=True) & nld.NLD_DEVERR_PAGE_RANGE
+    assert np.array_equal(kp, kv.k_bits), "nothing written"
+
+
+# ---------------------------------------------------------------------------
 # logits -> (argmax id, confidence)
 # ---------------------------------------------------------------------------
 
