@@ -77,6 +77,10 @@ class Oracle:
         lib.nldo_logits_argmax.restype = None
         lib.nldo_kv_commit.argtypes = [P, P, P, P, P, I, P, P, I, I, I, I, I, I, I]
         lib.nldo_kv_commit.restype = None
+        lib.nldo_block_attn_masked.argtypes = [P, P, P, P, P, I, I, I, I, I, I, I, I, P, D, P, P, P, Lg]
+        lib.nldo_block_attn_masked.restype = I
+        lib.nldo_quadss_mask.argtypes = [I, P]
+        lib.nldo_quadss_mask.restype = I
         lib.nldo_max_threads.argtypes = []
         lib.nldo_max_threads.restype = I
         self.lib = lib
@@ -182,6 +186,37 @@ class Oracle:
         conf = np.zeros((rows,), dtype=np.float64)
         self.lib.nldo_logits_argmax(self._p(lb), rows, vocab, ld, self._p(ids), self._p(conf))
         return ids, conf
+
+    def quadss_mask(self, k):
+        """uint32 [1 + k + k^2] block masks of quadratic self-speculation (bit j: slot j visible)."""
+        out = np.zeros((32,), dtype=np.uint32)
+        n = self.lib.nldo_quadss_mask(int(k), self._p(out))
+        if n < 0:
+            raise ValueError(f"k={k}: block of 1 + k + k^2 slots exceeds 32")
+        return out[:n].copy()
+
+    def block_attn_masked(self, q_bits, k_bits, v_bits, page_table, prefix_lens, num_q_heads, num_kv_heads,
+                          block_len, block_mask, scale, want_probs=False):
+        """Block attention whose block part follows block_mask (uint32 [bl]);
+        (out [B, bl, Hq, D], lse [B, Hq, bl], probs or None) in fp64."""
+        q = np.ascontiguousarray(q_bits, dtype=np.uint16)
+        k = np.ascontiguousarray(k_bits, dtype=np.uint16)
+        v = np.ascontiguousarray(v_bits, dtype=np.uint16)
+        table = np.ascontiguousarray(page_table, dtype=np.int32)
+        pl = np.ascontiguousarray(prefix_lens, dtype=np.int32)
+        bm = np.ascontiguousarray(block_mask, dtype=np.uint32)
+        B, bl, Hq, D = q.shape
+        num_pages, Hkv, P, _ = k.shape
+        out = np.zeros((B, bl, Hq, D), dtype=np.float64)
+        lse = np.zeros((B, Hq, bl), dtype=np.float64)
+        stride = int(pl.max() + bl) if B else 1
+        probs = np.zeros((B, Hq, bl, stride), dtype=np.float64) if want_probs else None
+        rc = self.lib.nldo_block_attn_masked(self._p(q), self._p(k), self._p(v), self._p(table), self._p(pl),
+                                             B, Hq, Hkv, D, P, num_pages, table.shape[1], bl, self._p(bm),
+                                             float(scale), self._p(out), self._p(lse), self._p(probs), stride)
+        if rc != 0:
+            raise RuntimeError(f"nldo_block_attn_masked failed ({rc})")
+        return out, lse, probs
 
     def kv_commit(self, k_new_bits, v_new_bits, counts, page_table, prefix_lens, k_bits, v_bits, advance):
         """Commit rows of a [B, bl, Hkv, D] K/V block into copies of the page

@@ -36,6 +36,9 @@
  *    inputs of the two decisions (Sec. 2; Sec. 5).
  *  - Block KV commit into the paged slots after the prefix, with the prefix
  *    advanced by the committed rows (Sec. 3 Mode 3; Sec. 2 block refresh).
+ *  - Block attention with a table mask over the block slots, and the
+ *    structured mask of quadratic self-speculation (Sec. 3 variant; appendix
+ *    Eq. quad_input) as one such table.
  *
  * Build: gcc -O2 -fopenmp -ffp-contract=off -shared -fPIC (see build.py).
  */
@@ -62,13 +65,17 @@ static double bf16_to_f64(uint16_t bits)
     return (double)f;
 }
 
-/* Mask of Sec. 2.2 / Sec. 3 for block row i (0-based) and logical key t. */
-static int key_visible(long t, long L, int bl, int i, int mode)
+/* Mask of Sec. 2.2 / Sec. 3 for block row i (0-based) and logical key t.
+ * Mode 2 takes the block part from a table: bit j of bm[i] makes block slot j
+ * visible to row i (the structured mask of quadratic self-speculation,
+ * Sec. 3 variant, is one such table). */
+static int key_visible(long t, long L, int bl, int i, int mode, const uint32_t *bm)
 {
     if (t < L) return 1;             /* clean prefix: always visible */
     long j = t - L;                  /* block slot of key t */
     if (j >= bl) return 0;           /* slots past the block hold nothing */
     if (mode == 0) return 1;         /* diffusion draft: bidirectional */
+    if (mode == 2) return (int)((bm[i] >> j) & 1u);
     return j <= i;                   /* AR verify: causal, self included */
 }
 
@@ -91,7 +98,7 @@ int nldo_max_threads(void)
 static int attn_row(const uint16_t *q, const uint16_t *k, const uint16_t *v,
                     const int32_t *page_table, long L, int b, int i, int h,
                     int Hq, int Hkv, int D, int P, int num_pages, int max_pages,
-                    int bl, int mode, double scale, long key_begin, long key_end,
+                    int bl, int mode, const uint32_t *bm, double scale, long key_begin, long key_end,
                     double *s, char *use, double *o, double *lse, double *probs)
 {
     const int G = Hq / Hkv;
@@ -102,7 +109,7 @@ static int attn_row(const uint16_t *q, const uint16_t *k, const uint16_t *v,
     long nuse = 0;
 
     for (long t = 0; t < N; ++t) {
-        use[t] = key_visible(t, L, bl, i, mode) && t >= key_begin && (key_end < 0 || t < key_end);
+        use[t] = key_visible(t, L, bl, i, mode, bm) && t >= key_begin && (key_end < 0 || t < key_end);
         if (!use[t]) continue;
         long lp = t / P;
         if (lp >= max_pages) return NLDO_ERR_PAGE;
@@ -141,7 +148,7 @@ static int check_shape(int B, int Hq, int Hkv, int D, int P, int bl, int mode)
 {
     if (B < 0 || Hq <= 0 || Hkv <= 0 || D <= 0 || P <= 0 || bl <= 0) return 0;
     if (Hq % Hkv != 0) return 0;
-    if (mode != 0 && mode != 1) return 0;
+    if (mode != 0 && mode != 1 && !(mode == 2 && bl <= 32)) return 0;
     return 1;
 }
 
@@ -151,13 +158,14 @@ static int check_shape(int B, int Hq, int Hkv, int D, int P, int bl, int mode)
  * out [B, bl, Hq, D], lse [B, Hq, bl] (fp64). probs: NULL, or
  * [B, Hq, bl, probs_stride] with probs_stride >= max_b (L_b + bl).
  */
-int nldo_block_attn(const uint16_t *q, const uint16_t *k, const uint16_t *v,
-                    const int32_t *page_table, const int32_t *prefix_lens,
-                    int B, int Hq, int Hkv, int D, int P, int num_pages, int max_pages,
-                    int bl, int mode, double scale, long key_begin, long key_end,
-                    double *out, double *lse, double *probs, long probs_stride)
+static int block_attn_all(const uint16_t *q, const uint16_t *k, const uint16_t *v,
+                          const int32_t *page_table, const int32_t *prefix_lens,
+                          int B, int Hq, int Hkv, int D, int P, int num_pages, int max_pages,
+                          int bl, int mode, const uint32_t *bm, double scale, long key_begin, long key_end,
+                          double *out, double *lse, double *probs, long probs_stride)
 {
     if (!check_shape(B, Hq, Hkv, D, P, bl, mode)) return NLDO_ERR_ARGS;
+    if (mode == 2 && bm == NULL) return NLDO_ERR_ARGS;
     long maxN = 0;
     for (int b = 0; b < B; ++b) {
         if (prefix_lens[b] < 0) return NLDO_ERR_ARGS;
@@ -182,7 +190,7 @@ int nldo_block_attn(const uint16_t *q, const uint16_t *k, const uint16_t *v,
                     double l_out;
                     double *p = probs ? probs + ((bh * bl) + i) * probs_stride : NULL;
                     int rc = attn_row(q, k, v, page_table, prefix_lens[b], b, i, h, Hq, Hkv, D, P,
-                                      num_pages, max_pages, bl, mode, scale, key_begin, key_end,
+                                      num_pages, max_pages, bl, mode, bm, scale, key_begin, key_end,
                                       s, use, o, &l_out, p);
                     if (rc != NLDO_OK) {
 #pragma omp atomic write
@@ -200,6 +208,30 @@ int nldo_block_attn(const uint16_t *q, const uint16_t *k, const uint16_t *v,
     return status;
 }
 
+int nldo_block_attn(const uint16_t *q, const uint16_t *k, const uint16_t *v,
+                    const int32_t *page_table, const int32_t *prefix_lens,
+                    int B, int Hq, int Hkv, int D, int P, int num_pages, int max_pages,
+                    int bl, int mode, double scale, long key_begin, long key_end,
+                    double *out, double *lse, double *probs, long probs_stride)
+{
+    if (mode == 2) return NLDO_ERR_ARGS;  /* the table form has its own entry */
+    return block_attn_all(q, k, v, page_table, prefix_lens, B, Hq, Hkv, D, P, num_pages, max_pages, bl,
+                          mode, NULL, scale, key_begin, key_end, out, lse, probs, probs_stride);
+}
+
+/* Block attention whose block part follows a table: bit j of block_mask[i]
+ * makes block slot j visible to block row i (bl <= 32); the prefix is
+ * fully visible as in every mode. */
+int nldo_block_attn_masked(const uint16_t *q, const uint16_t *k, const uint16_t *v,
+                           const int32_t *page_table, const int32_t *prefix_lens,
+                           int B, int Hq, int Hkv, int D, int P, int num_pages, int max_pages,
+                           int bl, const uint32_t *block_mask, double scale,
+                           double *out, double *lse, double *probs, long probs_stride)
+{
+    return block_attn_all(q, k, v, page_table, prefix_lens, B, Hq, Hkv, D, P, num_pages, max_pages, bl,
+                          2, block_mask, scale, 0, -1, out, lse, probs, probs_stride);
+}
+
 /*
  * Block attention for selected rows only: rows[r] = (b, i, h) triples.
  * out [nrows, D], lse [nrows].
@@ -210,7 +242,7 @@ int nldo_block_attn_rows(const uint16_t *q, const uint16_t *k, const uint16_t *v
                          int bl, int mode, double scale, long nsel, const int32_t *rows,
                          double *out, double *lse)
 {
-    if (!check_shape(B, Hq, Hkv, D, P, bl, mode)) return NLDO_ERR_ARGS;
+    if (!check_shape(B, Hq, Hkv, D, P, bl, mode) || mode == 2) return NLDO_ERR_ARGS;
     long maxN = 0;
     for (int b = 0; b < B; ++b)
         if ((long)prefix_lens[b] + bl > maxN) maxN = (long)prefix_lens[b] + bl;
@@ -232,7 +264,7 @@ int nldo_block_attn_rows(const uint16_t *q, const uint16_t *k, const uint16_t *v
                     continue;
                 }
                 int rc = attn_row(q, k, v, page_table, prefix_lens[b], b, i, h, Hq, Hkv, D, P,
-                                  num_pages, max_pages, bl, mode, scale, 0, -1,
+                                  num_pages, max_pages, bl, mode, NULL, scale, 0, -1,
                                   s, use, out + r * (long)D, lse + r, NULL);
                 if (rc != NLDO_OK) {
 #pragma omp atomic write
@@ -455,4 +487,50 @@ void nldo_kv_commit(const uint16_t *k_new, const uint16_t *v_new, const int32_t 
         }
         if (advance) prefix_lens[b] = (int32_t)(L + count);
     }
+}
+
+/*
+ * The block layout and mask of quadratic self-speculation (Sec. 3 variant;
+ * appendix, Eq. quad_input): after the verified prefix come the AR token
+ * x_{n+1}, then k groups, each a speculative token x^t_{n+g+1} followed by k
+ * fresh mask tokens: 1 + k + k^2 block slots. Reading of the structured
+ * mask: the speculative chain (x_{n+1} and the k speculative tokens) is
+ * causal among itself and sees no mask token, so its predictions verify the
+ * previous drafts; the k masks of group g see the chain up to their own
+ * speculative token and, bidirectionally, the masks of their group, so they
+ * draft the next block for the case that verification accepts up to that
+ * token. Writes masks[0 .. 1+k+k^2-1] (bit j: slot j visible); returns the
+ * block length, or -1 when it exceeds 32 slots.
+ */
+int nldo_quadss_mask(int k, uint32_t *masks)
+{
+    const int n = 1 + k + k * k;
+    if (k < 1 || n > 32) return -1;
+    /* group of slot j: 0 for the AR token, g for the speculative token of
+     * group g and for its masks; chain slots are the AR and speculative ones */
+    int group[32], chain[32];
+    group[0] = 0;
+    chain[0] = 1;
+    for (int g = 1; g <= k; ++g) {
+        const int spec = 1 + (g - 1) * (k + 1);
+        group[spec] = g;
+        chain[spec] = 1;
+        for (int r = 1; r <= k; ++r) {
+            group[spec + r] = g;
+            chain[spec + r] = 0;
+        }
+    }
+    for (int i = 0; i < n; ++i) {
+        uint32_t bits = 0;
+        for (int j = 0; j < n; ++j) {
+            int vis;
+            if (chain[i])
+                vis = chain[j] && j <= i;
+            else
+                vis = (chain[j] && group[j] <= group[i]) || (!chain[j] && group[j] == group[i]);
+            if (vis) bits |= 1u << j;
+        }
+        masks[i] = bits;
+    }
+    return n;
 }

@@ -707,6 +707,93 @@ def pin_commit_rollback_chain(orc):
         assert np.array_equal(got, np.array(history[b]).reshape(got.shape))
 
 
+# --------------------------------------------------------------------------
+# table-mask attention and the quadratic self-speculation mask
+# --------------------------------------------------------------------------
+
+def pin_quadss_layout(orc):
+    """Eq. quad_input: 1 + k + k^2 block slots, k^2 of them masks. Chain slots
+    (the AR token and the k speculative tokens) see only chain slots, causally;
+    the masks of a group see the chain through their speculative token and
+    exactly the k masks of their group; every slot sees itself."""
+    for k in range(1, 6):
+        m = orc.quadss_mask(k)
+        n = 1 + k + k * k
+        assert len(m) == n
+        bits = [[(int(m[i]) >> j) & 1 for j in range(n)] for i in range(n)]
+        spec = [0] + [1 + (g - 1) * (k + 1) for g in range(1, k + 1)]
+        masks = [j for j in range(n) if j not in spec]
+        assert len(masks) == k * k
+        for i in range(n):
+            assert bits[i][i] == 1
+            if i in spec:
+                assert [j for j in range(n) if bits[i][j]] == [j for j in spec if j <= i]
+            else:
+                g = (i - 1) // (k + 1) + 1
+                own = [spec[g] + r for r in range(1, k + 1)]
+                assert [j for j in masks if bits[i][j]] == own
+                assert [j for j in spec if bits[i][j]] == spec[:g + 1]
+    assert all(orc.quadss_mask(5) < 2 ** 31) and len(orc.quadss_mask(5)) == 31
+    try:
+        orc.quadss_mask(6)
+        raise AssertionError("k=6 (43 slots) must be refused")
+    except ValueError:
+        pass
+
+
+def pin_masked_reduces_to_modes(orc):
+    """A table of all ones is the diffusion pass; the lower-triangular table
+    is the verify pass (bit-identical: same arithmetic in the same order)."""
+    for seed, prefix in ((41, (7, 12)), (42, (0, 5))):
+        case = small_case(seed, prefix=prefix)
+        bl = case.block_len
+        full = np.full(bl, (1 << bl) - 1, dtype=np.uint32)
+        tril = np.array([(2 << i) - 1 for i in range(bl)], dtype=np.uint32)
+        for table, mode, qb in ((full, DIFF, case.q_draft_bits), (tril, VER, case.q_verify_bits)):
+            ref, rl = orc.block_attn(qb, case.kv.k_bits, case.kv.v_bits, case.kv.page_table, case.kv.prefix_lens,
+                                     case.num_q_heads, case.num_kv_heads, bl, mode, case.scale)
+            got, gl, _ = orc.block_attn_masked(qb, case.kv.k_bits, case.kv.v_bits, case.kv.page_table,
+                                               case.kv.prefix_lens, case.num_q_heads, case.num_kv_heads, bl,
+                                               table, case.scale)
+            assert np.array_equal(got, ref) and np.array_equal(gl, rl), f"mode {mode}"
+
+
+def pin_quadss_against_sdpa(orc):
+    """Quadratic-SS attention row by row against fp64 SDPA on exactly the keys
+    the reading names: a chain row = causal attention along the prefix and
+    the chain; a mask row of group g = unmasked attention over the prefix, the
+    chain through its speculative token and its group's masks."""
+    for k, prefix in ((2, (5, 9)), (3, (0, 14)), (5, (6, 1))):
+        bl = 1 + k + k * k
+        case = W.make_block_attn_case("quadss", 2, 4, 2, 16, bl, 4, list(prefix), 60 + k, shuffle_pages=True)
+        table = orc.quadss_mask(k)
+        out, _, _ = orc.block_attn_masked(case.q_draft_bits, case.kv.k_bits, case.kv.v_bits, case.kv.page_table,
+                                          case.kv.prefix_lens, case.num_q_heads, case.num_kv_heads, bl, table,
+                                          case.scale)
+        G = case.num_q_heads // case.num_kv_heads
+        for b in range(case.batch):
+            L = int(case.kv.prefix_lens[b])
+            kf, vf = gather_contiguous(case, b)  # [Hkv, L + bl, D]
+            q = np.transpose(q_f64(case.q_draft_bits[b]), (1, 0, 2))  # [Hq, bl, D]
+            for i in range(bl):
+                keys = list(range(L)) + [L + j for j in range(bl) if (int(table[i]) >> j) & 1]
+                ref = sdpa(q[:, i:i + 1], repeat_heads(kf[:, keys], G), repeat_heads(vf[:, keys], G), case.scale)
+                assert_close(out[b, i], ref[:, 0], 1e-12, f"quadss k={k} b={b} row {i}")
+
+
+def pin_masked_empty_row(orc):
+    """With no prefix, a row whose table entry is empty sees no key: o = 0, lse = -inf."""
+    case = small_case(43, prefix=(0, 0))
+    bl = case.block_len
+    table = np.array([(2 << i) - 1 for i in range(bl)], dtype=np.uint32)
+    table[2] = 0
+    out, lse, _ = orc.block_attn_masked(case.q_draft_bits, case.kv.k_bits, case.kv.v_bits, case.kv.page_table,
+                                        case.kv.prefix_lens, case.num_q_heads, case.num_kv_heads, bl, table,
+                                        case.scale)
+    assert np.all(out[:, 2] == 0) and np.all(lse[:, :, 2] == -np.inf)
+    assert np.all(np.isfinite(lse[:, :, [0, 1, 3]]))
+
+
 ATTENTION_PINS = [pin_decode_bl1, pin_diffusion_full_attention, pin_verify_causal_tail, pin_lse_logsumexp,
                   pin_softmax_rows, pin_page_permutation, pin_block_permutation, pin_closed_forms,
                   pin_golden_uniform, pin_split_combine]
@@ -715,4 +802,5 @@ DECISION_PINS = [pin_accept_golden, pin_accept_brute, pin_accept_statistics, pin
                  pin_threshold_limits, pin_greedy_golden, pin_greedy_brute, pin_greedy_chain]
 LOGITS_PINS = [pin_logits_golden, pin_logits_scipy, pin_logits_closed_forms, pin_logits_brute]
 COMMIT_PINS = [pin_commit_gather, pin_commit_then_attention, pin_commit_rollback_chain]
-ALL_PINS = ATTENTION_PINS + DECISION_PINS + LOGITS_PINS + COMMIT_PINS
+MASK_PINS = [pin_quadss_layout, pin_masked_reduces_to_modes, pin_quadss_against_sdpa, pin_masked_empty_row]
+ALL_PINS = ATTENTION_PINS + DECISION_PINS + LOGITS_PINS + COMMIT_PINS + MASK_PINS

@@ -86,6 +86,14 @@ MUTANTS = {
     # commit: pool written as [page, slot, head] instead of [page, head, slot]
     "commit_layout": ("const long dst = ((page * Hkv + g) * P + slot) * D;",
                       "const long dst = ((page * P + slot) * Hkv + g) * D;"),
+    # quadratic SS: the chain also sees mask slots
+    "quadss_chain_sees_masks": ("vis = chain[j] && j <= i;", "vis = j <= i;"),
+    # quadratic SS: a mask sees the masks of every group
+    "quadss_all_groups": ("(!chain[j] && group[j] == group[i])", "(!chain[j])"),
+    # quadratic SS: a mask sees the whole chain
+    "quadss_whole_chain": ("(chain[j] && group[j] <= group[i])", "chain[j]"),
+    # table mode ignores the table
+    "masked_ignores_table": ("if (mode == 2) return (int)((bm[i] >> j) & 1u);", "if (mode == 2) return 1;"),
     # unmask: ascending order
     "unmask_ascending": ("if (ca > cb) return 1;\n    if (ca < cb) return 0;",
                          "if (ca < cb) return 1;\n    if (ca > cb) return 0;"),
