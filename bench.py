@@ -46,7 +46,7 @@ PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_HBM_GBS = 6800.0
 TRAFFIC_NOTE = os.path.join(ROOT, "profiles", "block_attn_8b_b1_L4096_bl16.md")
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2607_05722_gb300", "csrc", f)
-                  for f in ("block_attn_tc.cu", "nld_internal.cuh")]
+                  for f in ("block_attn_tc.cuh", "nld_internal.cuh")]
 
 
 def parse_args():
@@ -425,6 +425,7 @@ def run_ours(args, world, rank, local):
         line["decisions"] = run_decisions(torch, nld, dev, stream)
         line["logits_argmax"] = run_logits(torch, nld, dev, stream, peak, l2)
         line["kv_commit"] = run_kv_commit(torch, nld, dev, stream)
+        line["quadss_pass"] = run_quadss(torch, nld, dev, stream, peak, l2)
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, budget_s=12.0)
     print(json.dumps(line), flush=True)
@@ -519,6 +520,45 @@ def time_graph(torch, stream, body, nsteps, reps):
         e1.record(stream)
     torch.cuda.synchronize()
     return e0.elapsed_time(e1) / (reps * nsteps)
+
+
+def run_quadss(torch, nld, dev, stream, peak, l2):
+    """One quadratic self-speculation pass (Sec. 3 variant: drafting and
+    verification in one forward with the structured mask) at the 8B shape
+    (B=1, 32/8 heads, D=128, 4096-token prefix) for k = 3 and 5 (13 and 31
+    block slots), next to a verify pass of the same block length: us per
+    pass and KV GB/s over rotating cold pools."""
+    res = {}
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(17)
+    B, Hq, Hkv, D, P, L = 1, 32, 8, 128, 16, 4096
+    for k in (3, 5):
+        bl = 1 + k + k * k
+        pages = (L + bl + P - 1) // P
+        kvb = (L + bl) * Hkv * D * 2 * 2
+        npool = int(max(2, np.ceil(3 * l2 / kvb)))
+        pools = [(torch.randn((pages, Hkv, P, D), generator=gen, device=dev).to(torch.bfloat16),
+                  torch.randn((pages, Hkv, P, D), generator=gen, device=dev).to(torch.bfloat16)) for _ in range(npool)]
+        table = torch.randperm(pages, generator=gen, device=dev).to(torch.int32).view(1, pages)
+        prefix = torch.full((B,), L, dtype=torch.int32, device=dev)
+        q = torch.randn((B, bl, Hq, D), generator=gen, device=dev).to(torch.bfloat16)
+        out = torch.empty_like(q)
+        p = nld.make_params(B, Hq, Hkv, D, P, pages, pages, 0, 0.0, 0)
+        ws = torch.empty(max(16, nld.nld_block_attn_workspace_size(p, bl)), dtype=torch.uint8, device=dev)
+        bm = torch.from_numpy(nld.nld_quadss_block_mask(k).view(np.int32)).to(dev)
+        masked = lambda i: nld.nld_block_attn_masked(p, q, pools[i % npool][0], pools[i % npool][1], table, prefix, bl,
+                                                     bm, out, None, ws)
+        verify = lambda i: nld.nld_block_attn(p, q, pools[i % npool][0], pools[i % npool][1], table, prefix, bl,
+                                              nld.NLD_MODE_VERIFY, out, None, ws)
+        us_m = time_graph(torch, stream, masked, 2 * npool, 10) * 1e3
+        us_v = time_graph(torch, stream, verify, 2 * npool, 10) * 1e3
+        res[f"k{k}_bl{bl}"] = {"quadss_us_per_pass": round(us_m, 3), "verify_us_per_pass": round(us_v, 3),
+                               "quadss_kv_gbs": round(kvb / (us_m * 1e-6) / 1e9, 1),
+                               "quadss_pct_of_hbm_peak": round(100 * kvb / (us_m * 1e-6) / 1e9 / peak, 2),
+                               "kv_bytes_per_pass": kvb}
+        del pools
+    res["timing"] = "CUDA graph of back-to-back passes over rotating cold KV pools (attention + combine)"
+    return res
 
 
 def run_kv_commit(torch, nld, dev, stream):

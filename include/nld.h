@@ -169,6 +169,36 @@ nld_status_t nld_block_attn_partials(const nld_attn_params_t *params, const void
                                      cudaStream_t stream);
 
 /*
+ * nld_block_attn with the block part of the mask from a table, for
+ * structured masks such as quadratic self-speculation's (Sec. 3 variant):
+ * key t is visible to block row i when t < L_b (the prefix, as always), or
+ * t = L_b + j with bit j of block_mask[i] set. A row that sees no key (no
+ * prefix and an empty table entry) gets out = 0 and lse = -inf.
+ *
+ *   block_mask  uint32 [block_len] on the device (block_len <= 32)
+ *   other arguments as for nld_block_attn
+ */
+nld_status_t nld_block_attn_masked(const nld_attn_params_t *params, const void *q_block,
+                                   const void *k_pages, const void *v_pages,
+                                   const int32_t *page_table, const int32_t *prefix_lens,
+                                   int block_len, const uint32_t *block_mask, void *out, float *lse,
+                                   void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/*
+ * The block layout and table mask of quadratic self-speculation (Sec. 3
+ * variant; appendix Eq. quad_input), host side: after the prefix come the AR
+ * token x_{n+1} (slot 0) and k groups, each a speculative token followed by
+ * k fresh mask tokens (slots 1+g(k+1) .. 1+g(k+1)+k): 1 + k + k^2 slots.
+ * The speculative chain (the AR token and the speculative tokens) is causal
+ * and sees no mask token (its predictions verify the previous drafts); the
+ * masks of a group see the chain up to their speculative token and their
+ * own group's masks (they draft the next block in case verification accepts
+ * up to that token). Writes masks[0 .. 1+k+k^2-1]; returns 1+k+k^2, or -1
+ * when k < 1 or the block would exceed 32 slots (k > 5).
+ */
+int nld_quadss_block_mask(int k, uint32_t *masks);
+
+/*
  * nld_block_attn for callers that cannot allocate device memory (the paper
  * has no counterpart: this is a deployment convenience of this library).
  * Plugins running inside another runtime's enqueue step, code bound to a

@@ -1,835 +1,9 @@
-// Block attention over a paged bf16 KV cache on the 5th-generation tensor
-// cores (tcgen05, accumulators in tensor memory), for up to 256 packed query
-// rows (Sec. 2.2 mask; Sec. 3 Modes 2 and 3).
-//
-// One CTA serves one (KV split, KV head g, sequence b): its G = Hq/Hkv query
-// heads times the bl block tokens form R = G*bl <= 256 query rows in one or
-// two 128-row MMA tiles, so each K/V page leaves HBM once per (b, g).
-//
-// Warp roles (9 warps):
-//   warps 0-2, 8  TMA producers: the boxes of each 64-token K/V tile (16 tokens
-//             x 64 dims each) dealt four ways into a 4-stage ring (produce_kv);
-//             TMA issue cost is per warp, so four issuing warps land a tile
-//             sooner.
-//   warp 3    allocates the TMEM columns; lane 0 issues every MMA:
-//               S_k = Q K_k^T   (M=128 rows, N=64 tokens, K=D; double-buffered in TMEM)
-//               O  += P_k V_k   (M=128 rows, N=D, K=64 tokens; V read MN-major)
-//             S_{k+1} is issued before O += P_k V_k so the tensor core computes
-//             the next scores while the softmax warps work on the current ones.
-//   warps 4-7 softmax: thread t owns TMEM lane 32*(warp%4)+lane, one query
-//             row. It loads its S row, applies the mask and the base-2 scale,
-//             keeps the running max and sum, writes P (bf16) to shared memory
-//             for the PV MMA, and at the end reads O from TMEM, divides by the
-//             sum and stages its row in the freed K/V ring, from where one
-//             bulk copy per row writes it (bf16 output or fp32 split partial).
-//             With at most 64 (32) packed rows, Q is replicated into the idle
-//             lane quadrants (REP = 2 or 4): each copy of a row takes a 64/REP-
-//             token slice of every tile with its own running max and sum, so
-//             every softmax warp works and each does 1/REP of the exponentials;
-//             the slices are merged once, before the epilogue.
-// When the KV range of a (sequence, KV head) is split over a thread-block
-// cluster, the CTAs stage their normalised rows in shared memory and merge
-// them through distributed shared memory (a cluster barrier, then each CTA
-// combines a slice of rows from all peers): the final output, or one partial
-// per cluster, leaves the kernel instead of one partial per split.
-// The running max is raised lazily: O is rescaled in TMEM only when a row's
-// max grows by more than 2^8 (P then stays below 256, exact enough in bf16);
-// the final division by the matching sum removes the reference max.
-#include "nld_internal.cuh"
+// Block attention on the tcgen05 tensor cores: the draft and verify passes
+// (the kernel and its launch templates are in block_attn_tc.cuh; the
+// table-mask instantiations live in block_attn_tc_masked.cu).
+#include "block_attn_tc.cuh"
 
 namespace nld {
-namespace {
-
-constexpr int kProducers = 4;
-constexpr int kMmaWarp = 3;
-constexpr int kSoftmaxWarp0 = 4;
-
-// MT 128-row M tiles per CTA (MT = 2 for 129..256 packed rows); 4*MT
-// softmax warps; TPS 64-token K/V tiles per score product. TPS = 2 (one M
-// tile, a split short enough to sit in the ring whole): N = 128 products,
-// which the tensor core runs at full rate (N = 64 at about half), half as
-// many steps in the chain S -> softmax -> PV, and four P buffers so that the
-// softmax of one pair never waits for the PV products of the last. A long
-// split streams with TPS = 1, where a stage frees after each tile and more
-// of the ring stays in flight. With two M tiles the ring shrinks to 3
-// stages, so that two Q tiles and 2x2 P buffers fit.
-template <int MT, int TPS>
-struct TcCfg {
-  static_assert(TPS == 1 || (TPS == 2 && MT == 1), "paired score products with one M tile");
-  static constexpr int kStages = MT == 1 ? 4 : 3;
-  static constexpr int kTPS = TPS;               // K/V tiles per score product
-  static constexpr int kSTok = kTPS * kTileTok;  // tokens (N) of a score product
-  static constexpr int kPBufs = 2 * kTPS;        // P buffers per M tile
-  static constexpr int kWarps = 5 + 4 * MT;      // 4 producers, 1 MMA, 4*MT softmax
-  static constexpr int kThreads = 32 * kWarps;
-  static constexpr uint32_t kTmemCols = 512;     // MT x (S0 | S1), then MT x O
-  static_assert(kStages % kTPS == 0, "a score product never wraps around the ring");
-  static_assert(2 * MT * kSTok + MT * 128 <= 512, "TMEM columns");
-};
-
-// producer index of a warp, or -1: warps 0-2 and the last warp
-template <int MT>
-__device__ __forceinline__ int producer_index(int warp) {
-  return warp < 3 ? warp : (warp == TcCfg<MT, 1>::kWarps - 1 ? 3 : -1);
-}
-constexpr float kRescaleLog2 = 8.0f;
-
-// Epilogue staging in the freed K/V ring and Q tiles: 128*MT rows of D fp32
-// (padded pitch), then 128*MT log2-sum-exp values, then the cluster merge
-// weights [rows][8] and merged lse per row.
-template <int D>
-__host__ __device__ constexpr int merge_pitch() { return D * 4 + 16; }
-
-// K/V ring: the K tiles column-block-major ([column block][stage], so that
-// the K tiles of consecutive stages form one operand of 128 rows), then the
-// V tiles stage-major ([stage][column block]).
-template <int D, int MT, int TPS>
-struct TcLayout {
-  using Geo = TileGeom<D>;
-  static constexpr int kStages = TcCfg<MT, TPS>::kStages;
-  static constexpr int kPBufs = TcCfg<MT, TPS>::kPBufs;
-  static constexpr int kVOff = kStages * Geo::kTileBytes;       // V tiles after the K tiles
-  static constexpr int kQBytes = Geo::kColBlocks * 128 * 128;  // one 128-row Q tile, bf16
-  static constexpr int kPBytes = 128 * kTileTok * 2;             // one 128-row x 64-token P buffer, bf16
-  static constexpr int kQOff = kStages * Geo::kStageBytes;
-  static constexpr int kPOff = kQOff + MT * kQBytes;
-  static constexpr int kBarOff = kPOff + MT * kPBufs * kPBytes;
-  // kv_full[st], kv_empty[st], s_full[2], s_free[2], p_full[P], o_done[P], q_ready, drain, tmem slot
-  static constexpr int kNumBars = 2 * kStages + 4 + 2 * kPBufs + 2;
-  static constexpr int kBytes = kBarOff + kNumBars * 8 + 16;
-  static_assert(kBytes + 1024 <= 232448, "shared memory per CTA");
-  static constexpr int kMergeRows = 128 * MT;
-  static constexpr int kLseOff = kMergeRows * merge_pitch<D>();
-  static constexpr int kWtsOff = kLseOff + kMergeRows * 4;
-  static constexpr int kLseOutOff = kWtsOff + kMergeRows * 8 * 4;
-  static_assert(kLseOutOff + kMergeRows * 4 <= kPOff, "epilogue staging overlaps the live buffers");
-};
-
-template <int D, int MT, int REP, int TPS>
-__global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
-    block_attn_tc_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
-                         const AttnArgs a) {
-  static_assert(REP == 1 || REP == 2 || REP == 4, "replication of 1, 2 or 4");
-  static_assert(MT == 1 || REP == 1, "replication only with one M tile");
-  using Geo = TileGeom<D>;
-  using Cfg = TcCfg<MT, TPS>;
-  using Lay = TcLayout<D, MT, TPS>;
-  constexpr int kTcStages = Lay::kStages;
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* q_s = smem + Lay::kQOff;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Lay::kBarOff);
-  uint64_t* kv_full = bars;
-  uint64_t* kv_empty = bars + kTcStages;
-  uint64_t* s_full = bars + 2 * kTcStages;
-  uint64_t* s_free = s_full + 2;
-  uint64_t* p_full = s_free + 2;
-  uint64_t* o_done = p_full + Cfg::kPBufs;
-  uint64_t* q_ready = o_done + Cfg::kPBufs;
-  uint64_t* drain = q_ready + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
-
-  const int warp = threadIdx.x >> 5;
-  const int lane = threadIdx.x & 31;
-  const int split = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
-
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < kTcStages; ++s) {
-      mbar_init(&kv_full[s], kProducers);  // one expect_tx arrival per producer warp
-      mbar_init(&kv_empty[s], 1);
-    }
-    for (int j = 0; j < 2; ++j) {
-      mbar_init(&s_full[j], 1);
-      mbar_init(&s_free[j], 4 * MT);
-    }
-    for (int j = 0; j < Cfg::kPBufs; ++j) {
-      mbar_init(&p_full[j], 4 * MT);
-      mbar_init(&o_done[j], 1);
-    }
-    mbar_init(q_ready, 4 * MT);
-    mbar_init(drain, 1);
-    fence_mbar_init();
-  }
-  if (warp == 0 && lane == 0) {
-    prefetch_tensormap(&tmk);
-    prefetch_tensormap(&tmv);
-  }
-  if (warp == kMmaWarp) {
-    tmem_alloc(tmem_slot, Cfg::kTmemCols);
-    tc_fence_before();
-  }
-  // Without NLD_ATTN_PREFIX_READY nothing global is read before the
-  // dependency wait. With it, the page table, the prefix lengths and
-  // prefix-only K/V tiles are read first, and only the block slots, Q and the
-  // outputs wait (producers: in produce_kv; softmax warps: before Q).
-  const bool early = a.prefix_ready != 0;
-  grid_launch_dependents();  // dependents launch early; they wait on this grid themselves
-  if (!early) grid_dependency_wait();
-  const int t_begin = split * a.chunk;
-  // The producers' first page-id loads and the prefix-length load are
-  // independent, so they are in flight together.
-  PagePrefetch first;
-  first.raw = 0;
-  if (producer_index<MT>(warp) >= 0) first.load(a, b, t_begin, 0, lane);
-  int L = __ldg(a.prefix_lens + b);
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
-  // TMEM columns: S of M tile mt, buffer j at (2*mt + j)*kSTok; O of tile mt after all S buffers.
-  constexpr int kTPS = Cfg::kTPS;
-  constexpr int kSTok = Cfg::kSTok;
-  constexpr int kPBufs = Cfg::kPBufs;
-  auto tS = [&](int mt, int j) -> uint32_t { return tmem + static_cast<uint32_t>((2 * mt + j) * kSTok); };
-  auto tO = [&](int mt) -> uint32_t { return tmem + static_cast<uint32_t>(2 * MT * kSTok + mt * D); };
-
-  const int lmax = a.max_pages * a.page_size - a.bl;
-  if (L < 0 || L > lmax) {
-    if (threadIdx.x == 0) atomicOr(a.err, NLD_DEVERR_PREFIX_RANGE);
-    L = min(max(L, 0), lmax);
-  }
-  const int N = L + a.bl;
-  const float scl = a.scale_log2;
-  const bool diff_mode = a.mode == NLD_MODE_DIFFUSION;
-  const int t_end = min(t_begin + a.chunk, N);
-  const int ntiles = t_begin < t_end ? (t_end - t_begin + kTileTok - 1) / kTileTok : 0;
-
-  if (ntiles == 0) {
-    // This split lies past the sequence: its partials carry no keys.
-    if (early) grid_dependency_wait();
-    if (a.csize > 1) {
-      float* lse_stage = reinterpret_cast<float*>(smem + Lay::kLseOff);
-      for (int r = threadIdx.x; r < Lay::kMergeRows; r += blockDim.x) lse_stage[r] = -INFINITY;
-    } else {
-      for (int r = threadIdx.x; r < a.R; r += blockDim.x) {
-        const int i = r / a.G, h = g * a.G + (r - i * a.G);
-        a.lse_part[((static_cast<size_t>(split) * a.B + b) * a.Hq + h) * a.bl + i] = -INFINITY;
-      }
-    }
-  } else if (producer_index<MT>(warp) >= 0) {
-    // ---------------- producers ----------------
-    int early_tiles = 0;  // leading tiles made of prefix tokens only
-    if (early) {
-      while (early_tiles < kTcStages && early_tiles < ntiles &&
-             min(t_begin + (early_tiles + 1) * kTileTok, t_end) <= L)
-        ++early_tiles;
-      if (early_tiles == 0) grid_dependency_wait();
-    }
-    const int issued = produce_kv<D>(a, &tmk, &tmv, smem, kv_full, kv_empty, kTcStages, g, b, t_begin, t_end,
-                                     ntiles, lane, producer_index<MT>(warp), kProducers, first, early_tiles);
-    if (lane == 0 && issued < ntiles) {
-      // Stopped early on a wait timeout: let the copies already issued land
-      // before the CTA exits (bounded).
-      for (int k = max(0, issued - kTcStages); k < issued; ++k)
-        mbar_wait(&kv_full[k % kTcStages], (k / kTcStages) & 1, a.err);
-    }
-  } else if (warp == kMmaWarp) {
-    // ---------------- MMA issuer ----------------
-    if (lane == 0) {
-      bool ok = mbar_wait(q_ready, 0, a.err);
-      tc_fence_after();
-      const uint32_t q_addr = smem_u32(q_s);
-      const uint32_t idesc_s = umma_idesc_bf16(128, kSTok, false);
-      const uint32_t idesc_o = umma_idesc_bf16(128, D, true);
-      // Score product j: tiles kTPS*j .. kTPS*j+kTPS-1, whose K tiles sit in
-      // consecutive stages (one operand of kSTok rows per column block). If
-      // the last product has a single tile, its second half reads a stage
-      // no tile of this CTA still needs; those columns are never used.
-      auto issue_s = [&](int j) {
-        const int st = (j * kTPS) % kTcStages;
-        const uint32_t k_addr = smem_u32(smem) + static_cast<uint32_t>(st * Geo::kColBlockBytes);
-#pragma unroll
-        for (int mt = 0; mt < MT; ++mt) {
-          const uint32_t d = tS(mt, j & 1);
-#pragma unroll
-          for (int kk = 0; kk < D / 16; ++kk) {
-            const uint32_t koff = (kk & 3) * 32;  // 16 elements along the 128-byte row
-            const int cb = kk >> 2;               // 64-dim column block
-            const uint64_t ad = sw128_desc(q_addr + mt * Lay::kQBytes + cb * (128 * 128) + koff, 0, 1024);
-            const uint64_t bd = sw128_desc(k_addr + cb * kTcStages * Geo::kColBlockBytes + koff, 0, 1024);
-            umma_bf16(d, ad, bd, idesc_s, kk > 0 ? 1u : 0u);
-          }
-        }
-        umma_commit(&s_full[j & 1]);
-      };
-      auto issue_pv = [&](int k) {
-        const int st = k % kTcStages;
-        const uint32_t v_addr = smem_u32(smem + Lay::kVOff + st * Geo::kTileBytes);
-#pragma unroll
-        for (int mt = 0; mt < MT; ++mt) {
-        const uint32_t p_addr = smem_u32(smem + Lay::kPOff + (mt * kPBufs + k % kPBufs) * Lay::kPBytes);
-#pragma unroll
-        for (int kt = 0; kt < kTileTok / 16; ++kt) {
-          // A = P rows (K-major, one 128-byte block of 64 tokens); B = V (MN-major:
-          // 64-dim atoms LBO apart, 8-token row groups SBO apart).
-          const uint64_t ad = sw128_desc(p_addr + kt * 32, 0, 1024);
-          const uint64_t bd = sw128_desc(v_addr + kt * 16 * 128, Geo::kColBlockBytes, 1024);
-          umma_bf16(tO(mt), ad, bd, idesc_o, (k > 0 || kt > 0) ? 1u : 0u);
-        }
-        }
-        umma_commit(&o_done[k % kPBufs]);
-        umma_commit(&kv_empty[st]);
-      };
-      // Event-driven issue: score product j needs its K tiles and a free S
-      // buffer (the softmax warps have read product j-2), and waits until
-      // the PV products of product j-2 are issued; PV_k needs P_k. Whichever
-      // is ready goes first, so a late K/V tile never holds back a ready PV.
-      // (Letting scores run further ahead measured slower: they queue in
-      // front of the PV products on the tensor core.)
-      const int nprod = (ntiles + kTPS - 1) / kTPS;
-      int next_s = 0, next_pv = 0;
-      const uint64_t t_start = global_timer_ns();
-      uint32_t spins = 0;
-      while (ok && next_pv < ntiles) {
-        bool progressed = false;
-        const int t0 = next_s * kTPS;  // first tile of the next score product
-        if (next_s < nprod && t0 - kTPS <= next_pv &&
-            mbar_test(&kv_full[t0 % kTcStages], (t0 / kTcStages) & 1) &&
-            (kTPS == 1 || t0 + 1 >= ntiles || mbar_test(&kv_full[(t0 + 1) % kTcStages], ((t0 + 1) / kTcStages) & 1)) &&
-            (next_s < 2 || mbar_test(&s_free[next_s & 1], ((next_s - 2) >> 1) & 1))) {
-          tc_fence_after();
-          issue_s(next_s++);
-          progressed = true;
-        }
-        if (next_pv < next_s * kTPS && mbar_test(&p_full[next_pv % kPBufs], (next_pv / kPBufs) & 1)) {
-          tc_fence_after();
-          issue_pv(next_pv++);
-          progressed = true;
-        }
-        if (!progressed) {
-          __nanosleep(20);  // this warp shares an SM sub-partition with a softmax warp
-          if ((++spins & 255u) == 0 && global_timer_ns() - t_start > kWaitLimitNs) {
-            atomicOr(a.err, NLD_DEVERR_WAIT_TIMEOUT);
-            ok = false;
-          }
-        }
-      }
-      if (!ok) {
-        // Let every MMA already issued finish before TMEM is released (bounded).
-        umma_commit(drain);
-        mbar_wait(drain, 0, a.err);
-      }
-    }
-    __syncwarp();
-  } else {
-    // ---------------- softmax warps ----------------
-    // Warp `quad` reads TMEM lanes 32*quad..+31. With REP > 1 those lanes hold
-    // a copy of row block rq = quad % kRowQuads and the warp takes the token
-    // slice cp = quad / kRowQuads (columns c0 .. c0+kCols-1) of every tile.
-    constexpr int kRowQuads = 4 / REP;
-    constexpr int kCols = kTileTok / REP;           // S columns per thread and tile
-    const int quad = warp & 3;
-    const int mt = (warp - kSoftmaxWarp0) >> 2;     // M tile of this warp
-    const int rq = quad % kRowQuads;                // row block
-    const int cp = quad / kRowQuads;                // token slice
-    const int c0 = cp * kCols;
-    const int r_loc = quad * 32 + lane;             // TMEM lane == row of the Q and P tiles
-    const int r = mt * 128 + rq * 32 + lane;        // packed query row
-    const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
-    const bool warp_rows = mt * 128 + rq * 32 < a.R;  // warp-uniform: the warp holds a real row
-    const bool row_ok = r < a.R;
-    const int row_i = r / a.G;
-    const int row_h = g * a.G + (r - row_i * a.G);
-    const int sm_tid = threadIdx.x - 32 * kSoftmaxWarp0;  // 0 .. 128*MT-1 across the softmax warps
-    const int swz = r_loc & 7;                      // 128-byte swizzle phase of this tile row
-    uint8_t* q_tile = q_s + mt * Lay::kQBytes;
-    auto p_buf = [&](int j) -> uint8_t* { return smem + Lay::kPOff + (mt * kPBufs + j) * Lay::kPBytes; };
-
-    // Q row -> shared memory in the 128-byte-swizzled K-major layout (padding
-    // rows zero); slice 0 loads it once and writes every copy. The columns of
-    // P a thread never writes (other slices' tokens, or all of a padding row)
-    // are zeroed once in every buffer.
-    if (early) grid_dependency_wait();
-    {
-      if (cp == 0) {
-        const uint4* qrow = reinterpret_cast<const uint4*>(
-            a.q + ((static_cast<size_t>(b) * a.bl + row_i) * a.Hq + row_h) * D);
-        uint4 v[D / 8];
-#pragma unroll
-        for (int c = 0; c < D / 8; ++c) v[c] = row_ok ? __ldg(qrow + c) : make_uint4(0, 0, 0, 0);
-#pragma unroll
-        for (int q = 0; q < REP; ++q) {
-          const int rl = r_loc + q * kRowQuads * 32;  // TMEM lane of copy q (same swizzle phase)
-#pragma unroll
-          for (int c = 0; c < D / 8; ++c)
-            *reinterpret_cast<uint4*>(q_tile + (c >> 3) * (128 * 128) + rl * 128 + (((c & 7) ^ swz) << 4)) = v[c];
-        }
-      }
-#pragma unroll
-      for (int j = 0; j < kPBufs; ++j)
-#pragma unroll
-        for (int c = 0; c < 8; ++c)
-          if (!row_ok || c < c0 / 8 || c >= (c0 + kCols) / 8)
-            *reinterpret_cast<uint4*>(p_buf(j) + r_loc * 128 + ((c ^ swz) << 4)) = make_uint4(0, 0, 0, 0);
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(q_ready);
-    }
-
-    // The keys this row may see inside [t_begin, t_end) are exactly t < lim
-    // (Sec. 2.2: the whole prefix; in the draft pass every block slot, in the
-    // verify pass the block slots up to the row's own), so the mask is one
-    // compare per element on every tile, with no separate code path.
-    const int lim = diff_mode ? t_end : min(t_end, L + row_i + 1);
-    // A wait that gives up does so for the whole warp, so that no lane skips
-    // a warp-collective TMEM instruction the others execute.
-    auto warp_wait = [&](uint64_t* bar, uint32_t parity) {
-      return __all_sync(0xffffffffu, mbar_wait(bar, parity, a.err));
-    };
-    float m_run = -INFINITY, l_run = 0.f;
-    bool ok = true;
-    for (int k = 0; k < ntiles; ++k) {
-      const int j = k / kTPS, half = k % kTPS;  // score product and its 64-token half
-      const int buf = k % kPBufs;               // P buffer
-      const int st = k % kTcStages;
-      const int tile_t0 = t_begin + k * kTileTok;
-      const int valid = t_end - tile_t0;
-      if (half == 0 && !warp_wait(&s_full[j & 1], (j >> 1) & 1)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      float s[kCols];
-      if (warp_rows) {
-        const uint32_t ts = tS(mt, j & 1) + lane_off + static_cast<uint32_t>(half * kTileTok + c0);
-        if constexpr (kCols == 64) {
-          tmem_ld64(ts, s);
-        } else if constexpr (kCols == 32) {
-          tmem_ld32(ts, s);
-        } else {
-          tmem_ld16(ts, s);
-        }
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0 && (half == kTPS - 1 || k == ntiles - 1)) mbar_arrive(&s_free[j & 1]);
-
-      float alpha = 1.f;
-      bool rescale = false;
-      if (warp_rows) {
-        // Mask, base-2 scale and row max, branch-free.
-        const int nv = lim - (tile_t0 + c0);
-        float mx = -INFINITY;
-#pragma unroll
-        for (int j = 0; j < kCols; ++j) {
-          s[j] = j < nv ? s[j] * scl : -INFINITY;
-          mx = fmaxf(mx, s[j]);
-        }
-        if (m_run == -INFINITY) {
-          m_run = mx;  // nothing accumulated for this row yet
-        } else if (mx > m_run + kRescaleLog2) {
-          alpha = ex2(m_run - mx);
-          m_run = mx;
-          l_run *= alpha;
-          rescale = true;
-        }
-      }
-      if (__any_sync(0xffffffffu, rescale)) {
-        // O holds P_0..P_{k-1} V: wait for the last PV, then scale this warp's rows.
-        if (!warp_wait(&o_done[(k - 1) % kPBufs], ((k - 1) / kPBufs) & 1)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-#pragma unroll 1
-        for (int c = 0; c < D / 32; ++c) {
-          float o[32];
-          tmem_ld32(tO(mt) + lane_off + c * 32, o);
-#pragma unroll
-          for (int j = 0; j < 32; ++j) o[j] *= alpha;
-          tmem_st32(tO(mt) + lane_off + c * 32, o);
-        }
-      }
-      // P buffer `buf` is free once the PV of tile k-kPBufs has completed.
-      if (k >= kPBufs && !warp_wait(&o_done[buf], ((k / kPBufs) - 1) & 1)) {
-        ok = false;
-        break;
-      }
-      if (warp_rows) {
-        const float mu = m_run == -INFINITY ? 0.f : m_run;
-        uint8_t* prow = p_buf(buf) + r_loc * 128;
-#pragma unroll
-        for (int c = 0; c < kCols / 8; ++c) {
-          uint32_t w[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float p0 = ex2(s[c * 8 + 2 * e] - mu);
-            const float p1 = ex2(s[c * 8 + 2 * e + 1] - mu);
-            l_run += p0 + p1;
-            w[e] = pack_bf16(p0, p1);
-          }
-          const int chunk = c0 / 8 + c;
-          *reinterpret_cast<uint4*>(prow + ((chunk ^ swz) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
-        }
-      }
-      if (valid < kTileTok && (valid & (kGroupTok - 1))) {
-        // Cache slots past the sequence end inside its last page may hold
-        // stale or uninitialised data; P is 0 there but 0 * NaN = NaN, so
-        // zero those V rows before the PV MMA reads them.
-        if (!warp_wait(&kv_full[st], (k / kTcStages) & 1)) {
-          ok = false;
-          break;
-        }
-        const int r0 = valid, r1 = (valid + kGroupTok - 1) & ~(kGroupTok - 1);
-        uint8_t* vt = smem + Lay::kVOff + st * Geo::kTileBytes;
-        for (int idx = sm_tid; idx < (r1 - r0) * (D / 8); idx += 128 * MT) {
-          const int row = r0 + idx / (D / 8), c = idx % (D / 8);
-          *reinterpret_cast<uint4*>(vt + kv_swz(row, c)) = make_uint4(0, 0, 0, 0);
-        }
-      }
-      fence_proxy_async_smem();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&p_full[buf]);
-    }
-
-    // ---------------- epilogue ----------------
-    // Every PV has completed once o_done of the last tile fires, so the K/V
-    // ring is free for staging.
-    // Warp-uniform, like every condition around the warp-collective TMEM
-    // loads and stores below.
-    const bool o_ready =
-        __all_sync(0xffffffffu, ok && mbar_wait(&o_done[(ntiles - 1) % kPBufs], ((ntiles - 1) / kPBufs) & 1, a.err));
-    // Weights of the token slices of each row, by the split-combine rule
-    // (Sec. 3 Mode 2, here on one SM): slices cp > 0 leave their max, sum and
-    // unscaled O row in the freed ring (rows 32*kRowQuads.. of it); slice 0
-    // weighs them against its own and adds them in as it stages its output.
-    float w_self = 1.f;
-    float w_rep[REP > 1 ? REP - 1 : 1];
-    w_rep[0] = 0.f;
-    if constexpr (REP > 1) {
-      float* part_ml = reinterpret_cast<float*>(smem + Lay::kWtsOff);  // [TMEM lane][max, sum]
-      if (o_ready) tc_fence_after();
-      if (cp > 0) {
-        part_ml[2 * r_loc] = o_ready ? m_run : -INFINITY;  // a slice cut short by a timeout is dropped
-        part_ml[2 * r_loc + 1] = l_run;
-        if (warp_rows && o_ready) {
-          uint8_t* xrow = smem + r_loc * merge_pitch<D>();
-#pragma unroll 1
-          for (int c = 0; c < D / 32; ++c) {
-            float o[32];
-            tmem_ld32(tO(mt) + lane_off + c * 32, o);
-#pragma unroll
-            for (int q4 = 0; q4 < 8; ++q4)
-              *reinterpret_cast<float4*>(xrow + c * 128 + q4 * 16) =
-                  make_float4(o[4 * q4], o[4 * q4 + 1], o[4 * q4 + 2], o[4 * q4 + 3]);
-          }
-        }
-      }
-      named_bar_sync(2, 128);  // the four softmax warps
-      if (cp == 0) {
-        float m = m_run, mp[REP - 1], lp[REP - 1];
-#pragma unroll
-        for (int q = 0; q < REP - 1; ++q) {
-          const int lq = ((q + 1) * kRowQuads + rq) * 32 + lane;
-          mp[q] = part_ml[2 * lq];
-          lp[q] = part_ml[2 * lq + 1];
-          m = fmaxf(m, mp[q]);
-        }
-        // A row that saw no key in any slice (possible in the verify pass)
-        // keeps m = -inf, sum 0 and weight 0 everywhere.
-        w_self = m_run == -INFINITY ? 0.f : ex2(m_run - m);
-        float l = w_self * l_run;
-#pragma unroll
-        for (int q = 0; q < REP - 1; ++q) {
-          w_rep[q] = mp[q] == -INFINITY ? 0.f : ex2(mp[q] - m);
-          l += w_rep[q] * lp[q];
-        }
-        if (m != -INFINITY) {
-          m_run = m;
-          l_run = l;
-        }
-      }
-    }
-    // Unnormalised O of this thread's row, columns 64c..64c+63: its own TMEM
-    // lane plus, with REP > 1, the other slices of the row. Warp-collective.
-    auto load_o = [&](int c, float* o) {
-      tmem_ld64(tO(mt) + lane_off + c * 64, o);
-      if constexpr (REP > 1) {
-#pragma unroll
-        for (int j = 0; j < 64; ++j) o[j] *= w_self;
-#pragma unroll
-        for (int q = 0; q < REP - 1; ++q) {
-          if (w_rep[q] == 0.f) continue;  // a slice without keys never wrote its row
-          const uint8_t* xrow = smem + ((q + 1) * kRowQuads * 32 + rq * 32 + lane) * merge_pitch<D>() + c * 256;
-#pragma unroll
-          for (int q4 = 0; q4 < 16; ++q4) {
-            const float4 x = *reinterpret_cast<const float4*>(xrow + q4 * 16);
-            o[4 * q4] += w_rep[q] * x.x;
-            o[4 * q4 + 1] += w_rep[q] * x.y;
-            o[4 * q4 + 2] += w_rep[q] * x.z;
-            o[4 * q4 + 3] += w_rep[q] * x.w;
-          }
-        }
-      }
-    };
-    // One thread per output row from here on (slice 0 of each row).
-    const bool out_warp = warp_rows && cp == 0;
-    const bool out_row = row_ok && cp == 0;
-    if (a.csize > 1) {
-      // Cluster: stage this CTA's normalised rows and their log2-sum-exp in
-      // the freed ring for the merge across the cluster (rows without keys,
-      // or after a timeout, carry lse = -inf and are skipped by the merge).
-      if (o_ready) tc_fence_after();
-      float* lse_stage = reinterpret_cast<float*>(smem + Lay::kLseOff);
-      const float l = l_run;
-      const bool has = o_ready && out_row && l > 0.f;
-      if (cp == 0) lse_stage[r] = has ? m_run + lg2(l) : -INFINITY;
-      if (out_warp && o_ready) {
-        const float inv = l > 0.f ? 1.f / l : 0.f;
-        uint8_t* my = smem + r * merge_pitch<D>();
-#pragma unroll 1
-        for (int c = 0; c < D / 64; ++c) {
-          float o[64];
-          load_o(c, o);
-#pragma unroll
-          for (int q4 = 0; q4 < 16; ++q4)
-            *reinterpret_cast<float4*>(my + c * 256 + q4 * 16) =
-                make_float4(o[4 * q4] * inv, o[4 * q4 + 1] * inv, o[4 * q4 + 2] * inv, o[4 * q4 + 3] * inv);
-        }
-      }
-    } else if (o_ready) {
-      // Each thread stages its row (padded pitch, no bank conflicts) and
-      // hands it to the TMA engine as one bulk copy.
-      tc_fence_after();
-      if (out_warp) {
-        const float l = l_run;
-        const float inv = l > 0.f ? 1.f / l : 0.f;
-        const float lse_v = l > 0.f ? (m_run + lg2(l)) * kLn2 : -INFINITY;
-        const bool split_out = a.o_part != nullptr;
-        const int row_bytes = split_out ? D * 4 : D * 2;
-        uint8_t* my = smem + (mt * 128 + r_loc) * (row_bytes + 16);
-#pragma unroll 1
-        for (int c = 0; c < D / 64; ++c) {
-          float o[64];
-          load_o(c, o);
-#pragma unroll
-          for (int j = 0; j < 64; ++j) o[j] *= inv;
-          if (split_out) {
-#pragma unroll
-            for (int q4 = 0; q4 < 16; ++q4)
-              *reinterpret_cast<float4*>(my + c * 256 + q4 * 16) =
-                  make_float4(o[4 * q4], o[4 * q4 + 1], o[4 * q4 + 2], o[4 * q4 + 3]);
-          } else {
-#pragma unroll
-            for (int q4 = 0; q4 < 8; ++q4) {
-              const int j = q4 * 8;
-              *reinterpret_cast<uint4*>(my + c * 128 + q4 * 16) =
-                  make_uint4(pack_bf16(o[j], o[j + 1]), pack_bf16(o[j + 2], o[j + 3]), pack_bf16(o[j + 4], o[j + 5]),
-                             pack_bf16(o[j + 6], o[j + 7]));
-            }
-          }
-        }
-        // Output row (unsplit) or partial row; partial rows without keys are
-        // not written (their lse is -inf and the combine skips them).
-        if (row_ok && (!split_out || l > 0.f)) {
-          const size_t grow = split_out ? ((static_cast<size_t>(split) * a.B + b) * a.Hq + row_h) * a.bl + row_i
-                                        : (static_cast<size_t>(b) * a.bl + row_i) * a.Hq + row_h;
-          uint8_t* gbase = split_out ? reinterpret_cast<uint8_t*>(a.o_part) : reinterpret_cast<uint8_t*>(a.out);
-          fence_proxy_async_smem();  // this thread's staged row, visible to the TMA engine
-          bulk_store(gbase + grow * row_bytes, my, static_cast<uint32_t>(row_bytes));
-        }
-        if (row_ok) {
-          if (!split_out) {
-            if (a.lse != nullptr) a.lse[(static_cast<size_t>(b) * a.Hq + row_h) * a.bl + row_i] = lse_v;
-          } else {
-            a.lse_part[((static_cast<size_t>(split) * a.B + b) * a.Hq + row_h) * a.bl + row_i] = lse_v;
-          }
-        }
-        bulk_store_wait_read();  // the staged row stays in place until the copy has read it
-      }
-    }
-    tc_fence_before();
-  }
-
-  if (a.csize > 1) {
-    // Merge across the cluster (the splits of this sequence and KV head):
-    // CTA `rank` combines rows [rank*Rc, (rank+1)*Rc) from every peer's
-    // staged rows through distributed shared memory, by the same rule as the
-    // split combine, and writes the final output (one cluster per sequence
-    // and KV head) or this cluster's partial.
-    cluster_sync();
-    if (warp >= kSoftmaxWarp0 && warp < kSoftmaxWarp0 + 4 * MT) {
-      const uint32_t rank = cluster_ctarank();
-      const int Rc = (a.R + a.csize - 1) / a.csize;
-      const int r0 = static_cast<int>(rank) * Rc;
-      const int nrows = max(0, min(a.R, r0 + Rc) - r0);
-      const uint32_t stage_u32 = smem_u32(smem);
-      const uint32_t lse_u32 = stage_u32 + Lay::kLseOff;
-      // this CTA's merge weights, local: [row][peer] and the merged lse per row
-      float* wts = reinterpret_cast<float*>(smem + Lay::kWtsOff);
-      float* lse_out = reinterpret_cast<float*>(smem + Lay::kLseOutOff);
-      const int tid = threadIdx.x - 32 * kSoftmaxWarp0;
-      // 1) per-row weights: one thread per row, the peers' lse loads in flight together
-      if (tid < nrows) {
-        const int r = r0 + tid;
-        float lp[8];
-        float m = -INFINITY;
-#pragma unroll
-        for (int p = 0; p < 8; ++p) lp[p] = p < a.csize ? ld_dsmem_f32(dsmem_addr(lse_u32 + r * 4, p)) : -INFINITY;
-#pragma unroll
-        for (int p = 0; p < 8; ++p) m = fmaxf(m, lp[p]);
-        float w[8];
-        float wsum = 0.f;
-#pragma unroll
-        for (int p = 0; p < 8; ++p) {
-          w[p] = (m != -INFINITY && lp[p] != -INFINITY) ? ex2(lp[p] - m) : 0.f;
-          wsum += w[p];
-        }
-        const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
-#pragma unroll
-        for (int p = 0; p < 8; ++p) wts[tid * 8 + p] = w[p] * inv;
-        lse_out[tid] = wsum > 0.f ? (m + lg2(wsum)) * kLn2 : -INFINITY;
-      }
-      named_bar_sync(1, 128 * MT);
-      // 2) rows: two (row, 4-dim) items per thread per round, every peer load in flight
-      const bool final_out = a.num_partials == 1;
-      const int pidx = split / a.csize;
-      const int items = nrows * (D / 4);
-      for (int base = tid; base < items; base += 2 * 128 * MT) {
-        float4 acc[2];
-        int ridx[2], d4[2];
-        bool live[2];
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          const int idx = base + u * 128 * MT;
-          live[u] = idx < items;
-          ridx[u] = live[u] ? idx / (D / 4) : 0;
-          d4[u] = idx % (D / 4);
-          acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-        float4 o[2][8];
-#pragma unroll
-        for (int u = 0; u < 2; ++u)
-#pragma unroll
-          for (int p = 0; p < 8; ++p)
-            if (live[u] && p < a.csize && wts[ridx[u] * 8 + p] > 0.f)  // rows without keys are never read
-              o[u][p] = ld_dsmem_f4(dsmem_addr(stage_u32 + (r0 + ridx[u]) * merge_pitch<D>() + d4[u] * 16, p));
-            else
-              o[u][p] = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-#pragma unroll
-          for (int p = 0; p < 8; ++p) {
-            const float w = p < a.csize ? wts[ridx[u] * 8 + p] : 0.f;
-            acc[u].x += w * o[u][p].x; acc[u].y += w * o[u][p].y;
-            acc[u].z += w * o[u][p].z; acc[u].w += w * o[u][p].w;
-          }
-          if (!live[u]) continue;
-          const int r = r0 + ridx[u];
-          const int i = r / a.G, h = g * a.G + (r - i * a.G);
-          const float lse_v = lse_out[ridx[u]];
-          if (final_out) {
-            __nv_bfloat16* orow = a.out + ((static_cast<size_t>(b) * a.bl + i) * a.Hq + h) * D;
-            *reinterpret_cast<uint2*>(orow + d4[u] * 4) =
-                make_uint2(pack_bf16(acc[u].x, acc[u].y), pack_bf16(acc[u].z, acc[u].w));
-            if (d4[u] == 0 && a.lse != nullptr) a.lse[(static_cast<size_t>(b) * a.Hq + h) * a.bl + i] = lse_v;
-          } else {
-            const size_t prow = ((static_cast<size_t>(pidx) * a.B + b) * a.Hq + h) * a.bl + i;
-            if (lse_v != -INFINITY) *reinterpret_cast<float4*>(a.o_part + prow * D + d4[u] * 4) = acc[u];
-            if (d4[u] == 0) a.lse_part[prow] = lse_v;
-          }
-        }
-      }
-    }
-    cluster_sync();  // peers keep their shared memory until every merge has read it
-  }
-
-  __syncthreads();
-  if (warp == kMmaWarp) {
-    tc_fence_after();
-    tmem_dealloc(tmem, Cfg::kTmemCols);
-  }
-}
-
-template <int D, int MT, int REP, int TPS>
-cudaError_t configure_tc(int dev) {
-  static int configured[64] = {0};
-  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if (!__atomic_load_n(&configured[dev], __ATOMIC_ACQUIRE)) {
-    cudaError_t e = cudaFuncSetAttribute(block_attn_tc_kernel<D, MT, REP, TPS>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(TcLayout<D, MT, TPS>::kBytes + 1024));
-    if (e != cudaSuccess) return e;
-    __atomic_store_n(&configured[dev], 1, __ATOMIC_RELEASE);
-  }
-  return cudaSuccess;
-}
-
-template <int D, int MT, int REP, int TPS>
-cudaError_t launch_tc_t(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, cudaStream_t stream) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  if ((e = configure_tc<D, MT, REP, TPS>(dev)) != cudaSuccess) return e;
-  dim3 grid(a.num_splits, a.Hkv, a.B);
-  return launch_kernel_cluster(block_attn_tc_kernel<D, MT, REP, TPS>, grid, dim3(TcCfg<MT, TPS>::kThreads),
-                               TcLayout<D, MT, TPS>::kBytes + 1024, stream, a.csize, tmk, tmv, a);
-}
-
-// With one CTA per SM either way, cluster residency is the same for both
-// score-product widths; the query uses TPS = 1.
-template <int D, int MT, int REP>
-int max_active_clusters_t(int csize) {
-  static int cache[64][4];  // [device][cluster size 2/4/8] + 1 (0 = not queried)
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
-  const int slot = csize == 2 ? 0 : csize == 4 ? 1 : csize == 8 ? 2 : 3;
-  int v = __atomic_load_n(&cache[dev][slot], __ATOMIC_ACQUIRE);
-  if (v) return v - 1;
-  if (configure_tc<D, MT, REP, 1>(dev) != cudaSuccess) return 0;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(csize, 1, 1);
-  cfg.blockDim = dim3(TcCfg<MT, 1>::kThreads);
-  cfg.dynamicSmemBytes = TcLayout<D, MT, 1>::kBytes + 1024;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = csize;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, block_attn_tc_kernel<D, MT, REP, 1>, &cfg) != cudaSuccess) {
-    cudaGetLastError();
-    n = 0;
-  }
-  __atomic_store_n(&cache[dev][slot], n + 1, __ATOMIC_RELEASE);
-  return n;
-}
-
-// Copies of each Q row in the 128 TMEM lanes of one M tile: 4 for up to 32
-// packed rows, 2 for up to 64, else 1 (and 1 with two M tiles).
-int tc_replication(int rows) { return rows <= 32 ? 4 : rows <= 64 ? 2 : 1; }
-
-template <int D>
-int max_active_clusters_d(int csize, int rows) {
-  if (rows > 128) return max_active_clusters_t<D, 2, 1>(csize);
-  switch (tc_replication(rows)) {
-    case 4: return max_active_clusters_t<D, 1, 4>(csize);
-    case 2: return max_active_clusters_t<D, 1, 2>(csize);
-    default: return max_active_clusters_t<D, 1, 1>(csize);
-  }
-}
-
-template <int D, int TPS>
-cudaError_t launch_tc_rep(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, cudaStream_t stream) {
-  switch (tc_replication(a.R)) {
-    case 4: return launch_tc_t<D, 1, 4, TPS>(a, tmk, tmv, stream);
-    case 2: return launch_tc_t<D, 1, 2, TPS>(a, tmk, tmv, stream);
-    default: return launch_tc_t<D, 1, 1, TPS>(a, tmk, tmv, stream);
-  }
-}
-
-// Paired score products when a split fits in the ring whole (it is then
-// latency-bound: fewer, wider steps help); single tiles when it streams.
-template <int D>
-cudaError_t launch_tc_d(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, cudaStream_t stream) {
-  if (a.R > 128) return launch_tc_t<D, 2, 1, 1>(a, tmk, tmv, stream);
-  if (a.chunk <= TcCfg<1, 2>::kStages * kTileTok) return launch_tc_rep<D, 2>(a, tmk, tmv, stream);
-  return launch_tc_rep<D, 1>(a, tmk, tmv, stream);
-}
-
-}  // namespace
 
 bool tc_supports(int R, int head_dim) { return R <= 256 && (head_dim == 64 || head_dim == 128); }
 
@@ -839,7 +13,8 @@ int tc_max_active_clusters(int csize, int head_dim, int rows) {
 
 cudaError_t launch_block_attn_tc(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, int head_dim,
                                  cudaStream_t stream) {
-  return head_dim == 128 ? launch_tc_d<128>(a, tmk, tmv, stream) : launch_tc_d<64>(a, tmk, tmv, stream);
+  if (a.mode == kModeBlockMask) return launch_block_attn_tc_masked(a, tmk, tmv, head_dim, stream);
+  return head_dim == 128 ? launch_tc_d<128, false>(a, tmk, tmv, stream) : launch_tc_d<64, false>(a, tmk, tmv, stream);
 }
 
 }  // namespace nld

@@ -226,11 +226,13 @@ namespace {
 
 nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_block, const void* k_pages,
                              const void* v_pages, const int32_t* page_table, const int32_t* prefix_lens,
-                             int block_len, nld_mode_t mode, void* out, float* lse, void* workspace,
-                             size_t workspace_bytes, bool run_combine, cudaStream_t stream) {
+                             int block_len, int mode, const uint32_t* block_mask, void* out, float* lse,
+                             void* workspace, size_t workspace_bytes, bool run_combine, cudaStream_t stream) {
   nld_status_t st = check_params(params, block_len);
   if (st != NLD_OK) return st;
-  if (mode != NLD_MODE_DIFFUSION && mode != NLD_MODE_VERIFY) return NLD_ERR_INVALID_ARG;
+  if (mode != NLD_MODE_DIFFUSION && mode != NLD_MODE_VERIFY && mode != nld::kModeBlockMask)
+    return NLD_ERR_INVALID_ARG;
+  if (mode == nld::kModeBlockMask && !aligned(block_mask, 4)) return NLD_ERR_INVALID_ARG;
   if (!aligned(q_block, 16) || !aligned(k_pages, 16) || !aligned(v_pages, 16) || !aligned(out, 16) ||
       !aligned(page_table, 4) || !aligned(prefix_lens, 4))
     return NLD_ERR_INVALID_ARG;
@@ -276,7 +278,8 @@ nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_bloc
   a.chunk = plan.chunk;
   a.csize = plan.csize;
   a.num_partials = plan.partials;
-  a.mode = static_cast<int>(mode);
+  a.mode = mode;
+  a.block_mask = mode == nld::kModeBlockMask ? block_mask : nullptr;
   a.scale_log2 = scale * nld::kLog2e;
   a.prefix_ready = (params->flags & NLD_ATTN_PREFIX_READY) ? 1 : 0;
   if (plan.partials > 1) {
@@ -300,16 +303,43 @@ nld_status_t nld_block_attn(const nld_attn_params_t* params, const void* q_block
                             const void* v_pages, const int32_t* page_table, const int32_t* prefix_lens,
                             int block_len, nld_mode_t mode, void* out, float* lse, void* workspace,
                             size_t workspace_bytes, cudaStream_t stream) {
-  return block_attn_impl(params, q_block, k_pages, v_pages, page_table, prefix_lens, block_len, mode, out, lse,
-                         workspace, workspace_bytes, true, stream);
+  return block_attn_impl(params, q_block, k_pages, v_pages, page_table, prefix_lens, block_len, mode, nullptr, out,
+                         lse, workspace, workspace_bytes, true, stream);
+}
+
+nld_status_t nld_block_attn_masked(const nld_attn_params_t* params, const void* q_block, const void* k_pages,
+                                   const void* v_pages, const int32_t* page_table, const int32_t* prefix_lens,
+                                   int block_len, const uint32_t* block_mask, void* out, float* lse, void* workspace,
+                                   size_t workspace_bytes, cudaStream_t stream) {
+  return block_attn_impl(params, q_block, k_pages, v_pages, page_table, prefix_lens, block_len, nld::kModeBlockMask,
+                         block_mask, out, lse, workspace, workspace_bytes, true, stream);
+}
+
+int nld_quadss_block_mask(int k, uint32_t* masks) {
+  // Slot order (Eq. quad_input): the AR token, then for each of the k
+  // speculative tokens that token followed by its k masks. The chain (AR
+  // and speculative tokens) is causal and sees no mask; the masks of a
+  // speculative token see the chain up to it and their own k masks.
+  const int n = 1 + k + k * k;
+  if (k < 1 || n > nld::kMaxBlock || masks == nullptr) return -1;
+  uint32_t chain = 1u;  // chain slots seen so far (the AR token, slot 0)
+  masks[0] = chain;
+  for (int g = 0; g < k; ++g) {
+    const int spec = 1 + g * (k + 1);
+    chain |= 1u << spec;
+    masks[spec] = chain;
+    const uint32_t group = ((1u << k) - 1u) << (spec + 1);  // this token's k masks
+    for (int r = 1; r <= k; ++r) masks[spec + r] = chain | group;
+  }
+  return n;
 }
 
 nld_status_t nld_block_attn_partials(const nld_attn_params_t* params, const void* q_block, const void* k_pages,
                                      const void* v_pages, const int32_t* page_table, const int32_t* prefix_lens,
                                      int block_len, nld_mode_t mode, void* out, float* lse, void* workspace,
                                      size_t workspace_bytes, cudaStream_t stream) {
-  return block_attn_impl(params, q_block, k_pages, v_pages, page_table, prefix_lens, block_len, mode, out, lse,
-                         workspace, workspace_bytes, false, stream);
+  return block_attn_impl(params, q_block, k_pages, v_pages, page_table, prefix_lens, block_len, mode, nullptr, out,
+                         lse, workspace, workspace_bytes, false, stream);
 }
 
 nld_status_t nld_split_kv_combine(const float* o_part, const float* lse_part, int num_splits, int batch,

@@ -16,6 +16,7 @@ namespace nld {
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kMaxSplits = 128;
+constexpr int kModeBlockMask = 2;  // block part of the mask from a per-row table
 constexpr int kMaxRows = 256;   // (Hq / Hkv) * block_len handled by one CTA (two 128-row M tiles)
 constexpr int kMaxBlock = 32;   // block_len and the decision width n
 constexpr int kTileTok = 64;    // KV tokens per pipeline stage
@@ -34,7 +35,8 @@ struct AttnArgs {
   int B, Hq, Hkv, G, bl, R;    // R = G * bl query rows per CTA
   int page_size, log2_page, num_pages, max_pages;
   int num_splits, chunk;       // splits and tokens per split (multiple of 16)
-  int mode;                    // NLD_MODE_DIFFUSION or NLD_MODE_VERIFY
+  int mode;                    // NLD_MODE_DIFFUSION, NLD_MODE_VERIFY or kModeBlockMask
+  const uint32_t* block_mask;  // [bl] row masks over the block slots (kModeBlockMask only)
   float scale_log2;            // softmax scale * log2(e)
   int prefix_ready;            // NLD_ATTN_PREFIX_READY: prefix K/V may be read before the dependency wait
   int csize;                   // thread-block cluster size along the splits (1 = no cluster)
@@ -46,6 +48,9 @@ struct AttnArgs {
 bool tc_supports(int R, int head_dim);
 cudaError_t launch_block_attn_tc(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv,
                                  int head_dim, cudaStream_t stream);
+// The same for a table mask (a.mode == kModeBlockMask; block_attn_tc_masked.cu).
+cudaError_t launch_block_attn_tc_masked(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv,
+                                        int head_dim, cudaStream_t stream);
 cudaError_t launch_combine(const float* o_part, const float* lse_part, int S, int B, int Hq, int bl,
                            int D, __nv_bfloat16* out, float* lse, cudaStream_t stream);
 cudaError_t launch_accept(const int32_t* draft, const int32_t* verify, int B, int n, int32_t* acc,

@@ -13,6 +13,7 @@ import os
 import re
 from typing import Optional
 
+import numpy as np
 import torch
 
 from . import build as _build
@@ -78,6 +79,10 @@ def lib(path: Optional[str] = None):
     L.nld_logits_argmax.restype = I
     L.nld_kv_commit.argtypes = [PP, V, V, V, V, V, I, I, V, V, V]
     L.nld_kv_commit.restype = I
+    L.nld_block_attn_masked.argtypes = [PP, V, V, V, V, V, I, V, V, V, V, Sz, V]
+    L.nld_block_attn_masked.restype = I
+    L.nld_quadss_block_mask.argtypes = [I, V]
+    L.nld_quadss_block_mask.restype = I
     L.nld_unmask.restype = I
     L.nld_status_string.argtypes = [I]
     L.nld_status_string.restype = ctypes.c_char_p
@@ -193,6 +198,40 @@ def nld_block_attn_partials(params: AttnParams, q_block, k_pages, v_pages, page_
     nld_block_attn(params, q_block, k_pages, v_pages, page_table, prefix_lens, block_len, mode, out, lse,
                    workspace, stream, _entry="nld_block_attn_partials")
 
+
+
+def nld_block_attn_masked(params: AttnParams, q_block, k_pages, v_pages, page_table, prefix_lens, block_len: int,
+                          block_mask, out, lse=None, workspace=None, stream=None):
+    """nld_block_attn with the block part of the mask from block_mask (uint32
+    [block_len] as int32 on the device; bit j: block slot j visible)."""
+    B, Hq, Hkv, D, P = params.batch, params.num_q_heads, params.num_kv_heads, params.head_dim, params.page_size
+    _expect(q_block, torch.bfloat16, (B, block_len, Hq, D), "q_block")
+    _expect(k_pages, torch.bfloat16, (params.num_pages, Hkv, P, D), "k_pages")
+    _expect(v_pages, torch.bfloat16, (params.num_pages, Hkv, P, D), "v_pages")
+    _expect(page_table, torch.int32, (B, params.max_pages_per_seq), "page_table")
+    _expect(prefix_lens, torch.int32, (B,), "prefix_lens")
+    _expect(block_mask, torch.int32, (block_len,), "block_mask")
+    _expect(out, torch.bfloat16, (B, block_len, Hq, D), "out")
+    if lse is not None:
+        _expect(lse, torch.float32, (B, Hq, block_len), "lse")
+    ws_bytes = 0
+    if workspace is not None:
+        if not workspace.is_cuda or not workspace.is_contiguous():
+            raise ValueError("workspace: must be a contiguous CUDA tensor")
+        ws_bytes = workspace.numel() * workspace.element_size()
+    st = lib().nld_block_attn_masked(ctypes.byref(params), _ptr(q_block), _ptr(k_pages), _ptr(v_pages),
+                                     _ptr(page_table), _ptr(prefix_lens), int(block_len), _ptr(block_mask),
+                                     _ptr(out), _ptr(lse), _ptr(workspace), ws_bytes, _stream(stream))
+    _check(st, "nld_block_attn_masked")
+
+
+def nld_quadss_block_mask(k: int):
+    """The quadratic self-speculation table: numpy uint32 [1 + k + k^2]."""
+    out = np.zeros((32,), dtype=np.uint32)
+    n = lib().nld_quadss_block_mask(int(k), out.ctypes.data)
+    if n < 0:
+        raise ValueError(f"k={k}: 1 + k + k^2 slots must be at most 32")
+    return out[:n].copy()
 
 def nld_block_attn_static_scratch(params: AttnParams, q_block, k_pages, v_pages, page_table, prefix_lens,
                                   block_len: int, mode: int, out, lse=None, stream=None):

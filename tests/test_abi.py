@@ -4,6 +4,7 @@ CUDA call (the checks below return before the library touches a device)."""
 import ctypes
 import os
 
+import numpy as np
 import pytest
 
 from paper_2607_05722_gb300 import build, nld
@@ -113,6 +114,16 @@ def test_decisions_reject_bad_sizes(L):
     assert L.nld_greedy_accept(FAKE, FAKE, FAKE, 1, 8, FAKE, ctypes.c_void_p(0x10002), None) == 1
     assert L.nld_split_kv_combine(FAKE, FAKE, 0, 1, 4, 8, 128, FAKE, None, None) == 1
     assert L.nld_split_kv_combine(FAKE, FAKE, 2, 1, 4, 8, 80, FAKE, None, None) == 2
+
+
+def test_quadss_table_matches_oracle(L, orc):
+    """The library's host-side table of quadratic self-speculation (written on
+    its own) equals the oracle's; k beyond 5 (more than 32 slots) is refused."""
+    for k in range(1, 6):
+        assert np.array_equal(nld.nld_quadss_block_mask(k), orc.quadss_mask(k)), f"k={k}"
+    for k in (0, 6):
+        with pytest.raises(ValueError):
+            nld.nld_quadss_block_mask(k)
 
 
 def test_no_cpu_fallback_without_library(tmp_path):

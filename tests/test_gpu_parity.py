@@ -515,6 +515,78 @@ def test_partials_entry_point_then_combine(orc, spec, splits):
         compare_attn(out, lse, ro, rl, f"{name} partials mode={mode} S={splits}")
 
 
+# ---------------------------------------------------------------------------
+# table-mask attention (quadratic self-speculation)
+# ---------------------------------------------------------------------------
+
+def run_masked(dc, table, splits=0, q=None):
+    c = dc.case
+    p = dc.params(splits)
+    q = dc.q[DIFF] if q is None else q
+    out = torch.empty((c.batch, c.block_len, c.num_q_heads, c.head_dim), dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty((c.batch, c.num_q_heads, c.block_len), dtype=torch.float32, device="cuda")
+    ws = torch.empty(max(16, nld.nld_block_attn_workspace_size(p, c.block_len)), dtype=torch.uint8, device="cuda")
+    bm = torch.from_numpy(np.asarray(table, dtype=np.uint32).view(np.int32)).cuda()
+    nld.nld_block_attn_masked(p, q, dc.k, dc.v, dc.table, dc.prefix, c.block_len, bm, out, lse, ws)
+    return out, lse
+
+
+@pytest.mark.parametrize("spec", [SMALL[1], SMALL[3], SMALL[10], SMALL[8]], ids=[SMALL[i][0] for i in (1, 3, 10, 8)])
+def test_masked_tables_reduce_to_modes(spec):
+    """An all-ones table runs the draft pass and the lower-triangular table
+    the verify pass: bit-identical to nld_block_attn."""
+    name, B, Hq, Hkv, D, P, bl, prefix = spec
+    case = W.make_block_attn_case(name, B, Hq, Hkv, D, block_len=bl, page_size=P, prefix_lens=prefix,
+                                  seed=sum(prefix) + 3 * bl)
+    dc = DeviceCase(case)
+    full = np.full(bl, (1 << bl) - 1, dtype=np.uint64).astype(np.uint32)
+    tril = np.array([(2 << i) - 1 for i in range(bl)], dtype=np.uint64).astype(np.uint32)
+    for splits in (0, 1, 3):
+        for table, mode in ((full, DIFF), (tril, VER)):
+            ref_o, ref_l = dc.run(mode, splits)
+            got_o, got_l = run_masked(dc, table, splits, q=dc.q[mode])
+            assert torch.equal(got_o, ref_o) and torch.equal(got_l, ref_l), f"{name} mode={mode} S={splits}"
+
+
+@pytest.mark.parametrize("k,G,D,prefix", [(1, 4, 128, [100]), (2, 8, 64, [0, 37]), (3, 4, 128, [300, 5]),
+                                          (4, 6, 128, [64]), (5, 4, 128, [1000, 17]), (5, 8, 64, [250])])
+def test_quadss_attention_matches_oracle(orc, k, G, D, prefix):
+    bl = 1 + k + k * k
+    Hkv = 2
+    case = W.make_block_attn_case(f"quadss{k}", len(prefix), G * Hkv, Hkv, D, block_len=bl, page_size=16,
+                                  prefix_lens=prefix, seed=90 + k + G)
+    dc = DeviceCase(case)
+    table = nld.nld_quadss_block_mask(k)
+    ro, rl, _ = orc.block_attn_masked(case.q_draft_bits, case.kv.k_bits, case.kv.v_bits, case.kv.page_table,
+                                      case.kv.prefix_lens, case.num_q_heads, case.num_kv_heads, bl, table, case.scale)
+    for splits in (0, 1, 3):
+        out, lse = run_masked(dc, table, splits)
+        compare_attn(out, lse, ro, rl, f"quadss k={k} G={G} S={splits}")
+
+
+def test_masked_random_tables_and_empty_row(orc):
+    rng = np.random.default_rng(91)
+    for prefix in ([0, 0], [33, 7]):
+        case = W.make_block_attn_case("randmask", 2, 8, 2, 128, block_len=20, page_size=16, prefix_lens=prefix,
+                                      seed=sum(prefix) + 91)
+        dc = DeviceCase(case)
+        table = rng.integers(0, 1 << 20, size=20, dtype=np.uint64).astype(np.uint32)
+        table[3] = 0  # with no prefix this row sees nothing
+        ro, rl, _ = orc.block_attn_masked(case.q_draft_bits, case.kv.k_bits, case.kv.v_bits, case.kv.page_table,
+                                          case.kv.prefix_lens, case.num_q_heads, case.num_kv_heads, 20, table,
+                                          case.scale)
+        for splits in (0, 2):
+            out, lse = run_masked(dc, table, splits)
+            o = out.float().cpu().numpy()
+            l = lse.cpu().numpy()
+            if prefix[0] == 0:
+                assert np.all(o[0, 3] == 0) and np.all(l[0, :, 3] == -np.inf)
+            fin = np.isfinite(rl)
+            assert np.array_equal(np.isfinite(l), fin)
+            compare_attn(out, None, ro, rl, f"random table prefix={prefix} S={splits}")
+            assert np.max(np.abs(l[fin] - rl[fin])) <= 2e-3
+
+
 def test_attention_tail_slots_hold_nan(orc):
     """Cache slots past the block inside the last page may be uninitialised;
     NaN there must not reach the output."""
