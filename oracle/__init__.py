@@ -81,6 +81,8 @@ class Oracle:
         lib.nldo_block_attn_masked.restype = I
         lib.nldo_quadss_mask.argtypes = [I, P]
         lib.nldo_quadss_mask.restype = I
+        lib.nldo_ensemble_argmax.argtypes = [P, P, Lg, I, Lg, D, P, P]
+        lib.nldo_ensemble_argmax.restype = None
         lib.nldo_max_threads.argtypes = []
         lib.nldo_max_threads.restype = I
         self.lib = lib
@@ -185,6 +187,17 @@ class Oracle:
         ids = np.zeros((rows,), dtype=np.int32)
         conf = np.zeros((rows,), dtype=np.float64)
         self.lib.nldo_logits_argmax(self._p(lb), rows, vocab, ld, self._p(ids), self._p(conf))
+        return ids, conf
+
+    def ensemble_argmax(self, ar_bits, diff_bits, lam, vocab=None):
+        """(ids [rows] int32, conf [rows] fp64) of lam * softmax(ar) + (1 - lam) * softmax(diff)."""
+        a = np.ascontiguousarray(ar_bits, dtype=np.uint16)
+        d = np.ascontiguousarray(diff_bits, dtype=np.uint16)
+        rows, ld = a.shape
+        vocab = ld if vocab is None else int(vocab)
+        ids = np.zeros((rows,), dtype=np.int32)
+        conf = np.zeros((rows,), dtype=np.float64)
+        self.lib.nldo_ensemble_argmax(self._p(a), self._p(d), rows, vocab, ld, float(lam), self._p(ids), self._p(conf))
         return ids, conf
 
     def quadss_mask(self, k):

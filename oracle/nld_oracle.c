@@ -39,6 +39,8 @@
  *  - Block attention with a table mask over the block slots, and the
  *    structured mask of quadratic self-speculation (Sec. 3 variant; appendix
  *    Eq. quad_input) as one such table.
+ *  - The AR-diffusion ensemble verifier: argmax and max of the mixture of
+ *    the two predicted distributions (appendix, quadratic SS details).
  *
  * Build: gcc -O2 -fopenmp -ffp-contract=off -shared -fPIC (see build.py).
  */
@@ -533,4 +535,54 @@ int nldo_quadss_mask(int k, uint32_t *masks)
         masks[i] = bits;
     }
     return n;
+}
+
+/* softmax of one bf16 row into p[0..vocab) (fp64); all zero when no logit is above -inf */
+static void softmax_row(const uint16_t *row, int vocab, double *p)
+{
+    double m = -INFINITY;
+    for (int v = 0; v < vocab; ++v) {
+        const double l = bf16_to_f64(row[v]);
+        if (l > m) m = l;
+    }
+    if (m == -INFINITY) {
+        for (int v = 0; v < vocab; ++v) p[v] = 0.0;
+        return;
+    }
+    double sum = 0.0;
+    for (int v = 0; v < vocab; ++v) sum += (p[v] = exp(bf16_to_f64(row[v]) - m));
+    for (int v = 0; v < vocab; ++v) p[v] /= sum;
+}
+
+/*
+ * AR-diffusion ensemble verifier (appendix, verification with the ensemble):
+ * p_ens = lambda p_AR + (1 - lambda) p_diff over the vocabulary, from the
+ * causal logits at a speculative token and the denoising logits at the mask
+ * that follows it; ids = the lowest argmax of p_ens, conf = max p_ens.
+ * A distribution with no logit above -inf contributes nothing. Logits are
+ * finite or -inf. ar, diff bf16 bits [rows, ld].
+ */
+void nldo_ensemble_argmax(const uint16_t *ar, const uint16_t *diff, long rows, int vocab, long ld,
+                          double lambda, int32_t *ids, double *conf)
+{
+    #pragma omp parallel
+    {
+        double *pa = (double *)malloc(sizeof(double) * (vocab > 0 ? vocab : 1));
+        double *pb = (double *)malloc(sizeof(double) * (vocab > 0 ? vocab : 1));
+        #pragma omp for schedule(dynamic, 1)
+        for (long r = 0; r < rows; ++r) {
+            softmax_row(ar + r * ld, vocab, pa);
+            softmax_row(diff + r * ld, vocab, pb);
+            double best = -1.0;
+            int id = 0;
+            for (int v = 0; v < vocab; ++v) {
+                const double p = lambda * pa[v] + (1.0 - lambda) * pb[v];
+                if (p > best) { best = p; id = v; }
+            }
+            ids[r] = id;
+            conf[r] = best;
+        }
+        free(pa);
+        free(pb);
+    }
 }

@@ -794,6 +794,55 @@ def pin_masked_empty_row(orc):
     assert np.all(np.isfinite(lse[:, :, [0, 1, 3]]))
 
 
+# --------------------------------------------------------------------------
+# AR-diffusion ensemble verifier pins
+# --------------------------------------------------------------------------
+
+def pin_ensemble_golden(orc):
+    for ar, df, lam, idx, cf in read_golden("ensemble_cases.txt"):
+        a = _bf16_rows(np.array([[float(v) for v in ar.split()]], np.float32))
+        d = _bf16_rows(np.array([[float(v) for v in df.split()]], np.float32))
+        ids, conf = orc.ensemble_argmax(a, d, float(lam))
+        assert int(ids[0]) == int(idx) and abs(conf[0] - float(cf)) < 1e-15, f"{ar} | {df} | {lam}: {ids[0]} {conf[0]}"
+
+
+def pin_ensemble_limits(orc):
+    """lambda = 1 is the AR verifier alone, lambda = 0 the diffusion one: the
+    pinned logits rule on each input."""
+    rng = np.random.default_rng(71)
+    a = _bf16_rows(rng.standard_normal((20, 500)).astype(np.float32) * 3)
+    d = _bf16_rows(rng.standard_normal((20, 500)).astype(np.float32) * 3)
+    for lam, src in ((1.0, a), (0.0, d)):
+        ids, conf = orc.ensemble_argmax(a, d, lam)
+        ri, rc = orc.logits_argmax(src)
+        assert np.array_equal(ids, ri) and np.allclose(conf, rc, rtol=1e-14, atol=0)
+
+
+def pin_ensemble_scipy(orc):
+    """Against scipy.special.softmax mixtures (ids where the top two are apart)."""
+    rng = np.random.default_rng(72)
+    for V, lam in ((7, 0.3), (1000, 0.5), (32000, 0.8)):
+        a = _bf16_rows(rng.standard_normal((16, V)).astype(np.float32) * 3)
+        d = _bf16_rows(rng.standard_normal((16, V)).astype(np.float32) * 3)
+        p = (lam * scipy.special.softmax(W.bf16_bits_to_f32(a).astype(np.float64), axis=1)
+             + (1 - lam) * scipy.special.softmax(W.bf16_bits_to_f32(d).astype(np.float64), axis=1))
+        ids, conf = orc.ensemble_argmax(a, d, lam)
+        assert np.allclose(conf, p.max(axis=1), rtol=1e-12, atol=0)
+        top2 = np.sort(p, axis=1)[:, -2:]
+        clear = top2[:, 1] - top2[:, 0] > 1e-12
+        assert np.array_equal(ids[clear], np.argmax(p, axis=1)[clear])
+
+
+def pin_ensemble_empty_side(orc):
+    """A distribution with nothing above -inf contributes nothing."""
+    rng = np.random.default_rng(73)
+    d = _bf16_rows(rng.standard_normal((8, 64)).astype(np.float32))
+    a = _bf16_rows(np.full((8, 64), -np.inf, np.float32))
+    ids, conf = orc.ensemble_argmax(a, d, 0.3)
+    ri, rc = orc.logits_argmax(d)
+    assert np.array_equal(ids, ri) and np.allclose(conf, 0.7 * rc, rtol=1e-14, atol=0)
+
+
 ATTENTION_PINS = [pin_decode_bl1, pin_diffusion_full_attention, pin_verify_causal_tail, pin_lse_logsumexp,
                   pin_softmax_rows, pin_page_permutation, pin_block_permutation, pin_closed_forms,
                   pin_golden_uniform, pin_split_combine]
@@ -803,4 +852,5 @@ DECISION_PINS = [pin_accept_golden, pin_accept_brute, pin_accept_statistics, pin
 LOGITS_PINS = [pin_logits_golden, pin_logits_scipy, pin_logits_closed_forms, pin_logits_brute]
 COMMIT_PINS = [pin_commit_gather, pin_commit_then_attention, pin_commit_rollback_chain]
 MASK_PINS = [pin_quadss_layout, pin_masked_reduces_to_modes, pin_quadss_against_sdpa, pin_masked_empty_row]
-ALL_PINS = ATTENTION_PINS + DECISION_PINS + LOGITS_PINS + COMMIT_PINS + MASK_PINS
+ENSEMBLE_PINS = [pin_ensemble_golden, pin_ensemble_limits, pin_ensemble_scipy, pin_ensemble_empty_side]
+ALL_PINS = ATTENTION_PINS + DECISION_PINS + LOGITS_PINS + COMMIT_PINS + MASK_PINS + ENSEMBLE_PINS

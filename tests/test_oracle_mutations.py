@@ -94,6 +94,13 @@ MUTANTS = {
     "quadss_whole_chain": ("(chain[j] && group[j] <= group[i])", "chain[j]"),
     # table mode ignores the table
     "masked_ignores_table": ("if (mode == 2) return (int)((bm[i] >> j) & 1u);", "if (mode == 2) return 1;"),
+    # ensemble: the weights swapped
+    "ensemble_lambda_swapped": ("const double p = lambda * pa[v] + (1.0 - lambda) * pb[v];",
+                                "const double p = (1.0 - lambda) * pa[v] + lambda * pb[v];"),
+    # ensemble: ties to the last index
+    "ensemble_ties_last": ("if (p > best) { best = p; id = v; }", "if (p >= best) { best = p; id = v; }"),
+    # ensemble: mixes unnormalised weights
+    "ensemble_unnormalised": ("for (int v = 0; v < vocab; ++v) p[v] /= sum;", ""),
     # unmask: ascending order
     "unmask_ascending": ("if (ca > cb) return 1;\n    if (ca < cb) return 0;",
                          "if (ca < cb) return 1;\n    if (ca > cb) return 0;"),
