@@ -610,6 +610,14 @@ def run_logits(torch, nld, dev, stream, peak, l2):
         gbs = nbytes / (us * 1e-6) / 1e9
         res[f"rows{rows}_v{V}"] = {"us_per_call": round(us, 3), "logits_gbs": round(gbs, 1),
                                    "pct_of_hbm_peak": round(100 * gbs / peak, 2), "buffers": nbuf}
+        if rows <= 512:
+            # the ensemble verifier reads two logits rows per position (AR and diffusion)
+            npair = max(1, nbuf // 2)
+            us_e = time_graph(torch, stream, lambda i: nld.nld_logits_ensemble_argmax(
+                bufs[(2 * i) % (2 * npair)], bufs[(2 * i + 1) % (2 * npair)], 0.5, ids, conf), max(npair, 8), 10) * 1e3
+            gbs_e = 2 * nbytes / (us_e * 1e-6) / 1e9
+            res[f"ensemble_rows{rows}_v{V}"] = {"us_per_call": round(us_e, 3), "logits_gbs": round(gbs_e, 1),
+                                               "pct_of_hbm_peak": round(100 * gbs_e / peak, 2)}
         del bufs
     res["timing"] = "CUDA graph of back-to-back calls over rotating buffers, events around 10 replays"
     return res

@@ -319,6 +319,26 @@ nld_status_t nld_logits_argmax(const void *logits, int rows, int vocab, int ld, 
                                float *conf, cudaStream_t stream);
 
 /*
+ * AR-diffusion ensemble verifier (appendix, quadratic self-speculation:
+ * verification with the ensemble): per row r,
+ *   p = lambda softmax(ar_logits[r]) + (1 - lambda) softmax(diff_logits[r]),
+ *   ids[r] = the lowest v with p_v = max p,  conf[r] = max p,
+ * from the causal logits at a speculative token and the denoising logits at
+ * the mask that follows it. A row whose logits are all -inf contributes
+ * nothing; logits are finite or -inf. fp32 arithmetic: two rows whose
+ * mixture values lie within a few 1e-6 (relative) of each other may be taken
+ * in either order.
+ *
+ *   ar_logits, diff_logits  bf16 [rows, ld], first `vocab` entries used;
+ *                           ld >= vocab, a multiple of 8; 16-byte aligned
+ *   lambda                  in [0, 1]
+ *   ids int32 [rows], conf fp32 [rows]
+ */
+nld_status_t nld_logits_ensemble_argmax(const void *ar_logits, const void *diff_logits, int rows,
+                                        int vocab, int ld, float lambda, int32_t *ids, float *conf,
+                                        cudaStream_t stream);
+
+/*
  * Block KV commit into the paged cache (Sec. 3 Mode 3: the accepted drafts
  * are committed to the verified prefix and the verifier's cache is rebuilt
  * at the rejection point; Sec. 2: a completed diffusion block's KV cache is

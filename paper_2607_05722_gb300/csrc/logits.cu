@@ -210,9 +210,209 @@ __global__ void __launch_bounds__(kLgThreads)
   }
 }
 
+// ---------------------------------------------------------------------------
+// AR-diffusion ensemble verifier (appendix, verification with the ensemble):
+// p = lambda softmax(ar) + (1 - lambda) softmax(diff); id = lowest argmax,
+// conf = max p. Two passes over the row pair in one launch: the pieces of a
+// row pair first fold both rows into (max, sum), merge them across the
+// cluster (distributed shared memory), then re-read their pieces (now in L2)
+// to evaluate p and keep its lowest-index maximum.
+// ---------------------------------------------------------------------------
+
+constexpr int kEnThreads = 256;
+
+// (p, i) merge: the larger p, the lower index on ties.
+__device__ __forceinline__ void en_merge(float& p, int& i, float p2, int i2) {
+  if (p2 > p || (p2 == p && i2 < i)) {
+    p = p2;
+    i = i2;
+  }
+}
+
+__global__ void __launch_bounds__(kEnThreads)
+    ensemble_argmax_kernel(const __nv_bfloat16* __restrict__ ar, const __nv_bfloat16* __restrict__ diff, int vocab,
+                           long ld, int split, float lambda, int32_t* __restrict__ ids, float* __restrict__ conf) {
+  __shared__ float red[kEnThreads / 32][6];
+  __shared__ float tot[4];  // rank 0: m_a, s_a, m_b, s_b of the row pair
+  __shared__ float best[2];  // this CTA's (p, index)
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, t = threadIdx.x;
+  const int piece = static_cast<int>(blockIdx.x % split);
+  const long row = static_cast<long>(blockIdx.x / split);
+  const int nvec = vocab >> 3, tail = vocab & 7;
+  const int per = (nvec + split - 1) / split;
+  const int v0 = min(nvec, piece * per), v1 = min(nvec, v0 + per);
+  const bool has_tail = piece == split - 1 && t < tail;
+  grid_launch_dependents();
+  grid_dependency_wait();  // the logits come from earlier kernels
+  const uint4* ra = reinterpret_cast<const uint4*>(ar + row * ld);
+  const uint4* rb = reinterpret_cast<const uint4*>(diff + row * ld);
+  const uint16_t* ta = reinterpret_cast<const uint16_t*>(ar + row * ld) + nvec * 8;
+  const uint16_t* tb = reinterpret_cast<const uint16_t*>(diff + row * ld) + nvec * 8;
+
+  // ---- pass 1: (max, sum) of each row over this piece ----
+  float ma = -INFINITY, sa = 0.f, mb = -INFINITY, sb = 0.f;
+  int ia = 0, ib = 0;
+  for (int v = v0 + t; v < v1; v += kEnThreads) {
+    const uint4 wa = __ldg(ra + v), wb = __ldg(rb + v);
+    float xa[8], xb[8];
+    unpack_bf16(wa.x, xa[0], xa[1]); unpack_bf16(wa.y, xa[2], xa[3]);
+    unpack_bf16(wa.z, xa[4], xa[5]); unpack_bf16(wa.w, xa[6], xa[7]);
+    unpack_bf16(wb.x, xb[0], xb[1]); unpack_bf16(wb.y, xb[2], xb[3]);
+    unpack_bf16(wb.z, xb[4], xb[5]); unpack_bf16(wb.w, xb[6], xb[7]);
+    lg_fold(xa, v * 8, ma, sa, ia);
+    lg_fold(xb, v * 8, mb, sb, ib);
+  }
+  if (has_tail) {
+    const float xa[1] = {__uint_as_float(static_cast<uint32_t>(ta[t]) << 16)};
+    const float xb[1] = {__uint_as_float(static_cast<uint32_t>(tb[t]) << 16)};
+    lg_fold(xa, nvec * 8 + t, ma, sa, ia);
+    lg_fold(xb, nvec * 8 + t, mb, sb, ib);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    lg_merge(ma, sa, ia, __shfl_xor_sync(0xffffffffu, ma, off), __shfl_xor_sync(0xffffffffu, sa, off),
+             __shfl_xor_sync(0xffffffffu, ia, off));
+    lg_merge(mb, sb, ib, __shfl_xor_sync(0xffffffffu, mb, off), __shfl_xor_sync(0xffffffffu, sb, off),
+             __shfl_xor_sync(0xffffffffu, ib, off));
+  }
+  if (lane == 0) {
+    red[warp][0] = ma; red[warp][1] = sa; red[warp][2] = mb; red[warp][3] = sb;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    ma = lane < kEnThreads / 32 ? red[lane][0] : -INFINITY;
+    sa = lane < kEnThreads / 32 ? red[lane][1] : 0.f;
+    mb = lane < kEnThreads / 32 ? red[lane][2] : -INFINITY;
+    sb = lane < kEnThreads / 32 ? red[lane][3] : 0.f;
+#pragma unroll
+    for (int off = 4; off > 0; off >>= 1) {
+      lg_merge(ma, sa, ia, __shfl_xor_sync(0xffffffffu, ma, off), __shfl_xor_sync(0xffffffffu, sa, off), 0);
+      lg_merge(mb, sb, ib, __shfl_xor_sync(0xffffffffu, mb, off), __shfl_xor_sync(0xffffffffu, sb, off), 0);
+    }
+    if (lane == 0) {
+      tot[0] = ma; tot[1] = sa; tot[2] = mb; tot[3] = sb;
+    }
+  }
+  if (split > 1) {
+    cluster_sync();  // every piece's (max, sum) is in its shared memory
+    if (cluster_ctarank() == 0 && warp == 0) {
+      const uint32_t base = smem_u32(tot);
+      ma = -INFINITY; sa = 0.f; mb = -INFINITY; sb = 0.f;
+      if (lane < split) {
+        ma = ld_dsmem_f32(dsmem_addr(base, lane));
+        sa = ld_dsmem_f32(dsmem_addr(base + 4, lane));
+        mb = ld_dsmem_f32(dsmem_addr(base + 8, lane));
+        sb = ld_dsmem_f32(dsmem_addr(base + 12, lane));
+      }
+#pragma unroll
+      for (int off = 4; off > 0; off >>= 1) {
+        lg_merge(ma, sa, ia, __shfl_xor_sync(0xffffffffu, ma, off), __shfl_xor_sync(0xffffffffu, sa, off), 0);
+        lg_merge(mb, sb, ib, __shfl_xor_sync(0xffffffffu, mb, off), __shfl_xor_sync(0xffffffffu, sb, off), 0);
+      }
+    }
+    cluster_sync();  // every rank has read the pieces' states before rank 0 overwrites its own
+    if (cluster_ctarank() == 0 && threadIdx.x == 0) {
+      tot[0] = ma; tot[1] = sa; tot[2] = mb; tot[3] = sb;
+    }
+    cluster_sync();  // the row pair's totals are in rank 0's shared memory
+    const uint32_t base0 = dsmem_addr(smem_u32(tot), 0);
+    ma = ld_dsmem_f32(base0);
+    sa = ld_dsmem_f32(base0 + 4);
+    mb = ld_dsmem_f32(base0 + 8);
+    sb = ld_dsmem_f32(base0 + 12);
+  } else {
+    __syncthreads();
+    ma = tot[0]; sa = tot[1]; mb = tot[2]; sb = tot[3];
+  }
+  // An empty distribution (max -inf) gets weight 0 and a stand-in max of 0,
+  // so its terms are exp(-inf) * 0 = 0.
+  const float ca = ma == -INFINITY ? 0.f : lambda / sa;
+  const float cb = mb == -INFINITY ? 0.f : (1.f - lambda) / sb;
+  const float ma2 = (ma == -INFINITY ? 0.f : ma) * kLog2e;
+  const float mb2 = (mb == -INFINITY ? 0.f : mb) * kLog2e;
+
+  // ---- pass 2: p over this piece (re-read, now in L2), lowest-index max ----
+  float pbest = -1.f;
+  int ibest = 0;
+  for (int v = v0 + t; v < v1; v += kEnThreads) {
+    const uint4 wa = __ldg(ra + v), wb = __ldg(rb + v);
+    float xa[8], xb[8];
+    unpack_bf16(wa.x, xa[0], xa[1]); unpack_bf16(wa.y, xa[2], xa[3]);
+    unpack_bf16(wa.z, xa[4], xa[5]); unpack_bf16(wa.w, xa[6], xa[7]);
+    unpack_bf16(wb.x, xb[0], xb[1]); unpack_bf16(wb.y, xb[2], xb[3]);
+    unpack_bf16(wb.z, xb[4], xb[5]); unpack_bf16(wb.w, xb[6], xb[7]);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float p = ca * ex2(fmaf(xa[j], kLog2e, -ma2)) + cb * ex2(fmaf(xb[j], kLog2e, -mb2));
+      if (p > pbest) {
+        pbest = p;
+        ibest = v * 8 + j;
+      }
+    }
+  }
+  if (has_tail) {
+    const float a = __uint_as_float(static_cast<uint32_t>(ta[t]) << 16);
+    const float b = __uint_as_float(static_cast<uint32_t>(tb[t]) << 16);
+    const float p = ca * ex2(fmaf(a, kLog2e, -ma2)) + cb * ex2(fmaf(b, kLog2e, -mb2));
+    if (p > pbest) {
+      pbest = p;
+      ibest = nvec * 8 + t;
+    }
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1)
+    en_merge(pbest, ibest, __shfl_xor_sync(0xffffffffu, pbest, off), __shfl_xor_sync(0xffffffffu, ibest, off));
+  if (lane == 0) {
+    red[warp][4] = pbest;
+    red[warp][5] = __int_as_float(ibest);
+  }
+  __syncthreads();
+  if (warp == 0) {
+    pbest = lane < kEnThreads / 32 ? red[lane][4] : -1.f;
+    ibest = lane < kEnThreads / 32 ? __float_as_int(red[lane][5]) : 0;
+#pragma unroll
+    for (int off = 4; off > 0; off >>= 1)
+      en_merge(pbest, ibest, __shfl_xor_sync(0xffffffffu, pbest, off), __shfl_xor_sync(0xffffffffu, ibest, off));
+    if (lane == 0) {
+      best[0] = pbest;
+      best[1] = __int_as_float(ibest);
+    }
+  }
+  if (split > 1) {
+    cluster_sync();
+    if (cluster_ctarank() == 0 && warp == 0) {
+      const uint32_t base = smem_u32(best);
+      pbest = -1.f;
+      ibest = 0;
+      if (lane < split) {
+        pbest = ld_dsmem_f32(dsmem_addr(base, lane));
+        ibest = __float_as_int(ld_dsmem_f32(dsmem_addr(base + 4, lane)));
+      }
+#pragma unroll
+      for (int off = 4; off > 0; off >>= 1)
+        en_merge(pbest, ibest, __shfl_xor_sync(0xffffffffu, pbest, off), __shfl_xor_sync(0xffffffffu, ibest, off));
+      if (lane == 0) {
+        ids[row] = ibest;
+        conf[row] = pbest;
+      }
+    }
+    cluster_sync();  // the peers keep their shared memory until rank 0 has read it
+  } else if (threadIdx.x == 0) {
+    ids[row] = ibest;
+    conf[row] = pbest;
+  }
+}
+
 }  // namespace
 
 int logits_split_vectors() { return kLgStageVecs; }
+
+cudaError_t launch_ensemble_argmax(const __nv_bfloat16* ar, const __nv_bfloat16* diff, int rows, int vocab, long ld,
+                                   int split, float lambda, int32_t* ids, float* conf, cudaStream_t stream) {
+  const dim3 grid(static_cast<unsigned>(static_cast<long>(rows) * split));
+  return launch_kernel_cluster(ensemble_argmax_kernel, grid, dim3(kEnThreads), 0, stream, split, ar, diff, vocab, ld,
+                               split, lambda, ids, conf);
+}
 
 cudaError_t launch_logits_argmax(const __nv_bfloat16* logits, int rows, int vocab, long ld, int split, int32_t* ids,
                                  float* conf, unsigned int* err, cudaStream_t stream) {

@@ -421,6 +421,29 @@ nld_status_t nld_logits_argmax(const void* logits, int rows, int vocab, int ld, 
              : NLD_ERR_CUDA;
 }
 
+nld_status_t nld_logits_ensemble_argmax(const void* ar_logits, const void* diff_logits, int rows, int vocab, int ld,
+                                        float lambda, int32_t* ids, float* conf, cudaStream_t stream) {
+  if (rows < 1 || vocab < 1 || ld < vocab || ld % 8 != 0) return NLD_ERR_INVALID_ARG;
+  if (!(lambda >= 0.f && lambda <= 1.f)) return NLD_ERR_INVALID_ARG;  // also rejects NaN
+  if (!aligned(ar_logits, 16) || !aligned(diff_logits, 16) || !aligned(ids, 4) || !aligned(conf, 4))
+    return NLD_ERR_INVALID_ARG;
+  int sms = 0;
+  nld_status_t st = device_state(nullptr, &sms);
+  if (st != NLD_OK) return st;
+  int split = 1;
+  if (rows < sms) {
+    const int by_sms = sms / rows;
+    const int by_len = (vocab / 8) / nld::logits_split_vectors();
+    const int want = by_sms < by_len ? by_sms : by_len;
+    while (split * 2 <= want && split * 2 <= 8) split *= 2;
+  }
+  return nld::launch_ensemble_argmax(static_cast<const __nv_bfloat16*>(ar_logits),
+                                     static_cast<const __nv_bfloat16*>(diff_logits), rows, vocab, ld, split, lambda,
+                                     ids, conf, stream) == cudaSuccess
+             ? NLD_OK
+             : NLD_ERR_CUDA;
+}
+
 nld_status_t nld_kv_commit(const nld_attn_params_t* params, const void* k_new, const void* v_new,
                            const int32_t* counts, const int32_t* page_table, int32_t* prefix_lens, int block_len,
                            int advance, void* k_pages, void* v_pages, cudaStream_t stream) {

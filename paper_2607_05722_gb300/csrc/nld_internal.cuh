@@ -65,6 +65,9 @@ cudaError_t launch_greedy_accept(const int32_t* pred, const int32_t* target, con
 cudaError_t launch_logits_argmax(const __nv_bfloat16* logits, int rows, int vocab, long ld, int split, int32_t* ids,
                                  float* conf, unsigned int* err, cudaStream_t stream);
 int logits_split_vectors();  // 16-byte vectors a CTA streams per ring stage
+// AR-diffusion ensemble verifier: `split` CTAs per row pair (a cluster when > 1).
+cudaError_t launch_ensemble_argmax(const __nv_bfloat16* ar, const __nv_bfloat16* diff, int rows, int vocab, long ld,
+                                   int split, float lambda, int32_t* ids, float* conf, cudaStream_t stream);
 // Block KV commit (rows j < count_b to slots L_b + j), then L_b += count_b.
 cudaError_t launch_kv_commit(const __nv_bfloat16* k_new, const __nv_bfloat16* v_new, const int32_t* counts,
                              const int32_t* page_table, int32_t* prefix_lens, __nv_bfloat16* k_pages,

@@ -77,6 +77,8 @@ def lib(path: Optional[str] = None):
     L.nld_greedy_accept.restype = I
     L.nld_logits_argmax.argtypes = [V, I, I, I, V, V, V]
     L.nld_logits_argmax.restype = I
+    L.nld_logits_ensemble_argmax.argtypes = [V, V, I, I, I, ctypes.c_float, V, V, V]
+    L.nld_logits_ensemble_argmax.restype = I
     L.nld_kv_commit.argtypes = [PP, V, V, V, V, V, I, I, V, V, V]
     L.nld_kv_commit.restype = I
     L.nld_block_attn_masked.argtypes = [PP, V, V, V, V, V, I, V, V, V, V, Sz, V]
@@ -325,6 +327,21 @@ def nld_logits_argmax(logits, ids, conf, vocab=None, stream=None):
     _check(lib().nld_logits_argmax(_ptr(logits), rows, vocab, ld, _ptr(ids), _ptr(conf), _stream(stream)),
            "nld_logits_argmax")
 
+
+
+def nld_logits_ensemble_argmax(ar_logits, diff_logits, lam: float, ids, conf, vocab=None, stream=None):
+    """Lowest argmax and max of lam * softmax(ar) + (1 - lam) * softmax(diff) per row."""
+    for name, t in (("ar_logits", ar_logits), ("diff_logits", diff_logits)):
+        if t.dtype != torch.bfloat16 or t.dim() != 2 or not t.is_cuda or t.stride(1) != 1:
+            raise ValueError(f"{name}: a CUDA bf16 [rows, ld] tensor with unit column stride")
+    if ar_logits.shape != diff_logits.shape or ar_logits.stride(0) != diff_logits.stride(0):
+        raise ValueError("ar_logits and diff_logits: same shape and row stride")
+    rows, ld = ar_logits.shape[0], ar_logits.stride(0)
+    vocab = ar_logits.shape[1] if vocab is None else int(vocab)
+    _expect(ids, torch.int32, (rows,), "ids")
+    _expect(conf, torch.float32, (rows,), "conf")
+    _check(lib().nld_logits_ensemble_argmax(_ptr(ar_logits), _ptr(diff_logits), rows, vocab, ld, float(lam),
+                                            _ptr(ids), _ptr(conf), _stream(stream)), "nld_logits_ensemble_argmax")
 
 def nld_kv_commit(params: AttnParams, k_new, v_new, counts, page_table, prefix_lens, block_len: int, advance: bool,
                   k_pages, v_pages, stream=None):

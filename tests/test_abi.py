@@ -112,6 +112,10 @@ def test_decisions_reject_bad_sizes(L):
     assert L.nld_greedy_accept(FAKE, FAKE, FAKE, 0, 8, FAKE, None, None) == 1
     assert L.nld_greedy_accept(FAKE, None, FAKE, 1, 8, FAKE, None, None) == 1
     assert L.nld_greedy_accept(FAKE, FAKE, FAKE, 1, 8, FAKE, ctypes.c_void_p(0x10002), None) == 1
+    assert L.nld_logits_ensemble_argmax(FAKE, FAKE, 1, 8, 8, 1.5, FAKE, FAKE, None) == 1
+    assert L.nld_logits_ensemble_argmax(FAKE, FAKE, 1, 8, 8, float("nan"), FAKE, FAKE, None) == 1
+    assert L.nld_logits_ensemble_argmax(FAKE, FAKE, 1, 9, 12, 0.5, FAKE, FAKE, None) == 1
+    assert L.nld_logits_argmax(FAKE, 0, 8, 8, FAKE, FAKE, None) == 1
     assert L.nld_split_kv_combine(FAKE, FAKE, 0, 1, 4, 8, 128, FAKE, None, None) == 1
     assert L.nld_split_kv_combine(FAKE, FAKE, 2, 1, 4, 8, 80, FAKE, None, None) == 2
 

@@ -315,6 +315,59 @@ def test_logits_matches_oracle(orc, rows, vocab, ld):
     check_logits(gpu_logits(bits, vocab), orc.logits_argmax(bits, vocab), f"rows={rows} V={vocab} ld={ld}")
 
 
+def gpu_ensemble(a_bits, d_bits, lam, vocab=None):
+    rows = a_bits.shape[0]
+    ta = torch.from_numpy(np.ascontiguousarray(a_bits).view(np.int16)).view(torch.bfloat16).cuda()
+    td = torch.from_numpy(np.ascontiguousarray(d_bits).view(np.int16)).view(torch.bfloat16).cuda()
+    ids = torch.full((rows,), -7, dtype=torch.int32, device="cuda")
+    conf = torch.full((rows,), -7.0, dtype=torch.float32, device="cuda")
+    nld.nld_logits_ensemble_argmax(ta, td, lam, ids, conf, vocab=vocab)
+    return ids.cpu().numpy(), conf.cpu().numpy().astype(np.float64)
+
+
+def mixture_f64(a_bits, d_bits, lam, vocab):
+    def sm(bits):
+        x = W.bf16_bits_to_f32(bits[:, :vocab]).astype(np.float64)
+        m = x.max(axis=1, keepdims=True)
+        w = np.where(np.isfinite(m), np.exp(x - np.where(np.isfinite(m), m, 0)), 0.0)
+        s = w.sum(axis=1, keepdims=True)
+        return np.where(s > 0, w / np.where(s > 0, s, 1), 0.0)
+    return lam * sm(a_bits) + (1 - lam) * sm(d_bits)
+
+
+def test_ensemble_golden_cases():
+    for ar, df, lam, idx, cf in oracle_pins.read_golden("ensemble_cases.txt"):
+        a = W.f32_to_bf16_bits(np.array([[float(v) for v in ar.split()]], np.float32))
+        d = W.f32_to_bf16_bits(np.array([[float(v) for v in df.split()]], np.float32))
+        V = a.shape[1]
+        pa = np.zeros((1, 8), np.uint16); pa[0, :V] = a[0]
+        pd = np.zeros((1, 8), np.uint16); pd[0, :V] = d[0]
+        gi, gc = gpu_ensemble(pa, pd, float(lam), vocab=V)
+        assert int(gi[0]) == int(idx) and abs(gc[0] - float(cf)) <= LOGITS_RTOL * float(cf), f"{ar} | {df} | {lam}"
+
+
+@pytest.mark.parametrize("rows,vocab,ld,lam", [(16, 131072, 131072, 0.5), (5, 1001, 1008, 0.3), (300, 32000, 32000, 0.7),
+                                               (2, 131077, 131080, 1.0), (3, 9, 16, 0.0), (1, 7, 8, 0.25)])
+def test_ensemble_matches_oracle(orc, rows, vocab, ld, lam):
+    """ids: the oracle's where its two best mixture values are apart by more
+    than the fp32 error, else any position whose mixture value is within that
+    error of the max; conf within the logits bound."""
+    rng = np.random.default_rng(rows + vocab)
+    a = W.f32_to_bf16_bits((rng.standard_normal((rows, ld)) * 3).astype(np.float32))
+    d = W.f32_to_bf16_bits((rng.standard_normal((rows, ld)) * 3).astype(np.float32))
+    if rows >= 3:
+        a[1, :vocab] = W.f32_to_bf16_bits(np.full(vocab, -np.inf, np.float32))  # one side empty
+    gi, gc = gpu_ensemble(a, d, lam, vocab)
+    oi, oc = orc.ensemble_argmax(a, d, lam, vocab)
+    p = mixture_f64(a, d, lam, vocab)
+    assert np.all(np.abs(gc - oc) <= LOGITS_RTOL * oc)
+    tol = 2 * LOGITS_RTOL * oc
+    top2 = np.sort(p, axis=1)[:, -2:]
+    clear = top2[:, 1] - top2[:, 0] > tol
+    assert np.array_equal(gi[clear], oi[clear])
+    assert np.all(p[np.arange(rows), gi] >= oc - tol), "the GPU's id is a maximiser within the error"
+
+
 def test_logits_peaked_rows(orc):
     """Peaked rows (a confident prediction): the confidence near 1 is kept to
     the same relative bound."""
