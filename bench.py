@@ -62,6 +62,8 @@ def parse_args():
     ap.add_argument("--only-workload", default=None,
                     help="time only this named workload (device-drawn inputs), e.g. for a profiler")
     ap.add_argument("--workload-batch", type=int, default=None, help="batch override for --only-workload")
+    ap.add_argument("--only-section", default=None, choices=["decisions", "logits", "kv_commit", "quadss"],
+                    help="time only this section of the report (e.g. for a profiler)")
     ap.add_argument("--no-prefix-ready", action="store_true",
                     help="do not let attention stream prefix KV before its dependency wait")
     ap.add_argument("--seed", type=int, default=0)
@@ -185,6 +187,27 @@ def run_only_workload(args, local):
     stream = torch.cuda.Stream(device=dev)
     res = run_workloads(torch, nld, dev, stream, peak, l2, only=args.only_workload, batch=args.workload_batch)
     print(json.dumps({"workload": args.only_workload, "batch": args.workload_batch, **res[args.only_workload]}))
+
+
+def run_only_section(args, local):
+    """Time one auxiliary section of the report alone; prints one JSON line."""
+    import torch
+
+    from paper_2607_05722_gb300 import build as nld_build
+    from paper_2607_05722_gb300 import nld
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    nld_build.build()
+    nld.lib()
+    peak, _ = hbm_peak()
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    stream = torch.cuda.Stream(device=dev)
+    fn = {"decisions": lambda: run_decisions(torch, nld, dev, stream),
+          "logits": lambda: run_logits(torch, nld, dev, stream, peak, l2),
+          "kv_commit": lambda: run_kv_commit(torch, nld, dev, stream),
+          "quadss": lambda: run_quadss(torch, nld, dev, stream, peak, l2)}[args.only_section]
+    print(json.dumps({"section": args.only_section, **fn()}))
 
 
 def run_ours(args, world, rank, local):
@@ -814,6 +837,9 @@ def main():
         return
     if args.only_workload is not None:
         run_only_workload(args, local)
+        return
+    if args.only_section is not None:
+        run_only_section(args, local)
         return
     run_ours(args, world, rank, local)
 
