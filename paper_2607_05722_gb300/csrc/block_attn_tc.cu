@@ -11,10 +11,9 @@ int tc_max_active_clusters(int csize, int head_dim, int rows) {
   return head_dim == 128 ? max_active_clusters_d<128>(csize, rows) : max_active_clusters_d<64>(csize, rows);
 }
 
-cudaError_t launch_block_attn_tc(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, int head_dim,
-                                 cudaStream_t stream) {
-  if (a.mode == kModeBlockMask) return launch_block_attn_tc_masked(a, tmk, tmv, head_dim, stream);
-  return head_dim == 128 ? launch_tc_d<128, false>(a, tmk, tmv, stream) : launch_tc_d<64, false>(a, tmk, tmv, stream);
+cudaError_t launch_block_attn_tc(const AttnArgs& a, const TmaMaps& maps, int head_dim, cudaStream_t stream) {
+  if (a.mode == kModeBlockMask) return launch_block_attn_tc_masked(a, maps, head_dim, stream);
+  return head_dim == 128 ? launch_tc_d<128, false>(a, maps, stream) : launch_tc_d<64, false>(a, maps, stream);
 }
 
 }  // namespace nld

@@ -6,27 +6,29 @@
 // heads times the bl block tokens form R = G*bl <= 256 query rows in one or
 // two 128-row MMA tiles, so each K/V page leaves HBM once per (b, g).
 //
-// Warp roles (9 warps):
-//   warps 0-2, 8  TMA producers: the boxes of each 64-token K/V tile (16 tokens
-//             x 64 dims each) dealt four ways into a 4-stage ring (produce_kv);
-//             TMA issue cost is per warp, so four issuing warps land a tile
-//             sooner.
-//   warp 3    allocates the TMEM columns; lane 0 issues every MMA:
-//               S_k = Q K_k^T   (M=128 rows, N=64 tokens, K=D; double-buffered in TMEM)
+// Warp roles (5 + 4*MT warps):
+//   warps 0-2 and the last  TMA producers: the boxes of each 64-token K/V tile
+//             (16 tokens x 64 dims each) dealt four ways into a ring of up to
+//             8 stages (produce_kv); TMA issue cost is per warp, so four
+//             issuing warps land a tile sooner.
+//   warp 3    allocates the TMEM columns; lane 0 loads Q by TMA (one M tile)
+//             and issues every MMA:
+//               S_j = Q K^T     (M=128 rows, N=64*TPS tokens, K=D; double-buffered in TMEM)
 //               O  += P_k V_k   (M=128 rows, N=D, K=64 tokens; V read MN-major)
-//             S_{k+1} is issued before O += P_k V_k so the tensor core computes
-//             the next scores while the softmax warps work on the current ones.
-//   warps 4-7 softmax: thread t owns TMEM lane 32*(warp%4)+lane, one query
+//             S_{j+1} is issued before the PV products of S_j so the tensor
+//             core computes the next scores while the softmax warps work.
+//   warps 4.. softmax: thread t owns TMEM lane 32*(warp%4)+lane, one query
 //             row. It loads its S row, applies the mask and the base-2 scale,
 //             keeps the running max and sum, writes P (bf16) to shared memory
 //             for the PV MMA, and at the end reads O from TMEM, divides by the
-//             sum and stages its row in the freed K/V ring, from where one
-//             bulk copy per row writes it (bf16 output or fp32 split partial).
+//             sum and stages its row in the freed K/V ring in 128-byte-swizzled
+//             boxes, which one thread writes with tiled TMA stores (bf16 output
+//             or fp32 split partial; the CTA's rows are contiguous in both).
 //             With at most 64 (32) packed rows, Q is replicated into the idle
 //             lane quadrants (REP = 2 or 4): each copy of a row takes a 64/REP-
 //             token slice of every tile with its own running max and sum, so
 //             every softmax warp works and each does 1/REP of the exponentials;
-//             the slices are merged once, before the epilogue.
+//             the copies are merged once, each finalising 1/REP of the columns.
 // When the KV range of a (sequence, KV head) is split over a thread-block
 // cluster, the CTAs stage their normalised rows in shared memory and merge
 // them through distributed shared memory (a cluster barrier, then each CTA
@@ -52,19 +54,18 @@ constexpr int kSoftmaxWarp0 = 4;
 // many steps in the chain S -> softmax -> PV, and four P buffers so that the
 // softmax of one pair never waits for the PV products of the last. A long
 // split streams with TPS = 1, where a stage frees after each tile and more
-// of the ring stays in flight. With two M tiles the ring shrinks to 3
-// stages, so that two Q tiles and 2x2 P buffers fit.
+// of the ring stays in flight. The ring takes what shared memory the Q
+// tiles and P buffers leave (up to 8 stages): a streaming CTA's bandwidth is
+// the bytes it has in flight over the DRAM latency, so every stage counts.
 template <int MT, int TPS>
 struct TcCfg {
   static_assert(TPS == 1 || (TPS == 2 && MT == 1), "paired score products with one M tile");
-  static constexpr int kStages = MT == 1 ? 4 : 3;
   static constexpr int kTPS = TPS;               // K/V tiles per score product
   static constexpr int kSTok = kTPS * kTileTok;  // tokens (N) of a score product
   static constexpr int kPBufs = 2 * kTPS;        // P buffers per M tile
   static constexpr int kWarps = 5 + 4 * MT;      // 4 producers, 1 MMA, 4*MT softmax
   static constexpr int kThreads = 32 * kWarps;
   static constexpr uint32_t kTmemCols = 512;     // MT x (S0 | S1), then MT x O
-  static_assert(kStages % kTPS == 0, "a score product never wraps around the ring");
   static_assert(2 * MT * kSTok + MT * 128 <= 512, "TMEM columns");
 };
 
@@ -87,29 +88,38 @@ __host__ __device__ constexpr int merge_pitch() { return D * 4 + 16; }
 template <int D, int MT, int TPS>
 struct TcLayout {
   using Geo = TileGeom<D>;
-  static constexpr int kStages = TcCfg<MT, TPS>::kStages;
   static constexpr int kPBufs = TcCfg<MT, TPS>::kPBufs;
-  static constexpr int kVOff = kStages * Geo::kTileBytes;       // V tiles after the K tiles
   static constexpr int kQBytes = Geo::kColBlocks * 128 * 128;  // one 128-row Q tile, bf16
   static constexpr int kPBytes = 128 * kTileTok * 2;             // one 128-row x 64-token P buffer, bf16
+  // stages: what is left of 227 KB after Q, P, 512 bytes of barriers and the
+  // 1024-byte alignment slack, a multiple of TPS, at most 8
+  static constexpr int kFitStages =
+      (232448 - 1024 - 512 - MT * kQBytes - MT * kPBufs * kPBytes) / Geo::kStageBytes;
+  static constexpr int kStages = (kFitStages < 8 ? kFitStages : 8) / TPS * TPS;
+  static_assert(kStages >= 2 * TPS, "at least two score products in the ring");
+  static constexpr int kVOff = kStages * Geo::kTileBytes;       // V tiles after the K tiles
   static constexpr int kQOff = kStages * Geo::kStageBytes;
   static constexpr int kPOff = kQOff + MT * kQBytes;
   static constexpr int kBarOff = kPOff + MT * kPBufs * kPBytes;
-  // kv_full[st], kv_empty[st], s_full[2], s_free[2], p_full[P], o_done[P], q_ready, drain, tmem slot
-  static constexpr int kNumBars = 2 * kStages + 4 + 2 * kPBufs + 2;
+  // kv_full[st], kv_empty[st], s_full[2], s_free[2], p_full[P], o_done[P], q_ready, q_full, drain, tmem slot
+  static constexpr int kNumBars = 2 * kStages + 4 + 2 * kPBufs + 3;
   static constexpr int kBytes = kBarOff + kNumBars * 8 + 16;
+  static_assert(kNumBars * 8 + 16 <= 512, "barrier reserve");
   static_assert(kBytes + 1024 <= 232448, "shared memory per CTA");
   static constexpr int kMergeRows = 128 * MT;
   static constexpr int kLseOff = kMergeRows * merge_pitch<D>();
   static constexpr int kWtsOff = kLseOff + kMergeRows * 4;
   static constexpr int kLseOutOff = kWtsOff + kMergeRows * 8 * 4;
   static_assert(kLseOutOff + kMergeRows * 4 <= kPOff, "epilogue staging overlaps the live buffers");
+  // copies of a row (REP > 1) exchange their O column ranges here
+  static constexpr int kXchgOff = (kLseOutOff + kMergeRows * 4 + 15) / 16 * 16;
+  // output boxes for the tiled stores (128-byte rows, 1024-byte aligned)
+  static_assert(D / 32 * kMergeRows * 128 <= kPOff, "output staging");
 };
 
 template <int D, int MT, int REP, int TPS, bool MASKED>
 __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
-    block_attn_tc_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
-                         const AttnArgs a) {
+    block_attn_tc_kernel(const __grid_constant__ TmaMaps maps, const AttnArgs a) {
   static_assert(REP == 1 || REP == 2 || REP == 4, "replication of 1, 2 or 4");
   static_assert(MT == 1 || REP == 1, "replication only with one M tile");
   using Geo = TileGeom<D>;
@@ -127,7 +137,8 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
   uint64_t* p_full = s_free + 2;
   uint64_t* o_done = p_full + Cfg::kPBufs;
   uint64_t* q_ready = o_done + Cfg::kPBufs;
-  uint64_t* drain = q_ready + 1;
+  uint64_t* q_full = q_ready + 1;  // the Q tiles' TMA copies (one M tile)
+  uint64_t* drain = q_full + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
 
   const int warp = threadIdx.x >> 5;
@@ -148,12 +159,15 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
       mbar_init(&o_done[j], 1);
     }
     mbar_init(q_ready, 4 * MT);
+    mbar_init(q_full, 1);
     mbar_init(drain, 1);
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
-    prefetch_tensormap(&tmk);
-    prefetch_tensormap(&tmv);
+    prefetch_tensormap(&maps.k);
+    prefetch_tensormap(&maps.v);
+    prefetch_tensormap(&maps.o);
+    if (MT == 1) prefetch_tensormap(&maps.q);
   }
   if (warp == kMmaWarp) {
     tmem_alloc(tmem_slot, Cfg::kTmemCols);
@@ -215,7 +229,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
         ++early_tiles;
       if (early_tiles == 0) grid_dependency_wait();
     }
-    const int issued = produce_kv<D>(a, &tmk, &tmv, smem, kv_full, kv_empty, kTcStages, g, b, t_begin, t_end,
+    const int issued = produce_kv<D>(a, &maps.k, &maps.v, smem, kv_full, kv_empty, kTcStages, g, b, t_begin, t_end,
                                      ntiles, lane, producer_index<MT>(warp), kProducers, first, early_tiles);
     if (lane == 0 && issued < ntiles) {
       // Stopped early on a wait timeout: let the copies already issued land
@@ -226,7 +240,21 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
   } else if (warp == kMmaWarp) {
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
+      if constexpr (MT == 1) {
+        // Q by TMA, straight after the dependency wait: per column block one
+        // box of the CTA's R rows (G heads x bl slots, in packed row order),
+        // written once per copy.
+        if (early) grid_dependency_wait();
+        mbar_arrive_expect_tx(q_full, static_cast<uint32_t>(REP * (D / 64) * a.R * 128));
+#pragma unroll
+        for (int q = 0; q < REP; ++q)
+#pragma unroll
+          for (int cb = 0; cb < D / 64; ++cb)
+            tma_load_3d(q_s + cb * (128 * 128) + q * (128 / REP) * 128, &maps.q, q_full, cb * 64, g * a.G,
+                        b * a.bl);
+      }
       bool ok = mbar_wait(q_ready, 0, a.err);
+      if constexpr (MT == 1) ok = ok && mbar_wait(q_full, 0, a.err);
       tc_fence_after();
       const uint32_t q_addr = smem_u32(q_s);
       const uint32_t idesc_s = umma_idesc_bf16(128, kSTok, false);
@@ -339,9 +367,18 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     // rows zero); slice 0 loads it once and writes every copy. The columns of
     // P a thread never writes (other slices' tokens, or all of a padding row)
     // are zeroed once in every buffer.
-    if (early) grid_dependency_wait();
+    // One M tile: the MMA warp brings Q by TMA and the rows past R stay zero
+    // (written here, before the dependency wait). Two M tiles: the rows are
+    // loaded here after the wait.
+    if (MT == 1 && !row_ok) {
+#pragma unroll
+      for (int c = 0; c < D / 8; ++c)
+        *reinterpret_cast<uint4*>(q_tile + (c >> 3) * (128 * 128) + r_loc * 128 + (((c & 7) ^ swz) << 4)) =
+            make_uint4(0, 0, 0, 0);
+    }
+    if (MT == 2 && early) grid_dependency_wait();
     {
-      if (cp == 0) {
+      if (MT == 2 && cp == 0) {
         const uint4* qrow = reinterpret_cast<const uint4*>(
             a.q + ((static_cast<size_t>(b) * a.bl + row_i) * a.Hq + row_h) * D);
         uint4 v[D / 8];
@@ -365,6 +402,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(q_ready);
     }
+    if (MT == 1 && early) grid_dependency_wait();  // before the mask table and the outputs
 
     // The keys this row may see inside [t_begin, t_end) are exactly t < lim
     // (Sec. 2.2: the whole prefix; in the draft pass every block slot, in the
@@ -518,154 +556,197 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     // loads and stores below.
     const bool o_ready =
         __all_sync(0xffffffffu, ok && mbar_wait(&o_done[(ntiles - 1) % kPBufs], ((ntiles - 1) / kPBufs) & 1, a.err));
-    // Weights of the token slices of each row, by the split-combine rule
-    // (Sec. 3 Mode 2, here on one SM): slices cp > 0 leave their max, sum and
-    // unscaled O row in the freed ring (rows 32*kRowQuads.. of it); slice 0
-    // weighs them against its own and adds them in as it stages its output.
-    float w_self = 1.f;
-    float w_rep[REP > 1 ? REP - 1 : 1];
-    w_rep[0] = 0.f;
+    // Copies of a row (REP > 1) hold its O over disjoint token slices, merged
+    // by the split-combine rule (Sec. 3 Mode 2, here on one SM). The work is
+    // split by columns: copy c finalises output columns [c*kRange,
+    // (c+1)*kRange), so it leaves its (max, sum) and its unscaled O over the
+    // other copies' ranges in the freed ring and reads theirs over its own.
+    constexpr int kRange = D / REP;           // output columns this copy finalises
+    constexpr int kChunk = kRange < 64 ? kRange : 64;  // columns per TMEM load: 16, 32 or 64
+    static_assert(kChunk == 16 || kChunk == 32 || kChunk == 64, "TMEM load width");
+    auto ld_chunk = [&](uint32_t taddr, float* o) {
+      if constexpr (kChunk == 64) {
+        tmem_ld64(taddr, o);
+      } else if constexpr (kChunk == 32) {
+        tmem_ld32(taddr, o);
+      } else {
+        tmem_ld16(taddr, o);
+      }
+    };
+    constexpr int kXPitch = kRange * 4 + 16;  // exchange row pitch in bytes (padded: no bank conflicts)
+    // copy c's O over copy q's column range, for this thread's row
+    auto xchg_row = [&](int c, int q) -> uint8_t* {
+      const int slot = c * (REP - 1) + (q < c ? q : q - 1);
+      return smem + Lay::kXchgOff + (slot * 32 * kRowQuads + rq * 32 + lane) * kXPitch;
+    };
+    float wgt[REP];  // weight of each copy's O in this row's output, then with 1/sum folded in
+    float m_row = m_run, l_row = l_run;
+    wgt[0] = 1.f;
+    if (o_ready) tc_fence_after();
     if constexpr (REP > 1) {
+      static_assert(Lay::kXchgOff + REP * (REP - 1) * 32 * kRowQuads * kXPitch <= Lay::kPOff, "exchange buffers");
+      static_assert(D / 32 * (128 / REP) * 128 <= Lay::kWtsOff, "output staging below the copies' weights");
       float* part_ml = reinterpret_cast<float*>(smem + Lay::kWtsOff);  // [TMEM lane][max, sum]
-      if (o_ready) tc_fence_after();
-      if (cp > 0) {
-        part_ml[2 * r_loc] = o_ready ? m_run : -INFINITY;  // a slice cut short by a timeout is dropped
-        part_ml[2 * r_loc + 1] = l_run;
-        if (warp_rows && o_ready) {
-          uint8_t* xrow = smem + r_loc * merge_pitch<D>();
+      part_ml[2 * r_loc] = o_ready ? m_run : -INFINITY;  // a copy cut short by a timeout is dropped
+      part_ml[2 * r_loc + 1] = l_run;
+      if (warp_rows && o_ready) {
 #pragma unroll 1
-          for (int c = 0; c < D / 32; ++c) {
-            float o[32];
-            tmem_ld32(tO(mt) + lane_off + c * 32, o);
+        for (int q = 0; q < REP; ++q) {
+          if (q == cp) continue;
+          uint8_t* x = xchg_row(cp, q);
+#pragma unroll 1
+          for (int cc = 0; cc < kRange / kChunk; ++cc) {
+            float o[kChunk];
+            ld_chunk(tO(mt) + lane_off + q * kRange + cc * kChunk, o);
 #pragma unroll
-            for (int q4 = 0; q4 < 8; ++q4)
-              *reinterpret_cast<float4*>(xrow + c * 128 + q4 * 16) =
+            for (int q4 = 0; q4 < kChunk / 4; ++q4)
+              *reinterpret_cast<float4*>(x + cc * kChunk * 4 + q4 * 16) =
                   make_float4(o[4 * q4], o[4 * q4 + 1], o[4 * q4 + 2], o[4 * q4 + 3]);
           }
         }
       }
       named_bar_sync(2, 128);  // the four softmax warps
-      if (cp == 0) {
-        float m = m_run, mp[REP - 1], lp[REP - 1];
+      float mc[REP], lc[REP];
+      float m = -INFINITY;
 #pragma unroll
-        for (int q = 0; q < REP - 1; ++q) {
-          const int lq = ((q + 1) * kRowQuads + rq) * 32 + lane;
-          mp[q] = part_ml[2 * lq];
-          lp[q] = part_ml[2 * lq + 1];
-          m = fmaxf(m, mp[q]);
-        }
-        // A row that saw no key in any slice (possible in the verify pass)
-        // keeps m = -inf, sum 0 and weight 0 everywhere.
-        w_self = m_run == -INFINITY ? 0.f : ex2(m_run - m);
-        float l = w_self * l_run;
-#pragma unroll
-        for (int q = 0; q < REP - 1; ++q) {
-          w_rep[q] = mp[q] == -INFINITY ? 0.f : ex2(mp[q] - m);
-          l += w_rep[q] * lp[q];
-        }
-        if (m != -INFINITY) {
-          m_run = m;
-          l_run = l;
-        }
+      for (int c = 0; c < REP; ++c) {
+        const int lq = (c * kRowQuads + rq) * 32 + lane;
+        mc[c] = part_ml[2 * lq];
+        lc[c] = part_ml[2 * lq + 1];
+        m = fmaxf(m, mc[c]);
       }
+      // A row that saw no key in any slice (possible in the verify pass)
+      // keeps m = -inf, sum 0 and weight 0 everywhere.
+      float l = 0.f;
+#pragma unroll
+      for (int c = 0; c < REP; ++c) {
+        wgt[c] = mc[c] == -INFINITY ? 0.f : ex2(mc[c] - m);
+        l += wgt[c] * lc[c];
+      }
+      m_row = m;
+      l_row = l;
     }
-    // Unnormalised O of this thread's row, columns 64c..64c+63: its own TMEM
-    // lane plus, with REP > 1, the other slices of the row. Warp-collective.
-    auto load_o = [&](int c, float* o) {
-      tmem_ld64(tO(mt) + lane_off + c * 64, o);
+    const float inv = l_row > 0.f ? 1.f / l_row : 0.f;
+#pragma unroll
+    for (int c = 0; c < REP; ++c) wgt[c] *= inv;
+    // Normalised output columns cp*kRange + cc*kChunk .. +kChunk-1 of this
+    // thread's row: its own TMEM lane plus the other copies' exchanged ranges.
+    // Warp-collective.
+    auto final_chunk = [&](int cc, float* o) {
+      const int col0 = cp * kRange + cc * kChunk;
+      ld_chunk(tO(mt) + lane_off + col0, o);
+      float w_own = wgt[0];
+#pragma unroll
+      for (int c = 1; c < REP; ++c) w_own = c == cp ? wgt[c] : w_own;  // no dynamic register index
+#pragma unroll
+      for (int j = 0; j < kChunk; ++j) o[j] *= w_own;
       if constexpr (REP > 1) {
 #pragma unroll
-        for (int j = 0; j < 64; ++j) o[j] *= w_self;
+        for (int c = 0; c < REP; ++c) {
+          if (c == cp || wgt[c] == 0.f) continue;  // a copy without keys never wrote its range
+          const uint8_t* x = xchg_row(c, cp) + cc * kChunk * 4;
 #pragma unroll
-        for (int q = 0; q < REP - 1; ++q) {
-          if (w_rep[q] == 0.f) continue;  // a slice without keys never wrote its row
-          const uint8_t* xrow = smem + ((q + 1) * kRowQuads * 32 + rq * 32 + lane) * merge_pitch<D>() + c * 256;
-#pragma unroll
-          for (int q4 = 0; q4 < 16; ++q4) {
-            const float4 x = *reinterpret_cast<const float4*>(xrow + q4 * 16);
-            o[4 * q4] += w_rep[q] * x.x;
-            o[4 * q4 + 1] += w_rep[q] * x.y;
-            o[4 * q4 + 2] += w_rep[q] * x.z;
-            o[4 * q4 + 3] += w_rep[q] * x.w;
+          for (int q4 = 0; q4 < kChunk / 4; ++q4) {
+            const float4 v = *reinterpret_cast<const float4*>(x + q4 * 16);
+            o[4 * q4] += wgt[c] * v.x;
+            o[4 * q4 + 1] += wgt[c] * v.y;
+            o[4 * q4 + 2] += wgt[c] * v.z;
+            o[4 * q4 + 3] += wgt[c] * v.w;
           }
         }
       }
+      if (!(l_row > 0.f)) {
+#pragma unroll
+        for (int j = 0; j < kChunk; ++j) o[j] = 0.f;  // a row without keys: zeros
+      }
     };
-    // One thread per output row from here on (slice 0 of each row).
-    const bool out_warp = warp_rows && cp == 0;
-    const bool out_row = row_ok && cp == 0;
     if (a.csize > 1) {
       // Cluster: stage this CTA's normalised rows and their log2-sum-exp in
       // the freed ring for the merge across the cluster (rows without keys,
       // or after a timeout, carry lse = -inf and are skipped by the merge).
-      if (o_ready) tc_fence_after();
       float* lse_stage = reinterpret_cast<float*>(smem + Lay::kLseOff);
-      const float l = l_run;
-      const bool has = o_ready && out_row && l > 0.f;
-      if (cp == 0) lse_stage[r] = has ? m_run + lg2(l) : -INFINITY;
-      if (out_warp && o_ready) {
-        const float inv = l > 0.f ? 1.f / l : 0.f;
+      const bool has = o_ready && row_ok && l_row > 0.f;
+      if (cp == 0) lse_stage[r] = has ? m_row + lg2(l_row) : -INFINITY;
+      if (warp_rows && o_ready) {
         uint8_t* my = smem + r * merge_pitch<D>();
 #pragma unroll 1
-        for (int c = 0; c < D / 64; ++c) {
-          float o[64];
-          load_o(c, o);
+        for (int cc = 0; cc < kRange / kChunk; ++cc) {
+          float o[kChunk];
+          final_chunk(cc, o);
+          uint8_t* dst = my + (cp * kRange + cc * kChunk) * 4;
 #pragma unroll
-          for (int q4 = 0; q4 < 16; ++q4)
-            *reinterpret_cast<float4*>(my + c * 256 + q4 * 16) =
-                make_float4(o[4 * q4] * inv, o[4 * q4 + 1] * inv, o[4 * q4 + 2] * inv, o[4 * q4 + 3] * inv);
+          for (int q4 = 0; q4 < kChunk / 4; ++q4)
+            *reinterpret_cast<float4*>(dst + q4 * 16) =
+                make_float4(o[4 * q4], o[4 * q4 + 1], o[4 * q4 + 2], o[4 * q4 + 3]);
         }
       }
-    } else if (o_ready) {
-      // Each thread stages its row (padded pitch, no bank conflicts) and
-      // hands it to the TMA engine as one bulk copy.
-      tc_fence_after();
-      if (out_warp) {
-        const float l = l_run;
-        const float inv = l > 0.f ? 1.f / l : 0.f;
-        const float lse_v = l > 0.f ? (m_run + lg2(l)) * kLn2 : -INFINITY;
-        const bool split_out = a.o_part != nullptr;
-        const int row_bytes = split_out ? D * 4 : D * 2;
-        uint8_t* my = smem + (mt * 128 + r_loc) * (row_bytes + 16);
+    } else {
+      // The CTA's rows are contiguous in the output: per (block slot, head)
+      // in the bf16 output, per (head, block slot) in the fp32 partials. Each
+      // thread stages its columns in 128-byte-swizzled boxes of 128-byte rows
+      // (no bank conflicts), in that order, and one thread stores the boxes
+      // with tiled TMA copies: D/64 (bf16) or D/32 (fp32) copies per CTA.
+      const bool split_out = a.o_part != nullptr;
+      const int srow = split_out ? (r - row_i * a.G) * a.bl + row_i : r;  // row within the boxes
+      const int box_stride = (a.R * 128 + 1023) & ~1023;
+      // kIters rounds (2 with one copy and D = 128, else 1): round cc stages
+      // columns [cc*D/kIters, (cc+1)*D/kIters) of every row, and their boxes
+      // are stored while the next round is staged.
+      constexpr int kIters = kRange / kChunk;
 #pragma unroll 1
-        for (int c = 0; c < D / 64; ++c) {
-          float o[64];
-          load_o(c, o);
+      for (int cc = 0; cc < kIters; ++cc) {
+        if (warp_rows && o_ready) {
+          float o[kChunk];
+          final_chunk(cc, o);
+          const int col0 = cp * kRange + cc * kChunk;
+          if (row_ok) {
+            if (split_out) {
 #pragma unroll
-          for (int j = 0; j < 64; ++j) o[j] *= inv;
-          if (split_out) {
+              for (int k4 = 0; k4 < kChunk / 4; ++k4) {
+                const int col = col0 + 4 * k4;
+                uint8_t* row = smem + (col >> 5) * box_stride + srow * 128;
+                const float* v = o + 4 * k4;
+                *reinterpret_cast<float4*>(row + ((((col & 31) >> 2) ^ (srow & 7)) << 4)) =
+                    make_float4(v[0], v[1], v[2], v[3]);
+              }
+            } else {
+              uint8_t* row = smem + (col0 >> 6) * box_stride + srow * 128;
+              const int ch0 = (col0 & 63) >> 3;
 #pragma unroll
-            for (int q4 = 0; q4 < 16; ++q4)
-              *reinterpret_cast<float4*>(my + c * 256 + q4 * 16) =
-                  make_float4(o[4 * q4], o[4 * q4 + 1], o[4 * q4 + 2], o[4 * q4 + 3]);
-          } else {
-#pragma unroll
-            for (int q4 = 0; q4 < 8; ++q4) {
-              const int j = q4 * 8;
-              *reinterpret_cast<uint4*>(my + c * 128 + q4 * 16) =
-                  make_uint4(pack_bf16(o[j], o[j + 1]), pack_bf16(o[j + 2], o[j + 3]), pack_bf16(o[j + 4], o[j + 5]),
-                             pack_bf16(o[j + 6], o[j + 7]));
+              for (int c8 = 0; c8 < kChunk / 8; ++c8) {
+                const float* v = o + c8 * 8;
+                *reinterpret_cast<uint4*>(row + (((ch0 + c8) ^ (srow & 7)) << 4)) =
+                    make_uint4(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]), pack_bf16(v[4], v[5]),
+                               pack_bf16(v[6], v[7]));
+              }
             }
           }
         }
-        // Output row (unsplit) or partial row; partial rows without keys are
-        // not written (their lse is -inf and the combine skips them).
-        if (row_ok && (!split_out || l > 0.f)) {
-          const size_t grow = split_out ? ((static_cast<size_t>(split) * a.B + b) * a.Hq + row_h) * a.bl + row_i
-                                        : (static_cast<size_t>(b) * a.bl + row_i) * a.Hq + row_h;
-          uint8_t* gbase = split_out ? reinterpret_cast<uint8_t*>(a.o_part) : reinterpret_cast<uint8_t*>(a.out);
-          fence_proxy_async_smem();  // this thread's staged row, visible to the TMA engine
-          bulk_store(gbase + grow * row_bytes, my, static_cast<uint32_t>(row_bytes));
-        }
-        if (row_ok) {
-          if (!split_out) {
-            if (a.lse != nullptr) a.lse[(static_cast<size_t>(b) * a.Hq + row_h) * a.bl + row_i] = lse_v;
+        fence_proxy_async_smem();     // the staged boxes, visible to the TMA engine
+        named_bar_sync(3, 128 * MT);  // every softmax warp, with rows or not
+        if (sm_tid == 0 && o_ready) {
+          if (split_out) {
+            const int row0 = ((split * a.B + b) * a.Hq + g * a.G) * a.bl;
+#pragma unroll
+            for (int x = cc * (D / 32 / kIters); x < (cc + 1) * (D / 32 / kIters); ++x)
+              tma_store_2d(&maps.o, smem + x * box_stride, x * 32, row0);
           } else {
-            a.lse_part[((static_cast<size_t>(split) * a.B + b) * a.Hq + row_h) * a.bl + row_i] = lse_v;
+#pragma unroll
+            for (int x = cc * (D / 64 / kIters); x < (cc + 1) * (D / 64 / kIters); ++x)
+              tma_store_3d(&maps.o, smem + x * box_stride, x * 64, g * a.G, b * a.bl);
           }
+          bulk_commit();
         }
-        bulk_store_wait_read();  // the staged row stays in place until the copy has read it
       }
+      if (warp_rows && o_ready && row_ok && cp == 0) {
+        const float lse_v = l_row > 0.f ? (m_row + lg2(l_row)) * kLn2 : -INFINITY;
+        if (!split_out) {
+          if (a.lse != nullptr) a.lse[(static_cast<size_t>(b) * a.Hq + row_h) * a.bl + row_i] = lse_v;
+        } else {
+          a.lse_part[((static_cast<size_t>(split) * a.B + b) * a.Hq + row_h) * a.bl + row_i] = lse_v;
+        }
+      }
+      if (sm_tid == 0 && o_ready) bulk_store_wait_read();  // the boxes stay in place until read
     }
     tc_fence_before();
   }
@@ -785,14 +866,14 @@ cudaError_t configure_tc(int dev) {
 }
 
 template <int D, int MT, int REP, int TPS, bool MASKED>
-cudaError_t launch_tc_t(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, cudaStream_t stream) {
+cudaError_t launch_tc_t(const AttnArgs& a, const TmaMaps& maps, cudaStream_t stream) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if ((e = configure_tc<D, MT, REP, TPS, MASKED>(dev)) != cudaSuccess) return e;
   dim3 grid(a.num_splits, a.Hkv, a.B);
   return launch_kernel_cluster(block_attn_tc_kernel<D, MT, REP, TPS, MASKED>, grid, dim3(TcCfg<MT, TPS>::kThreads),
-                               TcLayout<D, MT, TPS>::kBytes + 1024, stream, a.csize, tmk, tmv, a);
+                               TcLayout<D, MT, TPS>::kBytes + 1024, stream, a.csize, maps, a);
 }
 
 // With one CTA per SM either way, cluster residency is the same for both
@@ -841,21 +922,21 @@ int max_active_clusters_d(int csize, int rows) {
 }
 
 template <int D, int TPS, bool MASKED>
-cudaError_t launch_tc_rep(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, cudaStream_t stream) {
+cudaError_t launch_tc_rep(const AttnArgs& a, const TmaMaps& maps, cudaStream_t stream) {
   switch (tc_replication(a.R)) {
-    case 4: return launch_tc_t<D, 1, 4, TPS, MASKED>(a, tmk, tmv, stream);
-    case 2: return launch_tc_t<D, 1, 2, TPS, MASKED>(a, tmk, tmv, stream);
-    default: return launch_tc_t<D, 1, 1, TPS, MASKED>(a, tmk, tmv, stream);
+    case 4: return launch_tc_t<D, 1, 4, TPS, MASKED>(a, maps, stream);
+    case 2: return launch_tc_t<D, 1, 2, TPS, MASKED>(a, maps, stream);
+    default: return launch_tc_t<D, 1, 1, TPS, MASKED>(a, maps, stream);
   }
 }
 
 // Paired score products when a split fits in the ring whole (it is then
 // latency-bound: fewer, wider steps help); single tiles when it streams.
 template <int D, bool MASKED>
-cudaError_t launch_tc_d(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv, cudaStream_t stream) {
-  if (a.R > 128) return launch_tc_t<D, 2, 1, 1, MASKED>(a, tmk, tmv, stream);
-  if (a.chunk <= TcCfg<1, 2>::kStages * kTileTok) return launch_tc_rep<D, 2, MASKED>(a, tmk, tmv, stream);
-  return launch_tc_rep<D, 1, MASKED>(a, tmk, tmv, stream);
+cudaError_t launch_tc_d(const AttnArgs& a, const TmaMaps& maps, cudaStream_t stream) {
+  if (a.R > 128) return launch_tc_t<D, 2, 1, 1, MASKED>(a, maps, stream);
+  if (a.chunk <= TcLayout<D, 1, 2>::kStages * kTileTok) return launch_tc_rep<D, 2, MASKED>(a, maps, stream);
+  return launch_tc_rep<D, 1, MASKED>(a, maps, stream);
 }
 
 }  // namespace

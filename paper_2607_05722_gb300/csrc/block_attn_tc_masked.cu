@@ -6,9 +6,8 @@
 
 namespace nld {
 
-cudaError_t launch_block_attn_tc_masked(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv,
-                                        int head_dim, cudaStream_t stream) {
-  return head_dim == 128 ? launch_tc_d<128, true>(a, tmk, tmv, stream) : launch_tc_d<64, true>(a, tmk, tmv, stream);
+cudaError_t launch_block_attn_tc_masked(const AttnArgs& a, const TmaMaps& maps, int head_dim, cudaStream_t stream) {
+  return head_dim == 128 ? launch_tc_d<128, true>(a, maps, stream) : launch_tc_d<64, true>(a, maps, stream);
 }
 
 }  // namespace nld

@@ -1,6 +1,7 @@
 // C ABI of libnld (include/nld.h): host-side argument checks, KV split choice,
 // TMA descriptor encoding and kernel launches. Nothing here allocates device
 // memory or synchronises, except nld_device_error().
+#include <climits>
 #include <math.h>
 #include <stdio.h>
 #include <stdlib.h>
@@ -179,6 +180,40 @@ nld_status_t encode_pool_map(CUtensorMap* map, const void* base, const nld_attn_
   return r == CUDA_SUCCESS ? NLD_OK : NLD_ERR_CUDA;
 }
 
+// Map over a [B, bl, Hq, D] bf16 block (queries or output) whose box is one
+// CTA's R = G * bl rows of 64 dims (G heads x bl slots), 128-byte swizzle.
+nld_status_t encode_block_map(CUtensorMap* map, const void* base, const nld::AttnArgs& a, int D) {
+  EncodeTiledFn fn = encode_fn();
+  if (fn == nullptr) return NLD_ERR_CUDA;
+  cuuint32_t estr[3] = {1, 1, 1};
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(a.Hq), static_cast<cuuint64_t>(a.B) * a.bl};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(D) * 2, static_cast<cuuint64_t>(D) * 2 * a.Hq};
+  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(a.G), static_cast<cuuint32_t>(a.bl)};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? NLD_OK : NLD_ERR_CUDA;
+}
+
+// Map for the tiled output stores of one CTA's R = G * bl rows, 128-byte
+// swizzle. Split partials: fp32 rows [partials * B * Hq * bl, D], box 32 dims
+// x R rows. Final output [B, bl, Hq, D] bf16: box 64 dims x G heads x bl slots.
+nld_status_t encode_out_map(CUtensorMap* map, const nld::AttnArgs& a, int D) {
+  if (a.o_part == nullptr) return encode_block_map(map, a.out, a, D);
+  EncodeTiledFn fn = encode_fn();
+  if (fn == nullptr) return NLD_ERR_CUDA;
+  const long long rows = static_cast<long long>(a.num_partials) * a.B * a.Hq * a.bl;
+  if (rows > INT_MAX) return NLD_ERR_UNSUPPORTED;  // row coordinates are int
+  cuuint32_t estr[2] = {1, 1};
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(D) * 4};
+  cuuint32_t box[2] = {32, static_cast<cuuint32_t>(a.R)};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, a.o_part, dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? NLD_OK : NLD_ERR_CUDA;
+}
+
 }  // namespace
 
 namespace nld {
@@ -251,9 +286,9 @@ nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_bloc
   st = device_state(&err, nullptr);
   if (st != NLD_OK) return st;
 
-  CUtensorMap tmk, tmv;
-  if ((st = encode_pool_map(&tmk, k_pages, params)) != NLD_OK) return st;
-  if ((st = encode_pool_map(&tmv, v_pages, params)) != NLD_OK) return st;
+  nld::TmaMaps maps;
+  if ((st = encode_pool_map(&maps.k, k_pages, params)) != NLD_OK) return st;
+  if ((st = encode_pool_map(&maps.v, v_pages, params)) != NLD_OK) return st;
 
   const int G = params->num_q_heads / params->num_kv_heads;
   const float scale = params->softmax_scale > 0.f ? params->softmax_scale : 1.0f / sqrtf((float)params->head_dim);
@@ -286,7 +321,9 @@ nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_bloc
     a.o_part = static_cast<float*>(workspace);
     a.lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) + o_bytes);
   }
-  if (nld::launch_block_attn_tc(a, tmk, tmv, params->head_dim, stream) != cudaSuccess) return NLD_ERR_CUDA;
+  if ((st = encode_out_map(&maps.o, a, params->head_dim)) != NLD_OK) return st;
+  if ((st = encode_block_map(&maps.q, q_block, a, params->head_dim)) != NLD_OK) return st;
+  if (nld::launch_block_attn_tc(a, maps, params->head_dim, stream) != cudaSuccess) return NLD_ERR_CUDA;
   if (plan.partials > 1 && run_combine) {
     if (nld::launch_combine(a.o_part, a.lse_part, plan.partials, a.B, a.Hq, block_len, params->head_dim, a.out, lse,
                             stream) != cudaSuccess)

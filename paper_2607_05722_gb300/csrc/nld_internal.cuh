@@ -46,11 +46,15 @@ struct AttnArgs {
 // Launchers (defined next to their kernels). Return a CUDA error code.
 // tcgen05 kernel: query rows R <= 256 (one or two 128-row MMA tiles).
 bool tc_supports(int R, int head_dim);
-cudaError_t launch_block_attn_tc(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv,
-                                 int head_dim, cudaStream_t stream);
+// Tensor maps of one call: k/v the K/V page pools; q the query block and o
+// the output (bf16 rows) or, with split partials, the fp32 partial rows, in
+// boxes of one CTA's rows.
+struct TmaMaps {
+  CUtensorMap k, v, o, q;
+};
+cudaError_t launch_block_attn_tc(const AttnArgs& a, const TmaMaps& maps, int head_dim, cudaStream_t stream);
 // The same for a table mask (a.mode == kModeBlockMask; block_attn_tc_masked.cu).
-cudaError_t launch_block_attn_tc_masked(const AttnArgs& a, const CUtensorMap& tmk, const CUtensorMap& tmv,
-                                        int head_dim, cudaStream_t stream);
+cudaError_t launch_block_attn_tc_masked(const AttnArgs& a, const TmaMaps& maps, int head_dim, cudaStream_t stream);
 cudaError_t launch_combine(const float* o_part, const float* lse_part, int S, int B, int Hq, int bl,
                            int D, __nv_bfloat16* out, float* lse, cudaStream_t stream);
 cudaError_t launch_accept(const int32_t* draft, const int32_t* verify, int B, int n, int32_t* acc,
@@ -210,6 +214,16 @@ __device__ __forceinline__ void tma_load_4d(void* dst, const CUtensorMap* map, u
       : "memory");
 }
 
+// 3-D tiled TMA load into shared memory, completing on an mbarrier.
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, uint64_t* bar, int c0, int c1,
+                                            int c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2)
+      : "memory");
+}
+
 __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
@@ -305,6 +319,24 @@ __device__ __forceinline__ void bulk_store(void* gdst, const void* ssrc, uint32_
                : "memory");
 }
 __device__ __forceinline__ void bulk_store_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+
+// Tiled TMA stores shared -> global (one box at coordinates {c0, c1[, c2]},
+// the innermost coordinate a multiple of 16 bytes), in the issuing thread's
+// bulk group: close it with bulk_commit() and wait with bulk_store_wait_read()
+// before the source is overwritten or the CTA exits.
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int c0, int c1) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(smem_u32(src)), "r"(c0), "r"(c1)
+               : "memory");
+}
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void* src, int c0, int c1, int c2) {
+  asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(smem_u32(src)), "r"(c0), "r"(c1), "r"(c2)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
