@@ -681,13 +681,13 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
         }
       }
     } else {
-      // The CTA's rows are contiguous in the output: per (block slot, head)
-      // in the bf16 output, per (head, block slot) in the fp32 partials. Each
-      // thread stages its columns in 128-byte-swizzled boxes of 128-byte rows
-      // (no bank conflicts), in that order, and one thread stores the boxes
-      // with tiled TMA copies: D/64 (bf16) or D/32 (fp32) copies per CTA.
+      // Each thread stages its columns in 128-byte-swizzled boxes of 128-byte
+      // rows in packed row order (block slot major, so that any 8 consecutive
+      // lanes hit 8 different bank groups), and one thread stores the boxes
+      // with tiled TMA copies: D/64 (bf16 output) or D/32 (fp32 partials,
+      // whose map walks the heads before the block slots) copies per CTA.
       const bool split_out = a.o_part != nullptr;
-      const int srow = split_out ? (r - row_i * a.G) * a.bl + row_i : r;  // row within the boxes
+      const int srow = r;  // row within the boxes
       const int box_stride = (a.R * 128 + 1023) & ~1023;
       // kIters rounds (2 with one copy and D = 128, else 1): round cc stages
       // columns [cc*D/kIters, (cc+1)*D/kIters) of every row, and their boxes
@@ -726,10 +726,9 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
         named_bar_sync(3, 128 * MT);  // every softmax warp, with rows or not
         if (sm_tid == 0 && o_ready) {
           if (split_out) {
-            const int row0 = ((split * a.B + b) * a.Hq + g * a.G) * a.bl;
 #pragma unroll
             for (int x = cc * (D / 32 / kIters); x < (cc + 1) * (D / 32 / kIters); ++x)
-              tma_store_2d(&maps.o, smem + x * box_stride, x * 32, row0);
+              tma_store_4d(&maps.o, smem + x * box_stride, x * 32, g * a.G, 0, split * a.B + b);
           } else {
 #pragma unroll
             for (int x = cc * (D / 64 / kIters); x < (cc + 1) * (D / 64 / kIters); ++x)

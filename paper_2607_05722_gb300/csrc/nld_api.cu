@@ -196,19 +196,23 @@ nld_status_t encode_block_map(CUtensorMap* map, const void* base, const nld::Att
 }
 
 // Map for the tiled output stores of one CTA's R = G * bl rows, 128-byte
-// swizzle. Split partials: fp32 rows [partials * B * Hq * bl, D], box 32 dims
-// x R rows. Final output [B, bl, Hq, D] bf16: box 64 dims x G heads x bl slots.
+// swizzle, rows in packed order (block slot major). Final output [B, bl, Hq,
+// D] bf16: box 64 dims x G heads x bl slots. Split partials [partials * B,
+// Hq, bl, D] fp32: the map walks dims, heads (stride bl * D), block slots
+// (stride D), then (partial, sequence); box 32 dims x G heads x bl slots.
 nld_status_t encode_out_map(CUtensorMap* map, const nld::AttnArgs& a, int D) {
   if (a.o_part == nullptr) return encode_block_map(map, a.out, a, D);
   EncodeTiledFn fn = encode_fn();
   if (fn == nullptr) return NLD_ERR_CUDA;
-  const long long rows = static_cast<long long>(a.num_partials) * a.B * a.Hq * a.bl;
-  if (rows > INT_MAX) return NLD_ERR_UNSUPPORTED;  // row coordinates are int
-  cuuint32_t estr[2] = {1, 1};
-  cuuint64_t dims[2] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(rows)};
-  cuuint64_t strides[1] = {static_cast<cuuint64_t>(D) * 4};
-  cuuint32_t box[2] = {32, static_cast<cuuint32_t>(a.R)};
-  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, a.o_part, dims, strides, box, estr,
+  const long long units = static_cast<long long>(a.num_partials) * a.B;
+  if (units > INT_MAX) return NLD_ERR_UNSUPPORTED;  // coordinates are int
+  const cuuint64_t row = static_cast<cuuint64_t>(D) * 4;
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(a.Hq), static_cast<cuuint64_t>(a.bl),
+                        static_cast<cuuint64_t>(units)};
+  cuuint64_t strides[3] = {row * a.bl, row, row * a.bl * a.Hq};
+  cuuint32_t box[4] = {32, static_cast<cuuint32_t>(a.G), static_cast<cuuint32_t>(a.bl), 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, a.o_part, dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? NLD_OK : NLD_ERR_CUDA;
