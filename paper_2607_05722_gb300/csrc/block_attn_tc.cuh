@@ -343,14 +343,20 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     // ---------------- softmax warps ----------------
     // Warp `quad` reads TMEM lanes 32*quad..+31. With REP > 1 those lanes hold
     // a copy of row block rq = quad % kRowQuads and the warp takes the token
-    // slice cp = quad / kRowQuads (columns c0 .. c0+kCols-1) of every tile.
+    // slice cp = quad / kRowQuads (columns c0u .. c0u+kColsU-1) of every step.
     constexpr int kRowQuads = 4 / REP;
-    constexpr int kCols = kTileTok / REP;           // S columns per thread and tile
+    // Softmax steps: one tile, or with paired score products and copies
+    // (TPS = 2, REP >= 2) the whole product, so that a step's columns per
+    // thread stay at most 64 and its work is one max and one exponential pass.
+    constexpr int kU = (kTPS == 2 && REP >= 2) ? 2 : 1;  // tiles per softmax step
+    constexpr int kColsU = kU * kTileTok / REP;          // S columns per thread and step
     const int quad = warp & 3;
     const int mt = (warp - kSoftmaxWarp0) >> 2;     // M tile of this warp
     const int rq = quad % kRowQuads;                // row block
     const int cp = quad / kRowQuads;                // token slice
-    const int c0 = cp * kCols;
+    const int c0u = cp * kColsU;           // first column of this thread's slice of a step
+    const int h_own = c0u / kTileTok;      // the step's tile holding the slice
+    const int lc0 = c0u % kTileTok;        // first column of the slice within that tile
     const int r_loc = quad * 32 + lane;             // TMEM lane == row of the Q and P tiles
     const int r = mt * 128 + rq * 32 + lane;        // packed query row
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
@@ -396,18 +402,20 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
       for (int j = 0; j < kPBufs; ++j)
 #pragma unroll
         for (int c = 0; c < 8; ++c)
-          if (!row_ok || c < c0 / 8 || c >= (c0 + kCols) / 8)
+          if (!row_ok || j % kU != h_own || c < lc0 / 8 || c >= (lc0 + kColsU) / 8)
             *reinterpret_cast<uint4*>(p_buf(j) + r_loc * 128 + ((c ^ swz) << 4)) = make_uint4(0, 0, 0, 0);
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(q_ready);
     }
+
     if (MT == 1 && early) grid_dependency_wait();  // before the mask table and the outputs
 
     // The keys this row may see inside [t_begin, t_end) are exactly t < lim
     // (Sec. 2.2: the whole prefix; in the draft pass every block slot, in the
-    // verify pass the block slots up to the row's own), so the mask is one
-    // compare per element on every tile, with no separate code path.
+    // verify pass the block slots up to the row's own), so a step's visible
+    // columns are a leading run of them, one compare to find; a step whose
+    // columns a whole warp sees skips the mask.
     const int lim = diff_mode ? t_end : min(t_end, L + row_i + 1);
     // MASKED (a table mask, e.g. quadratic self-speculation's, Sec. 3): the
     // prefix and the block slots whose bit is set in this row's table entry;
@@ -417,12 +425,12 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     if constexpr (MASKED) rowbits = row_ok ? __ldg(a.block_mask + row_i) : 0u;
     const int plim = min(t_end, L);  // prefix keys of this split end here
     auto column_mask = [&](int col0) -> uint64_t {  // col0: token of this thread's first column
-      const int np = min(max(plim - col0, 0), kCols);
+      const int np = min(max(plim - col0, 0), kColsU);
       uint64_t vis = np >= 64 ? ~0ull : (1ull << np) - 1ull;
       const int off = col0 - L;  // block slot of column 0
-      if (off < a.bl && off + kCols > 0) {
+      if (off < a.bl && off + kColsU > 0) {
         uint64_t bb = off >= 0 ? static_cast<uint64_t>(rowbits) >> off : static_cast<uint64_t>(rowbits) << -off;
-        const int nvalid = min(max(t_end - col0, 0), kCols);
+        const int nvalid = min(max(t_end - col0, 0), kColsU);
         bb &= nvalid >= 64 ? ~0ull : (1ull << nvalid) - 1ull;
         vis |= bb;
       }
@@ -435,23 +443,23 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     };
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
-    for (int k = 0; k < ntiles; ++k) {
-      const int j = k / kTPS, half = k % kTPS;  // score product and its 64-token half
-      const int buf = k % kPBufs;               // P buffer
-      const int st = k % kTcStages;
-      const int tile_t0 = t_begin + k * kTileTok;
-      const int valid = t_end - tile_t0;
+    const int nsteps = (ntiles + kU - 1) / kU;
+    for (int u = 0; u < nsteps; ++u) {
+      const int k0 = u * kU;                      // first tile of the step
+      const int j = k0 / kTPS, half = k0 % kTPS;  // score product and the step's first 64-token half
+      const int step_t0 = t_begin + k0 * kTileTok;
+      const int k_own = k0 + h_own;               // the tile holding this thread's columns
       if (half == 0 && !warp_wait(&s_full[j & 1], (j >> 1) & 1)) {
         ok = false;
         break;
       }
       tc_fence_after();
-      float s[kCols];
+      float s[kColsU];
       if (warp_rows) {
-        const uint32_t ts = tS(mt, j & 1) + lane_off + static_cast<uint32_t>(half * kTileTok + c0);
-        if constexpr (kCols == 64) {
+        const uint32_t ts = tS(mt, j & 1) + lane_off + static_cast<uint32_t>(half * kTileTok + c0u);
+        if constexpr (kColsU == 64) {
           tmem_ld64(ts, s);
-        } else if constexpr (kCols == 32) {
+        } else if constexpr (kColsU == 32) {
           tmem_ld32(ts, s);
         } else {
           tmem_ld16(ts, s);
@@ -459,28 +467,35 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0 && (half == kTPS - 1 || k == ntiles - 1)) mbar_arrive(&s_free[j & 1]);
+      const int k_last = min(k0 + kU - 1, ntiles - 1);  // last tile of the step
+      if (lane == 0 && (k_last % kTPS == kTPS - 1 || k_last == ntiles - 1)) mbar_arrive(&s_free[j & 1]);
 
       float alpha = 1.f;
       bool rescale = false;
       if (warp_rows) {
-        // Mask, base-2 scale and row max, branch-free.
-        float mx = -INFINITY;
+        // Row max on the raw scores (the scale is positive, so it commutes
+        // with the max; it is applied in the exponent below), four partial
+        // maxima of three-input max instructions. A step whose columns this
+        // warp sees in full (nearly every prefix step) takes no mask.
+        uint64_t vis = ~0ull;
         if constexpr (MASKED) {
-          const uint64_t vis = column_mask(tile_t0 + c0);
-#pragma unroll
-          for (int j = 0; j < kCols; ++j) {
-            s[j] = ((vis >> j) & 1ull) ? s[j] * scl : -INFINITY;
-            mx = fmaxf(mx, s[j]);
-          }
+          vis = column_mask(step_t0 + c0u);
         } else {
-          const int nv = lim - (tile_t0 + c0);
-#pragma unroll
-          for (int j = 0; j < kCols; ++j) {
-            s[j] = j < nv ? s[j] * scl : -INFINITY;
-            mx = fmaxf(mx, s[j]);
-          }
+          const int nv = lim - (step_t0 + c0u);
+          vis = nv >= 64 ? ~0ull : nv <= 0 ? 0ull : (1ull << nv) - 1ull;
         }
+        constexpr uint64_t kAll = kColsU >= 64 ? ~0ull : (1ull << kColsU) - 1ull;
+        if (!__all_sync(0xffffffffu, (vis & kAll) == kAll)) {
+#pragma unroll
+          for (int e = 0; e < kColsU; ++e) s[e] = ((vis >> e) & 1ull) ? s[e] : -INFINITY;
+        }
+        float pm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+        for (int e = 0; e < kColsU; e += 8) {
+#pragma unroll
+          for (int q = 0; q < 4; ++q) pm[q] = fmax3(pm[q], s[e + 2 * q], s[e + 2 * q + 1]);
+        }
+        const float mx = fmax3(pm[0], pm[1], fmaxf(pm[2], pm[3])) * scl;  // base-2 units
         if (m_run == -INFINITY) {
           m_run = mx;  // nothing accumulated for this row yet
         } else if (mx > m_run + kRescaleLog2) {
@@ -491,8 +506,8 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
         }
       }
       if (__any_sync(0xffffffffu, rescale)) {
-        // O holds P_0..P_{k-1} V: wait for the last PV, then scale this warp's rows.
-        if (!warp_wait(&o_done[(k - 1) % kPBufs], ((k - 1) / kPBufs) & 1)) {
+        // O holds P_0..P_{k0-1} V: wait for the last PV, then scale this warp's rows.
+        if (!warp_wait(&o_done[(k0 - 1) % kPBufs], ((k0 - 1) / kPBufs) & 1)) {
           ok = false;
           break;
         }
@@ -502,51 +517,73 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
           float o[32];
           tmem_ld32(tO(mt) + lane_off + c * 32, o);
 #pragma unroll
-          for (int j = 0; j < 32; ++j) o[j] *= alpha;
+          for (int e = 0; e < 32; ++e) o[e] *= alpha;
           tmem_st32(tO(mt) + lane_off + c * 32, o);
         }
       }
-      // P buffer `buf` is free once the PV of tile k-kPBufs has completed.
-      if (k >= kPBufs && !warp_wait(&o_done[buf], ((k / kPBufs) - 1) & 1)) {
-        ok = false;
-        break;
-      }
-      if (warp_rows) {
-        const float mu = m_run == -INFINITY ? 0.f : m_run;
-        uint8_t* prow = p_buf(buf) + r_loc * 128;
-#pragma unroll
-        for (int c = 0; c < kCols / 8; ++c) {
-          uint32_t w[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float p0 = ex2(s[c * 8 + 2 * e] - mu);
-            const float p1 = ex2(s[c * 8 + 2 * e + 1] - mu);
-            l_run += p0 + p1;
-            w[e] = pack_bf16(p0, p1);
-          }
-          const int chunk = c0 / 8 + c;
-          *reinterpret_cast<uint4*>(prow + ((chunk ^ swz) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
-        }
-      }
-      if (valid < kTileTok && (valid & (kGroupTok - 1))) {
-        // Cache slots past the sequence end inside its last page may hold
-        // stale or uninitialised data; P is 0 there but 0 * NaN = NaN, so
-        // zero those V rows before the PV MMA reads them.
-        if (!warp_wait(&kv_full[st], (k / kTcStages) & 1)) {
+      if (k_own < ntiles) {
+        // P buffer of tile k_own is free once the PV of tile k_own-kPBufs has completed.
+        const int buf = k_own % kPBufs;
+        if (k_own >= kPBufs && !warp_wait(&o_done[buf], ((k_own / kPBufs) - 1) & 1)) {
           ok = false;
           break;
         }
-        const int r0 = valid, r1 = (valid + kGroupTok - 1) & ~(kGroupTok - 1);
-        uint8_t* vt = smem + Lay::kVOff + st * Geo::kTileBytes;
-        for (int idx = sm_tid; idx < (r1 - r0) * (D / 8); idx += 128 * MT) {
-          const int row = r0 + idx / (D / 8), c = idx % (D / 8);
-          *reinterpret_cast<uint4*>(vt + kv_swz(row, c)) = make_uint4(0, 0, 0, 0);
+        if (warp_rows) {
+          // p = 2^(s * scale * log2(e) - m): per pair of elements one paired
+          // FMA, two exponentials, one bf16 pack and one paired add.
+          const float nmu = m_run == -INFINITY ? 0.f : -m_run;
+          const float2 sc2 = make_float2(scl, scl), nm2 = make_float2(nmu, nmu);
+          uint8_t* prow = p_buf(buf) + r_loc * 128;
+          float2 ls[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+#pragma unroll
+          for (int c = 0; c < kColsU / 8; ++c) {
+            uint32_t w[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float2 x = fma2(make_float2(s[c * 8 + 2 * e], s[c * 8 + 2 * e + 1]), sc2, nm2);
+              const float2 pp = make_float2(ex2(x.x), ex2(x.y));
+              ls[e & 1] = add2(ls[e & 1], pp);
+              w[e] = pack_bf16(pp.x, pp.y);
+            }
+            const int chunk = lc0 / 8 + c;
+            *reinterpret_cast<uint4*>(prow + ((chunk ^ swz) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+          }
+          l_run += (ls[0].x + ls[0].y) + (ls[1].x + ls[1].y);
         }
       }
-      fence_proxy_async_smem();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&p_full[buf]);
+      // Hand the step's tiles to the MMA warp (every softmax warp arrives
+      // for every tile; P columns a warp does not own stay zero).
+      bool step_ok = true;
+#pragma unroll
+      for (int h = 0; h < kU; ++h) {
+        const int k = k0 + h;
+        if (k >= ntiles) break;
+        const int valid = t_end - (t_begin + k * kTileTok);
+        if (valid < kTileTok && (valid & (kGroupTok - 1))) {
+          // Cache slots past the sequence end inside its last page may hold
+          // stale or uninitialised data; P is 0 there but 0 * NaN = NaN, so
+          // zero those V rows before the PV MMA reads them.
+          const int st = k % kTcStages;
+          if (!warp_wait(&kv_full[st], (k / kTcStages) & 1)) {
+            step_ok = false;
+            break;
+          }
+          const int r0 = valid, r1 = (valid + kGroupTok - 1) & ~(kGroupTok - 1);
+          uint8_t* vt = smem + Lay::kVOff + st * Geo::kTileBytes;
+          for (int idx = sm_tid; idx < (r1 - r0) * (D / 8); idx += 128 * MT) {
+            const int row = r0 + idx / (D / 8), c = idx % (D / 8);
+            *reinterpret_cast<uint4*>(vt + kv_swz(row, c)) = make_uint4(0, 0, 0, 0);
+          }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&p_full[k % kPBufs]);
+      }
+      if (!step_ok) {
+        ok = false;
+        break;
+      }
     }
 
     // ---------------- epilogue ----------------
