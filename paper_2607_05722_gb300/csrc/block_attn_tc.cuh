@@ -62,7 +62,7 @@ struct TcCfg {
   static_assert(TPS == 1 || (TPS == 2 && MT == 1), "paired score products with one M tile");
   static constexpr int kTPS = TPS;               // K/V tiles per score product
   static constexpr int kSTok = kTPS * kTileTok;  // tokens (N) of a score product
-  static constexpr int kPBufs = 2 * kTPS;        // P buffers per M tile
+  static constexpr int kPBufs = 2 * kTPS;        // tiles in flight between the softmax and PV (barrier slots)
   static constexpr int kWarps = 5 + 4 * MT;      // 4 producers, 1 MMA, 4*MT softmax
   static constexpr int kThreads = 32 * kWarps;
   static constexpr uint32_t kTmemCols = 512;     // MT x (S0 | S1), then MT x O
@@ -90,17 +90,15 @@ struct TcLayout {
   using Geo = TileGeom<D>;
   static constexpr int kPBufs = TcCfg<MT, TPS>::kPBufs;
   static constexpr int kQBytes = Geo::kColBlocks * 128 * 128;  // one 128-row Q tile, bf16
-  static constexpr int kPBytes = 128 * kTileTok * 2;             // one 128-row x 64-token P buffer, bf16
-  // stages: what is left of 227 KB after Q, P, 512 bytes of barriers and the
-  // 1024-byte alignment slack, a multiple of TPS, at most 8
-  static constexpr int kFitStages =
-      (232448 - 1024 - 512 - MT * kQBytes - MT * kPBufs * kPBytes) / Geo::kStageBytes;
+  // stages: what is left of 227 KB after Q, 512 bytes of barriers and the
+  // 1024-byte alignment slack, a multiple of TPS, at most 8 (P lives in TMEM)
+  static constexpr int kFitStages = (232448 - 1024 - 512 - MT * kQBytes) / Geo::kStageBytes;
   static constexpr int kStages = (kFitStages < 8 ? kFitStages : 8) / TPS * TPS;
   static_assert(kStages >= 2 * TPS, "at least two score products in the ring");
   static constexpr int kVOff = kStages * Geo::kTileBytes;       // V tiles after the K tiles
   static constexpr int kQOff = kStages * Geo::kStageBytes;
-  static constexpr int kPOff = kQOff + MT * kQBytes;
-  static constexpr int kBarOff = kPOff + MT * kPBufs * kPBytes;
+  static constexpr int kPOff = kQOff + MT * kQBytes;  // end of the ring and Q tiles
+  static constexpr int kBarOff = kPOff;
   // kv_full[st], kv_empty[st], s_full[2], s_free[2], p_full[P], o_done[P], q_ready, q_full, drain, tmem slot
   static constexpr int kNumBars = 2 * kStages + 4 + 2 * kPBufs + 3;
   static constexpr int kBytes = kBarOff + kNumBars * 8 + 16;
@@ -285,15 +283,15 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
         const uint32_t v_addr = smem_u32(smem + Lay::kVOff + st * Geo::kTileBytes);
 #pragma unroll
         for (int mt = 0; mt < MT; ++mt) {
-        const uint32_t p_addr = smem_u32(smem + Lay::kPOff + (mt * kPBufs + k % kPBufs) * Lay::kPBytes);
+          // A = P in TMEM (bf16 pairs over the S columns of the tile's first
+          // half: 32 columns per 64-token tile); B = V (MN-major: 64-dim
+          // atoms LBO apart, 8-token row groups SBO apart).
+          const uint32_t p_tmem = tS(mt, (k / kTPS) & 1) + static_cast<uint32_t>((k % kTPS) * 32);
 #pragma unroll
-        for (int kt = 0; kt < kTileTok / 16; ++kt) {
-          // A = P rows (K-major, one 128-byte block of 64 tokens); B = V (MN-major:
-          // 64-dim atoms LBO apart, 8-token row groups SBO apart).
-          const uint64_t ad = sw128_desc(p_addr + kt * 32, 0, 1024);
-          const uint64_t bd = sw128_desc(v_addr + kt * 16 * 128, Geo::kColBlockBytes, 1024);
-          umma_bf16(tO(mt), ad, bd, idesc_o, (k > 0 || kt > 0) ? 1u : 0u);
-        }
+          for (int kt = 0; kt < kTileTok / 16; ++kt) {
+            const uint64_t bd = sw128_desc(v_addr + kt * 16 * 128, Geo::kColBlockBytes, 1024);
+            umma_bf16_ts(tO(mt), p_tmem + kt * 8, bd, idesc_o, (k > 0 || kt > 0) ? 1u : 0u);
+          }
         }
         umma_commit(&o_done[k % kPBufs]);
         umma_commit(&kv_empty[st]);
@@ -367,7 +365,6 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     const int sm_tid = threadIdx.x - 32 * kSoftmaxWarp0;  // 0 .. 128*MT-1 across the softmax warps
     const int swz = r_loc & 7;                      // 128-byte swizzle phase of this tile row
     uint8_t* q_tile = q_s + mt * Lay::kQBytes;
-    auto p_buf = [&](int j) -> uint8_t* { return smem + Lay::kPOff + (mt * kPBufs + j) * Lay::kPBytes; };
 
     // Q row -> shared memory in the 128-byte-swizzled K-major layout (padding
     // rows zero); slice 0 loads it once and writes every copy. The columns of
@@ -398,12 +395,6 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
             *reinterpret_cast<uint4*>(q_tile + (c >> 3) * (128 * 128) + rl * 128 + (((c & 7) ^ swz) << 4)) = v[c];
         }
       }
-#pragma unroll
-      for (int j = 0; j < kPBufs; ++j)
-#pragma unroll
-        for (int c = 0; c < 8; ++c)
-          if (!row_ok || j % kU != h_own || c < lc0 / 8 || c >= (lc0 + kColsU) / 8)
-            *reinterpret_cast<uint4*>(p_buf(j) + r_loc * 128 + ((c ^ swz) << 4)) = make_uint4(0, 0, 0, 0);
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(q_ready);
@@ -521,35 +512,45 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
           tmem_st32(tO(mt) + lane_off + c * 32, o);
         }
       }
-      if (k_own < ntiles) {
-        // P buffer of tile k_own is free once the PV of tile k_own-kPBufs has completed.
-        const int buf = k_own % kPBufs;
-        if (k_own >= kPBufs && !warp_wait(&o_done[buf], ((k_own / kPBufs) - 1) & 1)) {
-          ok = false;
-          break;
-        }
-        if (warp_rows) {
+      if (warp_rows) {
+        // P goes to TMEM over the consumed S columns: tile k of the product
+        // takes columns (k % TPS) * 32 .. +31 of its S buffer, bf16 pairs.
+        // This thread writes its slice of the tile k_own and zeros over the
+        // rest of the step's tiles (other copies' slices).
+        const uint32_t tbuf = tS(mt, j & 1) + lane_off;
+        if (k_own < ntiles) {
           // p = 2^(s * scale * log2(e) - m): per pair of elements one paired
           // FMA, two exponentials, one bf16 pack and one paired add.
           const float nmu = m_run == -INFINITY ? 0.f : -m_run;
           const float2 sc2 = make_float2(scl, scl), nm2 = make_float2(nmu, nmu);
-          uint8_t* prow = p_buf(buf) + r_loc * 128;
           float2 ls[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+          const uint32_t tp = tbuf + static_cast<uint32_t>((k_own % kTPS) * 32);
 #pragma unroll
-          for (int c = 0; c < kColsU / 8; ++c) {
-            uint32_t w[4];
+          for (int c = 0; c < kColsU / 16; ++c) {  // 16 columns (8 TMEM columns) per store
+            uint32_t w[8];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const float2 x = fma2(make_float2(s[c * 8 + 2 * e], s[c * 8 + 2 * e + 1]), sc2, nm2);
+            for (int e = 0; e < 8; ++e) {
+              const float2 x = fma2(make_float2(s[c * 16 + 2 * e], s[c * 16 + 2 * e + 1]), sc2, nm2);
               const float2 pp = make_float2(ex2(x.x), ex2(x.y));
               ls[e & 1] = add2(ls[e & 1], pp);
               w[e] = pack_bf16(pp.x, pp.y);
             }
-            const int chunk = lc0 / 8 + c;
-            *reinterpret_cast<uint4*>(prow + ((chunk ^ swz) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+            tmem_st_u32<8>(tp + static_cast<uint32_t>(lc0 / 2 + c * 8), w);
           }
           l_run += (ls[0].x + ls[0].y) + (ls[1].x + ls[1].y);
+          if constexpr (kColsU < kTileTok) {
+#pragma unroll
+            for (int q = 0; q < kTileTok / kColsU; ++q)
+              if (q != lc0 / kColsU) tmem_st_zero<kColsU / 2>(tp + static_cast<uint32_t>(q * (kColsU / 2)));
+          }
         }
+        if constexpr (kU > 1) {
+#pragma unroll
+          for (int h = 0; h < kU; ++h)
+            if (h != h_own && k0 + h < ntiles)
+              tmem_st_zero<32>(tbuf + static_cast<uint32_t>(((k0 + h) % kTPS) * 32));
+        }
+        tmem_wait_st();
       }
       // Hand the step's tiles to the MMA warp (every softmax warp arrives
       // for every tile; P columns a warp does not own stay zero).
