@@ -62,6 +62,8 @@ def parse_args():
     ap.add_argument("--only-workload", default=None,
                     help="time only this named workload (device-drawn inputs), e.g. for a profiler")
     ap.add_argument("--workload-batch", type=int, default=None, help="batch override for --only-workload")
+    ap.add_argument("--split-sweep", action="store_true",
+                    help="with --only-workload: also time a verify pass for explicit split counts 1..64")
     ap.add_argument("--only-section", default=None, choices=["decisions", "logits", "kv_commit", "quadss"],
                     help="time only this section of the report (e.g. for a profiler)")
     ap.add_argument("--no-prefix-ready", action="store_true",
@@ -185,7 +187,8 @@ def run_only_workload(args, local):
     peak, _ = hbm_peak()
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size
     stream = torch.cuda.Stream(device=dev)
-    res = run_workloads(torch, nld, dev, stream, peak, l2, only=args.only_workload, batch=args.workload_batch)
+    res = run_workloads(torch, nld, dev, stream, peak, l2, only=args.only_workload, batch=args.workload_batch,
+                        sweep_splits=args.split_sweep)
     print(json.dumps({"workload": args.only_workload, "batch": args.workload_batch, **res[args.only_workload]}))
 
 
@@ -716,7 +719,7 @@ def run_decisions(torch, nld, dev, stream):
     return res
 
 
-def run_workloads(torch, nld, dev, stream, peak, l2, only=None, batch=None):
+def run_workloads(torch, nld, dev, stream, peak, l2, only=None, batch=None, sweep_splits=False):
     """Each named workload's step (SURVEY-style sequences: passes, then the
     decisions), inputs drawn on the device, pools rotated past L2 where the
     KV is smaller than three times L2."""
@@ -764,7 +767,7 @@ def run_workloads(torch, nld, dev, stream, peak, l2, only=None, batch=None):
                  "kv_bytes_per_pass": kvb, "kv_partials": parts,
                  "l2": ("cold: %d rotating pools" % npool) if npool * kvb >= 3 * l2 else
                        "warm: KV fits in L2 (%d pools, launch-bound shape)" % npool}
-        if name.startswith("long") and only is None:
+        if (name.startswith("long") and only is None) or sweep_splits:
             sweep = {}
             for S in (1, 2, 4, 8, 16, 32, 64):
                 pS = nld.make_params(B, Hq, Hkv, D, w["page"], w["num_pages"], w["max_pages"], S, 0.0,
