@@ -50,13 +50,13 @@ constexpr int kSoftmaxWarp0 = 4;
 // MT 128-row M tiles per CTA (MT = 2 for 129..256 packed rows); 4*MT
 // softmax warps; TPS 64-token K/V tiles per score product. TPS = 2 (one M
 // tile, a split short enough to sit in the ring whole): N = 128 products,
-// which the tensor core runs at full rate (N = 64 at about half), half as
-// many steps in the chain S -> softmax -> PV, and four P buffers so that the
-// softmax of one pair never waits for the PV products of the last. A long
-// split streams with TPS = 1, where a stage frees after each tile and more
-// of the ring stays in flight. The ring takes what shared memory the Q
-// tiles and P buffers leave (up to 8 stages): a streaming CTA's bandwidth is
-// the bytes it has in flight over the DRAM latency, so every stage counts.
+// which the tensor core runs at full rate (N = 64 at about half), and half
+// as many steps in the chain S -> softmax -> PV. A long split streams with
+// TPS = 1, where a stage frees after each tile and more of the ring stays
+// in flight. P lives in TMEM over its consumed S columns, so the ring takes
+// what shared memory the Q tiles leave (up to 8 stages): a streaming CTA's
+// bandwidth is the bytes it has in flight over the DRAM latency, so every
+// stage counts.
 template <int MT, int TPS>
 struct TcCfg {
   static_assert(TPS == 1 || (TPS == 2 && MT == 1), "paired score products with one M tile");
@@ -99,7 +99,7 @@ struct TcLayout {
   static constexpr int kQOff = kStages * Geo::kStageBytes;
   static constexpr int kPOff = kQOff + MT * kQBytes;  // end of the ring and Q tiles
   static constexpr int kBarOff = kPOff;
-  // kv_full[st], kv_empty[st], s_full[2], s_free[2], p_full[P], o_done[P], q_ready, q_full, drain, tmem slot
+  // kv_full[st], kv_empty[st], s_full[2], s_free[2], p_full[kPBufs], o_done[kPBufs], q_ready, q_full, drain, tmem slot
   static constexpr int kNumBars = 2 * kStages + 4 + 2 * kPBufs + 3;
   static constexpr int kBytes = kBarOff + kNumBars * 8 + 16;
   static_assert(kNumBars * 8 + 16 <= 512, "barrier reserve");
