@@ -115,7 +115,28 @@ struct TcLayout {
   static_assert(D / 32 * kMergeRows * 128 <= kPOff, "output staging");
 };
 
-template <int D, int MT, int REP, int TPS, bool MASKED>
+// The sequence of rank blockIdx.z by prefix length (descending, ties by
+// index), computed by the whole CTA in `scratch` (2 * B ints of shared
+// memory). Out of line, so that kernels that never take it keep their code.
+__device__ __noinline__ int sequence_by_length_rank(const AttnArgs& a, int* scratch) {
+  int* lens = scratch;
+  int* order = scratch + a.B;
+  for (int t = threadIdx.x; t < a.B; t += blockDim.x) lens[t] = __ldg(a.prefix_lens + t);
+  __syncthreads();
+  for (int t = threadIdx.x; t < a.B; t += blockDim.x) {
+    const int lt = lens[t];
+    int rank = 0;
+    for (int u = 0; u < a.B; ++u) {
+      const int lu = lens[u];
+      rank += (lu > lt || (lu == lt && u < t)) ? 1 : 0;
+    }
+    order[rank] = t;
+  }
+  __syncthreads();
+  return order[blockIdx.z];
+}
+
+template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED>
 __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     block_attn_tc_kernel(const __grid_constant__ TmaMaps maps, const AttnArgs a) {
   static_assert(REP == 1 || REP == 2 || REP == 4, "replication of 1, 2 or 4");
@@ -141,7 +162,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int split = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+  const int split = blockIdx.x, g = blockIdx.y;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kTcStages; ++s) {
@@ -178,6 +199,12 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
   const bool early = a.prefix_ready != 0;
   grid_launch_dependents();  // dependents launch early; they wait on this grid themselves
   if (!early) grid_dependency_wait();
+  // ORDERED (one split per sequence and more (sequence, KV head) units than
+  // SMs): CTAs start in z order, so CTA z takes the sequence of rank z by
+  // prefix length and the last wave holds the short ones. The ranks are
+  // computed in the K/V ring, before any copy into it. A separate
+  // instantiation, so the other kernels keep b = blockIdx.z.
+  const int b = ORDERED ? sequence_by_length_rank(a, reinterpret_cast<int*>(smem)) : static_cast<int>(blockIdx.z);
   const int t_begin = split * a.chunk;
   // The producers' first page-id loads and the prefix-length load are
   // independent, so they are in flight together.
@@ -888,12 +915,12 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
   }
 }
 
-template <int D, int MT, int REP, int TPS, bool MASKED>
+template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED = false>
 cudaError_t configure_tc(int dev) {
   static int configured[64] = {0};
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   if (!__atomic_load_n(&configured[dev], __ATOMIC_ACQUIRE)) {
-    cudaError_t e = cudaFuncSetAttribute(block_attn_tc_kernel<D, MT, REP, TPS, MASKED>,
+    cudaError_t e = cudaFuncSetAttribute(block_attn_tc_kernel<D, MT, REP, TPS, MASKED, ORDERED>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(TcLayout<D, MT, TPS>::kBytes + 1024));
     if (e != cudaSuccess) return e;
@@ -902,15 +929,26 @@ cudaError_t configure_tc(int dev) {
   return cudaSuccess;
 }
 
-template <int D, int MT, int REP, int TPS, bool MASKED>
-cudaError_t launch_tc_t(const AttnArgs& a, const TmaMaps& maps, cudaStream_t stream) {
+template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED>
+cudaError_t launch_tc_o(const AttnArgs& a, const TmaMaps& maps, cudaStream_t stream) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  if ((e = configure_tc<D, MT, REP, TPS, MASKED>(dev)) != cudaSuccess) return e;
+  if ((e = configure_tc<D, MT, REP, TPS, MASKED, ORDERED>(dev)) != cudaSuccess) return e;
   dim3 grid(a.num_splits, a.Hkv, a.B);
-  return launch_kernel_cluster(block_attn_tc_kernel<D, MT, REP, TPS, MASKED>, grid, dim3(TcCfg<MT, TPS>::kThreads),
-                               TcLayout<D, MT, TPS>::kBytes + 1024, stream, a.csize, maps, a);
+  return launch_kernel_cluster(block_attn_tc_kernel<D, MT, REP, TPS, MASKED, ORDERED>, grid,
+                               dim3(TcCfg<MT, TPS>::kThreads), TcLayout<D, MT, TPS>::kBytes + 1024, stream, a.csize,
+                               maps, a);
+}
+
+// The longest-first order only for the unmasked passes (the table-mask
+// passes run at the block shapes of one sequence).
+template <int D, int MT, int REP, int TPS, bool MASKED>
+cudaError_t launch_tc_t(const AttnArgs& a, const TmaMaps& maps, cudaStream_t stream) {
+  if constexpr (!MASKED) {
+    if (a.order_by_length) return launch_tc_o<D, MT, REP, TPS, false, true>(a, maps, stream);
+  }
+  return launch_tc_o<D, MT, REP, TPS, MASKED, false>(a, maps, stream);
 }
 
 // With one CTA per SM either way, cluster residency is the same for both
@@ -923,7 +961,7 @@ int max_active_clusters_t(int csize) {
   const int slot = csize == 2 ? 0 : csize == 4 ? 1 : csize == 8 ? 2 : 3;
   int v = __atomic_load_n(&cache[dev][slot], __ATOMIC_ACQUIRE);
   if (v) return v - 1;
-  if (configure_tc<D, MT, REP, 1, false>(dev) != cudaSuccess) return 0;
+  if (configure_tc<D, MT, REP, 1, false, false>(dev) != cudaSuccess) return 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(csize, 1, 1);
   cfg.blockDim = dim3(TcCfg<MT, 1>::kThreads);
@@ -936,7 +974,7 @@ int max_active_clusters_t(int csize) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, block_attn_tc_kernel<D, MT, REP, 1, false>, &cfg) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveClusters(&n, block_attn_tc_kernel<D, MT, REP, 1, false, false>, &cfg) != cudaSuccess) {
     cudaGetLastError();
     n = 0;
   }

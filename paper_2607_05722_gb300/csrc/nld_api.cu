@@ -321,6 +321,16 @@ nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_bloc
   a.block_mask = mode == nld::kModeBlockMask ? block_mask : nullptr;
   a.scale_log2 = scale * nld::kLog2e;
   a.prefix_ready = (params->flags & NLD_ATTN_PREFIX_READY) ? 1 : 0;
+  {
+    // Longest sequences first when one split each leaves more units than SMs
+    // (several waves): the last wave then holds the short sequences.
+    int sms = 0;
+    if ((st = device_state(nullptr, &sms)) != NLD_OK) return st;
+    a.order_by_length = (plan.splits == 1 && plan.csize == 1 && a.B > 1 && a.B <= 1024 &&
+                         static_cast<long long>(a.B) * a.Hkv > sms)
+                            ? 1
+                            : 0;
+  }
   if (plan.partials > 1) {
     a.o_part = static_cast<float*>(workspace);
     a.lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) + o_bytes);

@@ -39,6 +39,7 @@ struct AttnArgs {
   const uint32_t* block_mask;  // [bl] row masks over the block slots (kModeBlockMask only)
   float scale_log2;            // softmax scale * log2(e)
   int prefix_ready;            // NLD_ATTN_PREFIX_READY: prefix K/V may be read before the dependency wait
+  int order_by_length;         // CTA z takes the sequence of rank z by prefix length (longest first)
   int csize;                   // thread-block cluster size along the splits (1 = no cluster)
   int num_partials;            // partials written per (b, h, i): num_splits / csize (1 = final output)
 };
