@@ -525,6 +525,32 @@ def test_attention_small_all_rows(orc, spec, mode, splits):
     compare_attn(out, lse, ro, rl, f"{name} mode={mode} S={splits}")
 
 
+@pytest.mark.parametrize("mode", [DIFF, VER], ids=["diffusion", "verify"])
+@pytest.mark.parametrize("D", [64, 128])
+def test_attention_multiwave_longest_first(orc, mode, D):
+    """More (sequence, KV head) units than SMs with one split each: the CTAs
+    take the sequences longest first (a permutation by prefix length, ties by
+    index); every row still lands in its own sequence's output."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    B, Hq, Hkv, bl, P = 48, 16, 4, 8, 16
+    assert B * Hkv > sms
+    rng = np.random.Generator(np.random.PCG64(2024 + D))
+    prefix = [int(x) for x in rng.integers(0, 400, size=B)]
+    prefix[5] = prefix[17] = prefix[30] = 257  # ties
+    prefix[0] = 0
+    case = W.make_block_attn_case("multiwave", B, Hq, Hkv, D, block_len=bl, page_size=P, prefix_lens=prefix,
+                                  seed=77 + D)
+    dc = DeviceCase(case)
+    assert nld.nld_block_attn_num_splits(dc.params(0), bl) == 1
+    ro, rl = oracle_full(orc, case, mode)
+    for splits in (0, 1):
+        out, lse = dc.run(mode, num_splits=splits)
+        compare_attn(out, lse, ro, rl, f"multiwave D={D} mode={mode} S={splits}")
+    for flags in (0, nld.NLD_ATTN_PREFIX_READY):
+        o2, l2 = dc.run(mode, 0, flags=flags)
+        compare_attn(o2, l2, ro, rl, f"multiwave D={D} mode={mode} flags={flags}")
+
+
 @pytest.mark.parametrize("spec", SMALL, ids=[s[0] for s in SMALL])
 def test_prefix_ready_flag_same_result(orc, spec):
     """NLD_ATTN_PREFIX_READY only moves prefix loads before the dependency
