@@ -393,13 +393,10 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     const int swz = r_loc & 7;                      // 128-byte swizzle phase of this tile row
     uint8_t* q_tile = q_s + mt * Lay::kQBytes;
 
-    // Q row -> shared memory in the 128-byte-swizzled K-major layout (padding
-    // rows zero); slice 0 loads it once and writes every copy. The columns of
-    // P a thread never writes (other slices' tokens, or all of a padding row)
-    // are zeroed once in every buffer.
-    // One M tile: the MMA warp brings Q by TMA and the rows past R stay zero
-    // (written here, before the dependency wait). Two M tiles: the rows are
-    // loaded here after the wait.
+    // Q rows in shared memory, 128-byte-swizzled K-major (padding rows zero).
+    // One M tile: the MMA warp brings Q by TMA and the rows past R are zeroed
+    // here, before the dependency wait. Two M tiles: slice 0 of each row loads
+    // it here after the wait and writes every copy.
     if (MT == 1 && !row_ok) {
 #pragma unroll
       for (int c = 0; c < D / 8; ++c)
@@ -437,7 +434,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     const int lim = diff_mode ? t_end : min(t_end, L + row_i + 1);
     // MASKED (a table mask, e.g. quadratic self-speculation's, Sec. 3): the
     // prefix and the block slots whose bit is set in this row's table entry;
-    // per tile one 64-bit column mask, tested bit by bit. A separate
+    // per step one 64-bit column mask, tested bit by bit. A separate
     // instantiation, so the two passes above keep their one compare.
     uint32_t rowbits = 0u;
     if constexpr (MASKED) rowbits = row_ok ? __ldg(a.block_mask + row_i) : 0u;
@@ -580,7 +577,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
         tmem_wait_st();
       }
       // Hand the step's tiles to the MMA warp (every softmax warp arrives
-      // for every tile; P columns a warp does not own stay zero).
+      // for every tile; the P columns of other copies' slices are zero).
       bool step_ok = true;
 #pragma unroll
       for (int h = 0; h < kU; ++h) {
