@@ -40,16 +40,23 @@ __global__ void __launch_bounds__(kDecideWarps * 32)
   if (b >= B) return;
   const float c = lane < n ? __ldg(conf + b * n + lane) : -INFINITY;
   const bool elig = lane < n && !isnan(c) && c != -INFINITY;
-  int rank = 0;
-  for (int j = 0; j < n; ++j) {
-    const float cj = __shfl_sync(0xffffffffu, c, j);
-    const bool ej = !isnan(cj) && cj != -INFINITY;  // j < n here
-    rank += (ej && (cj > c || (cj == c && j < lane))) ? 1 : 0;
-  }
   const int count = __popc(__ballot_sync(0xffffffffu, elig));
   const int sel = count < k ? count : k;
   int32_t* prow = positions + b * k;
-  if (elig && rank < k) prow[rank] = lane;
+  // Selection by warp max: each confidence as an unsigned key in the order
+  // of the floats (+0 and -0 equal; ineligible lanes 0, below every eligible
+  // key), then sel rounds of (max key, lowest lane holding it), the chosen
+  // lane dropping out. Rank order: confidence descending, index ascending.
+  const uint32_t bits = __float_as_uint(c == 0.f ? 0.f : c);
+  uint32_t key = elig ? ((bits & 0x80000000u) ? ~bits : (bits | 0x80000000u)) : 0u;
+  for (int r = 0; r < sel; ++r) {
+    const uint32_t top = __reduce_max_sync(0xffffffffu, key);
+    const int who = __ffs(__ballot_sync(0xffffffffu, key == top)) - 1;
+    if (lane == who) {
+      prow[r] = lane;
+      key = 0u;
+    }
+  }
   if (lane >= sel && lane < k) prow[lane] = -1;
   if (lane == 0 && num_selected != nullptr) num_selected[b] = sel;
 }
