@@ -493,7 +493,9 @@ def run_e2e(args, torch, nld, dev, stream, wl, params, splits, kv_bytes, world):
               "small": torch.empty(off, dtype=torch.uint8, device=dev),
               "out": torch.empty(out_bytes, dtype=torch.uint8, device=dev)}
         for name, (o, a) in offs.items():
-            ds[name] = ds["small"][o:o + a.nbytes].view(torch.from_numpy(a[:0].copy()).dtype).view(a.shape)
+            dt = {np.dtype(np.int16): torch.int16, np.dtype(np.int32): torch.int32,
+                  np.dtype(np.float32): torch.float32}[a.dtype]
+            ds[name] = ds["small"][o:o + a.nbytes].view(dt).view(a.shape)
         o = 0
         for name, n, dt, shape in (("out_d", B * bl * Hq * D * 2, torch.bfloat16, (B, bl, Hq, D)),
                                    ("out_v", B * bl * Hq * D * 2, torch.bfloat16, (B, bl, Hq, D)),
@@ -720,9 +722,9 @@ def run_decisions(torch, nld, dev, stream):
 
 
 def run_workloads(torch, nld, dev, stream, peak, l2, only=None, batch=None, sweep_splits=False):
-    """Each named workload's step (SURVEY-style sequences: passes, then the
-    decisions), inputs drawn on the device, pools rotated past L2 where the
-    KV is smaller than three times L2."""
+    """Each named workload's step (its attention passes, then its decisions),
+    inputs drawn on the device, pools rotated past L2 where the KV is smaller
+    than three times L2."""
     res = {}
     for name in W.WORKLOADS:
         if (only is None and name == WORKLOAD) or (only is not None and name != only):
