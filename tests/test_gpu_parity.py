@@ -700,6 +700,25 @@ def test_attention_split_sweep(orc):
         compare_attn(out, lse, ro, rl, f"S={S}")
 
 
+_CLUSTER_SPECS = [SMALL[0], SMALL[8], SMALL[10], SMALL[13], SMALL[11]]
+
+
+@pytest.mark.parametrize("spec", _CLUSTER_SPECS, ids=[s[0] for s in _CLUSTER_SPECS])
+def test_attention_cluster_merges(orc, spec):
+    """Explicit split counts of 2/4/8 (one thread-block cluster merging
+    through distributed shared memory) and 16 (clusters of 8, two partials):
+    row copies, one and two M tiles, D = 64 and 128, both passes."""
+    name, B, Hq, Hkv, D, P, bl, prefix = spec
+    case = W.make_block_attn_case(name, B, Hq, Hkv, D, block_len=bl, page_size=P, prefix_lens=prefix,
+                                  seed=sum(prefix) + 11 * bl)
+    dc = DeviceCase(case)
+    for mode in (DIFF, VER):
+        ro, rl = oracle_full(orc, case, mode)
+        for S in (2, 4, 8, 16):
+            out, lse = dc.run(mode, num_splits=S)
+            compare_attn(out, lse, ro, rl, f"{name} cluster mode={mode} S={S}")
+
+
 # ---------------------------------------------------------------------------
 # attention: self-consistency on the GPU
 # ---------------------------------------------------------------------------
