@@ -213,6 +213,32 @@ def run_only_section(args, local):
     print(json.dumps({"section": args.only_section, **fn()}))
 
 
+# ---------------------------------------------------------------------------
+# multi-GPU host logic (weak scaling: one rank per GPU, each on its own
+# sequences; the timing reduce is the only collective)
+# ---------------------------------------------------------------------------
+
+def rank_seed(base_seed: int, rank: int) -> int:
+    """Seed of a rank's workload: every rank draws its own sequences."""
+    return base_seed + rank
+
+
+def max_over_ranks(value: float, world: int, device=None) -> float:
+    """The job's time is its slowest rank's: the max over the ranks."""
+    if world <= 1:
+        return float(value)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_kv_gbs(kv_bytes_per_pass: int, passes: int, world: int, ms_per_step: float) -> float:
+    """Whole-job KV GB/s: every rank's passes over its own KV per step time."""
+    return passes * kv_bytes_per_pass * world / (ms_per_step * 1e-3) / 1e9
+
+
 def run_ours(args, world, rank, local):
     import torch
     import torch.distributed as dist
@@ -227,7 +253,7 @@ def run_ours(args, world, rank, local):
     nld_build.build()
     nld.lib()
 
-    wl = W.make_workload(WORKLOAD, seed=args.seed + rank)
+    wl = W.make_workload(WORKLOAD, seed=rank_seed(args.seed, rank))
     c = wl.attn
     kv = c.kv
     B, bl, Hq, Hkv, D = c.batch, c.block_len, c.num_q_heads, c.num_kv_heads, c.head_dim
@@ -322,11 +348,7 @@ def run_ours(args, world, rank, local):
     t_host1 = time.time()
     if world > 1:
         dist.barrier()
-    ms = ev0.elapsed_time(ev1)
-    if world > 1:
-        t = torch.tensor([ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ev0.elapsed_time(ev1), world, dev)
     clocks = None
     if sampler is not None:
         time.sleep(0.1)
@@ -399,8 +421,7 @@ def run_ours(args, world, rank, local):
         return
     peak, peak_kind = hbm_peak()
     ms_step = ms / args.steps
-    total_kv = 2 * kv_bytes * world
-    value = total_kv / (ms_step * 1e-3) / 1e9
+    value = job_kv_gbs(kv_bytes, 2, world, ms_step)
     attn_gbs = kv_bytes / (attn_ms * 1e-3) / 1e9
     line = {
         "metric": METRIC,
