@@ -19,11 +19,12 @@
 //             core computes the next scores while the softmax warps work.
 //   warps 4.. softmax: thread t owns TMEM lane 32*(warp%4)+lane, one query
 //             row. It loads its S row, applies the mask and the base-2 scale,
-//             keeps the running max and sum, writes P (bf16) to shared memory
-//             for the PV MMA, and at the end reads O from TMEM, divides by the
-//             sum and stages its row in the freed K/V ring in 128-byte-swizzled
-//             boxes, which one thread writes with tiled TMA stores (bf16 output
-//             or fp32 split partial; the CTA's rows are contiguous in both).
+//             keeps the running max and sum, writes P (bf16) back to TMEM
+//             over the consumed S columns as the PV MMA's A operand, and at
+//             the end reads O from TMEM, divides by the sum and stages its row
+//             in the freed K/V ring in 128-byte-swizzled boxes, which one
+//             thread writes with tiled TMA stores (bf16 output or fp32 split
+//             partials, in packed row order).
 //             With at most 64 (32) packed rows, Q is replicated into the idle
 //             lane quadrants (REP = 2 or 4): each copy of a row takes a 64/REP-
 //             token slice of every tile with its own running max and sum, so
