@@ -375,6 +375,16 @@ nld_status_t nld_kv_commit(const nld_attn_params_t *params, const void *k_new, c
                            int block_len, int advance, void *k_pages, void *v_pages,
                            cudaStream_t stream);
 
+/*
+ * Failure-detection check: launches one thread that waits, with the same
+ * bounded wait every pipeline uses, on an mbarrier nothing ever arrives on.
+ * After limit_ns nanoseconds (1 .. 1e9) the wait gives up, sets
+ * NLD_DEVERR_WAIT_TIMEOUT in the device error word and the kernel returns;
+ * the context stays usable. For tests and diagnostics.
+ * Errors: NLD_ERR_INVALID_ARG (limit out of range), NLD_ERR_CUDA (launch).
+ */
+nld_status_t nld_check_wait_timeout(uint64_t limit_ns, cudaStream_t stream);
+
 /* A static, human-readable name for a status code. */
 const char *nld_status_string(nld_status_t status);
 

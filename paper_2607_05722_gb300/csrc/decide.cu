@@ -138,6 +138,24 @@ cudaError_t launch_unmask_threshold(const float* conf, int B, int n, float thres
                        threshold, pos, nsel);
 }
 
+// One thread initialises an mbarrier that expects one arrival, never
+// arrives, and waits on it with the pipelines' bounded wait: the wait gives
+// up after limit_ns and records NLD_DEVERR_WAIT_TIMEOUT, as any kernel's
+// wait would, and the kernel returns.
+__global__ void __launch_bounds__(32) wait_timeout_check_kernel(uint64_t limit_ns, unsigned int* err) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+    mbar_wait_for(&bar, 0, err, limit_ns);
+  }
+}
+
+cudaError_t launch_wait_timeout_check(uint64_t limit_ns, unsigned int* err, cudaStream_t stream) {
+  wait_timeout_check_kernel<<<1, 32, 0, stream>>>(limit_ns, err);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_greedy_accept(const int32_t* pred, const int32_t* target, const float* conf, int B, int n,
                                  int32_t* pos, int32_t* nsel, cudaStream_t stream) {
   const unsigned blocks = static_cast<unsigned>((B + kDecideWarps - 1) / kDecideWarps);

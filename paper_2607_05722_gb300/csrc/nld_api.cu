@@ -515,6 +515,14 @@ nld_status_t nld_kv_commit(const nld_attn_params_t* params, const void* k_new, c
              : NLD_ERR_CUDA;
 }
 
+nld_status_t nld_check_wait_timeout(uint64_t limit_ns, cudaStream_t stream) {
+  if (limit_ns == 0 || limit_ns > nld::kWaitLimitNs) return NLD_ERR_INVALID_ARG;
+  unsigned int* err = nullptr;
+  nld_status_t st = device_state(&err, nullptr);
+  if (st != NLD_OK) return st;
+  return nld::launch_wait_timeout_check(limit_ns, err, stream) == cudaSuccess ? NLD_OK : NLD_ERR_CUDA;
+}
+
 nld_status_t nld_device_error(uint32_t* bits, int clear) {
   if (bits == nullptr) return NLD_ERR_INVALID_ARG;
   unsigned int* err = nullptr;

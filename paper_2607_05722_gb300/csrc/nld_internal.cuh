@@ -56,6 +56,8 @@ struct TmaMaps {
 cudaError_t launch_block_attn_tc(const AttnArgs& a, const TmaMaps& maps, int head_dim, cudaStream_t stream);
 // The same for a table mask (a.mode == kModeBlockMask; block_attn_tc_masked.cu).
 cudaError_t launch_block_attn_tc_masked(const AttnArgs& a, const TmaMaps& maps, int head_dim, cudaStream_t stream);
+// A kernel whose one mbarrier wait can never complete (decide.cu).
+cudaError_t launch_wait_timeout_check(uint64_t limit_ns, unsigned int* err, cudaStream_t stream);
 cudaError_t launch_combine(const float* o_part, const float* lse_part, int S, int B, int Hq, int bl,
                            int D, __nv_bfloat16* out, float* lse, cudaStream_t stream);
 cudaError_t launch_accept(const int32_t* draft, const int32_t* verify, int B, int n, int32_t* acc,
@@ -193,16 +195,20 @@ __device__ __forceinline__ uint64_t global_timer_ns() {
 // Wait for an mbarrier phase with a time limit. On timeout, records
 // NLD_DEVERR_WAIT_TIMEOUT and returns false instead of spinning forever.
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s: microsecond kernels never get near it
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, unsigned int* err) {
+__device__ __forceinline__ bool mbar_wait_for(uint64_t* bar, uint32_t parity, unsigned int* err,
+                                              uint64_t limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
   for (uint32_t it = 0;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 255u) == 255u && global_timer_ns() - t0 > kWaitLimitNs) {
+    if ((it & 255u) == 255u && global_timer_ns() - t0 > limit_ns) {
       atomicOr(err, NLD_DEVERR_WAIT_TIMEOUT);
       return false;
     }
   }
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, unsigned int* err) {
+  return mbar_wait_for(bar, parity, err, kWaitLimitNs);
 }
 
 // 4-D tiled TMA load into shared memory, completing on an mbarrier.

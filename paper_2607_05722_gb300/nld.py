@@ -90,6 +90,8 @@ def lib(path: Optional[str] = None):
     L.nld_status_string.restype = ctypes.c_char_p
     L.nld_device_error.argtypes = [ctypes.POINTER(ctypes.c_uint32), I]
     L.nld_device_error.restype = I
+    L.nld_check_wait_timeout.argtypes = [ctypes.c_uint64, V]
+    L.nld_check_wait_timeout.restype = I
     if path is None:
         _lib = L
     return L
@@ -359,6 +361,13 @@ def nld_kv_commit(params: AttnParams, k_new, v_new, counts, page_table, prefix_l
     _check(lib().nld_kv_commit(ctypes.byref(params), _ptr(k_new), _ptr(v_new), _ptr(counts), _ptr(page_table),
                                _ptr(prefix_lens), int(block_len), int(bool(advance)), _ptr(k_pages), _ptr(v_pages),
                                _stream(stream)), "nld_kv_commit")
+
+def nld_check_wait_timeout(limit_ns: int, stream=None) -> None:
+    """Launch the bounded-wait check: one wait that nothing completes gives up
+    after limit_ns and sets NLD_DEVERR_WAIT_TIMEOUT."""
+    _check(lib().nld_check_wait_timeout(ctypes.c_uint64(int(limit_ns)), _stream(stream)),
+           "nld_check_wait_timeout")
+
 
 def nld_device_error(clear: bool = False) -> int:
     bits = ctypes.c_uint32(0)

@@ -21,7 +21,8 @@ def L():
 def test_header_declares_the_abi():
     names = nld.header_functions()
     for f in ("nld_block_attn", "nld_block_attn_partials", "nld_block_attn_workspace_size", "nld_block_attn_num_splits",
-              "nld_split_kv_combine", "nld_accept", "nld_unmask", "nld_status_string", "nld_device_error"):
+              "nld_split_kv_combine", "nld_accept", "nld_unmask", "nld_status_string", "nld_device_error",
+              "nld_check_wait_timeout"):
         assert f in names, f
 
 
@@ -133,3 +134,9 @@ def test_quadss_table_matches_oracle(L, orc):
 def test_no_cpu_fallback_without_library(tmp_path):
     with pytest.raises(RuntimeError):
         nld.lib(str(tmp_path / "missing.so"))
+
+
+def test_wait_timeout_check_rejects_bad_limits(L):
+    # argument checks come before any device use
+    assert L.nld_check_wait_timeout(0, None) == 1
+    assert L.nld_check_wait_timeout(2_000_000_000, None) == 1

@@ -769,6 +769,24 @@ def test_device_clamps_bad_prefix_and_page_ids():
     assert nld.nld_device_error(clear=True) & nld.NLD_DEVERR_PAGE_RANGE
 
 
+def test_wait_timeout_is_reported_and_context_survives(orc):
+    """Failure detection without a fault: a bounded wait that nothing
+    completes gives up, sets NLD_DEVERR_WAIT_TIMEOUT and returns; the next
+    attention call on the same context is correct and raises no error."""
+    nld.nld_device_error(clear=True)
+    nld.nld_check_wait_timeout(2_000_000)  # 2 ms
+    torch.cuda.synchronize()
+    assert nld.nld_device_error(clear=True) & nld.NLD_DEVERR_WAIT_TIMEOUT
+    name, B, Hq, Hkv, D, P, bl, prefix = SMALL[1]
+    case = W.make_block_attn_case(name, B, Hq, Hkv, D, block_len=bl, page_size=P, prefix_lens=prefix, seed=5)
+    dc = DeviceCase(case)
+    out, lse = dc.run(VER)
+    torch.cuda.synchronize()
+    assert nld.nld_device_error(clear=True) == 0
+    ro, rl = oracle_full(orc, case, VER)
+    compare_attn(out, lse, ro, rl, "after a wait timeout")
+
+
 def test_workspace_too_small_launches_nothing():
     case = W.make_block_attn_case("ws", 1, 8, 2, 128, 16, 16, [500], seed=7)
     dc = DeviceCase(case)
