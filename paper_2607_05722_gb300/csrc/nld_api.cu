@@ -138,6 +138,10 @@ nld_status_t plan_splits(const nld_attn_params_t* p, int block_len, SplitPlan* o
     const long long c2 = (chunk + 2 * nld::kTileTok - 1) / (2 * nld::kTileTok) * (2 * nld::kTileTok);
     const long long s2 = (max_tokens + c2 - 1) / c2;
     if (s2 * 100 >= static_cast<long long>(want) * 85) chunk = c2;
+  } else if (automatic && csize == 1 && tc) {
+    // Streaming splits end on a whole tile when that keeps their number.
+    const long long c1 = (chunk + nld::kTileTok - 1) / nld::kTileTok * nld::kTileTok;
+    if ((max_tokens + c1 - 1) / c1 == (max_tokens + chunk - 1) / chunk) chunk = c1;
   }
   long long splits = (max_tokens + chunk - 1) / chunk;
   splits = (splits + csize - 1) / csize * csize;  // trailing empty splits complete a cluster
