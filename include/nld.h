@@ -111,6 +111,15 @@ typedef struct {
 int nld_block_attn_num_splits(const nld_attn_params_t *params, int block_len);
 
 /*
+ * Host-only view of the split plan for a device with sm_count SMs, cluster
+ * plans left out (their residency is a device query): plan[0] splits per
+ * (sequence, KV head), plan[1] tokens per split, plan[2] cluster size (1),
+ * plan[3] partials. Returns 0, or -1 for invalid parameters. Touches no
+ * device; for tests and capacity planning.
+ */
+int nld_block_attn_plan(const nld_attn_params_t *params, int block_len, int sm_count, int32_t plan[4]);
+
+/*
  * Workspace bytes nld_block_attn needs (0 when it runs unsplit). The
  * workspace holds fp32 split partials: O_part [S, B, Hq, bl, D] then
  * LSE_part [S, B, Hq, bl] at the next 256-byte boundary.

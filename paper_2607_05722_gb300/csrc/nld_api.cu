@@ -88,7 +88,11 @@ struct SplitPlan {
 // (the ring holds at least 6 tiles at head_dim 128).
 constexpr long long kPairedChunk = 384;
 
-nld_status_t plan_splits(const nld_attn_params_t* p, int block_len, SplitPlan* out) {
+// The plan for `sms` SMs; `clusters_resident(cs)` says how many clusters of
+// cs CTAs can be resident at once (0: none considered).
+template <typename ClustersResident>
+void plan_splits_for(const nld_attn_params_t* p, int block_len, int sms, ClustersResident clusters_resident,
+                     SplitPlan* out) {
   const long long max_tokens = static_cast<long long>(p->max_pages_per_seq) * p->page_size;
   const long long units = static_cast<long long>(p->batch) * p->num_kv_heads;
   const bool tc = nld::tc_supports((p->num_q_heads / p->num_kv_heads) * block_len, p->head_dim);
@@ -96,9 +100,6 @@ nld_status_t plan_splits(const nld_attn_params_t* p, int block_len, SplitPlan* o
   int want = p->num_splits;
   int csize = 1;
   if (automatic) {
-    int sms = 0;
-    nld_status_t st = device_state(nullptr, &sms);
-    if (st != NLD_OK) return st;
     // Fill the SMs once; when the (sequence, KV head) units fit in one wave,
     // also cut long ranges into pieces of at most kMaxAutoChunk tokens: with
     // ragged lengths (not known on the host) the longest sequence would
@@ -116,7 +117,7 @@ nld_status_t plan_splits(const nld_attn_params_t* p, int block_len, SplitPlan* o
     want = static_cast<int>(s);
     if (tc && want >= 2 && want <= 8) {
       const int cs = want >= 8 ? 8 : want >= 4 ? 4 : 2;
-      if (units <= nld::tc_max_active_clusters(cs, p->head_dim, (p->num_q_heads / p->num_kv_heads) * block_len)) {
+      if (units <= clusters_resident(cs)) {
         want = cs;
         csize = cs;
       }
@@ -149,6 +150,18 @@ nld_status_t plan_splits(const nld_attn_params_t* p, int block_len, SplitPlan* o
   out->splits = static_cast<int>(splits);
   out->csize = csize;
   out->partials = static_cast<int>(splits / csize);
+}
+
+nld_status_t plan_splits(const nld_attn_params_t* p, int block_len, SplitPlan* out) {
+  int sms = 0;
+  if (p->num_splits == 0) {
+    nld_status_t st = device_state(nullptr, &sms);
+    if (st != NLD_OK) return st;
+  }
+  const int rows = (p->num_q_heads / p->num_kv_heads) * block_len;
+  plan_splits_for(
+      p, block_len, sms, [&](int cs) { return static_cast<long long>(nld::tc_max_active_clusters(cs, p->head_dim, rows)); },
+      out);
   return NLD_OK;
 }
 
@@ -258,6 +271,18 @@ const char* nld_status_string(nld_status_t s) {
     case NLD_ERR_CUDA: return "NLD_ERR_CUDA";
   }
   return "NLD_ERR_UNKNOWN";
+}
+
+int nld_block_attn_plan(const nld_attn_params_t* params, int block_len, int sm_count, int32_t plan[4]) {
+  if (plan == nullptr || sm_count < 1) return -1;
+  if (check_params(params, block_len) != NLD_OK) return -1;
+  SplitPlan sp;
+  plan_splits_for(params, block_len, sm_count, [](int) { return 0LL; }, &sp);
+  plan[0] = sp.splits;
+  plan[1] = sp.chunk;
+  plan[2] = sp.csize;
+  plan[3] = sp.partials;
+  return 0;
 }
 
 int nld_block_attn_num_splits(const nld_attn_params_t* params, int block_len) {

@@ -92,6 +92,8 @@ def lib(path: Optional[str] = None):
     L.nld_device_error.restype = I
     L.nld_check_wait_timeout.argtypes = [ctypes.c_uint64, V]
     L.nld_check_wait_timeout.restype = I
+    L.nld_block_attn_plan.argtypes = [PP, I, I, ctypes.POINTER(ctypes.c_int32)]
+    L.nld_block_attn_plan.restype = I
     if path is None:
         _lib = L
     return L
@@ -361,6 +363,14 @@ def nld_kv_commit(params: AttnParams, k_new, v_new, counts, page_table, prefix_l
     _check(lib().nld_kv_commit(ctypes.byref(params), _ptr(k_new), _ptr(v_new), _ptr(counts), _ptr(page_table),
                                _ptr(prefix_lens), int(block_len), int(bool(advance)), _ptr(k_pages), _ptr(v_pages),
                                _stream(stream)), "nld_kv_commit")
+
+def nld_block_attn_plan(params: AttnParams, block_len: int, sm_count: int) -> dict:
+    """Host-only split plan for sm_count SMs (cluster plans left out)."""
+    out = (ctypes.c_int32 * 4)()
+    if lib().nld_block_attn_plan(ctypes.byref(params), block_len, sm_count, out) != 0:
+        raise NldError(1, "nld_block_attn_plan")
+    return {"splits": out[0], "chunk": out[1], "cluster": out[2], "partials": out[3]}
+
 
 def nld_check_wait_timeout(limit_ns: int, stream=None) -> None:
     """Launch the bounded-wait check: one wait that nothing completes gives up

@@ -140,3 +140,62 @@ def test_wait_timeout_check_rejects_bad_limits(L):
     # argument checks come before any device use
     assert L.nld_check_wait_timeout(0, None) == 1
     assert L.nld_check_wait_timeout(2_000_000_000, None) == 1
+
+
+# ---------------------------------------------------------------------------
+# the split plan (host logic, no device): 152 SMs as on GB300
+# ---------------------------------------------------------------------------
+
+def _plan(B, Hq, Hkv, D, P, prefix_max, bl, splits=0, sms=152):
+    pages = (prefix_max + bl + P - 1) // P
+    p = nld.make_params(B, Hq, Hkv, D, P, B * pages, pages, splits, 0.0, 0)
+    return nld.nld_block_attn_plan(p, bl, sms), pages * P
+
+
+def test_plan_8b_shape_takes_whole_paired_products(L):
+    plan, tokens = _plan(1, 32, 8, 128, 16, 4096, 16)
+    assert plan == {"splits": 17, "chunk": 256, "cluster": 1, "partials": 17}
+    assert plan["splits"] * 8 <= 152
+
+
+def test_plan_long_prefix_streams_whole_tiles(L):
+    plan, tokens = _plan(1, 32, 8, 128, 16, 32768, 32)
+    assert plan["splits"] == 19 and plan["chunk"] % 64 == 0
+    assert (plan["splits"] - 1) * plan["chunk"] < tokens <= plan["splits"] * plan["chunk"]
+
+
+def test_plan_many_units_one_split(L):
+    plan, _ = _plan(32, 32, 8, 128, 16, 8192, 8)  # 256 units > 152 SMs
+    assert plan["splits"] == 1 and plan["partials"] == 1
+
+
+def test_plan_ragged_batch_caps_pieces_at_2048_tokens(L):
+    # 64 units fit one wave: floor(152/64) = 2 splits, raised so that no piece
+    # of the 8208-token range exceeds 2048 tokens; pieces end on whole tiles
+    plan, tokens = _plan(8, 32, 8, 128, 16, 8192, 8)
+    assert tokens == 8208
+    assert plan["splits"] == -(-tokens // 2048) == 5
+    assert plan["chunk"] % 64 == 0 and plan["chunk"] <= 2048
+
+
+@pytest.mark.parametrize("B,Hq,Hkv,D,P,L_,bl", [(1, 4, 1, 64, 256, 256, 8), (2, 8, 2, 128, 16, 300, 16),
+                                               (3, 4, 2, 64, 32, 200, 5), (16, 40, 8, 128, 16, 16384, 32),
+                                               (1, 16, 2, 64, 16, 100, 32), (5, 12, 4, 128, 64, 1000, 20)])
+def test_plan_invariants(L, B, Hq, Hkv, D, P, L_, bl):
+    for sms in (1, 8, 148, 152, 160):
+        for S in (0, 1, 3, 7, 19):
+            plan, tokens = _plan(B, Hq, Hkv, D, P, L_, bl, splits=S, sms=sms)
+            assert plan["chunk"] % 16 == 0 and plan["chunk"] > 0
+            assert plan["splits"] * plan["chunk"] >= tokens
+            assert (plan["splits"] - 1) * plan["chunk"] < tokens
+            assert 1 <= plan["splits"] <= 128 and plan["partials"] == plan["splits"] // plan["cluster"]
+            if S:
+                assert plan["splits"] <= S
+
+
+def test_plan_rejects_bad_arguments(L):
+    p = nld.make_params(1, 32, 8, 128, 16, 300, 300, 0, 0.0, 0)
+    with pytest.raises(nld.NldError):
+        nld.nld_block_attn_plan(p, 16, 0)
+    with pytest.raises(nld.NldError):
+        nld.nld_block_attn_plan(p, 33, 152)
