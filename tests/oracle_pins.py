@@ -306,6 +306,48 @@ def pin_split_combine(orc):
             assert_close(lse, np.transpose(lse_full, (0, 2, 1)).reshape(-1), 1e-12, "split lse")
 
 
+def _sdpa_row(case, qbits, mode, b, i, h):
+    """One output row (b, i, h) and its lse, from torch SDPA in fp64 over the
+    keys the row sees (Sec. 2.2: the whole prefix, then every block slot in
+    the draft pass or block slots 0..i in the verify pass)."""
+    G = case.num_q_heads // case.num_kv_heads
+    L = int(case.kv.prefix_lens[b])
+    k, v = gather_contiguous(case, b)
+    n_vis = L + (case.block_len if mode == DIFF else i + 1)
+    q = q_f64(qbits[b, i, h])[None, None, :]  # [1, 1, D]
+    kk, vv = k[h // G, :n_vis][None], v[h // G, :n_vis][None]
+    o = sdpa(q, kk, vv, case.scale)[0, 0]
+    lse = scipy.special.logsumexp(q[0, 0] @ kk[0].T * case.scale)
+    return o, lse
+
+
+def pin_block_attn_rows(orc):
+    """The selected-rows entry (the oracle of every full-size GPU parity run):
+    rows listed as (b, i, h) triples, in any order and with repeats, each
+    equal to torch SDPA over the keys that row sees, bit-identical to the
+    same row of the all-rows entry, and written at its own list position."""
+    rng = np.random.default_rng(91)
+    # ragged batch, G = 3 (query head h reads KV head h // 3), bl = Hq so that
+    # a swapped (i, h) stays in range and is caught by value, not by bounds
+    case = W.make_block_attn_case("rows", 3, 6, 2, 16, 6, 4, [0, 9, 14], 92, shuffle_pages=True)
+    B, bl, Hq = case.batch, case.block_len, case.num_q_heads
+    trip = np.array([(b, i, h) for b in range(B) for i in range(bl) for h in range(Hq)], np.int32)
+    sel = np.concatenate([trip[rng.permutation(len(trip))[:40]], trip[[5, 5, len(trip) - 1]]])
+    kv = case.kv
+    for mode, qbits in ((DIFF, case.q_draft_bits), (VER, case.q_verify_bits)):
+        full, lse_full = orc.block_attn(qbits, kv.k_bits, kv.v_bits, kv.page_table, kv.prefix_lens, Hq,
+                                        case.num_kv_heads, bl, mode, case.scale)
+        out, lse = orc.block_attn_rows(qbits, kv.k_bits, kv.v_bits, kv.page_table, kv.prefix_lens, Hq,
+                                       case.num_kv_heads, bl, mode, case.scale, sel)
+        assert out.shape == (len(sel), case.head_dim) and lse.shape == (len(sel),)
+        for r, (b, i, h) in enumerate(sel):
+            o_ref, l_ref = _sdpa_row(case, qbits, mode, b, i, h)
+            assert_close(out[r], o_ref, 1e-12, f"rows mode={mode} r={r} (b,i,h)=({b},{i},{h})")
+            assert abs(lse[r] - l_ref) <= 1e-12, f"rows lse mode={mode} r={r}"
+            assert np.array_equal(out[r], full[b, i, h]), f"rows vs all rows mode={mode} r={r}"
+            assert lse[r] == lse_full[b, h, i], f"rows lse vs all rows mode={mode} r={r}"
+
+
 # --------------------------------------------------------------------------
 # decision pins
 # --------------------------------------------------------------------------
@@ -845,7 +887,7 @@ def pin_ensemble_empty_side(orc):
 
 ATTENTION_PINS = [pin_decode_bl1, pin_diffusion_full_attention, pin_verify_causal_tail, pin_lse_logsumexp,
                   pin_softmax_rows, pin_page_permutation, pin_block_permutation, pin_closed_forms,
-                  pin_golden_uniform, pin_split_combine]
+                  pin_golden_uniform, pin_split_combine, pin_block_attn_rows]
 DECISION_PINS = [pin_accept_golden, pin_accept_brute, pin_accept_statistics, pin_unmask_golden,
                  pin_unmask_brute, pin_unmask_lexsort, pin_threshold_golden, pin_threshold_brute,
                  pin_threshold_limits, pin_greedy_golden, pin_greedy_brute, pin_greedy_chain]

@@ -101,6 +101,15 @@ MUTANTS = {
     "ensemble_ties_last": ("if (p > best) { best = p; id = v; }", "if (p >= best) { best = p; id = v; }"),
     # ensemble: mixes unnormalised weights
     "ensemble_unnormalised": ("for (int v = 0; v < vocab; ++v) p[v] /= sum;", ""),
+    # selected rows: the triple read as (b, h, i)
+    "rows_triple_bhi": ("int b = rows[3 * r], i = rows[3 * r + 1], h = rows[3 * r + 2];",
+                        "int b = rows[3 * r], h = rows[3 * r + 1], i = rows[3 * r + 2];"),
+    # selected rows: each result written one list position later (wrapping, in bounds)
+    "rows_out_shifted": ("s, use, out + r * (long)D, lse + r, NULL);",
+                         "s, use, out + ((r + 1) % nsel) * (long)D, lse + (r + 1) % nsel, NULL);"),
+    # selected rows: lse written in reverse list order
+    "rows_lse_reversed": ("s, use, out + r * (long)D, lse + r, NULL);",
+                          "s, use, out + r * (long)D, lse + (nsel - 1 - r), NULL);"),
     # unmask: ascending order
     "unmask_ascending": ("if (ca > cb) return 1;\n    if (ca < cb) return 0;",
                          "if (ca < cb) return 1;\n    if (ca > cb) return 0;"),
