@@ -46,7 +46,7 @@ PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_HBM_GBS = 6800.0
 TRAFFIC_NOTE = os.path.join(ROOT, "profiles", "block_attn_8b_b1_L4096_bl16.md")
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2607_05722_gb300", "csrc", f)
-                  for f in ("block_attn_tc.cuh", "nld_internal.cuh")]
+                  for f in ("block_attn_tc.cuh", "nld_internal.cuh", "nld_api.cu")]
 
 
 def parse_args():

@@ -111,11 +111,17 @@ typedef struct {
 int nld_block_attn_num_splits(const nld_attn_params_t *params, int block_len);
 
 /*
- * Host-only view of the split plan for a device with sm_count SMs, cluster
- * plans left out (their residency is a device query): plan[0] splits per
- * (sequence, KV head), plan[1] tokens per split, plan[2] cluster size (1),
- * plan[3] partials. Returns 0, or -1 for invalid parameters. Touches no
- * device; for tests and capacity planning.
+ * Host-only view of the split plan for a device with sm_count SMs: plan[0]
+ * splits per (sequence, KV head), plan[1] tokens per split, plan[2] cluster
+ * size, plan[3] partials per output row. An explicit params->num_splits
+ * divisible by 8, 4 or 2 runs as clusters of that size (plan[2] = 8, 4 or
+ * 2), exactly as nld_block_attn launches it. An automatic plan
+ * (num_splits = 0) is given as if no cluster were resident: on a device
+ * where the plan's 2..8 pieces per (sequence, KV head) fit as resident
+ * clusters, the launched plan instead uses one cluster of 2, 4 or 8 per
+ * (sequence, KV head) and one partial, and nld_block_attn_num_splits
+ * reports that. Returns 0, or -1 for invalid parameters. Touches no device;
+ * for tests and capacity planning.
  */
 int nld_block_attn_plan(const nld_attn_params_t *params, int block_len, int sm_count, int32_t plan[4]);
 

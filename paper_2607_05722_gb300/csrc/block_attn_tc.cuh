@@ -332,7 +332,9 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
       // front of the PV products on the tensor core.)
       const int nprod = (ntiles + kTPS - 1) / kTPS;
       int next_s = 0, next_pv = 0;
-      const uint64_t t_start = global_timer_ns();
+      // The time limit bounds one stall, not the split: it restarts whenever
+      // an MMA group is issued.
+      uint64_t t_start = global_timer_ns();
       uint32_t spins = 0;
       while (ok && next_pv < ntiles) {
         bool progressed = false;
@@ -350,7 +352,12 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
           issue_pv(next_pv++);
           progressed = true;
         }
-        if (!progressed) {
+        if (progressed) {
+          if (spins != 0) {
+            spins = 0;
+            t_start = global_timer_ns();
+          }
+        } else {
           __nanosleep(20);  // this warp shares an SM sub-partition with a softmax warp
           if ((++spins & 255u) == 0 && global_timer_ns() - t_start > kWaitLimitNs) {
             atomicOr(a.err, NLD_DEVERR_WAIT_TIMEOUT);

@@ -1,10 +1,12 @@
 // Token decisions of tri-mode decoding, one warp per sequence (n <= 32).
 //  - accept (Sec. 3, Mode 3): ballot of draft != verify over the n positions;
 //    the lowest set bit is the first mismatch j*, the accepted length.
-//  - unmask (Sec. 3, Mode 2): lane i holds confidence c_i; its rank is
-//    #{j eligible: c_j > c_i} + #{j < i eligible: c_j == c_i}, so ranks of
-//    the eligible lanes are a permutation and the k smallest are written in
-//    rank order. -inf and NaN are not eligible.
+//  - unmask (Sec. 3, Mode 2): lane i holds confidence c_i as an unsigned key
+//    in the order of the floats (ineligible lanes: 0); k rounds of a warp max
+//    reduction each pick the largest key and the lowest lane holding it,
+//    which writes its position at that rank and drops out, so positions come
+//    out by (confidence descending, position ascending). -inf and NaN are not
+//    eligible.
 //  - threshold unmasking (Sec. 2, confidence-based sampling) and greedy
 //    parallel acceptance (Sec. 5, diffusion SOL): the committed set is a
 //    ballot (confidence > threshold; prediction == serial target), each member

@@ -365,7 +365,8 @@ def nld_kv_commit(params: AttnParams, k_new, v_new, counts, page_table, prefix_l
                                _stream(stream)), "nld_kv_commit")
 
 def nld_block_attn_plan(params: AttnParams, block_len: int, sm_count: int) -> dict:
-    """Host-only split plan for sm_count SMs (cluster plans left out)."""
+    """Host-only split plan for sm_count SMs: explicit split counts as launched
+    (clusters included); automatic plans as if no cluster were resident."""
     out = (ctypes.c_int32 * 4)()
     if lib().nld_block_attn_plan(ctypes.byref(params), block_len, sm_count, out) != 0:
         raise NldError(1, "nld_block_attn_plan")
