@@ -410,6 +410,18 @@ const char *nld_status_string(nld_status_t status);
  */
 nld_status_t nld_device_error(uint32_t *bits, int clear);
 
+/*
+ * Read the current device's count of running-max rescale events into
+ * *count; with clear != 0 reset it to 0. The attention kernels keep a
+ * row's running softmax maximum lazily (the online softmax of the scaled
+ * scores, Sec. 2.2 attention): the accumulated output is rescaled in tensor
+ * memory only when a later tile raises the row maximum by more than 2^8
+ * (base 2). Each warp that performs such a rescale adds 1. The count tells
+ * tests and diagnostics that this path ran; it does not change any result.
+ * Synchronises the device; not for the decode loop.
+ */
+nld_status_t nld_rescale_count(uint64_t *count, int clear);
+
 #ifdef __cplusplus
 }
 #endif

@@ -535,6 +535,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
           break;
         }
         tc_fence_after();
+        if (lane == 0) atomicAdd(a.rescales, 1ull);
 #pragma unroll 1
         for (int c = 0; c < D / 32; ++c) {
           float o[32];

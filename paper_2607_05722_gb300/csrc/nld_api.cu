@@ -14,31 +14,39 @@ namespace {
 
 using nld::AttnArgs;
 
-// Error word the kernels OR their NLD_DEVERR_* bits into.
+// Error word the kernels OR their NLD_DEVERR_* bits into, and the count of
+// running-max rescales (a diagnostic).
 __device__ unsigned int g_device_error;
+__device__ unsigned long long g_rescale_count;
 
 constexpr int kMaxDevices = 64;
 unsigned int* g_err_ptr[kMaxDevices];
+unsigned long long* g_rescale_ptr[kMaxDevices];
 int g_sm_count[kMaxDevices];
 std::mutex g_mu;
 
 bool aligned(const void* p, size_t a) { return p != nullptr && (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
-// Per-device state: address of the error word and SM count, looked up once.
-nld_status_t device_state(unsigned int** err, int* sms) {
+// Per-device state: addresses of the error word and the rescale counter and
+// the SM count, looked up once.
+nld_status_t device_state(unsigned int** err, int* sms, unsigned long long** rescales = nullptr) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return NLD_ERR_CUDA;
   std::lock_guard<std::mutex> lock(g_mu);
   if (g_err_ptr[dev] == nullptr) {
     void* p = nullptr;
+    void* c = nullptr;
     if (cudaGetSymbolAddress(&p, g_device_error) != cudaSuccess) return NLD_ERR_CUDA;
+    if (cudaGetSymbolAddress(&c, g_rescale_count) != cudaSuccess) return NLD_ERR_CUDA;
     int n = 0;
     if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return NLD_ERR_CUDA;
     g_sm_count[dev] = n;
+    g_rescale_ptr[dev] = static_cast<unsigned long long*>(c);
     g_err_ptr[dev] = static_cast<unsigned int*>(p);
   }
   if (err) *err = g_err_ptr[dev];
   if (sms) *sms = g_sm_count[dev];
+  if (rescales) *rescales = g_rescale_ptr[dev];
   return NLD_OK;
 }
 
@@ -329,7 +337,8 @@ nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_bloc
     if (!aligned(workspace, 16)) return NLD_ERR_INVALID_ARG;
   }
   unsigned int* err = nullptr;
-  st = device_state(&err, nullptr);
+  unsigned long long* rescales = nullptr;
+  st = device_state(&err, nullptr, &rescales);
   if (st != NLD_OK) return st;
 
   nld::TmaMaps maps;
@@ -345,6 +354,7 @@ nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_bloc
   a.out = static_cast<__nv_bfloat16*>(out);
   a.lse = lse;
   a.err = err;
+  a.rescales = rescales;
   a.B = params->batch;
   a.Hq = params->num_q_heads;
   a.Hkv = params->num_kv_heads;
@@ -576,6 +586,21 @@ nld_status_t nld_device_error(uint32_t* bits, int clear) {
   if (clear) {
     const unsigned int zero = 0;
     if (cudaMemcpy(err, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess) return NLD_ERR_CUDA;
+  }
+  return NLD_OK;
+}
+
+nld_status_t nld_rescale_count(uint64_t* count, int clear) {
+  if (count == nullptr) return NLD_ERR_INVALID_ARG;
+  unsigned long long* c = nullptr;
+  nld_status_t st = device_state(nullptr, nullptr, &c);
+  if (st != NLD_OK) return st;
+  unsigned long long v = 0;
+  if (cudaMemcpy(&v, c, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return NLD_ERR_CUDA;
+  *count = static_cast<uint64_t>(v);
+  if (clear) {
+    const unsigned long long zero = 0;
+    if (cudaMemcpy(c, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess) return NLD_ERR_CUDA;
   }
   return NLD_OK;
 }

@@ -32,6 +32,7 @@ struct AttnArgs {
   float* o_part;               // [S, B, Hq, bl, D]    (split; null when unsplit)
   float* lse_part;             // [S, B, Hq, bl]
   unsigned int* err;           // device error word
+  unsigned long long* rescales;  // running-max rescale events (diagnostic counter)
   int B, Hq, Hkv, G, bl, R;    // R = G * bl query rows per CTA
   int page_size, log2_page, num_pages, max_pages;
   int num_splits, chunk;       // splits and tokens per split (multiple of 16)

@@ -90,6 +90,8 @@ def lib(path: Optional[str] = None):
     L.nld_status_string.restype = ctypes.c_char_p
     L.nld_device_error.argtypes = [ctypes.POINTER(ctypes.c_uint32), I]
     L.nld_device_error.restype = I
+    L.nld_rescale_count.argtypes = [ctypes.POINTER(ctypes.c_uint64), I]
+    L.nld_rescale_count.restype = I
     L.nld_check_wait_timeout.argtypes = [ctypes.c_uint64, V]
     L.nld_check_wait_timeout.restype = I
     L.nld_block_attn_plan.argtypes = [PP, I, I, ctypes.POINTER(ctypes.c_int32)]
@@ -384,6 +386,13 @@ def nld_device_error(clear: bool = False) -> int:
     bits = ctypes.c_uint32(0)
     _check(lib().nld_device_error(ctypes.byref(bits), 1 if clear else 0), "nld_device_error")
     return int(bits.value)
+
+
+def nld_rescale_count(clear: bool = False) -> int:
+    """Running-max rescale events of the attention kernels on this device."""
+    n = ctypes.c_uint64(0)
+    _check(lib().nld_rescale_count(ctypes.byref(n), 1 if clear else 0), "nld_rescale_count")
+    return int(n.value)
 
 
 def nld_status_string(status: int) -> str:

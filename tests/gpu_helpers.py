@@ -34,14 +34,14 @@ class DeviceCase:
     def q_bits(self, mode):
         return self.case.q_draft_bits if mode == W.MODE_DIFFUSION else self.case.q_verify_bits
 
-    def params(self, num_splits=0, flags=0):
+    def params(self, num_splits=0, flags=0, softmax_scale=0.0):
         c = self.case
         return nld.make_params(c.batch, c.num_q_heads, c.num_kv_heads, c.head_dim, c.page_size,
-                               c.kv.num_pages, c.kv.max_pages, num_splits, 0.0, flags)
+                               c.kv.num_pages, c.kv.max_pages, num_splits, softmax_scale, flags)
 
-    def run(self, mode, num_splits=0, q=None, flags=0):
+    def run(self, mode, num_splits=0, q=None, flags=0, softmax_scale=0.0):
         c = self.case
-        p = self.params(num_splits, flags)
+        p = self.params(num_splits, flags, softmax_scale)
         q = self.q[mode] if q is None else q
         out = torch.empty((c.batch, c.block_len, c.num_q_heads, c.head_dim), dtype=torch.bfloat16, device=q.device)
         lse = torch.empty((c.batch, c.num_q_heads, c.block_len), dtype=torch.float32, device=q.device)
@@ -57,19 +57,37 @@ def oracle_full(orc, case: W.BlockAttnCase, mode):
                           case.num_q_heads, case.num_kv_heads, case.block_len, mode, case.scale)
 
 
-def compare_attn(out_gpu: torch.Tensor, lse_gpu: torch.Tensor, out_ref: np.ndarray, lse_ref: np.ndarray, what=""):
+def compare_attn(out_gpu: torch.Tensor, lse_gpu: torch.Tensor, out_ref: np.ndarray, lse_ref: np.ndarray, what="",
+                 max_abs=MAX_ABS):
     o = out_gpu.float().cpu().numpy().astype(np.float64)
     err = np.abs(o - out_ref)
+    bar = max_abs
     max_abs = float(err.max()) if err.size else 0.0
     rel = float(np.linalg.norm(o - out_ref) / max(np.linalg.norm(out_ref), 1e-30))
     assert np.all(np.isfinite(o)), f"{what}: non-finite output"
-    assert max_abs <= MAX_ABS, f"{what}: max abs err {max_abs:.3e}"
+    assert max_abs <= bar, f"{what}: max abs err {max_abs:.3e}"
     assert rel <= REL_L2, f"{what}: rel L2 err {rel:.3e}"
     if lse_gpu is not None:
         l = lse_gpu.cpu().numpy().astype(np.float64)
         lerr = float(np.max(np.abs(l - lse_ref))) if l.size else 0.0
         assert lerr <= LSE_ABS, f"{what}: lse err {lerr:.3e}"
     return max_abs, rel
+
+
+def rows_per_unit(case: W.BlockAttnCase, per_unit: int, seed: int):
+    """(b, i, h) rows: `per_unit` random rows of every (sequence, KV head),
+    i.e. of every CTA group of the launch, plus each sequence's first and
+    last block rows."""
+    rng = np.random.default_rng(seed)
+    G = case.num_q_heads // case.num_kv_heads
+    rows = set()
+    for b in range(case.batch):
+        rows.add((b, 0, 0))
+        rows.add((b, case.block_len - 1, case.num_q_heads - 1))
+        for g in range(case.num_kv_heads):
+            for _ in range(per_unit):
+                rows.add((b, int(rng.integers(case.block_len)), g * G + int(rng.integers(G))))
+    return np.array(sorted(rows), dtype=np.int32)
 
 
 def sample_rows(case: W.BlockAttnCase, n: int, seed: int):

@@ -13,7 +13,7 @@ import pytest
 import torch
 
 import oracle_pins
-from gpu_helpers import DeviceCase, compare_attn, oracle_full, sample_rows
+from gpu_helpers import DeviceCase, compare_attn, oracle_full, rows_per_unit, sample_rows
 from paper_2607_05722_gb300 import nld
 from paper_2607_05722_gb300 import workloads as W
 
@@ -802,15 +802,19 @@ def test_workspace_too_small_launches_nothing():
 
 
 # ---------------------------------------------------------------------------
-# attention: the named workloads at full size, sampled rows
+# attention: the named workloads at full size
 # ---------------------------------------------------------------------------
 
-FULL = ["tiny_b1_h4x1_d64_L256_bl8", "8b_b1_h32x8_d128_L4096_bl16", "long_b1_h32x8_d128_L32768_bl32",
-        "14b_b16_h40x8_d128_L8k-16k_bl32", "conc_b8_h32x8_d128_L512-8192_bl8", "conc_b128_h32x8_d128_L512-8192_bl8"]
+# every row of both passes where the oracle takes seconds; elsewhere four
+# rows of every (sequence, KV head), so every CTA group's output is checked
+FULL_ALL_ROWS = ["tiny_b1_h4x1_d64_L256_bl8", "8b_b1_h32x8_d128_L4096_bl16", "long_b1_h32x8_d128_L32768_bl32"]
+FULL = FULL_ALL_ROWS + ["14b_b16_h40x8_d128_L8k-16k_bl32", "conc_b8_h32x8_d128_L512-8192_bl8",
+                        "conc_b32_h32x8_d128_L512-8192_bl8", "conc_b64_h32x8_d128_L512-8192_bl8",
+                        "conc_b128_h32x8_d128_L512-8192_bl8"]
 
 
 @pytest.mark.parametrize("name", FULL)
-def test_full_size_workload_sampled_rows(orc, name):
+def test_full_size_workload(orc, name):
     wl = W.make_workload(name, seed=0)
     case = wl.attn
     dc = DeviceCase(case)
@@ -819,7 +823,11 @@ def test_full_size_workload_sampled_rows(orc, name):
             continue
         # automatic split count and the prefix-ready flag, as the bench runs it
         out, lse = dc.run(mode, flags=nld.NLD_ATTN_PREFIX_READY)
-        rows = sample_rows(case, 48, seed=mode + 1)
+        if name in FULL_ALL_ROWS:
+            ro, rl = oracle_full(orc, case, mode)
+            compare_attn(out, lse, ro, rl, f"{name} mode={mode} all rows")
+            continue
+        rows = rows_per_unit(case, 4, seed=mode + 1)
         qb = dc.q_bits(mode)
         ro, rl = orc.block_attn_rows(qb, case.kv.k_bits, case.kv.v_bits, case.kv.page_table, case.kv.prefix_lens,
                                      case.num_q_heads, case.num_kv_heads, case.block_len, mode, case.scale, rows)
