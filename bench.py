@@ -69,6 +69,8 @@ def parse_args():
     ap.add_argument("--no-prefix-ready", action="store_true",
                     help="do not let attention stream prefix KV before its dependency wait")
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--merge-in-grid", action="store_true",
+                    help="merge split partials inside the attention grid instead of with the combine kernel")
     return ap.parse_args()
 
 
@@ -275,10 +277,11 @@ def run_ours(args, world, rank, local):
     # The page table, prefix lengths and prefix KV are not written by the
     # kernels of the step, so each attention pass may start streaming its
     # prefix before waiting on the previous kernel (NLD_ATTN_PREFIX_READY).
+    merge_flag = nld.NLD_ATTN_MERGE_IN_GRID if args.merge_in_grid else 0
     params = nld.make_params(B, Hq, Hkv, D, c.page_size, kv.num_pages, kv.max_pages, args.splits, 0.0,
-                             0 if args.no_prefix_ready else nld.NLD_ATTN_PREFIX_READY)
+                             merge_flag | (0 if args.no_prefix_ready else nld.NLD_ATTN_PREFIX_READY))
     splits = nld.nld_block_attn_num_splits(params, bl)
-    ws = torch.empty(max(nld.nld_block_attn_workspace_size(params, bl), 16), dtype=torch.uint8, device=dev)
+    ws = torch.zeros(max(nld.nld_block_attn_workspace_size(params, bl), 16), dtype=torch.uint8, device=dev)
     out_d = torch.empty((B, bl, Hq, D), dtype=torch.bfloat16, device=dev)
     out_v = torch.empty_like(out_d)
     lse_d = torch.empty((B, Hq, bl), dtype=torch.float32, device=dev)
@@ -290,7 +293,8 @@ def run_ours(args, world, rank, local):
     acc = torch.empty((B,), dtype=torch.int32, device=dev)
     pos = torch.empty((B, k_unmask), dtype=torch.int32, device=dev)
     nsel = torch.empty((B,), dtype=torch.int32, device=dev)
-    launches_per_step = 2 * (1 + (splits > 1)) + 2
+    attn_kernels = nld.nld_block_attn_kernels(params, bl)  # 1: unsplit or merged in the grid; 2: + combine
+    launches_per_step = 2 * attn_kernels + 2
 
     def step(i, kd=None, vd=None, kvv=None, vv=None):
         kd, vd = (kd, vd) if kd is not None else pools[(2 * i) % npool]
@@ -363,10 +367,12 @@ def run_ours(args, world, rank, local):
     views = nld.workspace_views(params, bl, ws)
 
     def attn_launch(j, strm=None):
+        # the attention kernel alone: with the in-grid merge that is the whole
+        # call; otherwise the partials entry (the combine is timed apart)
         kp, vp = pools[j % npool]
         mode = nld.NLD_MODE_VERIFY if j % 2 else nld.NLD_MODE_DIFFUSION
-        nld.nld_block_attn_partials(params, q_v if j % 2 else q_d, kp, vp, table, prefix, bl, mode, out_v, lse_v,
-                                    ws, stream=strm)
+        fn = nld.nld_block_attn if attn_kernels == 1 else nld.nld_block_attn_partials
+        fn(params, q_v if j % 2 else q_d, kp, vp, table, prefix, bl, mode, out_v, lse_v, ws, stream=strm)
 
     g_attn = torch.cuda.CUDAGraph()
     with torch.cuda.stream(stream):
@@ -374,7 +380,7 @@ def run_ours(args, world, rank, local):
             for j in range(nker):
                 attn_launch(j)
     g_comb = None
-    if views is not None:
+    if views is not None and attn_kernels == 2:
         g_comb = torch.cuda.CUDAGraph()
         with torch.cuda.stream(stream):
             with torch.cuda.graph(g_comb, stream=stream):
@@ -410,7 +416,8 @@ def run_ours(args, world, rank, local):
     attn_iso_ms = float(np.mean([x.elapsed_time(y) for x, y in evs]))
 
     # ---- end to end through the API with host buffers ----
-    e2e_params = nld.make_params(B, Hq, Hkv, D, c.page_size, kv.num_pages, kv.max_pages, args.splits, 0.0, 0)
+    e2e_params = nld.make_params(B, Hq, Hkv, D, c.page_size, kv.num_pages, kv.max_pages, args.splits, 0.0,
+                                 merge_flag)
     e2e = run_e2e(args, torch, nld, dev, stream, wl, e2e_params, splits, kv_bytes, world)
 
     if world > 1:
@@ -440,7 +447,10 @@ def run_ours(args, world, rank, local):
             "workload": WORKLOAD,
             "batch_per_gpu": B, "q_heads": Hq, "kv_heads": Hkv, "head_dim": D, "prefix": int(kv.prefix_lens[0]),
             "block_len": bl, "page_size": c.page_size, "page_order": "random permutation",
-            "kv_partials": splits, "unmask_k": k_unmask, "prefix_ready_flag": not args.no_prefix_ready,
+            "kv_partials": splits, "attn_kernels_per_pass": attn_kernels,
+            "split_merge": ("in the attention grid" if attn_kernels == 1 and splits > 1 else
+                            "combine kernel" if attn_kernels == 2 else "none (one partial)"),
+            "unmask_k": k_unmask, "prefix_ready_flag": not args.no_prefix_ready,
             "step": "diffusion attention + unmask + verify attention + accept (one attention layer)",
             "l2": f"cold: each pass reads its own KV pool from a rotation of {npool} pools "
                   f"({npool * kv_bytes / 2**20:.0f} MiB > 3x L2 {l2 / 2**20:.0f} MiB)",
@@ -452,7 +462,7 @@ def run_ours(args, world, rank, local):
         "e2e": e2e,
         "gpu_launches": launches_per_step * args.steps,
         "roofline": {
-            "kernel": "block_attn_tc_kernel (attention; split partials when the plan has several)",
+            "kernel": "block_attn_tc_kernel (attention; with the in-grid split merge when the plan has one)",
             "bound": "hbm",
             "achieved": round(attn_gbs, 1),
             "peak": peak,
@@ -527,7 +537,7 @@ def run_e2e(args, torch, nld, dev, stream, wl, params, splits, kv_bytes, world):
 
     sets = [device_set(), device_set()]
     h_out = torch.empty(out_bytes, dtype=torch.uint8).pin_memory()
-    ws = torch.empty(max(nld.nld_block_attn_workspace_size(params, bl), 16), dtype=torch.uint8, device=dev)
+    ws = torch.zeros(max(nld.nld_block_attn_workspace_size(params, bl), 16), dtype=torch.uint8, device=dev)
     nsel = torch.empty((B,), dtype=torch.int32, device=dev)
     copy_stream = torch.cuda.Stream(device=dev)
 
@@ -635,7 +645,7 @@ def run_quadss(torch, nld, dev, stream, peak, l2):
         q = torch.randn((B, bl, Hq, D), generator=gen, device=dev).to(torch.bfloat16)
         out = torch.empty_like(q)
         p = nld.make_params(B, Hq, Hkv, D, P, pages, pages, 0, 0.0, 0)
-        ws = torch.empty(max(16, nld.nld_block_attn_workspace_size(p, bl)), dtype=torch.uint8, device=dev)
+        ws = torch.zeros(max(16, nld.nld_block_attn_workspace_size(p, bl)), dtype=torch.uint8, device=dev)
         bm = torch.from_numpy(nld.nld_quadss_block_mask(k).view(np.int32)).to(dev)
         masked = lambda i: nld.nld_block_attn_masked(p, q, pools[i % npool][0], pools[i % npool][1], table, prefix, bl,
                                                      bm, out, None, ws)
@@ -742,6 +752,47 @@ def run_decisions(torch, nld, dev, stream):
     return res
 
 
+SWEEP_SPLITS = (1, 2, 4, 8, 12, 16, 19, 24, 32, 48, 64)
+
+
+def split_sweep(torch, nld, stream, w, pools, out, lse, peak):
+    """Verify-pass time over explicit KV split counts, three ways: the
+    default plan (pieces of 2/4/8 dividing S merge as clusters), every piece
+    its own partial merged by the combine kernel, and every piece its own
+    partial merged inside the attention grid where the grid fits in one wave
+    (else by the combine kernel). `partial_bytes` = S x B x Hq x bl x (D+1)
+    x 4, written once and read once by the merge."""
+    B, bl, Hq, Hkv, D = w["batch"], w["bl"], w["hq"], w["hkv"], w["d"]
+    kvb = w["kv_bytes_per_pass"]
+    variants = (("clusters", 0), ("no_cluster", nld.NLD_ATTN_NO_CLUSTER),
+                ("no_cluster_in_grid_merge", nld.NLD_ATTN_NO_CLUSTER | nld.NLD_ATTN_MERGE_IN_GRID))
+    sweep = {}
+    for vname, vflags in variants:
+        curve = {}
+        for S in SWEEP_SPLITS:
+            pS = nld.make_params(B, Hq, Hkv, D, w["page"], w["num_pages"], w["max_pages"], S, 0.0,
+                                 nld.NLD_ATTN_PREFIX_READY | vflags)
+            plan = nld.nld_block_attn_plan(pS, bl, torch.cuda.get_device_properties(0).multi_processor_count)
+            wsS = torch.zeros(max(nld.nld_block_attn_workspace_size(pS, bl), 16), dtype=torch.uint8,
+                              device=out.device)
+
+            def one(i, pS=pS, wsS=wsS):
+                kp, vp = pools[i % len(pools)]
+                nld.nld_block_attn(pS, w["q_verify"], kp, vp, w["page_table"], w["prefix_lens"], bl,
+                                   nld.NLD_MODE_VERIFY, out, lse, wsS)
+            msS = time_graph(torch, stream, one, 16, reps=8)
+            parts = nld.nld_block_attn_num_splits(pS, bl)
+            gbs = kvb / (msS * 1e-3) / 1e9
+            curve[str(S)] = {"us_per_pass": round(msS * 1e3, 2), "kv_gbs": round(gbs, 1),
+                             "pct_of_hbm_peak": round(100 * gbs / peak, 2), "pieces": plan["splits"],
+                             "cluster": plan["cluster"], "kv_partials": parts,
+                             "kernels": nld.nld_block_attn_kernels(pS, bl),
+                             "partial_bytes": (parts * B * Hq * bl * (D + 1) * 4) if parts > 1 else 0}
+            del wsS
+        sweep[vname] = curve
+    return sweep
+
+
 def run_workloads(torch, nld, dev, stream, peak, l2, only=None, batch=None, sweep_splits=False):
     """Each named workload's step (its attention passes, then its decisions),
     inputs drawn on the device, pools rotated past L2 where the KV is smaller
@@ -758,7 +809,7 @@ def run_workloads(torch, nld, dev, stream, peak, l2, only=None, batch=None, swee
         params = nld.make_params(B, Hq, Hkv, D, w["page"], w["num_pages"], w["max_pages"], 0, 0.0,
                                  nld.NLD_ATTN_PREFIX_READY)
         parts = nld.nld_block_attn_num_splits(params, bl)
-        ws = torch.empty(max(nld.nld_block_attn_workspace_size(params, bl), 16), dtype=torch.uint8, device=dev)
+        ws = torch.zeros(max(nld.nld_block_attn_workspace_size(params, bl), 16), dtype=torch.uint8, device=dev)
         out = torch.empty((B, bl, Hq, D), dtype=torch.bfloat16, device=dev)
         lse = torch.empty((B, Hq, bl), dtype=torch.float32, device=dev)
         acc = torch.empty((B,), dtype=torch.int32, device=dev)
@@ -791,20 +842,7 @@ def run_workloads(torch, nld, dev, stream, peak, l2, only=None, batch=None, swee
                  "l2": ("cold: %d rotating pools" % npool) if npool * kvb >= 3 * l2 else
                        "warm: KV fits in L2 (%d pools, launch-bound shape)" % npool}
         if (name.startswith("long") and only is None) or sweep_splits:
-            sweep = {}
-            for S in (1, 2, 4, 8, 16, 32, 64):
-                pS = nld.make_params(B, Hq, Hkv, D, w["page"], w["num_pages"], w["max_pages"], S, 0.0,
-                                     nld.NLD_ATTN_PREFIX_READY)
-                wsS = torch.empty(max(nld.nld_block_attn_workspace_size(pS, bl), 16), dtype=torch.uint8, device=dev)
-
-                def one(i, pS=pS, wsS=wsS):
-                    kp, vp = pools[i % len(pools)]
-                    nld.nld_block_attn(pS, w["q_verify"], kp, vp, w["page_table"], w["prefix_lens"], bl,
-                                       nld.NLD_MODE_VERIFY, out, lse, wsS)
-                msS = time_graph(torch, stream, one, 16, reps=8)
-                sweep[str(S)] = {"us_per_pass": round(msS * 1e3, 2), "kv_gbs": round(kvb / (msS * 1e-3) / 1e9, 1),
-                                 "kv_partials": nld.nld_block_attn_num_splits(pS, bl)}
-            entry["verify_pass_split_sweep"] = sweep
+            entry["verify_pass_split_sweep"] = split_sweep(torch, nld, stream, w, pools, out, lse, peak)
         res[name] = entry
         del pools, w
         torch.cuda.empty_cache()

@@ -38,8 +38,15 @@
 // The running max is raised lazily: O is rescaled in TMEM only when a row's
 // max grows by more than 2^8 (P then stays below 256, exact enough in bf16);
 // the final division by the matching sum removes the reference max.
+// On request (NLD_ATTN_MERGE_IN_GRID), when a plan splits the KV range of
+// each (sequence, KV head) over CTAs of one wave, the split partials are
+// merged inside the grid: every split CTA publishes its fp32 partial, and
+// once all splits of its (sequence, KV head) have arrived it merges a slice
+// of that unit's rows into the final output (merge_unit_in_grid), so no
+// combine kernel follows.
 #pragma once
 #include "nld_internal.cuh"
+#include "split_merge.cuh"
 
 namespace nld {
 namespace {
@@ -135,6 +142,98 @@ __device__ __noinline__ int sequence_by_length_rank(const AttnArgs& a, int* scra
   }
   __syncthreads();
   return order[blockIdx.z];
+}
+
+// In-grid split merge for the (sequence b, KV head g) unit of this CTA, split
+// `split` of S (the split-combine rule of Sec. 3's passes over the whole
+// prefix: partials merge by their log-sum-exps). Run by every thread after a
+// barrier that follows this CTA's partial and lse writes; `leader` is the
+// thread that waited for the partial's TMA stores to complete, and `base`
+// the unit's base word it read after its dependency wait.
+// Unit words: [0] arrivals (only ever incremented), [1] base (the arrival
+// count when the current call started; arrivals == base between calls),
+// [2..5] give-up bits, one per split.
+//  1. The leader publishes the partial with a release increment of the
+//     arrival count (ticket t) and polls the count until it reaches
+//     base + S (every split of the unit has arrived), at most
+//     a.merge_wait_ns.
+//  2. If all arrived, the CTA merges rows [split*Rs, (split+1)*Rs) of the
+//     unit (Rs = ceil(R / S)) from every split's partial, one warp per row,
+//     with the combine kernel's row arithmetic, into out and lse.
+//  3. A CTA that waited in vain sets its split's give-up bit and looks once
+//     more; if all have arrived by then it merges its slice itself,
+//     otherwise it leaves. The last to arrive (t == base + S - 1) sets the
+//     base for the next call and takes the give-up bits (fence.sc on both
+//     sides: a CTA that saw the count short of base + S set its bit before
+//     the last arrival's read), merging those slices.
+// Nothing waits without a limit, and no step depends on the CTAs of a unit
+// being resident together. The plan uses this only when the grid fits in
+// one wave (one CTA per SM), where the wait is short.
+template <int D>
+__device__ __noinline__ void merge_unit_in_grid(const AttnArgs& a, uint8_t* smem, int b, int g, int split,
+                                                int leader, unsigned int base) {
+  grid_dependency_wait();  // every thread that writes the outputs has waited for earlier grids
+  const int S = a.num_splits;
+  const int Rs = (a.R + S - 1) / S;
+  const int r0 = min(a.R, split * Rs);
+  const int r1 = min(a.R, r0 + Rs);
+  unsigned int* ctr = a.merge_ctr + (static_cast<size_t>(b) * a.Hkv + g) * kMergeCtrWords;
+  // [0] all arrived, [1] last to arrive, [2..5] give-up bits taken by the last
+  volatile unsigned int* sh = reinterpret_cast<volatile unsigned int*>(smem);
+  const long R = static_cast<long>(a.B) * a.Hq * a.bl;
+  const int warp = static_cast<int>(threadIdx.x >> 5), nwarps = static_cast<int>(blockDim.x >> 5);
+  auto merge_rows = [&](int q0, int q1) {
+    for (int r = q0 + warp; r < q1; r += nwarps) {
+      const int i = r / a.G, h = g * a.G + (r - i * a.G);
+      merge_split_row<D, true>(a.o_part, a.lse_part, S, R, (static_cast<long>(b) * a.Hq + h) * a.bl + i, a.Hq,
+                               a.bl, a.out, a.lse);
+    }
+  };
+  if (static_cast<int>(threadIdx.x) == leader) {
+    const unsigned int target = base + static_cast<unsigned int>(S);
+    const unsigned int t = atom_add_release_gpu(&ctr[0], 1u);
+    bool all = false;
+    const uint64_t t0 = global_timer_ns();
+    for (uint32_t it = 0;; ++it) {
+      if (static_cast<int>(ld_acquire_gpu(&ctr[0]) - target) >= 0) {
+        all = true;
+        break;
+      }
+      if (a.merge_wait_ns == 0 || ((it & 15u) == 15u && global_timer_ns() - t0 >= a.merge_wait_ns)) break;
+      __nanosleep(32);
+    }
+    if (!all) {
+      atomicOr(&ctr[2 + split / 32], 1u << (split & 31));
+      fence_sc_gpu();
+      if (static_cast<int>(ld_acquire_gpu(&ctr[0]) - target) >= 0) {
+        all = true;  // every split arrived after all: merge this slice here
+        atomicAnd(&ctr[2 + split / 32], ~(1u << (split & 31)));
+      }
+    }
+    const bool last = t + 1u == target;
+    if (static_cast<unsigned int>(t - base) >= static_cast<unsigned int>(S)) atomicOr(a.err, NLD_DEVERR_MERGE_STATE);
+    if (last) {
+      st_relaxed_gpu(&ctr[1], target);
+      fence_sc_gpu();
+#pragma unroll
+      for (int w = 0; w < 4; ++w) sh[2 + w] = w * 32 < S ? atomicExch(&ctr[2 + w], 0u) : 0u;
+    }
+    sh[0] = all ? 1u : 0u;
+    sh[1] = last ? 1u : 0u;
+  }
+  __syncthreads();
+  if (sh[0] != 0u) merge_rows(r0, r1);
+  if (sh[1] != 0u) {
+    for (int w = 0; w < 4; ++w) {
+      unsigned int bits = sh[2 + w];
+      while (bits != 0u) {
+        const int s = 32 * w + __ffs(static_cast<int>(bits)) - 1;
+        bits &= bits - 1u;
+        const int q0 = min(a.R, s * Rs);
+        merge_rows(q0, min(a.R, q0 + Rs));
+      }
+    }
+  }
 }
 
 template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED>
@@ -234,9 +333,15 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
   const int t_end = min(t_begin + a.chunk, N);
   const int ntiles = t_begin < t_end ? (t_end - t_begin + kTileTok - 1) / kTileTok : 0;
 
+  // In-grid merge: the unit's base word, read by the merge leader (thread
+  // 32 * kSoftmaxWarp0) once it has waited for earlier grids.
+  unsigned int merge_base = 0u;
+  unsigned int* const merge_base_word =
+      a.merge_ctr != nullptr ? a.merge_ctr + (static_cast<size_t>(b) * a.Hkv + g) * kMergeCtrWords + 1 : nullptr;
   if (ntiles == 0) {
     // This split lies past the sequence: its partials carry no keys.
     if (early) grid_dependency_wait();
+    if (merge_base_word != nullptr && threadIdx.x == 32 * kSoftmaxWarp0) merge_base = ld_relaxed_gpu(merge_base_word);
     if (a.csize > 1) {
       float* lse_stage = reinterpret_cast<float*>(smem + Lay::kLseOff);
       for (int r = threadIdx.x; r < Lay::kMergeRows; r += blockDim.x) lse_stage[r] = -INFINITY;
@@ -433,6 +538,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     }
 
     if (MT == 1 && early) grid_dependency_wait();  // before the mask table and the outputs
+    if (merge_base_word != nullptr && sm_tid == 0) merge_base = ld_relaxed_gpu(merge_base_word);
 
     // The keys this row may see inside [t_begin, t_end) are exactly t < lim
     // (Sec. 2.2: the whole prefix; in the draft pass every block slot, in the
@@ -816,7 +922,16 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
           a.lse_part[((static_cast<size_t>(split) * a.B + b) * a.Hq + row_h) * a.bl + row_i] = lse_v;
         }
       }
-      if (sm_tid == 0 && o_ready) bulk_store_wait_read();  // the boxes stay in place until read
+      if (sm_tid == 0 && o_ready) {
+        if (a.merge_ctr != nullptr) {
+          // The partial is published to the other CTAs of the unit: its
+          // writes must be complete and ordered before the release.
+          bulk_store_wait_all();
+          fence_proxy_async_global();
+        } else {
+          bulk_store_wait_read();  // the boxes stay in place until read
+        }
+      }
     }
     tc_fence_before();
   }
@@ -914,6 +1029,10 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     cluster_sync();  // peers keep their shared memory until every merge has read it
   }
 
+  if (a.merge_ctr != nullptr) {
+    __syncthreads();  // this CTA's partial rows and lse values are written
+    merge_unit_in_grid<D>(a, smem, b, g, split, 32 * kSoftmaxWarp0, merge_base);
+  }
   __syncthreads();
   if (warp == kMmaWarp) {
     tc_fence_after();

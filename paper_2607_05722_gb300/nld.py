@@ -24,7 +24,12 @@ NLD_MODE_VERIFY = 1
 NLD_DEVERR_PREFIX_RANGE = 0x1
 NLD_DEVERR_PAGE_RANGE = 0x2
 NLD_DEVERR_WAIT_TIMEOUT = 0x4
+NLD_DEVERR_MERGE_STATE = 0x8
 NLD_ATTN_PREFIX_READY = 0x1
+NLD_ATTN_MERGE_IN_GRID = 0x2
+NLD_ATTN_NO_CLUSTER = 0x4
+NLD_ATTN_MERGE_NO_WAIT = 0x8
+MERGE_CTR_BYTES = 8192  # merge counters at the start of a split workspace
 
 HEADER = os.path.join(_build.INCLUDE, "nld.h")
 
@@ -94,6 +99,8 @@ def lib(path: Optional[str] = None):
     L.nld_rescale_count.restype = I
     L.nld_check_wait_timeout.argtypes = [ctypes.c_uint64, V]
     L.nld_check_wait_timeout.restype = I
+    L.nld_block_attn_kernels.argtypes = [PP, I]
+    L.nld_block_attn_kernels.restype = I
     L.nld_block_attn_plan.argtypes = [PP, I, I, ctypes.POINTER(ctypes.c_int32)]
     L.nld_block_attn_plan.restype = I
     if path is None:
@@ -155,6 +162,14 @@ def nld_block_attn_num_splits(params: AttnParams, block_len: int) -> int:
     return int(lib().nld_block_attn_num_splits(ctypes.byref(params), block_len))
 
 
+def nld_block_attn_kernels(params: AttnParams, block_len: int) -> int:
+    """Kernels one nld_block_attn call launches (1 or 2) on the current device."""
+    n = int(lib().nld_block_attn_kernels(ctypes.byref(params), block_len))
+    if n < 0:
+        raise NldError(1, "nld_block_attn_kernels")
+    return n
+
+
 def nld_block_attn_workspace_size(params: AttnParams, block_len: int) -> int:
     n = int(lib().nld_block_attn_workspace_size(ctypes.byref(params), block_len))
     if n == ctypes.c_size_t(-1).value:
@@ -170,11 +185,19 @@ def workspace_views(params: AttnParams, block_len: int, workspace):
         return None
     B, Hq, D = params.batch, params.num_q_heads, params.head_dim
     n_o = S * B * Hq * block_len * D
-    off = ((n_o * 4 + 255) // 256) * 256
+    o0 = MERGE_CTR_BYTES
+    l0 = o0 + ((n_o * 4 + 255) // 256) * 256
     flat = workspace.view(torch.uint8)
-    o_part = flat[:n_o * 4].view(torch.float32).view(S, B, Hq, block_len, D)
-    lse_part = flat[off:off + S * B * Hq * block_len * 4].view(torch.float32).view(S, B, Hq, block_len)
+    o_part = flat[o0:o0 + n_o * 4].view(torch.float32).view(S, B, Hq, block_len, D)
+    lse_part = flat[l0:l0 + S * B * Hq * block_len * 4].view(torch.float32).view(S, B, Hq, block_len)
     return o_part, lse_part
+
+
+def alloc_workspace(params: AttnParams, block_len: int, device="cuda"):
+    """A zeroed workspace for these parameters (None when the plan needs none):
+    the merge counters at its start must be zero before its first use."""
+    n = nld_block_attn_workspace_size(params, block_len)
+    return torch.zeros(n, dtype=torch.uint8, device=device) if n else None
 
 
 def nld_block_attn(params: AttnParams, q_block, k_pages, v_pages, page_table, prefix_lens, block_len: int,

@@ -46,7 +46,7 @@ class DeviceCase:
         out = torch.empty((c.batch, c.block_len, c.num_q_heads, c.head_dim), dtype=torch.bfloat16, device=q.device)
         lse = torch.empty((c.batch, c.num_q_heads, c.block_len), dtype=torch.float32, device=q.device)
         ws_bytes = nld.nld_block_attn_workspace_size(p, c.block_len)
-        ws = torch.empty(max(ws_bytes, 1), dtype=torch.uint8, device=q.device) if ws_bytes else None
+        ws = torch.zeros(max(ws_bytes, 1), dtype=torch.uint8, device=q.device) if ws_bytes else None
         nld.nld_block_attn(p, q, self.k, self.v, self.table, self.prefix, c.block_len, mode, out, lse, ws)
         return out, lse
 

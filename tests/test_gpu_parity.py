@@ -205,7 +205,7 @@ def test_kv_commit_staged_block_attention(orc):
         out = torch.empty((case.batch, case.block_len, case.num_q_heads, case.head_dim), dtype=torch.bfloat16,
                           device="cuda")
         lse = torch.empty((case.batch, case.num_q_heads, case.block_len), dtype=torch.float32, device="cuda")
-        ws = torch.empty(max(16, nld.nld_block_attn_workspace_size(p, case.block_len)), dtype=torch.uint8,
+        ws = torch.zeros(max(16, nld.nld_block_attn_workspace_size(p, case.block_len)), dtype=torch.uint8,
                          device="cuda")
         nld.nld_block_attn(p, bits_dev(qb), bits_dev(kp), bits_dev(vp), torch.from_numpy(kv.page_table).cuda(),
                            torch.from_numpy(kv.prefix_lens).cuda(), case.block_len, mode, out, lse, ws)
@@ -582,7 +582,7 @@ def test_partials_entry_point_then_combine(orc, spec, splits):
         pytest.skip("plan merges on chip: no partials")
     for mode in (DIFF, VER):
         ref_out, ref_lse = dc.run(mode, splits)
-        ws = torch.empty(nld.nld_block_attn_workspace_size(p, bl), dtype=torch.uint8, device="cuda")
+        ws = torch.zeros(nld.nld_block_attn_workspace_size(p, bl), dtype=torch.uint8, device="cuda")
         out = torch.full_like(ref_out, float("nan"))
         lse = torch.full_like(ref_lse, float("nan"))
         nld.nld_block_attn_partials(p, dc.q[mode], dc.k, dc.v, dc.table, dc.prefix, bl, mode, out, lse, ws)
@@ -604,7 +604,7 @@ def run_masked(dc, table, splits=0, q=None):
     q = dc.q[DIFF] if q is None else q
     out = torch.empty((c.batch, c.block_len, c.num_q_heads, c.head_dim), dtype=torch.bfloat16, device="cuda")
     lse = torch.empty((c.batch, c.num_q_heads, c.block_len), dtype=torch.float32, device="cuda")
-    ws = torch.empty(max(16, nld.nld_block_attn_workspace_size(p, c.block_len)), dtype=torch.uint8, device="cuda")
+    ws = torch.zeros(max(16, nld.nld_block_attn_workspace_size(p, c.block_len)), dtype=torch.uint8, device="cuda")
     bm = torch.from_numpy(np.asarray(table, dtype=np.uint32).view(np.int32)).cuda()
     nld.nld_block_attn_masked(p, q, dc.k, dc.v, dc.table, dc.prefix, c.block_len, bm, out, lse, ws)
     return out, lse
