@@ -69,8 +69,6 @@ def parse_args():
     ap.add_argument("--no-prefix-ready", action="store_true",
                     help="do not let attention stream prefix KV before its dependency wait")
     ap.add_argument("--seed", type=int, default=0)
-    ap.add_argument("--merge-in-grid", action="store_true",
-                    help="merge split partials inside the attention grid instead of with the combine kernel")
     return ap.parse_args()
 
 
@@ -277,9 +275,8 @@ def run_ours(args, world, rank, local):
     # The page table, prefix lengths and prefix KV are not written by the
     # kernels of the step, so each attention pass may start streaming its
     # prefix before waiting on the previous kernel (NLD_ATTN_PREFIX_READY).
-    merge_flag = nld.NLD_ATTN_MERGE_IN_GRID if args.merge_in_grid else 0
     params = nld.make_params(B, Hq, Hkv, D, c.page_size, kv.num_pages, kv.max_pages, args.splits, 0.0,
-                             merge_flag | (0 if args.no_prefix_ready else nld.NLD_ATTN_PREFIX_READY))
+                             0 if args.no_prefix_ready else nld.NLD_ATTN_PREFIX_READY)
     splits = nld.nld_block_attn_num_splits(params, bl)
     ws = torch.zeros(max(nld.nld_block_attn_workspace_size(params, bl), 16), dtype=torch.uint8, device=dev)
     out_d = torch.empty((B, bl, Hq, D), dtype=torch.bfloat16, device=dev)
@@ -293,7 +290,7 @@ def run_ours(args, world, rank, local):
     acc = torch.empty((B,), dtype=torch.int32, device=dev)
     pos = torch.empty((B, k_unmask), dtype=torch.int32, device=dev)
     nsel = torch.empty((B,), dtype=torch.int32, device=dev)
-    attn_kernels = nld.nld_block_attn_kernels(params, bl)  # 1: unsplit or merged in the grid; 2: + combine
+    attn_kernels = nld.nld_block_attn_kernels(params, bl)  # 1: unsplit or cluster-merged; 2: + combine
     launches_per_step = 2 * attn_kernels + 2
 
     def step(i, kd=None, vd=None, kvv=None, vv=None):
@@ -367,8 +364,8 @@ def run_ours(args, world, rank, local):
     views = nld.workspace_views(params, bl, ws)
 
     def attn_launch(j, strm=None):
-        # the attention kernel alone: with the in-grid merge that is the whole
-        # call; otherwise the partials entry (the combine is timed apart)
+        # the attention kernel alone: the whole call when it launches one
+        # kernel, else the partials entry (the combine is timed apart)
         kp, vp = pools[j % npool]
         mode = nld.NLD_MODE_VERIFY if j % 2 else nld.NLD_MODE_DIFFUSION
         fn = nld.nld_block_attn if attn_kernels == 1 else nld.nld_block_attn_partials
@@ -416,8 +413,7 @@ def run_ours(args, world, rank, local):
     attn_iso_ms = float(np.mean([x.elapsed_time(y) for x, y in evs]))
 
     # ---- end to end through the API with host buffers ----
-    e2e_params = nld.make_params(B, Hq, Hkv, D, c.page_size, kv.num_pages, kv.max_pages, args.splits, 0.0,
-                                 merge_flag)
+    e2e_params = nld.make_params(B, Hq, Hkv, D, c.page_size, kv.num_pages, kv.max_pages, args.splits, 0.0, 0)
     e2e = run_e2e(args, torch, nld, dev, stream, wl, e2e_params, splits, kv_bytes, world)
 
     if world > 1:
@@ -448,8 +444,7 @@ def run_ours(args, world, rank, local):
             "batch_per_gpu": B, "q_heads": Hq, "kv_heads": Hkv, "head_dim": D, "prefix": int(kv.prefix_lens[0]),
             "block_len": bl, "page_size": c.page_size, "page_order": "random permutation",
             "kv_partials": splits, "attn_kernels_per_pass": attn_kernels,
-            "split_merge": ("in the attention grid" if attn_kernels == 1 and splits > 1 else
-                            "combine kernel" if attn_kernels == 2 else "none (one partial)"),
+            "split_merge": "combine kernel" if attn_kernels == 2 else "none (one partial per row)",
             "unmask_k": k_unmask, "prefix_ready_flag": not args.no_prefix_ready,
             "step": "diffusion attention + unmask + verify attention + accept (one attention layer)",
             "l2": f"cold: each pass reads its own KV pool from a rotation of {npool} pools "
@@ -462,7 +457,7 @@ def run_ours(args, world, rank, local):
         "e2e": e2e,
         "gpu_launches": launches_per_step * args.steps,
         "roofline": {
-            "kernel": "block_attn_tc_kernel (attention; with the in-grid split merge when the plan has one)",
+            "kernel": "block_attn_tc_kernel (attention; split partials when the plan has several)",
             "bound": "hbm",
             "achieved": round(attn_gbs, 1),
             "peak": peak,
@@ -752,20 +747,18 @@ def run_decisions(torch, nld, dev, stream):
     return res
 
 
-SWEEP_SPLITS = (1, 2, 4, 8, 12, 16, 19, 24, 32, 48, 64)
+SWEEP_SPLITS = (1, 2, 4, 8, 12, 14, 16, 17, 18, 19, 20, 24, 32, 48, 64)
 
 
 def split_sweep(torch, nld, stream, w, pools, out, lse, peak):
-    """Verify-pass time over explicit KV split counts, three ways: the
-    default plan (pieces of 2/4/8 dividing S merge as clusters), every piece
-    its own partial merged by the combine kernel, and every piece its own
-    partial merged inside the attention grid where the grid fits in one wave
-    (else by the combine kernel). `partial_bytes` = S x B x Hq x bl x (D+1)
-    x 4, written once and read once by the merge."""
+    """Verify-pass time over explicit KV split counts, two ways: the default
+    plan (pieces of 2/4/8 dividing S merge as thread-block clusters) and
+    every piece its own partial merged by the combine kernel
+    (NLD_ATTN_NO_CLUSTER). `partial_bytes` = S x B x Hq x bl x (D+1) x 4,
+    written once by the attention kernel and read once by the combine."""
     B, bl, Hq, Hkv, D = w["batch"], w["bl"], w["hq"], w["hkv"], w["d"]
     kvb = w["kv_bytes_per_pass"]
-    variants = (("clusters", 0), ("no_cluster", nld.NLD_ATTN_NO_CLUSTER),
-                ("no_cluster_in_grid_merge", nld.NLD_ATTN_NO_CLUSTER | nld.NLD_ATTN_MERGE_IN_GRID))
+    variants = (("clusters", 0), ("no_cluster", nld.NLD_ATTN_NO_CLUSTER))
     sweep = {}
     for vname, vflags in variants:
         curve = {}

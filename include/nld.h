@@ -58,7 +58,6 @@ typedef enum {
 #define NLD_DEVERR_PREFIX_RANGE 0x1u /* a prefix length outside [0, max_pages*P - bl] was clamped */
 #define NLD_DEVERR_PAGE_RANGE 0x2u   /* a page id outside [0, num_pages) was clamped              */
 #define NLD_DEVERR_WAIT_TIMEOUT 0x4u /* a pipeline wait passed its time limit; output is invalid  */
-#define NLD_DEVERR_MERGE_STATE 0x8u  /* the workspace's split-merge counters were inconsistent at entry */
 
 /*
  * Shape of one block-attention call.
@@ -73,9 +72,8 @@ typedef enum {
  *                     into; 0 = choose from the SM count. Values above 128
  *                     are rejected.
  *   softmax_scale     score scale; 0 = 1/sqrt(head_dim)
- *   flags             0, or an OR of NLD_ATTN_PREFIX_READY,
- *                     NLD_ATTN_MERGE_IN_GRID, NLD_ATTN_NO_CLUSTER,
- *                     NLD_ATTN_MERGE_NO_WAIT
+ *   flags             0, or an OR of NLD_ATTN_PREFIX_READY and
+ *                     NLD_ATTN_NO_CLUSTER
  */
 typedef struct {
     int batch;
@@ -103,26 +101,11 @@ typedef struct {
 #define NLD_ATTN_PREFIX_READY 0x1u
 
 /*
- * NLD_ATTN_MERGE_IN_GRID: when the split plan leaves partials and the grid
- * fits in one wave, merge them inside the attention grid instead of with
- * the split combine kernel after it (see nld_block_attn): one kernel per
- * call instead of two, the same results to the bit. On a GB300 in a CUDA
- * graph the in-grid merge is slower (its exchange through L2 costs more
- * than the kernel boundary it removes); it saves one host launch per call
- * for callers that launch eagerly.
- *
  * NLD_ATTN_NO_CLUSTER: never run the splits of a (sequence, KV head) as a
  * thread-block cluster; every split writes its own partial. With explicit
  * split counts this makes num_splits the number of partials.
- *
- * NLD_ATTN_MERGE_NO_WAIT: in the in-grid merge, no CTA waits for the other
- * splits of its (sequence, KV head): the last CTA of each unit to arrive
- * merges every row. Same results to the bit, slower; it exercises the path
- * the merge falls back on when CTAs are not resident together.
  */
-#define NLD_ATTN_MERGE_IN_GRID 0x2u
 #define NLD_ATTN_NO_CLUSTER 0x4u
-#define NLD_ATTN_MERGE_NO_WAIT 0x8u
 
 /*
  * Number of split partials per output row that nld_block_attn leaves in the
@@ -137,9 +120,9 @@ int nld_block_attn_num_splits(const nld_attn_params_t *params, int block_len);
 
 /*
  * Kernels one nld_block_attn call with these parameters launches on the
- * current device: 1 (unsplit, cluster-merged, or split partials merged
- * inside the attention grid) or 2 (attention, then the split combine), or
- * -1 if the parameters are invalid. Host-side query; launches nothing.
+ * current device: 1 (unsplit, or split and merged in a thread-block
+ * cluster) or 2 (attention, then the split combine), or -1 if the
+ * parameters are invalid. Host-side query; launches nothing.
  */
 int nld_block_attn_kernels(const nld_attn_params_t *params, int block_len);
 
@@ -159,16 +142,11 @@ int nld_block_attn_kernels(const nld_attn_params_t *params, int block_len);
 int nld_block_attn_plan(const nld_attn_params_t *params, int block_len, int sm_count, int32_t plan[4]);
 
 /*
- * Workspace bytes nld_block_attn needs (0 when it runs unsplit). Layout:
- *   [0, 8192)        merge counters: 8 uint32 per (sequence, KV head)
- *   8192             O_part  fp32 [S, B, Hq, bl, D]
- *   next 256-byte    LSE_part fp32 [S, B, Hq, bl]
- * The counter region is used only with NLD_ATTN_MERGE_IN_GRID; it must
- * then hold zeros before the first such call (allocate the workspace zeroed
- * once). Every completed call leaves it
- * consistent (per unit: arrival count equal to its base word, give-up bits
- * clear), so a workspace is reused call after call without clearing. Calls
- * whose kernels may overlap on the GPU need separate workspaces.
+ * Workspace bytes nld_block_attn needs (0 when it runs unsplit). The
+ * workspace holds fp32 split partials: O_part [S, B, Hq, bl, D] then
+ * LSE_part [S, B, Hq, bl] at the next 256-byte boundary. Its contents need
+ * no initialisation. Calls whose kernels may overlap on the GPU need
+ * separate workspaces.
  * Returns (size_t)-1 if the parameters are invalid.
  */
 size_t nld_block_attn_workspace_size(const nld_attn_params_t *params, int block_len);
@@ -200,16 +178,7 @@ size_t nld_block_attn_workspace_size(const nld_attn_params_t *params, int block_
  * The block's own K/V must already be in the paged slots L_b .. L_b+bl-1.
  * When the plan splits the KV range into S > 1 partials (the workspace
  * holds them), the attention kernel is followed by the split combine (the
- * kernel nld_split_kv_combine runs). With NLD_ATTN_MERGE_IN_GRID, and when
- * all the CTAs fit in one wave on the device (splits x B x Hkv <= SMs,
- * B x Hkv <= 256), the partials are merged inside the attention grid
- * instead: each split CTA publishes its partial and, once every split of
- * its (sequence, KV head) has arrived, merges a slice of that unit's rows;
- * a CTA that waits in vain for more than 50 us leaves its slice to the last
- * CTA of the unit to arrive, so the merge never depends on the CTAs being
- * resident together. Both give the same bits. A workspace whose merge
- * counters were not consistent at entry (not zeroed before first use, or
- * shared by overlapping calls) is flagged as NLD_DEVERR_MERGE_STATE.
+ * kernel nld_split_kv_combine runs).
  */
 nld_status_t nld_block_attn(const nld_attn_params_t *params, const void *q_block,
                             const void *k_pages, const void *v_pages,
@@ -221,9 +190,8 @@ nld_status_t nld_block_attn(const nld_attn_params_t *params, const void *q_block
  * The attention kernel of nld_block_attn alone, same arguments. When the
  * split plan has one split it writes out and lse exactly as nld_block_attn
  * does. With S > 1 splits it writes only the fp32 partials into the
- * workspace (O_part at offset 8192, LSE_part at the next 256-byte boundary
- * after it; the layout of nld_block_attn_workspace_size) and leaves out/lse
- * untouched and the merge counters unused; the caller then
+ * workspace (O_part at offset 0, LSE_part at the next 256-byte boundary
+ * after S*B*Hq*bl*D*4 bytes) and leaves out/lse untouched; the caller then
  * merges them with nld_split_kv_combine (S = nld_block_attn_num_splits()).
  * This lets a caller time, overlap or reorder the two kernels.
  */
@@ -281,9 +249,6 @@ int nld_quadss_block_mask(int k, uint32_t *masks);
  *     address on that device; make it before any stream capture.
  *   - All calls on a device share the array. Calls whose kernels may overlap
  *     on the GPU (unordered streams) race on it; order them on one stream.
- *   - The array starts with the in-grid merge counters of the workspace
- *     layout; they are zero when the library loads and every completed call
- *     leaves them consistent for the next.
  */
 nld_status_t nld_block_attn_static_scratch(const nld_attn_params_t *params, const void *q_block,
                                            const void *k_pages, const void *v_pages,

@@ -38,15 +38,8 @@
 // The running max is raised lazily: O is rescaled in TMEM only when a row's
 // max grows by more than 2^8 (P then stays below 256, exact enough in bf16);
 // the final division by the matching sum removes the reference max.
-// On request (NLD_ATTN_MERGE_IN_GRID), when a plan splits the KV range of
-// each (sequence, KV head) over CTAs of one wave, the split partials are
-// merged inside the grid: every split CTA publishes its fp32 partial, and
-// once all splits of its (sequence, KV head) have arrived it merges a slice
-// of that unit's rows into the final output (merge_unit_in_grid), so no
-// combine kernel follows.
 #pragma once
 #include "nld_internal.cuh"
-#include "split_merge.cuh"
 
 namespace nld {
 namespace {
@@ -65,22 +58,34 @@ constexpr int kSoftmaxWarp0 = 4;
 // what shared memory the Q tiles leave (up to 8 stages): a streaming CTA's
 // bandwidth is the bytes it has in flight over the DRAM latency, so every
 // stage counts.
-template <int MT, int TPS>
+//
+// CG softmax groups per M tile: with CG = 2 (one M tile of up to 128 rows
+// without row copies, paired products) two groups of four warps share the
+// TMEM lanes; group c takes tile 2j + c of each product j, keeps its own
+// running max and sum and accumulates into its own O columns (PV of its
+// tile only), and the two are merged once before the epilogue, by the
+// split-combine rule. Per product the tensor core runs 8 score MMAs of N =
+// 128 and 8 PV MMAs, and each softmax thread does one 64-column tile: the
+// MMA issue and the softmax chain, which bound a streaming split with one
+// group, both shrink per tile.
+template <int MT, int TPS, int CG = 1>
 struct TcCfg {
   static_assert(TPS == 1 || (TPS == 2 && MT == 1), "paired score products with one M tile");
+  static_assert(CG == 1 || (CG == 2 && MT == 1 && TPS == 2), "two softmax groups: one M tile, paired products");
   static constexpr int kTPS = TPS;               // K/V tiles per score product
   static constexpr int kSTok = kTPS * kTileTok;  // tokens (N) of a score product
   static constexpr int kPBufs = 2 * kTPS;        // tiles in flight between the softmax and PV (barrier slots)
-  static constexpr int kWarps = 5 + 4 * MT;      // 4 producers, 1 MMA, 4*MT softmax
+  static constexpr int kSmWarps = 4 * MT * CG;   // softmax warps
+  static constexpr int kWarps = 5 + kSmWarps;    // 4 producers, 1 MMA, softmax
   static constexpr int kThreads = 32 * kWarps;
-  static constexpr uint32_t kTmemCols = 512;     // MT x (S0 | S1), then MT x O
-  static_assert(2 * MT * kSTok + MT * 128 <= 512, "TMEM columns");
+  static constexpr uint32_t kTmemCols = 512;     // MT x (S0 | S1), then MT x CG x O
+  static_assert(2 * MT * kSTok + MT * CG * 128 <= 512, "TMEM columns");
 };
 
 // producer index of a warp, or -1: warps 0-2 and the last warp
-template <int MT>
+template <int MT, int CG>
 __device__ __forceinline__ int producer_index(int warp) {
-  return warp < 3 ? warp : (warp == TcCfg<MT, 1>::kWarps - 1 ? 3 : -1);
+  return warp < 3 ? warp : (warp == 4 + 4 * MT * CG ? 3 : -1);
 }
 constexpr float kRescaleLog2 = 8.0f;
 
@@ -144,105 +149,14 @@ __device__ __noinline__ int sequence_by_length_rank(const AttnArgs& a, int* scra
   return order[blockIdx.z];
 }
 
-// In-grid split merge for the (sequence b, KV head g) unit of this CTA, split
-// `split` of S (the split-combine rule of Sec. 3's passes over the whole
-// prefix: partials merge by their log-sum-exps). Run by every thread after a
-// barrier that follows this CTA's partial and lse writes; `leader` is the
-// thread that waited for the partial's TMA stores to complete, and `base`
-// the unit's base word it read after its dependency wait.
-// Unit words: [0] arrivals (only ever incremented), [1] base (the arrival
-// count when the current call started; arrivals == base between calls),
-// [2..5] give-up bits, one per split.
-//  1. The leader publishes the partial with a release increment of the
-//     arrival count (ticket t) and polls the count until it reaches
-//     base + S (every split of the unit has arrived), at most
-//     a.merge_wait_ns.
-//  2. If all arrived, the CTA merges rows [split*Rs, (split+1)*Rs) of the
-//     unit (Rs = ceil(R / S)) from every split's partial, one warp per row,
-//     with the combine kernel's row arithmetic, into out and lse.
-//  3. A CTA that waited in vain sets its split's give-up bit and looks once
-//     more; if all have arrived by then it merges its slice itself,
-//     otherwise it leaves. The last to arrive (t == base + S - 1) sets the
-//     base for the next call and takes the give-up bits (fence.sc on both
-//     sides: a CTA that saw the count short of base + S set its bit before
-//     the last arrival's read), merging those slices.
-// Nothing waits without a limit, and no step depends on the CTAs of a unit
-// being resident together. The plan uses this only when the grid fits in
-// one wave (one CTA per SM), where the wait is short.
-template <int D>
-__device__ __noinline__ void merge_unit_in_grid(const AttnArgs& a, uint8_t* smem, int b, int g, int split,
-                                                int leader, unsigned int base) {
-  grid_dependency_wait();  // every thread that writes the outputs has waited for earlier grids
-  const int S = a.num_splits;
-  const int Rs = (a.R + S - 1) / S;
-  const int r0 = min(a.R, split * Rs);
-  const int r1 = min(a.R, r0 + Rs);
-  unsigned int* ctr = a.merge_ctr + (static_cast<size_t>(b) * a.Hkv + g) * kMergeCtrWords;
-  // [0] all arrived, [1] last to arrive, [2..5] give-up bits taken by the last
-  volatile unsigned int* sh = reinterpret_cast<volatile unsigned int*>(smem);
-  const long R = static_cast<long>(a.B) * a.Hq * a.bl;
-  const int warp = static_cast<int>(threadIdx.x >> 5), nwarps = static_cast<int>(blockDim.x >> 5);
-  auto merge_rows = [&](int q0, int q1) {
-    for (int r = q0 + warp; r < q1; r += nwarps) {
-      const int i = r / a.G, h = g * a.G + (r - i * a.G);
-      merge_split_row<D, true>(a.o_part, a.lse_part, S, R, (static_cast<long>(b) * a.Hq + h) * a.bl + i, a.Hq,
-                               a.bl, a.out, a.lse);
-    }
-  };
-  if (static_cast<int>(threadIdx.x) == leader) {
-    const unsigned int target = base + static_cast<unsigned int>(S);
-    const unsigned int t = atom_add_release_gpu(&ctr[0], 1u);
-    bool all = false;
-    const uint64_t t0 = global_timer_ns();
-    for (uint32_t it = 0;; ++it) {
-      if (static_cast<int>(ld_acquire_gpu(&ctr[0]) - target) >= 0) {
-        all = true;
-        break;
-      }
-      if (a.merge_wait_ns == 0 || ((it & 15u) == 15u && global_timer_ns() - t0 >= a.merge_wait_ns)) break;
-      __nanosleep(32);
-    }
-    if (!all) {
-      atomicOr(&ctr[2 + split / 32], 1u << (split & 31));
-      fence_sc_gpu();
-      if (static_cast<int>(ld_acquire_gpu(&ctr[0]) - target) >= 0) {
-        all = true;  // every split arrived after all: merge this slice here
-        atomicAnd(&ctr[2 + split / 32], ~(1u << (split & 31)));
-      }
-    }
-    const bool last = t + 1u == target;
-    if (static_cast<unsigned int>(t - base) >= static_cast<unsigned int>(S)) atomicOr(a.err, NLD_DEVERR_MERGE_STATE);
-    if (last) {
-      st_relaxed_gpu(&ctr[1], target);
-      fence_sc_gpu();
-#pragma unroll
-      for (int w = 0; w < 4; ++w) sh[2 + w] = w * 32 < S ? atomicExch(&ctr[2 + w], 0u) : 0u;
-    }
-    sh[0] = all ? 1u : 0u;
-    sh[1] = last ? 1u : 0u;
-  }
-  __syncthreads();
-  if (sh[0] != 0u) merge_rows(r0, r1);
-  if (sh[1] != 0u) {
-    for (int w = 0; w < 4; ++w) {
-      unsigned int bits = sh[2 + w];
-      while (bits != 0u) {
-        const int s = 32 * w + __ffs(static_cast<int>(bits)) - 1;
-        bits &= bits - 1u;
-        const int q0 = min(a.R, s * Rs);
-        merge_rows(q0, min(a.R, q0 + Rs));
-      }
-    }
-  }
-}
-
-template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED>
-__global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
+template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED, int CG>
+__global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
     block_attn_tc_kernel(const __grid_constant__ TmaMaps maps, const AttnArgs a) {
   static_assert(REP == 1 || REP == 2 || REP == 4, "replication of 1, 2 or 4");
   static_assert(MT == 1 || REP == 1, "replication only with one M tile");
+  static_assert(CG == 1 || REP == 1, "softmax groups without row copies");
   using Geo = TileGeom<D>;
-  using Cfg = TcCfg<MT, TPS>;
+  using Cfg = TcCfg<MT, TPS, CG>;
   using Lay = TcLayout<D, MT, TPS>;
   constexpr int kTcStages = Lay::kStages;
   extern __shared__ uint8_t smem_raw[];
@@ -271,13 +185,13 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     }
     for (int j = 0; j < 2; ++j) {
       mbar_init(&s_full[j], 1);
-      mbar_init(&s_free[j], 4 * MT);
+      mbar_init(&s_free[j], Cfg::kSmWarps);
     }
     for (int j = 0; j < Cfg::kPBufs; ++j) {
       mbar_init(&p_full[j], 4 * MT);
       mbar_init(&o_done[j], 1);
     }
-    mbar_init(q_ready, 4 * MT);
+    mbar_init(q_ready, Cfg::kSmWarps);
     mbar_init(q_full, 1);
     mbar_init(drain, 1);
     fence_mbar_init();
@@ -310,12 +224,13 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
   // independent, so they are in flight together.
   PagePrefetch first;
   first.raw = 0;
-  if (producer_index<MT>(warp) >= 0) first.load(a, b, t_begin, 0, lane);
+  if (producer_index<MT, CG>(warp) >= 0) first.load(a, b, t_begin, 0, lane);
   int L = __ldg(a.prefix_lens + b);
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  // TMEM columns: S of M tile mt, buffer j at (2*mt + j)*kSTok; O of tile mt after all S buffers.
+  // TMEM columns: S of M tile mt, buffer j at (2*mt + j)*kSTok; then the O
+  // accumulators, one per M tile (CG = 1) or per softmax group (CG = 2).
   constexpr int kTPS = Cfg::kTPS;
   constexpr int kSTok = Cfg::kSTok;
   constexpr int kPBufs = Cfg::kPBufs;
@@ -333,15 +248,9 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
   const int t_end = min(t_begin + a.chunk, N);
   const int ntiles = t_begin < t_end ? (t_end - t_begin + kTileTok - 1) / kTileTok : 0;
 
-  // In-grid merge: the unit's base word, read by the merge leader (thread
-  // 32 * kSoftmaxWarp0) once it has waited for earlier grids.
-  unsigned int merge_base = 0u;
-  unsigned int* const merge_base_word =
-      a.merge_ctr != nullptr ? a.merge_ctr + (static_cast<size_t>(b) * a.Hkv + g) * kMergeCtrWords + 1 : nullptr;
   if (ntiles == 0) {
     // This split lies past the sequence: its partials carry no keys.
     if (early) grid_dependency_wait();
-    if (merge_base_word != nullptr && threadIdx.x == 32 * kSoftmaxWarp0) merge_base = ld_relaxed_gpu(merge_base_word);
     if (a.csize > 1) {
       float* lse_stage = reinterpret_cast<float*>(smem + Lay::kLseOff);
       for (int r = threadIdx.x; r < Lay::kMergeRows; r += blockDim.x) lse_stage[r] = -INFINITY;
@@ -351,7 +260,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
         a.lse_part[((static_cast<size_t>(split) * a.B + b) * a.Hq + h) * a.bl + i] = -INFINITY;
       }
     }
-  } else if (producer_index<MT>(warp) >= 0) {
+  } else if (producer_index<MT, CG>(warp) >= 0) {
     // ---------------- producers ----------------
     int early_tiles = 0;  // leading tiles made of prefix tokens only
     if (early) {
@@ -361,7 +270,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
       if (early_tiles == 0) grid_dependency_wait();
     }
     const int issued = produce_kv<D>(a, &maps.k, &maps.v, smem, kv_full, kv_empty, kTcStages, g, b, t_begin, t_end,
-                                     ntiles, lane, producer_index<MT>(warp), kProducers, first, early_tiles);
+                                     ntiles, lane, producer_index<MT, CG>(warp), kProducers, first, early_tiles);
     if (lane == 0 && issued < ntiles) {
       // Stopped early on a wait timeout: let the copies already issued land
       // before the CTA exits (bounded).
@@ -418,12 +327,14 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
         for (int mt = 0; mt < MT; ++mt) {
           // A = P in TMEM (bf16 pairs over the S columns of the tile's first
           // half: 32 columns per 64-token tile); B = V (MN-major: 64-dim
-          // atoms LBO apart, 8-token row groups SBO apart).
+          // atoms LBO apart, 8-token row groups SBO apart). With two softmax
+          // groups tile k accumulates into O of group k % 2.
           const uint32_t p_tmem = tS(mt, (k / kTPS) & 1) + static_cast<uint32_t>((k % kTPS) * 32);
+          const uint32_t o_acc = tO(CG == 2 ? k % CG : mt);
 #pragma unroll
           for (int kt = 0; kt < kTileTok / 16; ++kt) {
             const uint64_t bd = sw128_desc(v_addr + kt * 16 * 128, Geo::kColBlockBytes, 1024);
-            umma_bf16_ts(tO(mt), p_tmem + kt * 8, bd, idesc_o, (k > 0 || kt > 0) ? 1u : 0u);
+            umma_bf16_ts(o_acc, p_tmem + kt * 8, bd, idesc_o, (k >= CG || kt > 0) ? 1u : 0u);
           }
         }
         umma_commit(&o_done[k % kPBufs]);
@@ -489,7 +400,11 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     constexpr int kU = (kTPS == 2 && REP >= 2) ? 2 : 1;  // tiles per softmax step
     constexpr int kColsU = kU * kTileTok / REP;          // S columns per thread and step
     const int quad = warp & 3;
-    const int mt = (warp - kSoftmaxWarp0) >> 2;     // M tile of this warp
+    const int wg = (warp - kSoftmaxWarp0) >> 2;
+    const int mt = CG == 1 ? wg : 0;                // M tile of this warp
+    const int cg = CG == 1 ? 0 : wg;                // softmax group: tiles k % CG == cg, O accumulator cg
+    const int oi = CG == 1 ? mt : cg;               // this warp's O accumulator
+    const int part = CG == 1 ? quad / kRowQuads : cg;  // this thread's share of a row's state (copy or group)
     const int rq = quad % kRowQuads;                // row block
     const int cp = quad / kRowQuads;                // token slice
     const int c0u = cp * kColsU;           // first column of this thread's slice of a step
@@ -502,7 +417,8 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     const bool row_ok = r < a.R;
     const int row_i = r / a.G;
     const int row_h = g * a.G + (r - row_i * a.G);
-    const int sm_tid = threadIdx.x - 32 * kSoftmaxWarp0;  // 0 .. 128*MT-1 across the softmax warps
+    const int sm_tid = threadIdx.x - 32 * kSoftmaxWarp0;  // 0 .. 32*kSmWarps-1 across the softmax warps
+    const int grp_tid = sm_tid - cg * 128 * MT;           // 0 .. 128*MT-1 within this softmax group
     const int swz = r_loc & 7;                      // 128-byte swizzle phase of this tile row
     uint8_t* q_tile = q_s + mt * Lay::kQBytes;
 
@@ -510,7 +426,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     // One M tile: the MMA warp brings Q by TMA and the rows past R are zeroed
     // here, before the dependency wait. Two M tiles: slice 0 of each row loads
     // it here after the wait and writes every copy.
-    if (MT == 1 && !row_ok) {
+    if (MT == 1 && !row_ok && cg == 0) {
 #pragma unroll
       for (int c = 0; c < D / 8; ++c)
         *reinterpret_cast<uint4*>(q_tile + (c >> 3) * (128 * 128) + r_loc * 128 + (((c & 7) ^ swz) << 4)) =
@@ -538,7 +454,6 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     }
 
     if (MT == 1 && early) grid_dependency_wait();  // before the mask table and the outputs
-    if (merge_base_word != nullptr && sm_tid == 0) merge_base = ld_relaxed_gpu(merge_base_word);
 
     // The keys this row may see inside [t_begin, t_end) are exactly t < lim
     // (Sec. 2.2: the whole prefix; in the draft pass every block slot, in the
@@ -572,13 +487,12 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     };
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
-    const int nsteps = (ntiles + kU - 1) / kU;
-    for (int u = 0; u < nsteps; ++u) {
-      const int k0 = u * kU;                      // first tile of the step
+    // This warp's steps start kU*CG tiles apart (CG = 2: the tiles of its group).
+    for (int k0 = cg * kU; k0 < ntiles; k0 += kU * CG) {  // k0: first tile of the step
       const int j = k0 / kTPS, half = k0 % kTPS;  // score product and the step's first 64-token half
       const int step_t0 = t_begin + k0 * kTileTok;
       const int k_own = k0 + h_own;               // the tile holding this thread's columns
-      if (half == 0 && !warp_wait(&s_full[j & 1], (j >> 1) & 1)) {
+      if ((CG == 2 || half == 0) && !warp_wait(&s_full[j & 1], (j >> 1) & 1)) {
         ok = false;
         break;
       }
@@ -597,7 +511,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
       tc_fence_before();
       __syncwarp();
       const int k_last = min(k0 + kU - 1, ntiles - 1);  // last tile of the step
-      if (lane == 0 && (k_last % kTPS == kTPS - 1 || k_last == ntiles - 1)) mbar_arrive(&s_free[j & 1]);
+      if (lane == 0 && (CG == 2 || k_last % kTPS == kTPS - 1 || k_last == ntiles - 1)) mbar_arrive(&s_free[j & 1]);
 
       float alpha = 1.f;
       bool rescale = false;
@@ -635,8 +549,9 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
         }
       }
       if (__any_sync(0xffffffffu, rescale)) {
-        // O holds P_0..P_{k0-1} V: wait for the last PV, then scale this warp's rows.
-        if (!warp_wait(&o_done[(k0 - 1) % kPBufs], ((k0 - 1) / kPBufs) & 1)) {
+        // This warp's O holds the PV of its earlier tiles, the last of them
+        // k0 - CG: wait for it, then scale this warp's rows.
+        if (!warp_wait(&o_done[(k0 - CG) % kPBufs], ((k0 - CG) / kPBufs) & 1)) {
           ok = false;
           break;
         }
@@ -645,10 +560,10 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
 #pragma unroll 1
         for (int c = 0; c < D / 32; ++c) {
           float o[32];
-          tmem_ld32(tO(mt) + lane_off + c * 32, o);
+          tmem_ld32(tO(oi) + lane_off + c * 32, o);
 #pragma unroll
           for (int e = 0; e < 32; ++e) o[e] *= alpha;
-          tmem_st32(tO(mt) + lane_off + c * 32, o);
+          tmem_st32(tO(oi) + lane_off + c * 32, o);
         }
       }
       if (warp_rows) {
@@ -710,7 +625,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
           }
           const int r0 = valid, r1 = (valid + kGroupTok - 1) & ~(kGroupTok - 1);
           uint8_t* vt = smem + Lay::kVOff + st * Geo::kTileBytes;
-          for (int idx = sm_tid; idx < (r1 - r0) * (D / 8); idx += 128 * MT) {
+          for (int idx = grp_tid; idx < (r1 - r0) * (D / 8); idx += 128 * MT) {
             const int row = r0 + idx / (D / 8), c = idx % (D / 8);
             *reinterpret_cast<uint4*>(vt + kv_swz(row, c)) = make_uint4(0, 0, 0, 0);
           }
@@ -738,8 +653,14 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     // split by columns: copy c finalises output columns [c*kRange,
     // (c+1)*kRange), so it leaves its (max, sum) and its unscaled O over the
     // other copies' ranges in the freed ring and reads theirs over its own.
-    constexpr int kRange = D / REP;           // output columns this copy finalises
-    constexpr int kChunk = kRange < 64 ? kRange : 64;  // columns per TMEM load: 16, 32 or 64
+    // With two softmax groups (CG = 2) the work is split the same way: group
+    // c finalises output columns [c*kRange, (c+1)*kRange), reading both
+    // groups' O over them from its own TMEM lanes.
+    constexpr int kParts = REP * CG;            // states per row: copies or softmax groups
+    constexpr int kRange = D / kParts;          // output columns this thread finalises
+    // columns per TMEM load: 16, 32 or 64 (32 at most with two groups, whose
+    // loads are paired)
+    constexpr int kChunk = CG > 1 ? (kRange < 32 ? kRange : 32) : (kRange < 64 ? kRange : 64);
     static_assert(kChunk == 16 || kChunk == 32 || kChunk == 64, "TMEM load width");
     auto ld_chunk = [&](uint32_t taddr, float* o) {
       if constexpr (kChunk == 64) {
@@ -756,7 +677,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
       const int slot = c * (REP - 1) + (q < c ? q : q - 1);
       return smem + Lay::kXchgOff + (slot * 32 * kRowQuads + rq * 32 + lane) * kXPitch;
     };
-    float wgt[REP];  // weight of each copy's O in this row's output, then with 1/sum folded in
+    float wgt[kParts];  // weight of each part's O in this row's output, then with 1/sum folded in
     float m_row = m_run, l_row = l_run;
     wgt[0] = 1.f;
     if (o_ready) tc_fence_after();
@@ -803,14 +724,52 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
       m_row = m;
       l_row = l;
     }
+    if constexpr (CG > 1) {
+      // The groups' (max, sum) per row, exchanged through the freed ring.
+      float* part_ml = reinterpret_cast<float*>(smem + Lay::kWtsOff);  // [group][TMEM lane][max, sum]
+      part_ml[2 * (cg * 128 + r_loc)] = o_ready ? m_run : -INFINITY;  // a group cut short is dropped
+      part_ml[2 * (cg * 128 + r_loc) + 1] = l_run;
+      named_bar_sync(2, 32 * Cfg::kSmWarps);
+      float mc[CG], lc[CG];
+      float m = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < CG; ++c) {
+        mc[c] = part_ml[2 * (c * 128 + r_loc)];
+        lc[c] = part_ml[2 * (c * 128 + r_loc) + 1];
+        m = fmaxf(m, mc[c]);
+      }
+      float l = 0.f;
+#pragma unroll
+      for (int c = 0; c < CG; ++c) {
+        wgt[c] = mc[c] == -INFINITY ? 0.f : ex2(mc[c] - m);
+        l += wgt[c] * lc[c];
+      }
+      m_row = m;
+      l_row = l;
+    }
     const float inv = l_row > 0.f ? 1.f / l_row : 0.f;
 #pragma unroll
-    for (int c = 0; c < REP; ++c) wgt[c] *= inv;
+    for (int c = 0; c < kParts; ++c) wgt[c] *= inv;
     // Normalised output columns cp*kRange + cc*kChunk .. +kChunk-1 of this
     // thread's row: its own TMEM lane plus the other copies' exchanged ranges.
     // Warp-collective.
     auto final_chunk = [&](int cc, float* o) {
-      const int col0 = cp * kRange + cc * kChunk;
+      const int col0 = part * kRange + cc * kChunk;
+      if constexpr (CG > 1) {
+        // Both groups' O over these columns; a group without keys for this
+        // row (weight 0) may hold stale TMEM, so it is selected away.
+        float o2[kChunk];
+        ld_chunk(tO(0) + lane_off + col0, o);
+        ld_chunk(tO(1) + lane_off + col0, o2);
+#pragma unroll
+        for (int j = 0; j < kChunk; ++j)
+          o[j] = (wgt[0] == 0.f ? 0.f : wgt[0] * o[j]) + (wgt[1] == 0.f ? 0.f : wgt[1] * o2[j]);
+        if (!(l_row > 0.f)) {
+#pragma unroll
+          for (int j = 0; j < kChunk; ++j) o[j] = 0.f;
+        }
+        return;
+      }
       ld_chunk(tO(mt) + lane_off + col0, o);
       float w_own = wgt[0];
 #pragma unroll
@@ -843,14 +802,14 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
       // or after a timeout, carry lse = -inf and are skipped by the merge).
       float* lse_stage = reinterpret_cast<float*>(smem + Lay::kLseOff);
       const bool has = o_ready && row_ok && l_row > 0.f;
-      if (cp == 0) lse_stage[r] = has ? m_row + lg2(l_row) : -INFINITY;
+      if (part == 0) lse_stage[r] = has ? m_row + lg2(l_row) : -INFINITY;
       if (warp_rows && o_ready) {
         uint8_t* my = smem + r * merge_pitch<D>();
 #pragma unroll 1
         for (int cc = 0; cc < kRange / kChunk; ++cc) {
           float o[kChunk];
           final_chunk(cc, o);
-          uint8_t* dst = my + (cp * kRange + cc * kChunk) * 4;
+          uint8_t* dst = my + (part * kRange + cc * kChunk) * 4;
 #pragma unroll
           for (int q4 = 0; q4 < kChunk / 4; ++q4)
             *reinterpret_cast<float4*>(dst + q4 * 16) =
@@ -875,7 +834,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
         if (warp_rows && o_ready) {
           float o[kChunk];
           final_chunk(cc, o);
-          const int col0 = cp * kRange + cc * kChunk;
+          const int col0 = part * kRange + cc * kChunk;
           if (row_ok) {
             if (split_out) {
 #pragma unroll
@@ -899,22 +858,29 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
             }
           }
         }
+        // One thread stores the boxes a round completed: with one softmax
+        // group round cc staged columns [cc*D/kIters, (cc+1)*D/kIters) of
+        // every row; with two groups each round staged a slice of both
+        // groups' ranges, so every box is stored after the last round.
+        if (CG > 1 && cc + 1 < kIters) continue;
+        constexpr int kStoreRounds = CG > 1 ? 1 : kIters;
+        const int sr = CG > 1 ? 0 : cc;
         fence_proxy_async_smem();     // the staged boxes, visible to the TMA engine
-        named_bar_sync(3, 128 * MT);  // every softmax warp, with rows or not
+        named_bar_sync(3, 32 * Cfg::kSmWarps);  // every softmax warp, with rows or not
         if (sm_tid == 0 && o_ready) {
           if (split_out) {
 #pragma unroll
-            for (int x = cc * (D / 32 / kIters); x < (cc + 1) * (D / 32 / kIters); ++x)
+            for (int x = sr * (D / 32 / kStoreRounds); x < (sr + 1) * (D / 32 / kStoreRounds); ++x)
               tma_store_4d(&maps.o, smem + x * box_stride, x * 32, g * a.G, 0, split * a.B + b);
           } else {
 #pragma unroll
-            for (int x = cc * (D / 64 / kIters); x < (cc + 1) * (D / 64 / kIters); ++x)
+            for (int x = sr * (D / 64 / kStoreRounds); x < (sr + 1) * (D / 64 / kStoreRounds); ++x)
               tma_store_3d(&maps.o, smem + x * box_stride, x * 64, g * a.G, b * a.bl);
           }
           bulk_commit();
         }
       }
-      if (warp_rows && o_ready && row_ok && cp == 0) {
+      if (warp_rows && o_ready && row_ok && part == 0) {
         const float lse_v = l_row > 0.f ? (m_row + lg2(l_row)) * kLn2 : -INFINITY;
         if (!split_out) {
           if (a.lse != nullptr) a.lse[(static_cast<size_t>(b) * a.Hq + row_h) * a.bl + row_i] = lse_v;
@@ -922,16 +888,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
           a.lse_part[((static_cast<size_t>(split) * a.B + b) * a.Hq + row_h) * a.bl + row_i] = lse_v;
         }
       }
-      if (sm_tid == 0 && o_ready) {
-        if (a.merge_ctr != nullptr) {
-          // The partial is published to the other CTAs of the unit: its
-          // writes must be complete and ordered before the release.
-          bulk_store_wait_all();
-          fence_proxy_async_global();
-        } else {
-          bulk_store_wait_read();  // the boxes stay in place until read
-        }
-      }
+      if (sm_tid == 0 && o_ready) bulk_store_wait_read();  // the boxes stay in place until read
     }
     tc_fence_before();
   }
@@ -943,7 +900,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     // split combine, and writes the final output (one cluster per sequence
     // and KV head) or this cluster's partial.
     cluster_sync();
-    if (warp >= kSoftmaxWarp0 && warp < kSoftmaxWarp0 + 4 * MT) {
+    if (warp >= kSoftmaxWarp0 && warp < kSoftmaxWarp0 + Cfg::kSmWarps) {
       const uint32_t rank = cluster_ctarank();
       const int Rc = (a.R + a.csize - 1) / a.csize;
       const int r0 = static_cast<int>(rank) * Rc;
@@ -975,18 +932,18 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
         for (int p = 0; p < 8; ++p) wts[tid * 8 + p] = w[p] * inv;
         lse_out[tid] = wsum > 0.f ? (m + lg2(wsum)) * kLn2 : -INFINITY;
       }
-      named_bar_sync(1, 128 * MT);
+      named_bar_sync(1, 32 * Cfg::kSmWarps);
       // 2) rows: two (row, 4-dim) items per thread per round, every peer load in flight
       const bool final_out = a.num_partials == 1;
       const int pidx = split / a.csize;
       const int items = nrows * (D / 4);
-      for (int base = tid; base < items; base += 2 * 128 * MT) {
+      for (int base = tid; base < items; base += 2 * 32 * Cfg::kSmWarps) {
         float4 acc[2];
         int ridx[2], d4[2];
         bool live[2];
 #pragma unroll
         for (int u = 0; u < 2; ++u) {
-          const int idx = base + u * 128 * MT;
+          const int idx = base + u * 32 * Cfg::kSmWarps;
           live[u] = idx < items;
           ridx[u] = live[u] ? idx / (D / 4) : 0;
           d4[u] = idx % (D / 4);
@@ -1029,10 +986,6 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
     cluster_sync();  // peers keep their shared memory until every merge has read it
   }
 
-  if (a.merge_ctr != nullptr) {
-    __syncthreads();  // this CTA's partial rows and lse values are written
-    merge_unit_in_grid<D>(a, smem, b, g, split, 32 * kSoftmaxWarp0, merge_base);
-  }
   __syncthreads();
   if (warp == kMmaWarp) {
     tc_fence_after();
@@ -1040,12 +993,12 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS>::kThreads, 1)
   }
 }
 
-template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED = false>
+template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED, int CG>
 cudaError_t configure_tc(int dev) {
   static int configured[64] = {0};
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   if (!__atomic_load_n(&configured[dev], __ATOMIC_ACQUIRE)) {
-    cudaError_t e = cudaFuncSetAttribute(block_attn_tc_kernel<D, MT, REP, TPS, MASKED, ORDERED>,
+    cudaError_t e = cudaFuncSetAttribute(block_attn_tc_kernel<D, MT, REP, TPS, MASKED, ORDERED, CG>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(TcLayout<D, MT, TPS>::kBytes + 1024));
     if (e != cudaSuccess) return e;
@@ -1054,31 +1007,33 @@ cudaError_t configure_tc(int dev) {
   return cudaSuccess;
 }
 
-template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED>
+template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED, int CG>
 cudaError_t launch_tc_o(const AttnArgs& a, const TmaMaps& maps, cudaStream_t stream) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  if ((e = configure_tc<D, MT, REP, TPS, MASKED, ORDERED>(dev)) != cudaSuccess) return e;
+  if ((e = configure_tc<D, MT, REP, TPS, MASKED, ORDERED, CG>(dev)) != cudaSuccess) return e;
   dim3 grid(a.num_splits, a.Hkv, a.B);
-  return launch_kernel_cluster(block_attn_tc_kernel<D, MT, REP, TPS, MASKED, ORDERED>, grid,
-                               dim3(TcCfg<MT, TPS>::kThreads), TcLayout<D, MT, TPS>::kBytes + 1024, stream, a.csize,
-                               maps, a);
+  return launch_kernel_cluster(block_attn_tc_kernel<D, MT, REP, TPS, MASKED, ORDERED, CG>, grid,
+                               dim3(TcCfg<MT, TPS, CG>::kThreads), TcLayout<D, MT, TPS>::kBytes + 1024, stream,
+                               a.csize, maps, a);
 }
 
 // The longest-first order only for the unmasked passes (the table-mask
 // passes run at the block shapes of one sequence).
-template <int D, int MT, int REP, int TPS, bool MASKED>
+template <int D, int MT, int REP, int TPS, bool MASKED, int CG = 1>
 cudaError_t launch_tc_t(const AttnArgs& a, const TmaMaps& maps, cudaStream_t stream) {
   if constexpr (!MASKED) {
-    if (a.order_by_length) return launch_tc_o<D, MT, REP, TPS, false, true>(a, maps, stream);
+    if (a.order_by_length) return launch_tc_o<D, MT, REP, TPS, false, true, CG>(a, maps, stream);
   }
-  return launch_tc_o<D, MT, REP, TPS, MASKED, false>(a, maps, stream);
+  return launch_tc_o<D, MT, REP, TPS, MASKED, false, CG>(a, maps, stream);
 }
 
-// With one CTA per SM either way, cluster residency is the same for both
-// score-product widths; the query uses TPS = 1.
-template <int D, int MT, int REP>
+// Resident clusters of the kernel a plan would launch (one CTA per SM
+// either way; row copies and score-product width do not change residency,
+// the thread count of two softmax groups does not either, but the query
+// uses the instantiation that runs).
+template <int D, int MT, int REP, int TPS, int CG>
 int max_active_clusters_t(int csize) {
   static int cache[64][4];  // [device][cluster size 2/4/8] + 1 (0 = not queried)
   int dev = 0;
@@ -1086,11 +1041,11 @@ int max_active_clusters_t(int csize) {
   const int slot = csize == 2 ? 0 : csize == 4 ? 1 : csize == 8 ? 2 : 3;
   int v = __atomic_load_n(&cache[dev][slot], __ATOMIC_ACQUIRE);
   if (v) return v - 1;
-  if (configure_tc<D, MT, REP, 1, false, false>(dev) != cudaSuccess) return 0;
+  if (configure_tc<D, MT, REP, TPS, false, false, CG>(dev) != cudaSuccess) return 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(csize, 1, 1);
-  cfg.blockDim = dim3(TcCfg<MT, 1>::kThreads);
-  cfg.dynamicSmemBytes = TcLayout<D, MT, 1>::kBytes + 1024;
+  cfg.blockDim = dim3(TcCfg<MT, TPS, CG>::kThreads);
+  cfg.dynamicSmemBytes = TcLayout<D, MT, TPS>::kBytes + 1024;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = csize;
@@ -1099,7 +1054,8 @@ int max_active_clusters_t(int csize) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, block_attn_tc_kernel<D, MT, REP, 1, false, false>, &cfg) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveClusters(&n, block_attn_tc_kernel<D, MT, REP, TPS, false, false, CG>, &cfg) !=
+      cudaSuccess) {
     cudaGetLastError();
     n = 0;
   }
@@ -1113,25 +1069,27 @@ int tc_replication(int rows) { return rows <= 32 ? 4 : rows <= 64 ? 2 : 1; }
 
 template <int D>
 int max_active_clusters_d(int csize, int rows) {
-  if (rows > 128) return max_active_clusters_t<D, 2, 1>(csize);
+  if (rows > 128) return max_active_clusters_t<D, 2, 1, 1, 1>(csize);
   switch (tc_replication(rows)) {
-    case 4: return max_active_clusters_t<D, 1, 4>(csize);
-    case 2: return max_active_clusters_t<D, 1, 2>(csize);
-    default: return max_active_clusters_t<D, 1, 1>(csize);
+    case 4: return max_active_clusters_t<D, 1, 4, 1, 1>(csize);
+    case 2: return max_active_clusters_t<D, 1, 2, 1, 1>(csize);
+    default: return max_active_clusters_t<D, 1, 1, 2, 2>(csize);
   }
 }
 
+// One M tile: rows copied 4 or 2 times (up to 64 rows), with paired score
+// products when a split fits in the ring whole (it is then latency-bound:
+// fewer, wider steps help) and single tiles when it streams; 65..128 rows
+// take paired products and two softmax groups, streaming or not.
 template <int D, int TPS, bool MASKED>
 cudaError_t launch_tc_rep(const AttnArgs& a, const TmaMaps& maps, cudaStream_t stream) {
   switch (tc_replication(a.R)) {
     case 4: return launch_tc_t<D, 1, 4, TPS, MASKED>(a, maps, stream);
     case 2: return launch_tc_t<D, 1, 2, TPS, MASKED>(a, maps, stream);
-    default: return launch_tc_t<D, 1, 1, TPS, MASKED>(a, maps, stream);
+    default: return launch_tc_t<D, 1, 1, 2, MASKED, 2>(a, maps, stream);
   }
 }
 
-// Paired score products when a split fits in the ring whole (it is then
-// latency-bound: fewer, wider steps help); single tiles when it streams.
 template <int D, bool MASKED>
 cudaError_t launch_tc_d(const AttnArgs& a, const TmaMaps& maps, cudaStream_t stream) {
   if (a.R > 128) return launch_tc_t<D, 2, 1, 1, MASKED>(a, maps, stream);

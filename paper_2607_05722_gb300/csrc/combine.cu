@@ -1,11 +1,102 @@
 // Split-KV combine: merge per-split softmax-normalised partial outputs and
-// their log-sum-exps into the full attention result, one warp per output row
-// (b, h, i); the row arithmetic is merge_split_row (split_merge.cuh), which
-// the attention kernel's in-grid merge runs as well.
-#include "split_merge.cuh"
+// their log-sum-exps into the full attention result.
+//   m = max_s lse_s, c_s = exp(lse_s - m), out = sum_s c_s o_s / sum_s c_s,
+//   lse = m + ln sum_s c_s.
+// One warp per output row (b, h, i); each lane owns D/32 consecutive dims, so
+// every partial row is read as one coalesced 256/512-byte segment; lane j
+// holds the lse of splits j, j+32, ... Partials of splits without keys
+// (lse = -inf) are never read.
+#include "nld_internal.cuh"
 
 namespace nld {
 namespace {
+
+// Row `row` of R = B*Hq*bl rows (partial row order [B, Hq, bl]); o_part
+// [S, R, D], lse_part [S, R] (natural log). Warp-collective.
+template <int D>
+__device__ __forceinline__ void merge_split_row(const float* __restrict__ o_part, const float* __restrict__ lse_part,
+                                                int S, long R, long row, int Hq, int bl,
+                                                __nv_bfloat16* __restrict__ out, float* __restrict__ lse) {
+  constexpr int V = D / 32;  // dims per lane (2 or 4)
+  const int lane = threadIdx.x & 31;
+  const int i = static_cast<int>(row % bl);
+  const long bh = row / bl;
+  const int h = static_cast<int>(bh % Hq);
+  const long b = bh / Hq;
+
+  // One memory round trip per 32 splits: each lane loads its share of the
+  // partial rows at the same time as the lse values.
+  constexpr int kMaxPerLane = kMaxSplits / 32;
+  constexpr int kRound = 32;
+  const long split_stride = R * static_cast<long>(D);
+  const float* base = o_part + row * D + lane * V;
+  float ls[kMaxPerLane];
+#pragma unroll
+  for (int u = 0; u < kMaxPerLane; ++u) {
+    const int s = lane + 32 * u;
+    ls[u] = s < S ? __ldg(lse_part + static_cast<long>(s) * R + row) : -INFINITY;
+  }
+  float x[kRound][V];
+  auto load_round = [&](int s0) {
+#pragma unroll
+    for (int u = 0; u < kRound; ++u) {
+      const int s = s0 + u;
+      if (s < S) {
+        const float* op = base + s * split_stride;
+        if constexpr (V == 4) {
+          const float4 t = __ldg(reinterpret_cast<const float4*>(op));
+          x[u][0] = t.x; x[u][1] = t.y; x[u][2] = t.z; x[u][3] = t.w;
+        } else {
+          const float2 t = __ldg(reinterpret_cast<const float2*>(op));
+          x[u][0] = t.x; x[u][1] = t.y;
+        }
+      }
+    }
+  };
+  load_round(0);
+  float m = -INFINITY;
+#pragma unroll
+  for (int u = 0; u < kMaxPerLane; ++u) m = fmaxf(m, ls[u]);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
+
+  float acc[V];
+#pragma unroll
+  for (int v = 0; v < V; ++v) acc[v] = 0.f;
+  float csum = 0.f;
+  if (m != -INFINITY) {
+    const float m2 = m * kLog2e;
+    float w[kMaxPerLane];  // weight of split lane + 32u; 0 for empty splits
+#pragma unroll
+    for (int u = 0; u < kMaxPerLane; ++u) {
+      w[u] = ls[u] == -INFINITY ? 0.f : ex2(fmaf(ls[u], kLog2e, -m2));
+      csum += w[u];
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) csum += __shfl_xor_sync(0xffffffffu, csum, off);
+    for (int s0 = 0; s0 < S; s0 += kRound) {
+      if (s0 > 0) load_round(s0);
+      const int blk = s0 >> 5;  // warp-uniform
+      const float wsrc = blk == 0 ? w[0] : blk == 1 ? w[1] : blk == 2 ? w[2] : w[3];
+#pragma unroll
+      for (int u = 0; u < kRound; ++u) {
+        const float wu = __shfl_sync(0xffffffffu, wsrc, u);
+        if (s0 + u < S && wu > 0.f) {
+#pragma unroll
+          for (int v = 0; v < V; ++v) acc[v] = fmaf(wu, x[u][v], acc[v]);
+        }
+      }
+    }
+  }
+  const float inv = csum > 0.f ? 1.f / csum : 0.f;
+  __nv_bfloat16* orow = out + ((b * bl + i) * Hq + h) * D + lane * V;
+#pragma unroll
+  for (int v = 0; v < V; v += 2)
+    *reinterpret_cast<uint32_t*>(orow + v) = pack_bf16(acc[v] * inv, acc[v + 1] * inv);
+  if (lse != nullptr && lane == 0)
+    lse[(b * Hq + h) * bl + i] = csum > 0.f ? fmaf(lg2(csum), kLn2, m) : -INFINITY;
+}
+
 
 constexpr int kCombineWarps = 8;
 
@@ -18,7 +109,7 @@ __global__ void __launch_bounds__(kCombineWarps * 32)
   const long row = static_cast<long>(blockIdx.x) * kCombineWarps + (threadIdx.x >> 5);
   const long R = static_cast<long>(B) * Hq * bl;
   if (row >= R) return;
-  merge_split_row<D, false>(o_part, lse_part, S, R, row, Hq, bl, out, lse);
+  merge_split_row<D>(o_part, lse_part, S, R, row, Hq, bl, out, lse);
 }
 
 }  // namespace

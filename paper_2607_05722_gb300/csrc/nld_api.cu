@@ -58,7 +58,7 @@ nld_status_t check_params(const nld_attn_params_t* p, int block_len) {
       p->max_pages_per_seq < 1 || p->num_splits < 0 || p->softmax_scale < 0.f || !isfinite(p->softmax_scale))
     return NLD_ERR_INVALID_ARG;
   if (p->num_q_heads % p->num_kv_heads != 0) return NLD_ERR_INVALID_ARG;
-  if (p->flags & ~(NLD_ATTN_PREFIX_READY | NLD_ATTN_MERGE_IN_GRID | NLD_ATTN_NO_CLUSTER | NLD_ATTN_MERGE_NO_WAIT))
+  if (p->flags & ~(NLD_ATTN_PREFIX_READY | NLD_ATTN_NO_CLUSTER))
     return NLD_ERR_INVALID_ARG;
   if (block_len < 1 || block_len > nld::kMaxBlock) return NLD_ERR_INVALID_ARG;
   if (p->num_splits > nld::kMaxSplits) return NLD_ERR_INVALID_ARG;
@@ -172,20 +172,6 @@ nld_status_t plan_splits(const nld_attn_params_t* p, int block_len, SplitPlan* o
   plan_splits_for(
       p, block_len, sms, [&](int cs) { return static_cast<long long>(nld::tc_max_active_clusters(cs, p->head_dim, rows)); },
       out);
-  return NLD_OK;
-}
-
-// Whether nld_block_attn merges the plan's partials inside the attention
-// grid: asked for, partials to merge, no cluster, the caller wants the final
-// output, and every CTA (one per SM) fits in one wave.
-nld_status_t merge_in_grid_for(const nld_attn_params_t* p, const SplitPlan& plan, bool run_combine, bool* out) {
-  *out = false;
-  if (!(p->flags & NLD_ATTN_MERGE_IN_GRID) || plan.partials <= 1 || plan.csize != 1 || !run_combine) return NLD_OK;
-  int sms = 0;
-  const nld_status_t st = device_state(nullptr, &sms);
-  if (st != NLD_OK) return st;
-  const long long units = static_cast<long long>(p->batch) * p->num_kv_heads;
-  *out = units <= nld::kMaxMergeUnits && units * plan.splits <= sms;
   return NLD_OK;
 }
 
@@ -320,10 +306,7 @@ int nld_block_attn_kernels(const nld_attn_params_t* params, int block_len) {
   if (check_params(params, block_len) != NLD_OK) return -1;
   SplitPlan plan;
   if (plan_splits(params, block_len, &plan) != NLD_OK) return -1;
-  if (plan.partials <= 1) return 1;
-  bool in_grid = false;
-  if (merge_in_grid_for(params, plan, true, &in_grid) != NLD_OK) return -1;
-  return in_grid ? 1 : 2;
+  return plan.partials <= 1 ? 1 : 2;
 }
 
 size_t nld_block_attn_workspace_size(const nld_attn_params_t* params, int block_len) {
@@ -331,7 +314,7 @@ size_t nld_block_attn_workspace_size(const nld_attn_params_t* params, int block_
   SplitPlan plan;
   if (plan_splits(params, block_len, &plan) != NLD_OK) return static_cast<size_t>(-1);
   if (plan.partials == 1) return 0;
-  return nld::kMergeCtrBytes + align256(partial_o_bytes(params, block_len, plan.partials)) +
+  return align256(partial_o_bytes(params, block_len, plan.partials)) +
          partial_lse_bytes(params, block_len, plan.partials);
 }
 
@@ -358,7 +341,7 @@ nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_bloc
   size_t o_bytes = 0;
   if (plan.partials > 1) {
     o_bytes = align256(partial_o_bytes(params, block_len, plan.partials));
-    const size_t need = nld::kMergeCtrBytes + o_bytes + partial_lse_bytes(params, block_len, plan.partials);
+    const size_t need = o_bytes + partial_lse_bytes(params, block_len, plan.partials);
     if (workspace == nullptr || workspace_bytes < need) return NLD_ERR_WORKSPACE;
     if (!aligned(workspace, 16)) return NLD_ERR_INVALID_ARG;
   }
@@ -409,21 +392,14 @@ nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_bloc
                             ? 1
                             : 0;
   }
-  bool merge_in_grid = false;
   if (plan.partials > 1) {
-    char* ws = static_cast<char*>(workspace);
-    a.o_part = reinterpret_cast<float*>(ws + nld::kMergeCtrBytes);
-    a.lse_part = reinterpret_cast<float*>(ws + nld::kMergeCtrBytes + o_bytes);
-    if ((st = merge_in_grid_for(params, plan, run_combine, &merge_in_grid)) != NLD_OK) return st;
-    if (merge_in_grid) {
-      a.merge_ctr = reinterpret_cast<unsigned int*>(ws);
-      a.merge_wait_ns = (params->flags & NLD_ATTN_MERGE_NO_WAIT) ? 0 : nld::kMergeWaitNs;
-    }
+    a.o_part = static_cast<float*>(workspace);
+    a.lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) + o_bytes);
   }
   if ((st = encode_out_map(&maps.o, a, params->head_dim)) != NLD_OK) return st;
   if ((st = encode_block_map(&maps.q, q_block, a, params->head_dim)) != NLD_OK) return st;
   if (nld::launch_block_attn_tc(a, maps, params->head_dim, stream) != cudaSuccess) return NLD_ERR_CUDA;
-  if (plan.partials > 1 && run_combine && !merge_in_grid) {
+  if (plan.partials > 1 && run_combine) {
     if (nld::launch_combine(a.o_part, a.lse_part, plan.partials, a.B, a.Hq, block_len, params->head_dim, a.out, lse,
                             stream) != cudaSuccess)
       return NLD_ERR_CUDA;

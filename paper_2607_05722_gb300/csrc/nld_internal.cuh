@@ -21,13 +21,6 @@ constexpr int kMaxRows = 256;   // (Hq / Hkv) * block_len handled by one CTA (tw
 constexpr int kMaxBlock = 32;   // block_len and the decision width n
 constexpr int kTileTok = 64;    // KV tokens per pipeline stage
 constexpr int kGroupTok = 16;   // KV tokens per TMA box (never crosses a page: P % 16 == 0)
-// In-grid split merge: counters at the start of the workspace, 8 words per
-// (sequence, KV head) unit (arrivals, base, 4 words of give-up bits, one per
-// split, 2 unused), for up to kMaxMergeUnits units.
-constexpr int kMergeCtrWords = 8;
-constexpr int kMaxMergeUnits = 256;
-constexpr size_t kMergeCtrBytes = static_cast<size_t>(kMaxMergeUnits) * kMergeCtrWords * 4;
-constexpr uint64_t kMergeWaitNs = 50000;  // a CTA waits at most 50 us for the other splits of its unit (default)
 
 // Arguments of the block-attention kernel (one CTA per (split, kv head, sequence)).
 struct AttnArgs {
@@ -50,8 +43,6 @@ struct AttnArgs {
   int order_by_length;         // CTA z takes the sequence of rank z by prefix length (longest first)
   int csize;                   // thread-block cluster size along the splits (1 = no cluster)
   int num_partials;            // partials written per (b, h, i): num_splits / csize (1 = final output)
-  unsigned int* merge_ctr;     // in-grid split merge: unit counters (kMergeCtrWords each), or null
-  uint64_t merge_wait_ns;      // how long a CTA waits for the other splits of its unit
 };
 
 // Launchers (defined next to their kernels). Return a CUDA error code.
@@ -365,34 +356,6 @@ __device__ __forceinline__ void bulk_store(void* gdst, const void* ssrc, uint32_
                : "memory");
 }
 __device__ __forceinline__ void bulk_store_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
-// Wait until this thread's bulk stores have completed (their writes done,
-// not only their shared-memory reads).
-__device__ __forceinline__ void bulk_store_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
-// Order this thread's completed async-proxy (TMA) global writes before its
-// later generic-proxy operations, e.g. a release that publishes them.
-__device__ __forceinline__ void fence_proxy_async_global() {
-  asm volatile("fence.proxy.async.global;" ::: "memory");
-}
-// Loads, stores and atomics with explicit scope and ordering (GPU scope).
-__device__ __forceinline__ unsigned int ld_acquire_gpu(const unsigned int* p) {
-  unsigned int v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
-}
-__device__ __forceinline__ unsigned int ld_relaxed_gpu(const unsigned int* p) {
-  unsigned int v;
-  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
-}
-__device__ __forceinline__ void st_relaxed_gpu(unsigned int* p, unsigned int v) {
-  asm volatile("st.relaxed.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
-}
-__device__ __forceinline__ unsigned int atom_add_release_gpu(unsigned int* p, unsigned int v) {
-  unsigned int old;
-  asm volatile("atom.release.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
-  return old;
-}
-__device__ __forceinline__ void fence_sc_gpu() { asm volatile("fence.sc.gpu;" ::: "memory"); }
 
 // Tiled TMA stores shared -> global (one box at coordinates {c0, c1[, c2]},
 // the innermost coordinate a multiple of 16 bytes), in the issuing thread's

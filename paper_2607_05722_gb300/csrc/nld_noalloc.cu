@@ -15,11 +15,9 @@
 // device address is looked up once per device, on the first call made with
 // that device current (cudaGetSymbolAddress); make that first call before
 // any stream capture. Every call on a device shares the one array and it
-// keeps the previous call's contents. Its first 8 KB hold the counters of
-// the in-grid split merge, which must start at zero: the array is zero when
-// the library loads, and every completed call leaves the counters
-// consistent for the next; the partials after them are rewritten before
-// they are read. Two
+// keeps the previous call's contents; nothing in it needs to start at zero,
+// because the attention kernel writes every partial that the combine reads.
+// Two
 // calls whose kernels overlap on the GPU (different streams without an
 // ordering between them) race on the array.
 #include <mutex>

@@ -24,12 +24,8 @@ NLD_MODE_VERIFY = 1
 NLD_DEVERR_PREFIX_RANGE = 0x1
 NLD_DEVERR_PAGE_RANGE = 0x2
 NLD_DEVERR_WAIT_TIMEOUT = 0x4
-NLD_DEVERR_MERGE_STATE = 0x8
 NLD_ATTN_PREFIX_READY = 0x1
-NLD_ATTN_MERGE_IN_GRID = 0x2
 NLD_ATTN_NO_CLUSTER = 0x4
-NLD_ATTN_MERGE_NO_WAIT = 0x8
-MERGE_CTR_BYTES = 8192  # merge counters at the start of a split workspace
 
 HEADER = os.path.join(_build.INCLUDE, "nld.h")
 
@@ -185,7 +181,7 @@ def workspace_views(params: AttnParams, block_len: int, workspace):
         return None
     B, Hq, D = params.batch, params.num_q_heads, params.head_dim
     n_o = S * B * Hq * block_len * D
-    o0 = MERGE_CTR_BYTES
+    o0 = 0
     l0 = o0 + ((n_o * 4 + 255) // 256) * 256
     flat = workspace.view(torch.uint8)
     o_part = flat[o0:o0 + n_o * 4].view(torch.float32).view(S, B, Hq, block_len, D)
@@ -194,8 +190,7 @@ def workspace_views(params: AttnParams, block_len: int, workspace):
 
 
 def alloc_workspace(params: AttnParams, block_len: int, device="cuda"):
-    """A zeroed workspace for these parameters (None when the plan needs none):
-    the merge counters at its start must be zero before its first use."""
+    """A workspace for these parameters (None when the plan needs none)."""
     n = nld_block_attn_workspace_size(params, block_len)
     return torch.zeros(n, dtype=torch.uint8, device=device) if n else None
 

@@ -50,14 +50,12 @@ def test_split_plan_and_workspace_size(L):
     # 4112 tokens / 19 -> 217 -> 224 per split -> 19 splits
     S, B, Hq, bl, D = 19, 1, 32, 16, 128
     o = S * B * Hq * bl * D * 4
-    ctr = 8192  # merge counters first: 8 uint32 for each of up to 256 (sequence, KV head) units
-    assert nld.MERGE_CTR_BYTES == ctr
-    assert nld.nld_block_attn_workspace_size(p, 16) == ctr + ((o + 255) // 256) * 256 + S * B * Hq * bl * 4
+    assert nld.nld_block_attn_workspace_size(p, 16) == ((o + 255) // 256) * 256 + S * B * Hq * bl * 4
     assert nld.nld_block_attn_workspace_size(params(num_splits=1), 16) == 0
     # 16 pieces run as two clusters of 8 (tcgen05 kernel, 64 packed rows): 2 partials
     assert nld.nld_block_attn_num_splits(params(num_splits=16), 16) == 2
     assert nld.nld_block_attn_workspace_size(params(num_splits=16), 16) == \
-        ctr + ((2 * Hq * bl * D * 4 + 255) // 256) * 256 + 2 * Hq * bl * 4
+        ((2 * Hq * bl * D * 4 + 255) // 256) * 256 + 2 * Hq * bl * 4
     # without clusters every piece is a partial
     assert nld.nld_block_attn_num_splits(params(num_splits=16, flags=nld.NLD_ATTN_NO_CLUSTER), 16) == 16
     # 4 pieces (chunk >= 16 tokens of 64) merge in one cluster: final output, no workspace
@@ -78,7 +76,8 @@ def test_split_plan_and_workspace_size(L):
     (dict(), 33, 1),                        # block_len > 32
     (dict(num_q_heads=72, num_kv_heads=8), 32, 2),  # 9 * 32 = 288 packed rows > 256
     (dict(batch=0), 16, 1),
-    (dict(flags=16), 16, 1),                # unknown flag bit
+    (dict(flags=2), 16, 1),                 # unknown flag bit
+    (dict(flags=8), 16, 1),                 # unknown flag bit
 ])
 def test_block_attn_rejects_bad_shapes(L, kw, bl, code):
     p = params(**kw)
@@ -211,8 +210,7 @@ def test_plan_without_clusters(L):
 
 
 def test_flags_accepted(L):
-    for f in (nld.NLD_ATTN_PREFIX_READY, nld.NLD_ATTN_MERGE_IN_GRID, nld.NLD_ATTN_NO_CLUSTER,
-              nld.NLD_ATTN_MERGE_NO_WAIT, 15):
+    for f in (nld.NLD_ATTN_PREFIX_READY, nld.NLD_ATTN_NO_CLUSTER, 5):
         assert nld.nld_block_attn_workspace_size(params(flags=f), 16) > 0
 
 
