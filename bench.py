@@ -25,6 +25,7 @@ from __future__ import annotations
 import argparse
 import hashlib
 import json
+import platform
 import os
 import re
 import subprocess
@@ -259,10 +260,7 @@ def run_ours(args, world, rank, local):
     B, bl, Hq, Hkv, D = c.batch, c.block_len, c.num_q_heads, c.num_kv_heads, c.head_dim
     kv_bytes = c.kv_bytes_per_pass()
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size
-    npool = max(args.pools, 2)
-    if npool * kv_bytes < 3 * l2:
-        npool = int(np.ceil(3 * l2 / kv_bytes)) + 1
-    npool += npool % 2
+    npool = pool_count(kv_bytes, l2, args.pools)
 
     def dev_bf16(bits):
         return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(dev)
@@ -439,18 +437,7 @@ def run_ours(args, world, rank, local):
         "vs_baseline": None,
         "dtype": "bf16",
         "data": "synthetic",
-        "config": {
-            "workload": WORKLOAD,
-            "batch_per_gpu": B, "q_heads": Hq, "kv_heads": Hkv, "head_dim": D, "prefix": int(kv.prefix_lens[0]),
-            "block_len": bl, "page_size": c.page_size, "page_order": "random permutation",
-            "kv_partials": splits, "attn_kernels_per_pass": attn_kernels,
-            "split_merge": "combine kernel" if attn_kernels == 2 else "none (one partial per row)",
-            "unmask_k": k_unmask, "prefix_ready_flag": not args.no_prefix_ready,
-            "step": "diffusion attention + unmask + verify attention + accept (one attention layer)",
-            "l2": f"cold: each pass reads its own KV pool from a rotation of {npool} pools "
-                  f"({npool * kv_bytes / 2**20:.0f} MiB > 3x L2 {l2 / 2**20:.0f} MiB)",
-            "timing": "CUDA graph of the steps, CUDA events on the launching stream",
-        },
+        "config": headline_config(wl, npool, l2, splits, attn_kernels, not args.no_prefix_ready),
         "steps_per_s": round(1e3 / ms_step, 1) * world,
         "pct_of_hbm_peak": round(100.0 * value / world / peak, 2),
         "clocks": clocks,
@@ -846,6 +833,51 @@ def run_workloads(torch, nld, dev, stream, peak, l2, only=None, batch=None, swee
 # CPU oracle timings
 # ---------------------------------------------------------------------------
 
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu, else /proc/cpuinfo), for the baseline records."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.split(":")[0].strip() in ("Model name", "Model"):
+                name = line.split(":", 1)[1].strip()
+                if name and not name.isdigit():
+                    return name
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith(("model name", "cpu model", "hardware")):
+                return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return platform.machine()
+
+
+def headline_config(wl, npool, l2, splits, attn_kernels, prefix_ready):
+    """The config dict of the headline workload, shared by both arms."""
+    c = wl.attn
+    kv_bytes = c.kv_bytes_per_pass()
+    return {
+        "workload": WORKLOAD,
+        "batch_per_gpu": c.batch, "q_heads": c.num_q_heads, "kv_heads": c.num_kv_heads, "head_dim": c.head_dim,
+        "prefix": int(c.kv.prefix_lens[0]), "block_len": c.block_len, "page_size": c.page_size,
+        "page_order": "random permutation", "kv_partials": splits, "attn_kernels_per_pass": attn_kernels,
+        "split_merge": "combine kernel" if attn_kernels == 2 else "none (one partial per row)",
+        "unmask_k": wl.unmask_k[0], "prefix_ready_flag": prefix_ready,
+        "step": "diffusion attention + unmask + verify attention + accept (one attention layer)",
+        "l2": f"cold: each pass reads its own KV pool from a rotation of {npool} pools "
+              f"({npool * kv_bytes / 2**20:.0f} MiB > 3x L2 {l2 / 2**20:.0f} MiB)",
+        "timing": "CUDA graph of the steps, CUDA events on the launching stream",
+    }
+
+
+def pool_count(kv_bytes, l2, pools_arg):
+    npool = max(pools_arg, 2)
+    if npool * kv_bytes < 3 * l2:
+        npool = int(np.ceil(3 * l2 / kv_bytes)) + 1
+    return npool + npool % 2
+
+
 def oracle_step(orc, wl, rows=None):
     """One draft+verify step on the oracle: both passes (all rows, or the
     given (b, i, h) rows), unmask and accept."""
@@ -876,9 +908,34 @@ def cpu_baseline(wl, budget_s: float):
             break
     dt = time.perf_counter() - t0
     return {"value": round(2 * kv_bytes * n / dt / 1e9, 4), "unit": "GB/s", "cores": orc.max_threads(),
-            "kind": "oracle", "steps_per_s": round(n / dt, 3),
+            "cpu_model": cpu_model(), "kind": "oracle", "steps_per_s": round(n / dt, 3),
             "sample": f"{n} full draft+verify steps (every row of both passes, unmask, accept) of {WORKLOAD}, "
                       f"fp64, OpenMP over (sequence, query head)"}
+
+
+def reference_config(args, wl):
+    """The GPU arm's config dict for the same workload: the split plan from
+    the host-only plan query for this machine's GPU (no device work), the pool
+    rotation from its L2 size."""
+    from paper_2607_05722_gb300 import build as nld_build
+    from paper_2607_05722_gb300 import nld
+    nld_build.build()  # the host-only plan query lives in the library (no kernel runs)
+    c = wl.attn
+    sms, l2 = 152, 129 << 20
+    try:
+        import torch
+        if torch.cuda.is_available():
+            prop = torch.cuda.get_device_properties(0)
+            sms, l2 = prop.multi_processor_count, prop.L2_cache_size
+    except Exception:  # noqa: BLE001 - the plan falls back to the GB300 figures
+        pass
+    prefix_ready = not args.no_prefix_ready
+    params = nld.make_params(c.batch, c.num_q_heads, c.num_kv_heads, c.head_dim, c.page_size, c.kv.num_pages,
+                             c.kv.max_pages, args.splits, 0.0, nld.NLD_ATTN_PREFIX_READY if prefix_ready else 0)
+    plan = nld.nld_block_attn_plan(params, c.block_len, sms)
+    kernels = 2 if plan["partials"] > 1 else 1
+    npool = pool_count(c.kv_bytes_per_pass(), l2, args.pools)
+    return headline_config(wl, npool, l2, plan["partials"], kernels, prefix_ready)
 
 
 def run_reference(args, world, rank):
@@ -916,11 +973,9 @@ def run_reference(args, world, rank):
         "metric": METRIC, "value": round(value, 4), "unit": "GB/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3 / frac, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
-        "config": {"workload": WORKLOAD, "batch_per_gpu": c.batch, "q_heads": c.num_q_heads,
-                   "kv_heads": c.num_kv_heads, "head_dim": c.head_dim, "prefix": int(c.kv.prefix_lens[0]),
-                   "block_len": c.block_len, "page_size": c.page_size},
-        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": orc.max_threads(), "kind": "oracle",
-                         "sample": desc},
+        "config": reference_config(args, wl),
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": orc.max_threads(),
+                         "cpu_model": cpu_model(), "kind": "oracle", "sample": desc},
         "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
