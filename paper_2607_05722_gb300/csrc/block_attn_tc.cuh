@@ -9,8 +9,10 @@
 // Warp roles (5 + 4*MT warps):
 //   warps 0-2 and the last  TMA producers: the boxes of each 64-token K/V tile
 //             (16 tokens x 64 dims each) dealt four ways into a ring of up to
-//             8 stages (produce_kv); TMA issue cost is per warp, so four
-//             issuing warps land a tile sooner.
+//             8 stages (produce_kv), warps 0-1 the K boxes, the others the V
+//             boxes, each kind with its own full/empty barriers so that a K
+//             slot refills once its score product is done; TMA issue cost is
+//             per warp, so four issuing warps land a tile sooner.
 //   warp 3    allocates the TMEM columns; lane 0 loads Q by TMA (one M tile)
 //             and issues every MMA:
 //               S_j = Q K^T     (M=128 rows, N=64*TPS tokens, K=D; double-buffered in TMEM)
@@ -112,8 +114,9 @@ struct TcLayout {
   static constexpr int kQOff = kStages * Geo::kStageBytes;
   static constexpr int kPOff = kQOff + MT * kQBytes;  // end of the ring and Q tiles
   static constexpr int kBarOff = kPOff;
-  // kv_full[st], kv_empty[st], s_full[2], s_free[2], p_full[kPBufs], o_done[kPBufs], q_ready, q_full, drain, tmem slot
-  static constexpr int kNumBars = 2 * kStages + 4 + 2 * kPBufs + 3;
+  // k_full[st], v_full[st], k_empty[st], v_empty[st], s_full[2], s_free[2], p_full[kPBufs], o_done[kPBufs],
+  // q_ready, q_full, drain, o_fin, tmem slot
+  static constexpr int kNumBars = 4 * kStages + 4 + 2 * kPBufs + 4;
   static constexpr int kBytes = kBarOff + kNumBars * 8 + 16;
   static_assert(kNumBars * 8 + 16 <= 512, "barrier reserve");
   static_assert(kBytes + 1024 <= 232448, "shared memory per CTA");
@@ -163,25 +166,38 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* q_s = smem + Lay::kQOff;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Lay::kBarOff);
-  uint64_t* kv_full = bars;
-  uint64_t* kv_empty = bars + kTcStages;
-  uint64_t* s_full = bars + 2 * kTcStages;
+  uint64_t* k_full = bars;                   // K slot of stage st landed
+  uint64_t* v_full = bars + kTcStages;       // V slot of stage st landed
+  uint64_t* k_empty = bars + 2 * kTcStages;  // the score product that read K of stage st completed
+  uint64_t* v_empty = bars + 3 * kTcStages;  // the PV product that read V of stage st completed
+  uint64_t* s_full = bars + 4 * kTcStages;
   uint64_t* s_free = s_full + 2;
   uint64_t* p_full = s_free + 2;
   uint64_t* o_done = p_full + Cfg::kPBufs;
   uint64_t* q_ready = o_done + Cfg::kPBufs;
   uint64_t* q_full = q_ready + 1;  // the Q tiles' TMA copies (one M tile)
   uint64_t* drain = q_full + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  // o_fin: every PV product has completed (committed once, after the last):
+  // a warp that ends its steps early (the group without the last tile) may
+  // be more than one phase behind on an o_done slot, so it never waits on
+  // one for the end of the split.
+  uint64_t* o_fin = drain + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_fin + 1);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int split = blockIdx.x, g = blockIdx.y;
+  // Block-slot chunks (a.nh = 2 for 129..256 packed rows): the two CTAs of
+  // a (split, KV head, sequence) are adjacent along x and hold block slots
+  // [hc*bl_c, (hc+1)*bl_c) of the G heads each, R = G*bl_c rows.
+  const int split = static_cast<int>(blockIdx.x) / a.nh, g = blockIdx.y;
+  const int slot0 = (static_cast<int>(blockIdx.x) - split * a.nh) * a.bl_c;  // first block slot of this CTA
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kTcStages; ++s) {
-      mbar_init(&kv_full[s], kProducers);  // one expect_tx arrival per producer warp
-      mbar_init(&kv_empty[s], 1);
+      mbar_init(&k_full[s], kProducers / 2);  // one expect_tx arrival per producer warp of the kind
+      mbar_init(&v_full[s], kProducers / 2);
+      mbar_init(&k_empty[s], 1);
+      mbar_init(&v_empty[s], 1);
     }
     for (int j = 0; j < 2; ++j) {
       mbar_init(&s_full[j], 1);
@@ -194,6 +210,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
     mbar_init(q_ready, Cfg::kSmWarps);
     mbar_init(q_full, 1);
     mbar_init(drain, 1);
+    mbar_init(o_fin, 1);
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
@@ -256,7 +273,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
       for (int r = threadIdx.x; r < Lay::kMergeRows; r += blockDim.x) lse_stage[r] = -INFINITY;
     } else {
       for (int r = threadIdx.x; r < a.R; r += blockDim.x) {
-        const int i = r / a.G, h = g * a.G + (r - i * a.G);
+        const int i = slot0 + r / a.G, h = g * a.G + (r - (r / a.G) * a.G);
         a.lse_part[((static_cast<size_t>(split) * a.B + b) * a.Hq + h) * a.bl + i] = -INFINITY;
       }
     }
@@ -269,13 +286,15 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
         ++early_tiles;
       if (early_tiles == 0) grid_dependency_wait();
     }
-    const int issued = produce_kv<D>(a, &maps.k, &maps.v, smem, kv_full, kv_empty, kTcStages, g, b, t_begin, t_end,
-                                     ntiles, lane, producer_index<MT, CG>(warp), kProducers, first, early_tiles);
+    const int pw = producer_index<MT, CG>(warp);
+    const int issued = produce_kv<D>(a, &maps.k, &maps.v, smem, k_full, v_full, k_empty, v_empty, kTcStages, g, b,
+                                     t_begin, t_end, ntiles, lane, pw, kProducers, first, early_tiles);
     if (lane == 0 && issued < ntiles) {
       // Stopped early on a wait timeout: let the copies already issued land
       // before the CTA exits (bounded).
+      uint64_t* full = pw >= kProducers / 2 ? v_full : k_full;
       for (int k = max(0, issued - kTcStages); k < issued; ++k)
-        mbar_wait(&kv_full[k % kTcStages], (k / kTcStages) & 1, a.err);
+        mbar_wait(&full[k % kTcStages], (k / kTcStages) & 1, a.err);
     }
   } else if (warp == kMmaWarp) {
     // ---------------- MMA issuer ----------------
@@ -291,7 +310,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
 #pragma unroll
           for (int cb = 0; cb < D / 64; ++cb)
             tma_load_3d(q_s + cb * (128 * 128) + q * (128 / REP) * 128, &maps.q, q_full, cb * 64, g * a.G,
-                        b * a.bl);
+                        b * a.bl + slot0);
       }
       bool ok = mbar_wait(q_ready, 0, a.err);
       if constexpr (MT == 1) ok = ok && mbar_wait(q_full, 0, a.err);
@@ -319,17 +338,26 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
           }
         }
         umma_commit(&s_full[j & 1]);
+        // The K slots of this product are free once it completes (a last
+        // product with one tile frees only that tile's slot).
+        umma_commit(&k_empty[st]);
+        if (kTPS == 2 && j * kTPS + 1 < ntiles) umma_commit(&k_empty[(st + 1) % kTcStages]);
       };
+      // P of tile h of a product starts at S column h*32 (one warp reads the
+      // whole product's columns before writing), or with two softmax groups,
+      // which share the TMEM lanes and read their tiles independently, at
+      // h*64: inside the columns of its own tile.
+      constexpr int kPCols = CG == 2 ? kTileTok : kTileTok / 2;
       auto issue_pv = [&](int k) {
         const int st = k % kTcStages;
         const uint32_t v_addr = smem_u32(smem + Lay::kVOff + st * Geo::kTileBytes);
 #pragma unroll
         for (int mt = 0; mt < MT; ++mt) {
-          // A = P in TMEM (bf16 pairs over the S columns of the tile's first
-          // half: 32 columns per 64-token tile); B = V (MN-major: 64-dim
+          // A = P in TMEM (bf16 pairs, 32 columns per 64-token tile, over S
+          // columns its tile's softmax has consumed); B = V (MN-major: 64-dim
           // atoms LBO apart, 8-token row groups SBO apart). With two softmax
           // groups tile k accumulates into O of group k % 2.
-          const uint32_t p_tmem = tS(mt, (k / kTPS) & 1) + static_cast<uint32_t>((k % kTPS) * 32);
+          const uint32_t p_tmem = tS(mt, (k / kTPS) & 1) + static_cast<uint32_t>((k % kTPS) * kPCols);
           const uint32_t o_acc = tO(CG == 2 ? k % CG : mt);
 #pragma unroll
           for (int kt = 0; kt < kTileTok / 16; ++kt) {
@@ -338,11 +366,13 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
           }
         }
         umma_commit(&o_done[k % kPBufs]);
-        umma_commit(&kv_empty[st]);
+        umma_commit(&v_empty[st]);
+        if (k == ntiles - 1) umma_commit(o_fin);
       };
       // Event-driven issue: score product j needs its K tiles and a free S
       // buffer (the softmax warps have read product j-2), and waits until
-      // the PV products of product j-2 are issued; PV_k needs P_k. Whichever
+      // the PV products of product j-2 are issued; PV_k needs P_k and the V
+      // tile of stage k. Whichever
       // is ready goes first, so a late K/V tile never holds back a ready PV.
       // (Letting scores run further ahead measured slower: they queue in
       // front of the PV products on the tensor core.)
@@ -356,14 +386,15 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
         bool progressed = false;
         const int t0 = next_s * kTPS;  // first tile of the next score product
         if (next_s < nprod && t0 - kTPS <= next_pv &&
-            mbar_test(&kv_full[t0 % kTcStages], (t0 / kTcStages) & 1) &&
-            (kTPS == 1 || t0 + 1 >= ntiles || mbar_test(&kv_full[(t0 + 1) % kTcStages], ((t0 + 1) / kTcStages) & 1)) &&
+            mbar_test(&k_full[t0 % kTcStages], (t0 / kTcStages) & 1) &&
+            (kTPS == 1 || t0 + 1 >= ntiles || mbar_test(&k_full[(t0 + 1) % kTcStages], ((t0 + 1) / kTcStages) & 1)) &&
             (next_s < 2 || mbar_test(&s_free[next_s & 1], ((next_s - 2) >> 1) & 1))) {
           tc_fence_after();
           issue_s(next_s++);
           progressed = true;
         }
-        if (next_pv < next_s * kTPS && mbar_test(&p_full[next_pv % kPBufs], (next_pv / kPBufs) & 1)) {
+        if (next_pv < next_s * kTPS && mbar_test(&p_full[next_pv % kPBufs], (next_pv / kPBufs) & 1) &&
+            mbar_test(&v_full[next_pv % kTcStages], (next_pv / kTcStages) & 1)) {
           tc_fence_after();
           issue_pv(next_pv++);
           progressed = true;
@@ -415,8 +446,8 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     const bool warp_rows = mt * 128 + rq * 32 < a.R;  // warp-uniform: the warp holds a real row
     const bool row_ok = r < a.R;
-    const int row_i = r / a.G;
-    const int row_h = g * a.G + (r - row_i * a.G);
+    const int row_i = slot0 + r / a.G;                    // block slot of this row
+    const int row_h = g * a.G + (r - (r / a.G) * a.G);
     const int sm_tid = threadIdx.x - 32 * kSoftmaxWarp0;  // 0 .. 32*kSmWarps-1 across the softmax warps
     const int grp_tid = sm_tid - cg * 128 * MT;           // 0 .. 128*MT-1 within this softmax group
     const int swz = r_loc & 7;                      // 128-byte swizzle phase of this tile row
@@ -568,17 +599,20 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
       }
       if (warp_rows) {
         // P goes to TMEM over the consumed S columns: tile k of the product
-        // takes columns (k % TPS) * 32 .. +31 of its S buffer, bf16 pairs.
-        // This thread writes its slice of the tile k_own and zeros over the
-        // rest of the step's tiles (other copies' slices).
+        // takes columns (k % TPS) * 32 .. +31 of its S buffer, bf16 pairs
+        // (with two softmax groups (k % TPS) * 64 .. +31: its own tile's
+        // columns, which the other group never reads). This thread writes
+        // its slice of the tile k_own and zeros over the rest of the step's
+        // tiles (other copies' slices).
         const uint32_t tbuf = tS(mt, j & 1) + lane_off;
+        constexpr int kPColsS = CG == 2 ? kTileTok : kTileTok / 2;
         if (k_own < ntiles) {
           // p = 2^(s * scale * log2(e) - m): per pair of elements one paired
           // FMA, two exponentials, one bf16 pack and one paired add.
           const float nmu = m_run == -INFINITY ? 0.f : -m_run;
           const float2 sc2 = make_float2(scl, scl), nm2 = make_float2(nmu, nmu);
           float2 ls[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-          const uint32_t tp = tbuf + static_cast<uint32_t>((k_own % kTPS) * 32);
+          const uint32_t tp = tbuf + static_cast<uint32_t>((k_own % kTPS) * kPColsS);
 #pragma unroll
           for (int c = 0; c < kColsU / 16; ++c) {  // 16 columns (8 TMEM columns) per store
             uint32_t w[8];
@@ -619,7 +653,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
           // stale or uninitialised data; P is 0 there but 0 * NaN = NaN, so
           // zero those V rows before the PV MMA reads them.
           const int st = k % kTcStages;
-          if (!warp_wait(&kv_full[st], (k / kTcStages) & 1)) {
+          if (!warp_wait(&v_full[st], (k / kTcStages) & 1)) {
             step_ok = false;
             break;
           }
@@ -642,12 +676,10 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
     }
 
     // ---------------- epilogue ----------------
-    // Every PV has completed once o_done of the last tile fires, so the K/V
-    // ring is free for staging.
-    // Warp-uniform, like every condition around the warp-collective TMEM
-    // loads and stores below.
-    const bool o_ready =
-        __all_sync(0xffffffffu, ok && mbar_wait(&o_done[(ntiles - 1) % kPBufs], ((ntiles - 1) / kPBufs) & 1, a.err));
+    // Every PV has completed once o_fin fires, so the K/V ring is free for
+    // staging. Warp-uniform, like every condition around the warp-collective
+    // TMEM loads and stores below.
+    const bool o_ready = __all_sync(0xffffffffu, ok && mbar_wait(o_fin, 0, a.err));
     // Copies of a row (REP > 1) hold its O over disjoint token slices, merged
     // by the split-combine rule (Sec. 3 Mode 2, here on one SM). The work is
     // split by columns: copy c finalises output columns [c*kRange,
@@ -871,11 +903,11 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
           if (split_out) {
 #pragma unroll
             for (int x = sr * (D / 32 / kStoreRounds); x < (sr + 1) * (D / 32 / kStoreRounds); ++x)
-              tma_store_4d(&maps.o, smem + x * box_stride, x * 32, g * a.G, 0, split * a.B + b);
+              tma_store_4d(&maps.o, smem + x * box_stride, x * 32, g * a.G, slot0, split * a.B + b);
           } else {
 #pragma unroll
             for (int x = sr * (D / 64 / kStoreRounds); x < (sr + 1) * (D / 64 / kStoreRounds); ++x)
-              tma_store_3d(&maps.o, smem + x * box_stride, x * 64, g * a.G, b * a.bl);
+              tma_store_3d(&maps.o, smem + x * box_stride, x * 64, g * a.G, b * a.bl + slot0);
           }
           bulk_commit();
         }
@@ -1013,7 +1045,7 @@ cudaError_t launch_tc_o(const AttnArgs& a, const TmaMaps& maps, cudaStream_t str
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if ((e = configure_tc<D, MT, REP, TPS, MASKED, ORDERED, CG>(dev)) != cudaSuccess) return e;
-  dim3 grid(a.num_splits, a.Hkv, a.B);
+  dim3 grid(a.num_splits * a.nh, a.Hkv, a.B);
   return launch_kernel_cluster(block_attn_tc_kernel<D, MT, REP, TPS, MASKED, ORDERED, CG>, grid,
                                dim3(TcCfg<MT, TPS, CG>::kThreads), TcLayout<D, MT, TPS>::kBytes + 1024, stream,
                                a.csize, maps, a);

@@ -91,7 +91,15 @@ struct SplitPlan {
   int chunk;     // tokens per split
   int csize;     // cluster size (1 = none)
   int partials;  // splits / csize
+  int nh;        // block-slot chunks: CTAs per (split, sequence, KV head) (1 or 2)
 };
+
+// 129..256 packed rows with an even block length run as two CTAs per
+// (split, sequence, KV head), each with half of the block slots (at most 128
+// rows: one M tile); the pair streams the same K/V tiles at the same time,
+// so the second read is served by L2. An odd block length keeps one CTA with
+// two M tiles.
+int slot_chunks(int rows, int block_len) { return rows > 128 && block_len % 2 == 0 ? 2 : 1; }
 
 // Longest split that still runs paired score products at both head sizes
 // (the ring holds at least 6 tiles at head_dim 128).
@@ -103,9 +111,11 @@ template <typename ClustersResident>
 void plan_splits_for(const nld_attn_params_t* p, int block_len, int sms, ClustersResident clusters_resident,
                      SplitPlan* out) {
   const long long max_tokens = static_cast<long long>(p->max_pages_per_seq) * p->page_size;
-  const long long units = static_cast<long long>(p->batch) * p->num_kv_heads;
-  const bool tc = nld::tc_supports((p->num_q_heads / p->num_kv_heads) * block_len, p->head_dim);
-  const bool clusters = tc && !(p->flags & NLD_ATTN_NO_CLUSTER);
+  const int rows = (p->num_q_heads / p->num_kv_heads) * block_len;
+  const int nh = slot_chunks(rows, block_len);
+  const long long units = static_cast<long long>(p->batch) * p->num_kv_heads * nh;  // CTAs per split
+  const bool tc = nld::tc_supports(rows, p->head_dim);
+  const bool clusters = tc && nh == 1 && !(p->flags & NLD_ATTN_NO_CLUSTER);
   const bool automatic = p->num_splits == 0;
   int want = p->num_splits;
   int csize = 1;
@@ -160,6 +170,7 @@ void plan_splits_for(const nld_attn_params_t* p, int block_len, int sms, Cluster
   out->splits = static_cast<int>(splits);
   out->csize = csize;
   out->partials = static_cast<int>(splits / csize);
+  out->nh = nh;
 }
 
 nld_status_t plan_splits(const nld_attn_params_t* p, int block_len, SplitPlan* out) {
@@ -228,7 +239,7 @@ nld_status_t encode_block_map(CUtensorMap* map, const void* base, const nld::Att
   cuuint32_t estr[3] = {1, 1, 1};
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(a.Hq), static_cast<cuuint64_t>(a.B) * a.bl};
   cuuint64_t strides[2] = {static_cast<cuuint64_t>(D) * 2, static_cast<cuuint64_t>(D) * 2 * a.Hq};
-  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(a.G), static_cast<cuuint32_t>(a.bl)};
+  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(a.G), static_cast<cuuint32_t>(a.bl_c)};
   CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -251,7 +262,7 @@ nld_status_t encode_out_map(CUtensorMap* map, const nld::AttnArgs& a, int D) {
   cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(a.Hq), static_cast<cuuint64_t>(a.bl),
                         static_cast<cuuint64_t>(units)};
   cuuint64_t strides[3] = {row * a.bl, row, row * a.bl * a.Hq};
-  cuuint32_t box[4] = {32, static_cast<cuuint32_t>(a.G), static_cast<cuuint32_t>(a.bl), 1};
+  cuuint32_t box[4] = {32, static_cast<cuuint32_t>(a.G), static_cast<cuuint32_t>(a.bl_c), 1};
   CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, a.o_part, dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -369,7 +380,9 @@ nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_bloc
   a.Hkv = params->num_kv_heads;
   a.G = G;
   a.bl = block_len;
-  a.R = G * block_len;
+  a.nh = plan.nh;
+  a.bl_c = block_len / plan.nh;
+  a.R = G * a.bl_c;
   a.page_size = params->page_size;
   a.log2_page = __builtin_ctz(static_cast<unsigned>(params->page_size));
   a.num_pages = params->num_pages;
@@ -388,7 +401,7 @@ nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_bloc
     int sms = 0;
     if ((st = device_state(nullptr, &sms)) != NLD_OK) return st;
     a.order_by_length = (plan.splits == 1 && plan.csize == 1 && a.B > 1 && a.B <= 1024 &&
-                         static_cast<long long>(a.B) * a.Hkv > sms)
+                         static_cast<long long>(a.B) * a.Hkv * a.nh > sms)
                             ? 1
                             : 0;
   }

@@ -33,7 +33,8 @@ struct AttnArgs {
   float* lse_part;             // [S, B, Hq, bl]
   unsigned int* err;           // device error word
   unsigned long long* rescales;  // running-max rescale events (diagnostic counter)
-  int B, Hq, Hkv, G, bl, R;    // R = G * bl query rows per CTA
+  int B, Hq, Hkv, G, bl, R;    // R = G * bl_c query rows per CTA
+  int nh, bl_c;                // block-slot chunks per (split, KV head, sequence) (1 or 2), slots per chunk
   int page_size, log2_page, num_pages, max_pages;
   int num_splits, chunk;       // splits and tokens per split (multiple of 16)
   int mode;                    // NLD_MODE_DIFFUSION, NLD_MODE_VERIFY or kModeBlockMask
@@ -576,19 +577,28 @@ struct PagePrefetch {
 // consecutive stages is contiguous per column block, then V tiles at
 // [stage][column block]. A tile has 4 groups x D/64 column blocks x {K, V} boxes
 // (16 tokens x 64 dims each); they are dealt to the producer warps in equal
-// shares and, within a warp, one box per lane. TMA issue cost is per warp, so
-// more producer warps land a tile sooner. A warp's expect_tx covers only its
-// own boxes, so `full` expects one arrival per producer warp. `first` holds
-// the page ids of the first 32 groups, already loaded. Returns tiles issued.
+// shares and, within a warp, one box per lane: the first half of the warps
+// load K, the second half V. K and V slots fill and free on their own
+// barriers (k_full/v_full, k_empty/v_empty), so a K slot is refilled as soon
+// as the score product that read it has completed, before the PV product
+// frees the V slot of the same tile. TMA issue cost is per warp, so more
+// producer warps land a tile sooner. A warp's expect_tx covers only its own
+// boxes, so a full barrier expects one arrival per warp of its kind. `first`
+// holds the page ids of the first 32 groups, already loaded. Returns tiles
+// issued.
 template <int D>
 __device__ __forceinline__ int produce_kv(const AttnArgs& a, const CUtensorMap* tmk, const CUtensorMap* tmv,
-                                          uint8_t* stages, uint64_t* full, uint64_t* empty, int nstage, int g,
-                                          int b, int t_begin, int t_end, int ntiles, int lane, int pw, int nprod,
-                                          const PagePrefetch& first, int early_tiles) {
+                                          uint8_t* stages, uint64_t* k_full, uint64_t* v_full, uint64_t* k_empty,
+                                          uint64_t* v_empty, int nstage, int g, int b, int t_begin, int t_end,
+                                          int ntiles, int lane, int pw, int nprod, const PagePrefetch& first,
+                                          int early_tiles) {
   using Geo = TileGeom<D>;
   constexpr int kGroups = kTileTok / kGroupTok;
   constexpr int kOpsPerTile = kGroups * 2 * Geo::kColBlocks;  // 16 (D=128) or 8 (D=64)
-  const int my_ops = kOpsPerTile / nprod;                     // nprod divides kOpsPerTile
+  const int my_ops = kOpsPerTile / nprod;                     // nprod divides kOpsPerTile (and its halves)
+  const bool warp_v = pw >= nprod / 2;                        // this warp's boxes are all V (else all K)
+  uint64_t* full = warp_v ? v_full : k_full;
+  uint64_t* empty = warp_v ? v_empty : k_empty;
   const uint32_t bytes = static_cast<uint32_t>(my_ops) * kGroupTok * 128;
   int page_cur = first.validate(a, t_begin, t_end, 0, lane);
   PagePrefetch nxt;

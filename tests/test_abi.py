@@ -61,8 +61,12 @@ def test_split_plan_and_workspace_size(L):
     # 4 pieces (chunk >= 16 tokens of 64) merge in one cluster: final output, no workspace
     assert nld.nld_block_attn_num_splits(params(num_splits=64, max_pages_per_seq=4), 8) == 1
     assert nld.nld_block_attn_workspace_size(params(num_splits=8), 16) == 0
-    # 160 packed rows use two M tiles of the tcgen05 kernel: 8 pieces merge in one cluster
-    assert nld.nld_block_attn_num_splits(params(num_q_heads=40, num_splits=8), 32) == 1
+    # 160 packed rows with an even block length: two CTAs per split (16 block
+    # slots each), no clusters, so 8 pieces leave 8 partials; with an odd
+    # block length (5 x 31 = 155 rows) one CTA with two M tiles, and 8 pieces
+    # merge in one cluster
+    assert nld.nld_block_attn_num_splits(params(num_q_heads=40, num_splits=8), 32) == 8
+    assert nld.nld_block_attn_num_splits(params(num_q_heads=40, num_splits=8), 31) == 1
 
 
 @pytest.mark.parametrize("kw,bl,code", [

@@ -509,6 +509,15 @@ SMALL = [
     ("d128_g6_bl30_180rows", 1, 6, 1, 128, 32, 30, [260]),
     ("d64_g5_bl32_160rows", 2, 10, 2, 64, 16, 32, [300, 45]),
     ("d64_g8_bl32_256rows", 1, 16, 2, 64, 16, 32, [100]),
+    # two softmax groups over an odd number of tiles longer than the ring
+    # (one split: 15 and 17 tiles): the group without the last tile reaches
+    # the epilogue early and must wait for every PV product
+    ("d128_g3_bl32_96rows_15tiles", 1, 6, 2, 128, 16, 32, [900]),
+    ("d128_g4_bl32_128rows_17tiles", 1, 8, 2, 128, 16, 32, [1060]),
+    # more than 128 rows with an odd block length: one CTA with two M tiles
+    # (an even block length splits the slots over two CTAs instead)
+    ("d128_g5_bl29_145rows", 1, 10, 2, 128, 16, 29, [300]),
+    ("d64_g8_bl31_248rows", 2, 16, 2, 64, 16, 31, [100, 37]),
 ]
 
 
