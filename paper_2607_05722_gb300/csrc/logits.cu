@@ -4,7 +4,10 @@
 //   m = max_v l_v, id = the lowest v with l_v = m,
 //   conf = max_v softmax(l)_v = 1 / sum_v exp(l_v - m).
 // A row is cut into `split` pieces, one CTA each (a thread-block cluster when
-// split > 1). In a CTA one producer warp streams the piece through a ring of
+// split > 1). Pieces of at most 2048 vectors (a few rows over many SMs, as
+// in a decode step) take logits_argmax_small_kernel: every thread loads its
+// vectors at once and folds them in one pass. Larger pieces stream: in a CTA
+// one producer warp streams the piece through a ring of
 // 16 KB stages with bulk copies (TMA engine) and eight warps fold each 8-logit
 // vector into a running (max, sum of exp(l - max), argmax): the vector max
 // comes first, so the rare rescale happens once per vector, then one exp per
@@ -207,6 +210,182 @@ __global__ void __launch_bounds__(kLgThreads)
       }
     }
     cluster_sync();
+  }
+}
+
+// Small pieces (at most kLsThreads * kLsMaxVecs 8-logit vectors per CTA: a
+// few rows over many SMs, the decode-step case): no ring. Every thread loads
+// all its vectors at once (one memory round trip), folds them in one pass
+// (the max of its logits first, then one exp per logit against it), and
+// the CTA merges the threads' states; the pieces of a row then push their
+// states into rank 0's shared memory with a remote store and a release
+// arrival on rank 0's mbarrier, and rank 0 merges them, so no peer waits
+// for another. Same rules as logits_argmax_kernel (ties to the lower index;
+// NaN never wins and makes the sum NaN; nothing above -inf: id 0, conf 0).
+constexpr int kLsThreads = 256;  // light enough for two CTAs per SM, so every cluster of 8 is resident at once
+constexpr int kLsMaxVecs = 8;  // vectors a thread holds in flight
+
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.aligned;" ::: "memory"); }
+__device__ __forceinline__ void st_dsmem_f32(uint32_t addr, float v) {
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_remote_release(uint32_t addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(addr) : "memory");
+}
+// Wait (bounded) with acquire at cluster scope, for arrivals made by peers.
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity, unsigned int* err) {
+  const uint64_t t0 = global_timer_ns();
+  for (uint32_t it = 0;; ++it) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    if (ok) return true;
+    if ((it & 255u) == 255u && global_timer_ns() - t0 > kWaitLimitNs) {
+      atomicOr(err, NLD_DEVERR_WAIT_TIMEOUT);
+      return false;
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kLsThreads)
+    logits_argmax_small_kernel(const __nv_bfloat16* __restrict__ logits, int vocab, long ld, int split,
+                               int32_t* __restrict__ ids, float* __restrict__ conf, unsigned int* err) {
+  __shared__ float red[kLsThreads / 32][3];
+  __shared__ float parts[8][3];  // rank 0: the pieces' (m, s, id)
+  __shared__ __align__(8) uint64_t arrived;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, t = threadIdx.x;
+  const int piece = static_cast<int>(blockIdx.x % split);
+  const long row = static_cast<long>(blockIdx.x / split);
+  const int nvec = vocab >> 3, tail = vocab & 7;
+  const int per = (nvec + split - 1) / split;
+  const int v0 = min(nvec, piece * per), v1 = min(nvec, v0 + per);
+  if (split > 1) {
+    if (t == 0) {
+      mbar_init(&arrived, static_cast<uint32_t>(split));
+      fence_mbar_init();
+    }
+    cluster_arrive_relaxed();  // rank 0's barrier is ready once every CTA has arrived (waited below)
+  }
+  grid_launch_dependents();  // dependents launch early; they wait on this grid themselves
+  grid_dependency_wait();    // the logits come from the previous kernel
+  const uint4* grow = reinterpret_cast<const uint4*>(logits + row * ld);
+  uint4 w[kLsMaxVecs];
+#pragma unroll
+  for (int j = 0; j < kLsMaxVecs; ++j) {
+    const int v = v0 + t + j * kLsThreads;
+    w[j] = v < v1 ? __ldg(grow + v) : make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u);  // -inf
+  }
+  // max of this thread's logits and the lowest index holding it
+  float m = -INFINITY;
+  int idx = 0;
+#pragma unroll
+  for (int j = 0; j < kLsMaxVecs; ++j) {
+    float x[8];
+    unpack_bf16(w[j].x, x[0], x[1]);
+    unpack_bf16(w[j].y, x[2], x[3]);
+    unpack_bf16(w[j].z, x[4], x[5]);
+    unpack_bf16(w[j].w, x[6], x[7]);
+    const int e0 = (v0 + t + j * kLsThreads) * 8;
+#pragma unroll
+    for (int e = 0; e < 8; ++e)
+      if (x[e] > m) {  // strictly greater: the first (lowest) index of the max stays; NaN never is
+        m = x[e];
+        idx = e0 + e;
+      }
+  }
+  float s = 0.f;
+#pragma unroll
+  for (int j = 0; j < kLsMaxVecs; ++j) {
+    float x[8];
+    unpack_bf16(w[j].x, x[0], x[1]);
+    unpack_bf16(w[j].y, x[2], x[3]);
+    unpack_bf16(w[j].z, x[4], x[5]);
+    unpack_bf16(w[j].w, x[6], x[7]);
+    if (m != -INFINITY) {
+#pragma unroll
+      for (int e = 0; e < 8; ++e) s += ex2((x[e] - m) * kLog2e);  // padding (-inf) adds 0; a NaN makes s NaN
+    } else {
+#pragma unroll
+      for (int e = 0; e < 8; ++e)
+        if (isnan(x[e])) s = NAN;
+    }
+  }
+  if (piece == split - 1 && t < tail) {  // the last vocab % 8 logits
+    const uint16_t bits = reinterpret_cast<const uint16_t*>(logits + row * ld)[nvec * 8 + t];
+    const float x[1] = {__uint_as_float(static_cast<uint32_t>(bits) << 16)};
+    lg_fold(x, nvec * 8 + t, m, s, idx);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+    const float s2 = __shfl_xor_sync(0xffffffffu, s, off);
+    const int i2 = __shfl_xor_sync(0xffffffffu, idx, off);
+    lg_merge(m, s, idx, m2, s2, i2);
+  }
+  if (lane == 0) {
+    red[warp][0] = m;
+    red[warp][1] = s;
+    red[warp][2] = __int_as_float(idx);
+  }
+  __syncthreads();
+  if (warp == 0) {
+    constexpr int kW = kLsThreads / 32;
+    m = lane < kW ? red[lane][0] : -INFINITY;
+    s = lane < kW ? red[lane][1] : 0.f;
+    idx = lane < kW ? __float_as_int(red[lane][2]) : 0;
+#pragma unroll
+    for (int off = kW / 2; off > 0; off >>= 1) {
+      const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+      const float s2 = __shfl_xor_sync(0xffffffffu, s, off);
+      const int i2 = __shfl_xor_sync(0xffffffffu, idx, off);
+      lg_merge(m, s, idx, m2, s2, i2);
+    }
+    if (split == 1 && lane == 0) {
+      ids[row] = idx;
+      conf[row] = m == -INFINITY ? 0.f : 1.f / s;
+    }
+  }
+  if (split > 1) {
+    cluster_wait();
+    if (t == 0) {
+      const uint32_t slot = smem_u32(&parts[piece][0]);
+      st_dsmem_f32(dsmem_addr(slot, 0), m);
+      st_dsmem_f32(dsmem_addr(slot + 4, 0), s);
+      st_dsmem_f32(dsmem_addr(slot + 8, 0), __int_as_float(idx));
+      mbar_arrive_remote_release(dsmem_addr(smem_u32(&arrived), 0));
+    }
+    if (cluster_ctarank() == 0 && warp == 0) {
+      bool ok = true;
+      if (lane == 0) ok = mbar_wait_cluster(&arrived, 0, err);
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      m = -INFINITY;
+      s = 0.f;
+      idx = 0;
+      if (ok && lane < split) {
+        m = parts[lane][0];
+        s = parts[lane][1];
+        idx = __float_as_int(parts[lane][2]);
+      }
+#pragma unroll
+      for (int off = 4; off > 0; off >>= 1) {
+        const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+        const float s2 = __shfl_xor_sync(0xffffffffu, s, off);
+        const int i2 = __shfl_xor_sync(0xffffffffu, idx, off);
+        lg_merge(m, s, idx, m2, s2, i2);
+      }
+      if (lane == 0 && ok) {
+        ids[row] = idx;
+        conf[row] = m == -INFINITY ? 0.f : 1.f / s;
+      }
+    }
   }
 }
 
@@ -427,6 +606,10 @@ cudaError_t launch_logits_argmax(const __nv_bfloat16* logits, int rows, int voca
     __atomic_store_n(&configured[dev], 1, __ATOMIC_RELEASE);
   }
   const dim3 grid(static_cast<unsigned>(static_cast<long>(rows) * split));
+  const long piece_vecs = ((vocab >> 3) + split - 1) / split;
+  if (piece_vecs <= static_cast<long>(kLsThreads) * kLsMaxVecs)
+    return launch_kernel_cluster(logits_argmax_small_kernel, grid, dim3(kLsThreads), 0, stream, split, logits, vocab,
+                                 ld, split, ids, conf, err);
   return launch_kernel_cluster(logits_argmax_kernel, grid, dim3(kLgThreads), kLgSmemBytes, stream, split, logits,
                                vocab, ld, split, ids, conf, err);
 }
