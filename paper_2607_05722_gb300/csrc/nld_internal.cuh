@@ -295,6 +295,12 @@ __device__ __forceinline__ void named_bar_sync(int id, int threads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
 }
 
+// Arrive on a named barrier without waiting (the other `threads` - 32*k
+// participants wait with named_bar_sync).
+__device__ __forceinline__ void named_bar_arrive(int id, int threads) {
+  asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(threads) : "memory");
+}
+
 // ---------------------------------------------------------------------------
 // Thread-block clusters and distributed shared memory
 // ---------------------------------------------------------------------------
@@ -584,7 +590,11 @@ struct PagePrefetch {
 // frees the V slot of the same tile. TMA issue cost is per warp, so more
 // producer warps land a tile sooner. A warp's expect_tx covers only its own
 // boxes, so a full barrier expects one arrival per warp of its kind. `first`
-// holds the page ids of the first 32 groups, already loaded. Returns tiles
+// holds the page ids of the first 32 groups, already loaded. The
+// `early_tiles` leading tiles issued before the dependency wait go out K
+// first: the V warps wait at a named barrier until the K warps have issued
+// the early K boxes, so the first score products' operands are not queued
+// behind V boxes that only the later PV products read. Returns tiles
 // issued.
 template <int D>
 __device__ __forceinline__ int produce_kv(const AttnArgs& a, const CUtensorMap* tmk, const CUtensorMap* tmv,
@@ -605,6 +615,11 @@ __device__ __forceinline__ int produce_kv(const AttnArgs& a, const CUtensorMap* 
   nxt.raw = 0;
   if (ntiles > 8) nxt.load(a, b, t_begin, 1, lane);
   int issued = 0;
+  // Named barrier 4: the nprod producer warps, once, before any wait of the
+  // loop (early_tiles <= nstage, so the K warps reach their arrival without
+  // waiting on a slot).
+  constexpr int kKFirstBar = 4;
+  if (warp_v && early_tiles > 0) named_bar_sync(kKFirstBar, 32 * nprod);
   for (int k = 0; k < ntiles; ++k) {
     const int st = k % nstage;
     // The first `early_tiles` tiles hold prefix tokens only and may be issued
@@ -639,6 +654,7 @@ __device__ __forceinline__ int produce_kv(const AttnArgs& a, const CUtensorMap* 
       tma_load_4d(dst, is_v ? tmv : tmk, &full[st], cb * 64, slot, g, page);
     }
     issued = k + 1;
+    if (!warp_v && k == early_tiles - 1) named_bar_arrive(kKFirstBar, 32 * nprod);
   }
   return issued;
 }
