@@ -584,19 +584,20 @@ struct PagePrefetch {
 // [stage][column block]. A tile has 4 groups x D/64 column blocks x {K, V} boxes
 // (16 tokens x 64 dims each); they are dealt to the producer warps in equal
 // shares and, within a warp, one box per lane: the first half of the warps
-// load K, the second half V. K and V slots fill and free on their own
-// barriers (k_full/v_full, k_empty/v_empty), so a K slot is refilled as soon
-// as the score product that read it has completed, before the PV product
-// frees the V slot of the same tile. TMA issue cost is per warp, so more
-// producer warps land a tile sooner. A warp's expect_tx covers only its own
-// boxes, so a full barrier expects one arrival per warp of its kind. `first`
-// holds the page ids of the first 32 groups, already loaded. The
-// `early_tiles` leading tiles issued before the dependency wait go out K
-// first: the V warps wait at a named barrier until the K warps have issued
-// the early K boxes, so the first score products' operands are not queued
-// behind V boxes that only the later PV products read. Returns tiles
-// issued.
-template <int D>
+// load K, the second half V. With kSplit, K and V slots fill and free on
+// their own barriers (k_full/v_full, k_empty/v_empty), so a K slot is
+// refilled as soon as the score product that read it has completed, before
+// the PV product frees the V slot of the same tile; without it a stage's K
+// and V fill on k_full and free on k_empty together. TMA issue cost is per
+// warp, so more producer warps land a tile sooner. A warp's expect_tx covers
+// only its own boxes, so a full barrier expects one arrival per warp (of its
+// kind, with kSplit). `first` holds the page ids of the first 32 groups,
+// already loaded. With kSplit the `early_tiles` leading tiles issued before
+// the dependency wait go out K first: the V warps wait at a named barrier
+// until the K warps have issued the early K boxes, so the first score
+// products' operands are not queued behind V boxes that only the later PV
+// products read. Returns tiles issued.
+template <int D, bool kSplit>
 __device__ __forceinline__ int produce_kv(const AttnArgs& a, const CUtensorMap* tmk, const CUtensorMap* tmv,
                                           uint8_t* stages, uint64_t* k_full, uint64_t* v_full, uint64_t* k_empty,
                                           uint64_t* v_empty, int nstage, int g, int b, int t_begin, int t_end,
@@ -607,8 +608,8 @@ __device__ __forceinline__ int produce_kv(const AttnArgs& a, const CUtensorMap* 
   constexpr int kOpsPerTile = kGroups * 2 * Geo::kColBlocks;  // 16 (D=128) or 8 (D=64)
   const int my_ops = kOpsPerTile / nprod;                     // nprod divides kOpsPerTile (and its halves)
   const bool warp_v = pw >= nprod / 2;                        // this warp's boxes are all V (else all K)
-  uint64_t* full = warp_v ? v_full : k_full;
-  uint64_t* empty = warp_v ? v_empty : k_empty;
+  uint64_t* full = kSplit && warp_v ? v_full : k_full;
+  uint64_t* empty = kSplit && warp_v ? v_empty : k_empty;
   const uint32_t bytes = static_cast<uint32_t>(my_ops) * kGroupTok * 128;
   int page_cur = first.validate(a, t_begin, t_end, 0, lane);
   PagePrefetch nxt;
@@ -619,7 +620,7 @@ __device__ __forceinline__ int produce_kv(const AttnArgs& a, const CUtensorMap* 
   // loop (early_tiles <= nstage, so the K warps reach their arrival without
   // waiting on a slot).
   constexpr int kKFirstBar = 4;
-  if (warp_v && early_tiles > 0) named_bar_sync(kKFirstBar, 32 * nprod);
+  if (kSplit && warp_v && early_tiles > 0) named_bar_sync(kKFirstBar, 32 * nprod);
   for (int k = 0; k < ntiles; ++k) {
     const int st = k % nstage;
     // The first `early_tiles` tiles hold prefix tokens only and may be issued
@@ -654,7 +655,7 @@ __device__ __forceinline__ int produce_kv(const AttnArgs& a, const CUtensorMap* 
       tma_load_4d(dst, is_v ? tmv : tmk, &full[st], cb * 64, slot, g, page);
     }
     issued = k + 1;
-    if (!warp_v && k == early_tiles - 1) named_bar_arrive(kKFirstBar, 32 * nprod);
+    if (kSplit && !warp_v && k == early_tiles - 1) named_bar_arrive(kKFirstBar, 32 * nprod);
   }
   return issued;
 }
