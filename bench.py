@@ -741,7 +741,7 @@ def split_sweep(torch, nld, stream, w, pools, out, lse, peak):
     """Verify-pass time over explicit KV split counts, two ways: the default
     plan (pieces of 2/4/8 dividing S merge as thread-block clusters) and
     every piece its own partial merged by the combine kernel
-    (NLD_ATTN_NO_CLUSTER). `partial_bytes` = S x B x Hq x bl x (D+1) x 4,
+    (NLD_ATTN_NO_CLUSTER). `partial_bytes` = S x B x Hq x bl x (2 D + 4) (bf16 rows, fp32 lse),
     written once by the attention kernel and read once by the combine."""
     B, bl, Hq, Hkv, D = w["batch"], w["bl"], w["hq"], w["hkv"], w["d"]
     kvb = w["kv_bytes_per_pass"]
@@ -767,7 +767,7 @@ def split_sweep(torch, nld, stream, w, pools, out, lse, peak):
                              "pct_of_hbm_peak": round(100 * gbs / peak, 2), "pieces": plan["splits"],
                              "cluster": plan["cluster"], "kv_partials": parts,
                              "kernels": nld.nld_block_attn_kernels(pS, bl),
-                             "partial_bytes": (parts * B * Hq * bl * (D + 1) * 4) if parts > 1 else 0}
+                             "partial_bytes": (parts * B * Hq * bl * (2 * D + 4)) if parts > 1 else 0}
             del wsS
         sweep[vname] = curve
     return sweep

@@ -143,9 +143,10 @@ int nld_block_attn_plan(const nld_attn_params_t *params, int block_len, int sm_c
 
 /*
  * Workspace bytes nld_block_attn needs (0 when it runs unsplit). The
- * workspace holds fp32 split partials: O_part [S, B, Hq, bl, D] then
- * LSE_part [S, B, Hq, bl] at the next 256-byte boundary. Its contents need
- * no initialisation. Calls whose kernels may overlap on the GPU need
+ * workspace holds the split partials: O_part bf16 [S, B, Hq, bl, D] (each
+ * row the partial output normalised by its own sum, so its values lie within
+ * the range of V) then LSE_part fp32 [S, B, Hq, bl] at the next 256-byte
+ * boundary. Its contents need no initialisation. Calls whose kernels may overlap on the GPU need
  * separate workspaces.
  * Returns (size_t)-1 if the parameters are invalid.
  */
@@ -189,9 +190,9 @@ nld_status_t nld_block_attn(const nld_attn_params_t *params, const void *q_block
 /*
  * The attention kernel of nld_block_attn alone, same arguments. When the
  * split plan has one split it writes out and lse exactly as nld_block_attn
- * does. With S > 1 splits it writes only the fp32 partials into the
- * workspace (O_part at offset 0, LSE_part at the next 256-byte boundary
- * after S*B*Hq*bl*D*4 bytes) and leaves out/lse untouched; the caller then
+ * does. With S > 1 splits it writes only the partials into the workspace
+ * (bf16 O_part at offset 0, fp32 LSE_part at the next 256-byte boundary
+ * after S*B*Hq*bl*D*2 bytes) and leaves out/lse untouched; the caller then
  * merges them with nld_split_kv_combine (S = nld_block_attn_num_splits()).
  * This lets a caller time, overlap or reorder the two kernels.
  */
@@ -263,15 +264,16 @@ nld_status_t nld_block_attn_static_scratch(const nld_attn_params_t *params, cons
  *   out = sum_s c_s o_s / sum_s c_s,  lse = m + ln sum_s c_s.
  * A partial with lse_s = -inf carries no keys: it gets weight 0 and its
  * o_s is not read. A row whose partials are all -inf gets out = 0 and
- * lse = -inf.
+ * lse = -inf. Weights, sums and the merged row are computed in fp32 from the
+ * bf16 partials; out is rounded to bf16 once.
  *
- *   o_part   fp32 [S, B, Hq, bl, D]
+ *   o_part   bf16 [S, B, Hq, bl, D] (16-byte aligned)
  *   lse_part fp32 [S, B, Hq, bl]
  *   out      bf16 [B, bl, Hq, D]
  *   lse      fp32 [B, Hq, bl], or NULL
  *   1 <= num_splits <= 128, head_dim 64 or 128, 1 <= block_len <= 32
  */
-nld_status_t nld_split_kv_combine(const float *o_part, const float *lse_part, int num_splits,
+nld_status_t nld_split_kv_combine(const void *o_part, const float *lse_part, int num_splits,
                                   int batch, int num_q_heads, int block_len, int head_dim,
                                   void *out, float *lse, cudaStream_t stream);
 

@@ -25,8 +25,8 @@
 //             over the consumed S columns as the PV MMA's A operand, and at
 //             the end reads O from TMEM, divides by the sum and stages its row
 //             in the freed K/V ring in 128-byte-swizzled boxes, which one
-//             thread writes with tiled TMA stores (bf16 output or fp32 split
-//             partials, in packed row order).
+//             thread writes with tiled TMA stores (the bf16 output or bf16
+//             split partials, in packed row order).
 //             With at most 64 (32) packed rows, Q is replicated into the idle
 //             lane quadrants (REP = 2 or 4): each copy of a row takes a 64/REP-
 //             token slice of every tile with its own running max and sum, so
@@ -128,7 +128,7 @@ struct TcLayout {
   // copies of a row (REP > 1) exchange their O column ranges here
   static constexpr int kXchgOff = (kLseOutOff + kMergeRows * 4 + 15) / 16 * 16;
   // output boxes for the tiled stores (128-byte rows, 1024-byte aligned)
-  static_assert(D / 32 * kMergeRows * 128 <= kPOff, "output staging");
+  static_assert(D / 64 * kMergeRows * 128 <= kPOff, "output staging");
 };
 
 // The sequence of rank blockIdx.z by prefix length (descending, ties by
@@ -733,7 +733,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
     if (o_ready) tc_fence_after();
     if constexpr (REP > 1) {
       static_assert(Lay::kXchgOff + REP * (REP - 1) * 32 * kRowQuads * kXPitch <= Lay::kPOff, "exchange buffers");
-      static_assert(D / 32 * (128 / REP) * 128 <= Lay::kWtsOff, "output staging below the copies' weights");
+      static_assert(D / 64 * (128 / REP) * 128 <= Lay::kWtsOff, "output staging below the copies' weights");
       float* part_ml = reinterpret_cast<float*>(smem + Lay::kWtsOff);  // [TMEM lane][max, sum]
       part_ml[2 * r_loc] = o_ready ? m_run : -INFINITY;  // a copy cut short by a timeout is dropped
       part_ml[2 * r_loc + 1] = l_run;
@@ -870,8 +870,9 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
       // Each thread stages its columns in 128-byte-swizzled boxes of 128-byte
       // rows in packed row order (block slot major, so that any 8 consecutive
       // lanes hit 8 different bank groups), and one thread stores the boxes
-      // with tiled TMA copies: D/64 (bf16 output) or D/32 (fp32 partials,
-      // whose map walks the heads before the block slots) copies per CTA.
+      // with tiled TMA copies: D/64 boxes of 64 bf16 columns per CTA (the
+      // output, or the split partials, whose map walks the heads before the
+      // block slots).
       const bool split_out = a.o_part != nullptr;
       const int srow = r;  // row within the boxes
       const int box_stride = (a.R * 128 + 1023) & ~1023;
@@ -886,25 +887,14 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
           final_chunk(cc, o);
           const int col0 = part * kRange + cc * kChunk;
           if (row_ok) {
-            if (split_out) {
+            uint8_t* row = smem + (col0 >> 6) * box_stride + srow * 128;
+            const int ch0 = (col0 & 63) >> 3;
 #pragma unroll
-              for (int k4 = 0; k4 < kChunk / 4; ++k4) {
-                const int col = col0 + 4 * k4;
-                uint8_t* row = smem + (col >> 5) * box_stride + srow * 128;
-                const float* v = o + 4 * k4;
-                *reinterpret_cast<float4*>(row + ((((col & 31) >> 2) ^ (srow & 7)) << 4)) =
-                    make_float4(v[0], v[1], v[2], v[3]);
-              }
-            } else {
-              uint8_t* row = smem + (col0 >> 6) * box_stride + srow * 128;
-              const int ch0 = (col0 & 63) >> 3;
-#pragma unroll
-              for (int c8 = 0; c8 < kChunk / 8; ++c8) {
-                const float* v = o + c8 * 8;
-                *reinterpret_cast<uint4*>(row + (((ch0 + c8) ^ (srow & 7)) << 4)) =
-                    make_uint4(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]), pack_bf16(v[4], v[5]),
-                               pack_bf16(v[6], v[7]));
-              }
+            for (int c8 = 0; c8 < kChunk / 8; ++c8) {
+              const float* v = o + c8 * 8;
+              *reinterpret_cast<uint4*>(row + (((ch0 + c8) ^ (srow & 7)) << 4)) =
+                  make_uint4(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]), pack_bf16(v[4], v[5]),
+                             pack_bf16(v[6], v[7]));
             }
           }
         }
@@ -918,13 +908,11 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
         fence_proxy_async_smem();     // the staged boxes, visible to the TMA engine
         named_bar_sync(3, 32 * Cfg::kSmWarps);  // every softmax warp, with rows or not
         if (sm_tid == 0 && o_ready) {
-          if (split_out) {
 #pragma unroll
-            for (int x = sr * (D / 32 / kStoreRounds); x < (sr + 1) * (D / 32 / kStoreRounds); ++x)
-              tma_store_4d(&maps.o, smem + x * box_stride, x * 32, g * a.G, slot0, split * a.B + b);
-          } else {
-#pragma unroll
-            for (int x = sr * (D / 64 / kStoreRounds); x < (sr + 1) * (D / 64 / kStoreRounds); ++x)
+          for (int x = sr * (D / 64 / kStoreRounds); x < (sr + 1) * (D / 64 / kStoreRounds); ++x) {
+            if (split_out)
+              tma_store_4d(&maps.o, smem + x * box_stride, x * 64, g * a.G, slot0, split * a.B + b);
+            else
               tma_store_3d(&maps.o, smem + x * box_stride, x * 64, g * a.G, b * a.bl + slot0);
           }
           bulk_commit();
@@ -1027,7 +1015,9 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
             if (d4[u] == 0 && a.lse != nullptr) a.lse[(static_cast<size_t>(b) * a.Hq + h) * a.bl + i] = lse_v;
           } else {
             const size_t prow = ((static_cast<size_t>(pidx) * a.B + b) * a.Hq + h) * a.bl + i;
-            if (lse_v != -INFINITY) *reinterpret_cast<float4*>(a.o_part + prow * D + d4[u] * 4) = acc[u];
+            if (lse_v != -INFINITY)
+              *reinterpret_cast<uint2*>(a.o_part + prow * D + d4[u] * 4) =
+                  make_uint2(pack_bf16(acc[u].x, acc[u].y), pack_bf16(acc[u].z, acc[u].w));
             if (d4[u] == 0) a.lse_part[prow] = lse_v;
           }
         }

@@ -189,7 +189,7 @@ nld_status_t plan_splits(const nld_attn_params_t* p, int block_len, SplitPlan* o
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 size_t partial_o_bytes(const nld_attn_params_t* p, int block_len, int splits) {
-  return static_cast<size_t>(splits) * p->batch * p->num_q_heads * block_len * p->head_dim * sizeof(float);
+  return static_cast<size_t>(splits) * p->batch * p->num_q_heads * block_len * p->head_dim * sizeof(__nv_bfloat16);
 }
 size_t partial_lse_bytes(const nld_attn_params_t* p, int block_len, int splits) {
   return static_cast<size_t>(splits) * p->batch * p->num_q_heads * block_len * sizeof(float);
@@ -247,23 +247,23 @@ nld_status_t encode_block_map(CUtensorMap* map, const void* base, const nld::Att
 }
 
 // Map for the tiled output stores of one CTA's R = G * bl rows, 128-byte
-// swizzle, rows in packed order (block slot major). Final output [B, bl, Hq,
-// D] bf16: box 64 dims x G heads x bl slots. Split partials [partials * B,
-// Hq, bl, D] fp32: the map walks dims, heads (stride bl * D), block slots
-// (stride D), then (partial, sequence); box 32 dims x G heads x bl slots.
+// swizzle, rows in packed order (block slot major), box 64 dims x G heads x
+// bl slots, bf16. Final output [B, bl, Hq, D]. Split partials [partials * B,
+// Hq, bl, D]: the map walks dims, heads (stride bl * D), block slots (stride
+// D), then (partial, sequence).
 nld_status_t encode_out_map(CUtensorMap* map, const nld::AttnArgs& a, int D) {
   if (a.o_part == nullptr) return encode_block_map(map, a.out, a, D);
   EncodeTiledFn fn = encode_fn();
   if (fn == nullptr) return NLD_ERR_CUDA;
   const long long units = static_cast<long long>(a.num_partials) * a.B;
   if (units > INT_MAX) return NLD_ERR_UNSUPPORTED;  // coordinates are int
-  const cuuint64_t row = static_cast<cuuint64_t>(D) * 4;
+  const cuuint64_t row = static_cast<cuuint64_t>(D) * 2;
   cuuint32_t estr[4] = {1, 1, 1, 1};
   cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(a.Hq), static_cast<cuuint64_t>(a.bl),
                         static_cast<cuuint64_t>(units)};
   cuuint64_t strides[3] = {row * a.bl, row, row * a.bl * a.Hq};
-  cuuint32_t box[4] = {32, static_cast<cuuint32_t>(a.G), static_cast<cuuint32_t>(a.bl_c), 1};
-  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, a.o_part, dims, strides, box, estr,
+  cuuint32_t box[4] = {64, static_cast<cuuint32_t>(a.G), static_cast<cuuint32_t>(a.bl_c), 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, a.o_part, dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? NLD_OK : NLD_ERR_CUDA;
@@ -406,15 +406,17 @@ nld_status_t block_attn_impl(const nld_attn_params_t* params, const void* q_bloc
                             : 0;
   }
   if (plan.partials > 1) {
-    a.o_part = static_cast<float*>(workspace);
+    a.o_part = static_cast<__nv_bfloat16*>(workspace);
     a.lse_part = reinterpret_cast<float*>(static_cast<char*>(workspace) + o_bytes);
   }
   if ((st = encode_out_map(&maps.o, a, params->head_dim)) != NLD_OK) return st;
   if ((st = encode_block_map(&maps.q, q_block, a, params->head_dim)) != NLD_OK) return st;
   if (nld::launch_block_attn_tc(a, maps, params->head_dim, stream) != cudaSuccess) return NLD_ERR_CUDA;
   if (plan.partials > 1 && run_combine) {
+    int sms = 0;
+    if ((st = device_state(nullptr, &sms)) != NLD_OK) return st;
     if (nld::launch_combine(a.o_part, a.lse_part, plan.partials, a.B, a.Hq, block_len, params->head_dim, a.out, lse,
-                            stream) != cudaSuccess)
+                            sms, stream) != cudaSuccess)
       return NLD_ERR_CUDA;
   }
   return NLD_OK;
@@ -467,7 +469,7 @@ nld_status_t nld_block_attn_partials(const nld_attn_params_t* params, const void
                          lse, workspace, workspace_bytes, false, stream);
 }
 
-nld_status_t nld_split_kv_combine(const float* o_part, const float* lse_part, int num_splits, int batch,
+nld_status_t nld_split_kv_combine(const void* o_part, const float* lse_part, int num_splits, int batch,
                                   int num_q_heads, int block_len, int head_dim, void* out, float* lse,
                                   cudaStream_t stream) {
   if (num_splits < 1 || num_splits > nld::kMaxSplits || batch < 1 || num_q_heads < 1 || block_len < 1 ||
@@ -476,8 +478,11 @@ nld_status_t nld_split_kv_combine(const float* o_part, const float* lse_part, in
   if (head_dim != 64 && head_dim != 128) return NLD_ERR_UNSUPPORTED;
   if (!aligned(o_part, 16) || !aligned(lse_part, 4) || !aligned(out, 16)) return NLD_ERR_INVALID_ARG;
   if (lse != nullptr && !aligned(lse, 4)) return NLD_ERR_INVALID_ARG;
-  if (nld::launch_combine(o_part, lse_part, num_splits, batch, num_q_heads, block_len, head_dim,
-                          static_cast<__nv_bfloat16*>(out), lse, stream) != cudaSuccess)
+  int sms = 0;
+  const nld_status_t st = device_state(nullptr, &sms);
+  if (st != NLD_OK) return st;
+  if (nld::launch_combine(static_cast<const __nv_bfloat16*>(o_part), lse_part, num_splits, batch, num_q_heads,
+                          block_len, head_dim, static_cast<__nv_bfloat16*>(out), lse, sms, stream) != cudaSuccess)
     return NLD_ERR_CUDA;
   return NLD_OK;
 }

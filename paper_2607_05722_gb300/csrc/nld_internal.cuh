@@ -29,7 +29,7 @@ struct AttnArgs {
   const int32_t* prefix_lens;  // [B]
   __nv_bfloat16* out;          // [B, bl, Hq, D]       (unsplit)
   float* lse;                  // [B, Hq, bl] or null  (unsplit)
-  float* o_part;               // [S, B, Hq, bl, D]    (split; null when unsplit)
+  __nv_bfloat16* o_part;       // [S, B, Hq, bl, D]    (split; null when unsplit), each row normalised
   float* lse_part;             // [S, B, Hq, bl]
   unsigned int* err;           // device error word
   unsigned long long* rescales;  // running-max rescale events (diagnostic counter)
@@ -50,7 +50,7 @@ struct AttnArgs {
 // tcgen05 kernel: query rows R <= 256 (one or two 128-row MMA tiles).
 bool tc_supports(int R, int head_dim);
 // Tensor maps of one call: k/v the K/V page pools; q the query block and o
-// the output (bf16 rows) or, with split partials, the fp32 partial rows, in
+// the output or, with split partials, the partial rows (bf16 both), in
 // boxes of one CTA's rows.
 struct TmaMaps {
   CUtensorMap k, v, o, q;
@@ -60,8 +60,8 @@ cudaError_t launch_block_attn_tc(const AttnArgs& a, const TmaMaps& maps, int hea
 cudaError_t launch_block_attn_tc_masked(const AttnArgs& a, const TmaMaps& maps, int head_dim, cudaStream_t stream);
 // A kernel whose one mbarrier wait can never complete (decide.cu).
 cudaError_t launch_wait_timeout_check(uint64_t limit_ns, unsigned int* err, cudaStream_t stream);
-cudaError_t launch_combine(const float* o_part, const float* lse_part, int S, int B, int Hq, int bl,
-                           int D, __nv_bfloat16* out, float* lse, cudaStream_t stream);
+cudaError_t launch_combine(const __nv_bfloat16* o_part, const float* lse_part, int S, int B, int Hq, int bl,
+                           int D, __nv_bfloat16* out, float* lse, int sm_count, cudaStream_t stream);
 cudaError_t launch_accept(const int32_t* draft, const int32_t* verify, int B, int n, int32_t* acc,
                           cudaStream_t stream);
 cudaError_t launch_unmask(const float* conf, int B, int n, int k, int32_t* pos, int32_t* nsel,

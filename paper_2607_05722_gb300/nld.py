@@ -174,17 +174,17 @@ def nld_block_attn_workspace_size(params: AttnParams, block_len: int) -> int:
 
 
 def workspace_views(params: AttnParams, block_len: int, workspace):
-    """(o_part [S,B,Hq,bl,D], lse_part [S,B,Hq,bl]) fp32 views of a workspace laid out as
-    include/nld.h documents, or None when the plan has one split."""
+    """(o_part bf16 [S,B,Hq,bl,D], lse_part fp32 [S,B,Hq,bl]) views of a workspace laid out
+    as include/nld.h documents, or None when the plan has one split."""
     S = nld_block_attn_num_splits(params, block_len)
     if S <= 1:
         return None
     B, Hq, D = params.batch, params.num_q_heads, params.head_dim
     n_o = S * B * Hq * block_len * D
     o0 = 0
-    l0 = o0 + ((n_o * 4 + 255) // 256) * 256
+    l0 = o0 + ((n_o * 2 + 255) // 256) * 256
     flat = workspace.view(torch.uint8)
-    o_part = flat[o0:o0 + n_o * 4].view(torch.float32).view(S, B, Hq, block_len, D)
+    o_part = flat[o0:o0 + n_o * 2].view(torch.bfloat16).view(S, B, Hq, block_len, D)
     lse_part = flat[l0:l0 + S * B * Hq * block_len * 4].view(torch.float32).view(S, B, Hq, block_len)
     return o_part, lse_part
 
@@ -279,9 +279,9 @@ def nld_block_attn_static_scratch(params: AttnParams, q_block, k_pages, v_pages,
 
 
 def nld_split_kv_combine(o_part, lse_part, out, lse=None, stream=None):
-    """Merge split partials o_part [S,B,Hq,bl,D], lse_part [S,B,Hq,bl] into out [B,bl,Hq,D]."""
+    """Merge split partials o_part bf16 [S,B,Hq,bl,D], lse_part fp32 [S,B,Hq,bl] into out [B,bl,Hq,D]."""
     S, B, Hq, bl, D = o_part.shape
-    _expect(o_part, torch.float32, (S, B, Hq, bl, D), "o_part")
+    _expect(o_part, torch.bfloat16, (S, B, Hq, bl, D), "o_part")
     _expect(lse_part, torch.float32, (S, B, Hq, bl), "lse_part")
     _expect(out, torch.bfloat16, (B, bl, Hq, D), "out")
     if lse is not None:

@@ -49,13 +49,13 @@ def test_split_plan_and_workspace_size(L):
     assert nld.nld_block_attn_num_splits(p, 16) == 19
     # 4112 tokens / 19 -> 217 -> 224 per split -> 19 splits
     S, B, Hq, bl, D = 19, 1, 32, 16, 128
-    o = S * B * Hq * bl * D * 4
+    o = S * B * Hq * bl * D * 2  # bf16 partial rows, then fp32 log-sum-exps
     assert nld.nld_block_attn_workspace_size(p, 16) == ((o + 255) // 256) * 256 + S * B * Hq * bl * 4
     assert nld.nld_block_attn_workspace_size(params(num_splits=1), 16) == 0
     # 16 pieces run as two clusters of 8 (tcgen05 kernel, 64 packed rows): 2 partials
     assert nld.nld_block_attn_num_splits(params(num_splits=16), 16) == 2
     assert nld.nld_block_attn_workspace_size(params(num_splits=16), 16) == \
-        ((2 * Hq * bl * D * 4 + 255) // 256) * 256 + 2 * Hq * bl * 4
+        ((2 * Hq * bl * D * 2 + 255) // 256) * 256 + 2 * Hq * bl * 4
     # without clusters every piece is a partial
     assert nld.nld_block_attn_num_splits(params(num_splits=16, flags=nld.NLD_ATTN_NO_CLUSTER), 16) == 16
     # 4 pieces (chunk >= 16 tokens of 64) merge in one cluster: final output, no workspace

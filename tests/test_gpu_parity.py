@@ -464,14 +464,18 @@ def test_unmask_denoising_chain(orc):
 def test_combine_matches_oracle(orc, S, D):
     rng = np.random.default_rng(S * 1000 + D)
     B, Hq, bl = 3, 8, 5
-    o = rng.standard_normal((S, B, Hq, bl, D)).astype(np.float32)
+    # partial rows in bf16 (the workspace format); the oracle merges the same
+    # bf16 values in fp64
+    o_bits = W.f32_to_bf16_bits(rng.standard_normal((S, B, Hq, bl, D)).astype(np.float32))
     l = (rng.standard_normal((S, B, Hq, bl)) * 3).astype(np.float32)
     l[rng.random(l.shape) < 0.3] = -np.inf
     l[:, 0, 0, 0] = -np.inf  # a row with no keys at all
-    o[np.broadcast_to((l == -np.inf)[..., None], o.shape)] = np.nan  # never read
+    o_bits[np.broadcast_to((l == -np.inf)[..., None], o_bits.shape)] = 0x7FC0  # NaN, never read
+    o = W.bf16_bits_to_f32(o_bits)
     out = torch.empty((B, bl, Hq, D), dtype=torch.bfloat16, device="cuda")
     lse = torch.empty((B, Hq, bl), dtype=torch.float32, device="cuda")
-    nld.nld_split_kv_combine(torch.from_numpy(o).cuda(), torch.from_numpy(l).cuda(), out, lse)
+    o_dev = torch.from_numpy(np.ascontiguousarray(o_bits).view(np.int16)).view(torch.bfloat16).cuda()
+    nld.nld_split_kv_combine(o_dev, torch.from_numpy(l).cuda(), out, lse)
     ro, rl = orc.combine(np.nan_to_num(o, nan=0.0).reshape(S, -1, D), l.reshape(S, -1))
     ro = ro.reshape(B, Hq, bl, D).transpose(0, 2, 1, 3)
     rl = rl.reshape(B, Hq, bl)
