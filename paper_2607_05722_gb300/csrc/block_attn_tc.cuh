@@ -152,7 +152,7 @@ __device__ __noinline__ int sequence_by_length_rank(const AttnArgs& a, int* scra
   return order[blockIdx.z];
 }
 
-template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED, int CG>
+template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED, int CG, bool JOINT = false>
 __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
     block_attn_tc_kernel(const __grid_constant__ TmaMaps maps, const AttnArgs a) {
   static_assert(REP == 1 || REP == 2 || REP == 4, "replication of 1, 2 or 4");
@@ -162,14 +162,17 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
   using Cfg = TcCfg<MT, TPS, CG>;
   using Lay = TcLayout<D, MT, TPS>;
   constexpr int kTcStages = Lay::kStages;
-  // Ring barriers. With two softmax groups (a long split of 65..128 rows) K
-  // and V slots fill and free on their own barriers, so a K slot is refilled
-  // as soon as the score product that read it has completed and the K boxes
-  // of the early tiles go out first; the kernels with one group (row copies,
-  // two M tiles) keep one barrier per stage for K and V together, freed by
-  // the PV product: each scheme measured faster on its own kernels (the
-  // split scheme: long prefix +4%; the joint one: concurrency sweep +6%).
-  constexpr bool kSplitKV = CG == 2;
+  // Ring barriers. With two softmax groups on a split of its own (65..128
+  // rows) K and V slots fill and free on their own barriers, so a K slot is
+  // refilled as soon as the score product that read it has completed and the
+  // K boxes of the early tiles go out first; the kernels with one group (row
+  // copies, two M tiles) and the block-slot chunk pairs (JOINT, whose second
+  // CTA reads each tile from L2 behind its partner) keep one barrier per
+  // stage for K and V together, freed by the PV product: each scheme measured
+  // faster on its own kernels (the split scheme: long prefix +4%; the joint
+  // one: concurrency sweep +6%, 14B chunk pairs +5%).
+  static_assert(!JOINT || CG == 2, "the joint variant of the two-group kernel");
+  constexpr bool kSplitKV = CG == 2 && !JOINT;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* q_s = smem + Lay::kQOff;
@@ -1033,12 +1036,12 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
   }
 }
 
-template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED, int CG>
+template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED, int CG, bool JOINT = false>
 cudaError_t configure_tc(int dev) {
   static int configured[64] = {0};
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   if (!__atomic_load_n(&configured[dev], __ATOMIC_ACQUIRE)) {
-    cudaError_t e = cudaFuncSetAttribute(block_attn_tc_kernel<D, MT, REP, TPS, MASKED, ORDERED, CG>,
+    cudaError_t e = cudaFuncSetAttribute(block_attn_tc_kernel<D, MT, REP, TPS, MASKED, ORDERED, CG, JOINT>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(TcLayout<D, MT, TPS>::kBytes + 1024));
     if (e != cudaSuccess) return e;
@@ -1047,26 +1050,26 @@ cudaError_t configure_tc(int dev) {
   return cudaSuccess;
 }
 
-template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED, int CG>
+template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED, int CG, bool JOINT = false>
 cudaError_t launch_tc_o(const AttnArgs& a, const TmaMaps& maps, cudaStream_t stream) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  if ((e = configure_tc<D, MT, REP, TPS, MASKED, ORDERED, CG>(dev)) != cudaSuccess) return e;
+  if ((e = configure_tc<D, MT, REP, TPS, MASKED, ORDERED, CG, JOINT>(dev)) != cudaSuccess) return e;
   dim3 grid(a.num_splits * a.nh, a.Hkv, a.B);
-  return launch_kernel_cluster(block_attn_tc_kernel<D, MT, REP, TPS, MASKED, ORDERED, CG>, grid,
+  return launch_kernel_cluster(block_attn_tc_kernel<D, MT, REP, TPS, MASKED, ORDERED, CG, JOINT>, grid,
                                dim3(TcCfg<MT, TPS, CG>::kThreads), TcLayout<D, MT, TPS>::kBytes + 1024, stream,
                                a.csize, maps, a);
 }
 
 // The longest-first order only for the unmasked passes (the table-mask
 // passes run at the block shapes of one sequence).
-template <int D, int MT, int REP, int TPS, bool MASKED, int CG = 1>
+template <int D, int MT, int REP, int TPS, bool MASKED, int CG = 1, bool JOINT = false>
 cudaError_t launch_tc_t(const AttnArgs& a, const TmaMaps& maps, cudaStream_t stream) {
   if constexpr (!MASKED) {
-    if (a.order_by_length) return launch_tc_o<D, MT, REP, TPS, false, true, CG>(a, maps, stream);
+    if (a.order_by_length) return launch_tc_o<D, MT, REP, TPS, false, true, CG, JOINT>(a, maps, stream);
   }
-  return launch_tc_o<D, MT, REP, TPS, MASKED, false, CG>(a, maps, stream);
+  return launch_tc_o<D, MT, REP, TPS, MASKED, false, CG, JOINT>(a, maps, stream);
 }
 
 // Resident clusters of the kernel a plan would launch (one CTA per SM
@@ -1126,7 +1129,10 @@ cudaError_t launch_tc_rep(const AttnArgs& a, const TmaMaps& maps, cudaStream_t s
   switch (tc_replication(a.R)) {
     case 4: return launch_tc_t<D, 1, 4, TPS, MASKED>(a, maps, stream);
     case 2: return launch_tc_t<D, 1, 2, TPS, MASKED>(a, maps, stream);
-    default: return launch_tc_t<D, 1, 1, 2, MASKED, 2>(a, maps, stream);
+    default:
+      // block-slot chunk pairs take the joint-barrier variant
+      if (a.nh > 1) return launch_tc_t<D, 1, 1, 2, MASKED, 2, true>(a, maps, stream);
+      return launch_tc_t<D, 1, 1, 2, MASKED, 2>(a, maps, stream);
   }
 }
 
