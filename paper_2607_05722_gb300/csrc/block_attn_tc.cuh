@@ -6,19 +6,23 @@
 // heads times the bl block tokens form R = G*bl <= 256 query rows in one or
 // two 128-row MMA tiles, so each K/V page leaves HBM once per (b, g).
 //
-// Warp roles (5 + 4*MT warps):
+// Warp roles (5 + 4*MT*CG warps):
 //   warps 0-2 and the last  TMA producers: the boxes of each 64-token K/V tile
 //             (16 tokens x 64 dims each) dealt four ways into a ring of up to
 //             8 stages (produce_kv), warps 0-1 the K boxes, the others the V
-//             boxes, each kind with its own full/empty barriers so that a K
-//             slot refills once its score product is done; TMA issue cost is
-//             per warp, so four issuing warps land a tile sooner.
+//             boxes (with two softmax groups each kind with its own full/empty
+//             barriers, so that a K slot refills once its score product is
+//             done); TMA issue cost is per warp, so four issuing warps land a
+//             tile sooner.
 //   warp 3    allocates the TMEM columns; lane 0 loads Q by TMA (one M tile)
 //             and issues every MMA:
 //               S_j = Q K^T     (M=128 rows, N=64*TPS tokens, K=D; double-buffered in TMEM)
 //               O  += P_k V_k   (M=128 rows, N=D, K=64 tokens; V read MN-major)
 //             S_{j+1} is issued before the PV products of S_j so the tensor
 //             core computes the next scores while the softmax warps work.
+//             Each MMA or commit instruction holds the issuing thread ~50
+//             cycles (measured), so the one issuing thread is a serial
+//             resource of the chain.
 //   warps 4.. softmax: thread t owns TMEM lane 32*(warp%4)+lane, one query
 //             row. It loads its S row, applies the mask and the base-2 scale,
 //             keeps the running max and sum, writes P (bf16) back to TMEM
@@ -32,6 +36,13 @@
 //             token slice of every tile with its own running max and sum, so
 //             every softmax warp works and each does 1/REP of the exponentials;
 //             the copies are merged once, each finalising 1/REP of the columns.
+//             With 65..128 rows (CG = 2) two groups of four softmax warps
+//             share the TMEM lanes: group c takes tile 2j + c of score
+//             product j. Both take the row max over both tiles (the other
+//             tile's columns read for the max only), so they hold the same
+//             running max and accumulate into one O; P has two TMEM buffers
+//             of its own, so a score product waits only for the softmax to
+//             have read the S buffer it overwrites, never for a PV product.
 // When the KV range of a (sequence, KV head) is split over a thread-block
 // cluster, the CTAs stage their normalised rows in shared memory and merge
 // them through distributed shared memory (a cluster barrier, then each CTA
@@ -63,13 +74,14 @@ constexpr int kSoftmaxWarp0 = 4;
 //
 // CG softmax groups per M tile: with CG = 2 (one M tile of up to 128 rows
 // without row copies, paired products) two groups of four warps share the
-// TMEM lanes; group c takes tile 2j + c of each product j, keeps its own
-// running max and sum and accumulates into its own O columns (PV of its
-// tile only), and the two are merged once before the epilogue, by the
-// split-combine rule. Per product the tensor core runs 8 score MMAs of N =
-// 128 and 8 PV MMAs, and each softmax thread does one 64-column tile: the
-// MMA issue and the softmax chain, which bound a streaming split with one
-// group, both shrink per tile.
+// TMEM lanes; group c takes tile 2j + c of each product j. Both groups take
+// each row's max over both tiles, so they keep the same running max and
+// accumulate into one O (each keeps the sum of its own tiles, added once
+// before the epilogue). TMEM: two S buffers, the one O, two P buffers of 64
+// columns. Per product the tensor core runs 8 score MMAs of N = 128 and 8
+// PV MMAs, each softmax thread exponentiates one 64-column tile, and a score
+// product waits only for the softmax warps to have read its S buffer: the
+// chain S -> softmax -> PV no longer holds the next score products back.
 template <int MT, int TPS, int CG = 1>
 struct TcCfg {
   static_assert(TPS == 1 || (TPS == 2 && MT == 1), "paired score products with one M tile");
@@ -152,7 +164,7 @@ __device__ __noinline__ int sequence_by_length_rank(const AttnArgs& a, int* scra
   return order[blockIdx.z];
 }
 
-template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED, int CG, bool JOINT = false>
+template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED, int CG>
 __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
     block_attn_tc_kernel(const __grid_constant__ TmaMaps maps, const AttnArgs a) {
   static_assert(REP == 1 || REP == 2 || REP == 4, "replication of 1, 2 or 4");
@@ -162,24 +174,23 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
   using Cfg = TcCfg<MT, TPS, CG>;
   using Lay = TcLayout<D, MT, TPS>;
   constexpr int kTcStages = Lay::kStages;
-  // Ring barriers. With two softmax groups on a split of its own (65..128
-  // rows) K and V slots fill and free on their own barriers, so a K slot is
-  // refilled as soon as the score product that read it has completed and the
-  // K boxes of the early tiles go out first; the kernels with one group (row
-  // copies, two M tiles) and the block-slot chunk pairs (JOINT, whose second
-  // CTA reads each tile from L2 behind its partner) keep one barrier per
-  // stage for K and V together, freed by the PV product: each scheme measured
-  // faster on its own kernels (the split scheme: long prefix +4%; the joint
-  // one: concurrency sweep +6%, 14B chunk pairs +5%).
-  static_assert(!JOINT || CG == 2, "the joint variant of the two-group kernel");
-  constexpr bool kSplitKV = CG == 2 && !JOINT;
+  // Ring barriers. With two softmax groups (65..128 rows, a split of its own
+  // or a block-slot chunk pair) K and V slots fill and free on their own
+  // barriers, so a K slot is refilled as soon as the score product that read
+  // it has completed and the K boxes of the early tiles go out first; the
+  // kernels with one group (row copies, two M tiles) keep one barrier per
+  // stage for K and V together, freed by the PV product. Each scheme
+  // measured faster on its own kernels (the split scheme: long prefix +4%,
+  // 14B chunk pairs +10% once the score products stopped waiting for the PV
+  // products; the joint one: concurrency sweep +6%).
+  constexpr bool kSplitKV = CG == 2;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* q_s = smem + Lay::kQOff;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Lay::kBarOff);
-  uint64_t* k_full = bars;                   // K (joint scheme: K and V) slot of stage st landed
+  uint64_t* k_full = bars;                   // K (one-group kernels: K and V) slot of stage st landed
   uint64_t* v_full = bars + kTcStages;       // V slot of stage st landed (split scheme)
-  uint64_t* k_empty = bars + 2 * kTcStages;  // the product that read K (joint: the PV product) of stage st completed
+  uint64_t* k_empty = bars + 2 * kTcStages;  // the product that read K (one group: the PV product) of stage st completed
   uint64_t* v_empty = bars + 3 * kTcStages;  // the PV product that read V of stage st completed (split scheme)
   uint64_t* s_full = bars + 4 * kTcStages;
   uint64_t* s_free = s_full + 2;
@@ -189,10 +200,8 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
   uint64_t* q_full = q_ready + 1;  // the Q tiles' TMA copies (one M tile)
   uint64_t* drain = q_full + 1;
   // o_fin (two softmax groups): every PV product has completed (committed
-  // once, after the last): a warp that ends its steps early (the group
-  // without the last tile) may be more than one phase behind on an o_done
-  // slot, so it never waits on one for the end of the split. With one group
-  // every softmax warp takes every step and waits on the last o_done phase.
+  // once, after the last). With one group every softmax warp waits on the
+  // last o_done phase.
   uint64_t* o_fin = drain + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_fin + 1);
 
@@ -221,7 +230,9 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
       mbar_init(&s_free[j], Cfg::kSmWarps);
     }
     for (int j = 0; j < Cfg::kPBufs; ++j) {
-      mbar_init(&p_full[j], 4 * MT);
+      // one group: the four warps of an M tile per tile; two groups: all
+      // eight softmax warps per score product (p_full[j % 2])
+      mbar_init(&p_full[j], CG == 2 ? Cfg::kSmWarps : 4 * MT);
       mbar_init(&o_done[j], 1);
     }
     mbar_init(q_ready, Cfg::kSmWarps);
@@ -264,12 +275,16 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   // TMEM columns: S of M tile mt, buffer j at (2*mt + j)*kSTok; then the O
-  // accumulators, one per M tile (CG = 1) or per softmax group (CG = 2).
+  // accumulators, one per M tile; with two softmax groups one O shared by
+  // both groups, then two P buffers of 64 columns (P of score product j in
+  // buffer j % 2, tile 2j + h at column h*32).
   constexpr int kTPS = Cfg::kTPS;
   constexpr int kSTok = Cfg::kSTok;
   constexpr int kPBufs = Cfg::kPBufs;
   auto tS = [&](int mt, int j) -> uint32_t { return tmem + static_cast<uint32_t>((2 * mt + j) * kSTok); };
   auto tO = [&](int mt) -> uint32_t { return tmem + static_cast<uint32_t>(2 * MT * kSTok + mt * D); };
+  auto tP = [&](int jb) -> uint32_t { return tmem + static_cast<uint32_t>(2 * kSTok + D + jb * kTileTok); };
+  static_assert(CG == 1 || 2 * kSTok + D + 2 * kTileTok <= static_cast<int>(Cfg::kTmemCols), "TMEM columns");
 
   const int lmax = a.max_pages * a.page_size - a.bl;
   if (L < 0 || L > lmax) {
@@ -362,11 +377,9 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
           if (kTPS == 2 && j * kTPS + 1 < ntiles) umma_commit(&k_empty[(st + 1) % kTcStages]);
         }
       };
-      // P of tile h of a product starts at S column h*32 (one warp reads the
-      // whole product's columns before writing), or with two softmax groups,
-      // which share the TMEM lanes and read their tiles independently, at
-      // h*64: inside the columns of its own tile.
-      constexpr int kPCols = CG == 2 ? kTileTok : kTileTok / 2;
+      // One softmax group: P of tile h of a product starts at S column h*32
+      // (one warp reads the whole product's columns before writing).
+      constexpr int kPCols = kTileTok / 2;
       auto issue_pv = [&](int k) {
         const int st = k % kTcStages;
         const uint32_t v_addr = smem_u32(smem + Lay::kVOff + st * Geo::kTileBytes);
@@ -374,19 +387,17 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
         for (int mt = 0; mt < MT; ++mt) {
           // A = P in TMEM (bf16 pairs, 32 columns per 64-token tile, over S
           // columns its tile's softmax has consumed); B = V (MN-major: 64-dim
-          // atoms LBO apart, 8-token row groups SBO apart). With two softmax
-          // groups tile k accumulates into O of group k % 2.
+          // atoms LBO apart, 8-token row groups SBO apart).
           const uint32_t p_tmem = tS(mt, (k / kTPS) & 1) + static_cast<uint32_t>((k % kTPS) * kPCols);
-          const uint32_t o_acc = tO(CG == 2 ? k % CG : mt);
+          const uint32_t o_acc = tO(mt);
 #pragma unroll
           for (int kt = 0; kt < kTileTok / 16; ++kt) {
             const uint64_t bd = sw128_desc(v_addr + kt * 16 * 128, Geo::kColBlockBytes, 1024);
-            umma_bf16_ts(o_acc, p_tmem + kt * 8, bd, idesc_o, (k >= CG || kt > 0) ? 1u : 0u);
+            umma_bf16_ts(o_acc, p_tmem + kt * 8, bd, idesc_o, (k > 0 || kt > 0) ? 1u : 0u);
           }
         }
         umma_commit(&o_done[k % kPBufs]);
         umma_commit(kSplitKV ? &v_empty[st] : &k_empty[st]);
-        if (CG == 2 && k == ntiles - 1) umma_commit(o_fin);
       };
       // Event-driven issue: score product j needs its K tiles and a free S
       // buffer (the softmax warps have read product j-2), and waits until
@@ -401,7 +412,67 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
       // an MMA group is issued.
       uint64_t t_start = global_timer_ns();
       uint32_t spins = 0;
-      while (ok && next_pv < ntiles) {
+      if constexpr (CG == 2) {
+        // Two softmax groups: P has TMEM columns of its own, so score product
+        // j waits only for its K tiles and for the softmax warps to have read
+        // product j - 2 from the S buffer it overwrites, and runs up to two
+        // products ahead of the softmax. The PV products of product j (both
+        // tiles into the one O) wait for P_j from all eight softmax warps and,
+        // split scheme, for the V tiles. Each tile's PV commits its stage's
+        // empty barrier, which the softmax warps also read as "PV of this
+        // tile completed".
+        auto issue_pv2 = [&](int j) {
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const int k = 2 * j + h;
+            if (k >= ntiles) break;
+            const int st = k % kTcStages;
+            const uint32_t v_addr = smem_u32(smem + Lay::kVOff + st * Geo::kTileBytes);
+            const uint32_t p_tmem = tP(j & 1) + static_cast<uint32_t>(h * (kTileTok / 2));
+#pragma unroll
+            for (int kt = 0; kt < kTileTok / 16; ++kt) {
+              const uint64_t bd = sw128_desc(v_addr + kt * 16 * 128, Geo::kColBlockBytes, 1024);
+              umma_bf16_ts(tO(0), p_tmem + kt * 8, bd, idesc_o, (k > 0 || kt > 0) ? 1u : 0u);
+            }
+            umma_commit(kSplitKV ? &v_empty[st] : &k_empty[st]);
+          }
+          if (j == nprod - 1) umma_commit(o_fin);
+        };
+        int next_p = 0;
+        while (ok && next_p < nprod) {
+          bool progressed = false;
+          const int t0 = 2 * next_s;
+          if (next_s < nprod && mbar_test(&k_full[t0 % kTcStages], (t0 / kTcStages) & 1) &&
+              (t0 + 1 >= ntiles || mbar_test(&k_full[(t0 + 1) % kTcStages], ((t0 + 1) / kTcStages) & 1)) &&
+              (next_s < 2 || mbar_test(&s_free[next_s & 1], ((next_s - 2) >> 1) & 1))) {
+            tc_fence_after();
+            issue_s(next_s++);
+            progressed = true;
+          }
+          const int p0 = 2 * next_p;
+          if (next_p < next_s && mbar_test(&p_full[next_p & 1], (next_p >> 1) & 1) &&
+              (!kSplitKV || (mbar_test(&v_full[p0 % kTcStages], (p0 / kTcStages) & 1) &&
+                             (p0 + 1 >= ntiles ||
+                              mbar_test(&v_full[(p0 + 1) % kTcStages], ((p0 + 1) / kTcStages) & 1))))) {
+            tc_fence_after();
+            issue_pv2(next_p++);
+            progressed = true;
+          }
+          if (progressed) {
+            if (spins != 0) {
+              spins = 0;
+              t_start = global_timer_ns();
+            }
+          } else {
+            __nanosleep(20);
+            if ((++spins & 255u) == 0 && global_timer_ns() - t_start > kWaitLimitNs) {
+              atomicOr(a.err, NLD_DEVERR_WAIT_TIMEOUT);
+              ok = false;
+            }
+          }
+        }
+      }
+      while (CG == 1 && ok && next_pv < ntiles) {
         bool progressed = false;
         const int t0 = next_s * kTPS;  // first tile of the next score product
         if (next_s < nprod && t0 - kTPS <= next_pv &&
@@ -452,8 +523,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
     const int quad = warp & 3;
     const int wg = (warp - kSoftmaxWarp0) >> 2;
     const int mt = CG == 1 ? wg : 0;                // M tile of this warp
-    const int cg = CG == 1 ? 0 : wg;                // softmax group: tiles k % CG == cg, O accumulator cg
-    const int oi = CG == 1 ? mt : cg;               // this warp's O accumulator
+    const int cg = CG == 1 ? 0 : wg;                // softmax group: tile 2j + cg of score product j
     const int part = CG == 1 ? quad / kRowQuads : cg;  // this thread's share of a row's state (copy or group)
     const int rq = quad % kRowQuads;                // row block
     const int cp = quad / kRowQuads;                // token slice
@@ -537,12 +607,171 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
     };
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
-    // This warp's steps start kU*CG tiles apart (CG = 2: the tiles of its group).
-    for (int k0 = cg * kU; k0 < ntiles; k0 += kU * CG) {  // k0: first tile of the step
+    if constexpr (CG == 2) {
+      // Two softmax groups over every score product j: group c takes tile
+      // 2j + c. The row max of a step is taken over both tiles of the product
+      // by each group (the other tile's columns are read for the max only),
+      // so the two groups hold the same running max and accumulate into one
+      // shared O; each keeps the sum of its own tiles. P_j goes to P buffer
+      // j % 2 once the PV products of product j - 2 (which read that buffer)
+      // have completed. The empty barrier of a tile's stage (committed after
+      // its PV product) tells the softmax warps that PV has completed; a
+      // parity wait on it is exact because every earlier phase of that
+      // barrier was waited for two steps before.
+      const int nprod = (ntiles + 1) / 2;
+      uint64_t* pv_done = kSplitKV ? v_empty : k_empty;
+      for (int j = 0; j < nprod; ++j) {
+        const int k = 2 * j + cg;        // this group's tile
+        const bool has = k < ntiles;     // warp-uniform (the last product may hold one tile)
+        const int t_own = t_begin + k * kTileTok;
+        const int t_oth = t_begin + (2 * j + 1 - cg) * kTileTok;
+        if (!warp_wait(&s_full[j & 1], (j >> 1) & 1)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        float s[kTileTok];
+        float pm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+        constexpr uint64_t kAll = ~0ull;
+        auto vis_of = [&](int col0) -> uint64_t {
+          if constexpr (MASKED) {
+            return column_mask(col0);
+          } else {
+            const int nv = lim - col0;
+            return nv >= 64 ? ~0ull : nv <= 0 ? 0ull : (1ull << nv) - 1ull;
+          }
+        };
+        if (warp_rows) {
+          const uint32_t ts = tS(0, j & 1) + lane_off;
+          if (has) tmem_ld64(ts + static_cast<uint32_t>(cg * kTileTok), s);
+          // The other tile, for the max only, 32 columns at a time.
+          const uint64_t vo = vis_of(t_oth);
+          const bool all_o = __all_sync(0xffffffffu, vo == kAll);
+#pragma unroll
+          for (int cc = 0; cc < 2; ++cc) {
+            float x[32];
+            tmem_ld32(ts + static_cast<uint32_t>((1 - cg) * kTileTok + cc * 32), x);
+            if (!all_o) {
+              const uint32_t bits = static_cast<uint32_t>(vo >> (32 * cc));
+#pragma unroll
+              for (int e = 0; e < 32; ++e) x[e] = ((bits >> e) & 1u) ? x[e] : -INFINITY;
+            }
+#pragma unroll
+            for (int e = 0; e < 32; e += 8) {
+#pragma unroll
+              for (int q = 0; q < 4; ++q) pm[q] = fmax3(pm[q], x[e + 2 * q], x[e + 2 * q + 1]);
+            }
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&s_free[j & 1]);
+
+        float alpha = 1.f;
+        bool rescale = false;
+        if (warp_rows) {
+          if (has) {
+            const uint64_t vis = vis_of(t_own);
+            if (!__all_sync(0xffffffffu, vis == kAll)) {
+#pragma unroll
+              for (int e = 0; e < kTileTok; ++e) s[e] = ((vis >> e) & 1ull) ? s[e] : -INFINITY;
+            }
+#pragma unroll
+            for (int e = 0; e < kTileTok; e += 8) {
+#pragma unroll
+              for (int q = 0; q < 4; ++q) pm[q] = fmax3(pm[q], s[e + 2 * q], s[e + 2 * q + 1]);
+            }
+          }
+          const float mx = fmax3(pm[0], pm[1], fmaxf(pm[2], pm[3])) * scl;  // base-2 units, both tiles
+          if (m_run == -INFINITY) {
+            m_run = mx;
+          } else if (mx > m_run + kRescaleLog2) {
+            alpha = ex2(m_run - mx);
+            m_run = mx;
+            l_run *= alpha;
+            rescale = true;
+          }
+        }
+        if (__any_sync(0xffffffffu, rescale)) {
+          // The shared O holds the PV products of products < j: wait for the
+          // last of them (tile 2j - 1; j >= 1 here), then this group scales
+          // its half of O's columns for this warp's rows.
+          const int kl = 2 * j - 1;
+          if (!warp_wait(&pv_done[kl % kTcStages], (kl / kTcStages) & 1)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          if (lane == 0 && cg == 0) atomicAdd(a.rescales, 1ull);
+#pragma unroll 1
+          for (int c = 0; c < D / 64; ++c) {
+            float o[32];
+            const uint32_t ta = tO(0) + lane_off + static_cast<uint32_t>(cg * (D / 2) + c * 32);
+            tmem_ld32(ta, o);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) o[e] *= alpha;
+            tmem_st32(ta, o);
+          }
+        }
+        if (warp_rows && has) {
+          if (j >= 2) {
+            const int kp = 2 * j - 3;  // last tile of product j - 2
+            if (!warp_wait(&pv_done[kp % kTcStages], (kp / kTcStages) & 1)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+          }
+          const float nmu = m_run == -INFINITY ? 0.f : -m_run;
+          const float2 sc2 = make_float2(scl, scl), nm2 = make_float2(nmu, nmu);
+          float2 ls[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+          const uint32_t tp = tP(j & 1) + lane_off + static_cast<uint32_t>(cg * (kTileTok / 2));
+#pragma unroll
+          for (int c = 0; c < kTileTok / 16; ++c) {
+            uint32_t w[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              const float2 x = fma2(make_float2(s[c * 16 + 2 * e], s[c * 16 + 2 * e + 1]), sc2, nm2);
+              const float2 pp = make_float2(ex2(x.x), ex2(x.y));
+              ls[e & 1] = add2(ls[e & 1], pp);
+              w[e] = pack_bf16(pp.x, pp.y);
+            }
+            tmem_st_u32<8>(tp + static_cast<uint32_t>(c * 8), w);
+          }
+          l_run += (ls[0].x + ls[0].y) + (ls[1].x + ls[1].y);
+          tmem_wait_st();
+        }
+        if (has) {
+          const int valid = t_end - t_own;
+          if (valid < kTileTok && (valid & (kGroupTok - 1))) {
+            // V rows past the sequence end inside its last page: zero them
+            // (P is 0 there, but 0 * NaN = NaN).
+            const int st = k % kTcStages;
+            if (!warp_wait(kSplitKV ? &v_full[st] : &k_full[st], (k / kTcStages) & 1)) {
+              ok = false;
+              break;
+            }
+            const int r0 = valid, r1 = (valid + kGroupTok - 1) & ~(kGroupTok - 1);
+            uint8_t* vt = smem + Lay::kVOff + st * Geo::kTileBytes;
+            for (int idx = grp_tid; idx < (r1 - r0) * (D / 8); idx += 128) {
+              const int row = r0 + idx / (D / 8), c = idx % (D / 8);
+              *reinterpret_cast<uint4*>(vt + kv_swz(row, c)) = make_uint4(0, 0, 0, 0);
+            }
+          }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&p_full[j & 1]);
+      }
+    }
+    // One softmax group: a step is one tile, or the whole product with row
+    // copies and paired products.
+    for (int k0 = 0; CG == 1 && k0 < ntiles; k0 += kU) {  // k0: first tile of the step
       const int j = k0 / kTPS, half = k0 % kTPS;  // score product and the step's first 64-token half
       const int step_t0 = t_begin + k0 * kTileTok;
       const int k_own = k0 + h_own;               // the tile holding this thread's columns
-      if ((CG == 2 || half == 0) && !warp_wait(&s_full[j & 1], (j >> 1) & 1)) {
+      if (half == 0 && !warp_wait(&s_full[j & 1], (j >> 1) & 1)) {
         ok = false;
         break;
       }
@@ -561,7 +790,7 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
       tc_fence_before();
       __syncwarp();
       const int k_last = min(k0 + kU - 1, ntiles - 1);  // last tile of the step
-      if (lane == 0 && (CG == 2 || k_last % kTPS == kTPS - 1 || k_last == ntiles - 1)) mbar_arrive(&s_free[j & 1]);
+      if (lane == 0 && (k_last % kTPS == kTPS - 1 || k_last == ntiles - 1)) mbar_arrive(&s_free[j & 1]);
 
       float alpha = 1.f;
       bool rescale = false;
@@ -600,8 +829,8 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
       }
       if (__any_sync(0xffffffffu, rescale)) {
         // This warp's O holds the PV of its earlier tiles, the last of them
-        // k0 - CG: wait for it, then scale this warp's rows.
-        if (!warp_wait(&o_done[(k0 - CG) % kPBufs], ((k0 - CG) / kPBufs) & 1)) {
+        // k0 - 1: wait for it, then scale this warp's rows.
+        if (!warp_wait(&o_done[(k0 - 1) % kPBufs], ((k0 - 1) / kPBufs) & 1)) {
           ok = false;
           break;
         }
@@ -610,21 +839,19 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
 #pragma unroll 1
         for (int c = 0; c < D / 32; ++c) {
           float o[32];
-          tmem_ld32(tO(oi) + lane_off + c * 32, o);
+          tmem_ld32(tO(mt) + lane_off + c * 32, o);
 #pragma unroll
           for (int e = 0; e < 32; ++e) o[e] *= alpha;
-          tmem_st32(tO(oi) + lane_off + c * 32, o);
+          tmem_st32(tO(mt) + lane_off + c * 32, o);
         }
       }
       if (warp_rows) {
         // P goes to TMEM over the consumed S columns: tile k of the product
-        // takes columns (k % TPS) * 32 .. +31 of its S buffer, bf16 pairs
-        // (with two softmax groups (k % TPS) * 64 .. +31: its own tile's
-        // columns, which the other group never reads). This thread writes
-        // its slice of the tile k_own and zeros over the rest of the step's
-        // tiles (other copies' slices).
+        // takes columns (k % TPS) * 32 .. +31 of its S buffer, bf16 pairs.
+        // This thread writes its slice of the tile k_own and zeros over the
+        // rest of the step's tiles (other copies' slices).
         const uint32_t tbuf = tS(mt, j & 1) + lane_off;
-        constexpr int kPColsS = CG == 2 ? kTileTok : kTileTok / 2;
+        constexpr int kPColsS = kTileTok / 2;
         if (k_own < ntiles) {
           // p = 2^(s * scale * log2(e) - m): per pair of elements one paired
           // FMA, two exponentials, one bf16 pack and one paired add.
@@ -809,18 +1036,11 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
     auto final_chunk = [&](int cc, float* o) {
       const int col0 = part * kRange + cc * kChunk;
       if constexpr (CG > 1) {
-        // Both groups' O over these columns; a group without keys for this
-        // row (weight 0) may hold stale TMEM, so it is selected away.
-        float o2[kChunk];
+        // The one O both groups accumulated (same running max), over the
+        // sum of both groups' sums.
         ld_chunk(tO(0) + lane_off + col0, o);
-        ld_chunk(tO(1) + lane_off + col0, o2);
 #pragma unroll
-        for (int j = 0; j < kChunk; ++j)
-          o[j] = (wgt[0] == 0.f ? 0.f : wgt[0] * o[j]) + (wgt[1] == 0.f ? 0.f : wgt[1] * o2[j]);
-        if (!(l_row > 0.f)) {
-#pragma unroll
-          for (int j = 0; j < kChunk; ++j) o[j] = 0.f;
-        }
+        for (int j = 0; j < kChunk; ++j) o[j] = l_row > 0.f ? o[j] * inv : 0.f;
         return;
       }
       ld_chunk(tO(mt) + lane_off + col0, o);
@@ -1036,12 +1256,12 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
   }
 }
 
-template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED, int CG, bool JOINT = false>
+template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED, int CG>
 cudaError_t configure_tc(int dev) {
   static int configured[64] = {0};
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   if (!__atomic_load_n(&configured[dev], __ATOMIC_ACQUIRE)) {
-    cudaError_t e = cudaFuncSetAttribute(block_attn_tc_kernel<D, MT, REP, TPS, MASKED, ORDERED, CG, JOINT>,
+    cudaError_t e = cudaFuncSetAttribute(block_attn_tc_kernel<D, MT, REP, TPS, MASKED, ORDERED, CG>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(TcLayout<D, MT, TPS>::kBytes + 1024));
     if (e != cudaSuccess) return e;
@@ -1050,26 +1270,26 @@ cudaError_t configure_tc(int dev) {
   return cudaSuccess;
 }
 
-template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED, int CG, bool JOINT = false>
+template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED, int CG>
 cudaError_t launch_tc_o(const AttnArgs& a, const TmaMaps& maps, cudaStream_t stream) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  if ((e = configure_tc<D, MT, REP, TPS, MASKED, ORDERED, CG, JOINT>(dev)) != cudaSuccess) return e;
+  if ((e = configure_tc<D, MT, REP, TPS, MASKED, ORDERED, CG>(dev)) != cudaSuccess) return e;
   dim3 grid(a.num_splits * a.nh, a.Hkv, a.B);
-  return launch_kernel_cluster(block_attn_tc_kernel<D, MT, REP, TPS, MASKED, ORDERED, CG, JOINT>, grid,
+  return launch_kernel_cluster(block_attn_tc_kernel<D, MT, REP, TPS, MASKED, ORDERED, CG>, grid,
                                dim3(TcCfg<MT, TPS, CG>::kThreads), TcLayout<D, MT, TPS>::kBytes + 1024, stream,
                                a.csize, maps, a);
 }
 
 // The longest-first order only for the unmasked passes (the table-mask
 // passes run at the block shapes of one sequence).
-template <int D, int MT, int REP, int TPS, bool MASKED, int CG = 1, bool JOINT = false>
+template <int D, int MT, int REP, int TPS, bool MASKED, int CG = 1>
 cudaError_t launch_tc_t(const AttnArgs& a, const TmaMaps& maps, cudaStream_t stream) {
   if constexpr (!MASKED) {
-    if (a.order_by_length) return launch_tc_o<D, MT, REP, TPS, false, true, CG, JOINT>(a, maps, stream);
+    if (a.order_by_length) return launch_tc_o<D, MT, REP, TPS, false, true, CG>(a, maps, stream);
   }
-  return launch_tc_o<D, MT, REP, TPS, MASKED, false, CG, JOINT>(a, maps, stream);
+  return launch_tc_o<D, MT, REP, TPS, MASKED, false, CG>(a, maps, stream);
 }
 
 // Resident clusters of the kernel a plan would launch (one CTA per SM
@@ -1129,10 +1349,7 @@ cudaError_t launch_tc_rep(const AttnArgs& a, const TmaMaps& maps, cudaStream_t s
   switch (tc_replication(a.R)) {
     case 4: return launch_tc_t<D, 1, 4, TPS, MASKED>(a, maps, stream);
     case 2: return launch_tc_t<D, 1, 2, TPS, MASKED>(a, maps, stream);
-    default:
-      // block-slot chunk pairs take the joint-barrier variant
-      if (a.nh > 1) return launch_tc_t<D, 1, 1, 2, MASKED, 2, true>(a, maps, stream);
-      return launch_tc_t<D, 1, 1, 2, MASKED, 2>(a, maps, stream);
+    default: return launch_tc_t<D, 1, 1, 2, MASKED, 2>(a, maps, stream);
   }
 }
 
