@@ -614,10 +614,12 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
       // so the two groups hold the same running max and accumulate into one
       // shared O; each keeps the sum of its own tiles. P_j goes to P buffer
       // j % 2 once the PV products of product j - 2 (which read that buffer)
-      // have completed. The empty barrier of a tile's stage (committed after
-      // its PV product) tells the softmax warps that PV has completed; a
-      // parity wait on it is exact because every earlier phase of that
-      // barrier was waited for two steps before.
+      // have completed; every warp waits for that before it hands product j
+      // over, so no warp is ever two products ahead on p_full. The empty
+      // barrier of a tile's stage (committed after its PV product) tells the
+      // softmax warps that PV has completed; a parity wait on it is exact
+      // because every earlier phase of that barrier was waited for two steps
+      // before.
       const int nprod = (ntiles + 1) / 2;
       uint64_t* pv_done = kSplitKV ? v_empty : k_empty;
       for (int j = 0; j < nprod; ++j) {
@@ -713,15 +715,20 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
             tmem_st32(ta, o);
           }
         }
-        if (warp_rows && has) {
-          if (j >= 2) {
-            const int kp = 2 * j - 3;  // last tile of product j - 2
-            if (!warp_wait(&pv_done[kp % kTcStages], (kp / kTcStages) & 1)) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
+        if (j >= 2) {
+          // P buffer j % 2 is free once the PV products of product j - 2
+          // (last tile 2j - 3) have completed. Every warp waits, with rows
+          // or not: a warp that skipped it could run ahead and arrive on
+          // p_full[j % 2] for product j + 2 before the others had arrived
+          // for product j, releasing PV_j early.
+          const int kp = 2 * j - 3;
+          if (!warp_wait(&pv_done[kp % kTcStages], (kp / kTcStages) & 1)) {
+            ok = false;
+            break;
           }
+          tc_fence_after();
+        }
+        if (warp_rows && has) {
           const float nmu = m_run == -INFINITY ? 0.f : -m_run;
           const float2 sc2 = make_float2(scl, scl), nm2 = make_float2(nmu, nmu);
           float2 ls[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};

@@ -564,6 +564,39 @@ def test_attention_multiwave_longest_first(orc, mode, D):
         compare_attn(o2, l2, ro, rl, f"multiwave D={D} mode={mode} flags={flags}")
 
 
+# Two softmax groups with a lane quadrant of padding rows (80 rows per
+# block-slot chunk, 96 rows) over splits longer than the ring: the warps of
+# the empty quadrant do no exponentials, so they are the first to hand each
+# score product over. A hand-off that let one of them run two products ahead
+# released a PV product before the other warps had written their P (the
+# output went wrong while the log-sum-exp stayed right). That interleaving
+# showed only under a slower softmax step (an experimental build), never with
+# the kernel as it was, so this test cannot prove its absence; it runs the
+# shapes that expose it repeatedly, after the other plans have run, both
+# passes, and the kernel now keeps every warp within one product of the
+# others by construction.
+HANDOFF = [
+    ("d128_g8_bl20_p128", 2, 16, 2, 128, 128, 20, [129, 1000]),
+    ("d128_g3_bl32_96rows", 1, 6, 2, 128, 16, 32, [900]),
+    ("d64_g5_bl32_160rows", 1, 10, 2, 64, 16, 32, [1500]),
+]
+
+
+@pytest.mark.parametrize("spec", HANDOFF, ids=[s[0] for s in HANDOFF])
+def test_two_group_handoff_repeated(orc, spec):
+    name, B, Hq, Hkv, D, P, bl, prefix = spec
+    case = W.make_block_attn_case(name, B, Hq, Hkv, D, block_len=bl, page_size=P, prefix_lens=prefix,
+                                  seed=sum(prefix) + bl + 5)
+    dc = DeviceCase(case)
+    ref = {mode: oracle_full(orc, case, mode) for mode in (DIFF, VER)}
+    for rep in range(6):
+        for splits in (0, 1, 3):
+            for mode in (DIFF, VER):
+                out, lse = dc.run(mode, num_splits=splits)
+                ro, rl = ref[mode]
+                compare_attn(out, lse, ro, rl, f"{name} mode={mode} S={splits} rep={rep}")
+
+
 @pytest.mark.parametrize("spec", SMALL, ids=[s[0] for s in SMALL])
 def test_prefix_ready_flag_same_result(orc, spec):
     """NLD_ATTN_PREFIX_READY only moves prefix loads before the dependency
