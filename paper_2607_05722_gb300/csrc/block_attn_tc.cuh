@@ -38,8 +38,8 @@
 //             the copies are merged once, each finalising 1/REP of the columns.
 //             With 65..128 rows (CG = 2) two groups of four softmax warps
 //             share the TMEM lanes: group c takes tile 2j + c of score
-//             product j. Both take the row max over both tiles (the other
-//             tile's columns read for the max only), so they hold the same
+//             product j. Both take the row max over both tiles (the groups'
+//             tile maxima exchanged through shared memory), so they hold the same
 //             running max and accumulate into one O; P has two TMEM buffers
 //             of its own, so a score product waits only for the softmax to
 //             have read the S buffer it overwrites, never for a PV product.
@@ -75,7 +75,8 @@ constexpr int kSoftmaxWarp0 = 4;
 // CG softmax groups per M tile: with CG = 2 (one M tile of up to 128 rows
 // without row copies, paired products) two groups of four warps share the
 // TMEM lanes; group c takes tile 2j + c of each product j. Both groups take
-// each row's max over both tiles, so they keep the same running max and
+// each row's max over both tiles (tile maxima exchanged through shared
+// memory every step), so they keep the same running max and
 // accumulate into one O (each keeps the sum of its own tiles, added once
 // before the epilogue). TMEM: two S buffers, the one O, two P buffers of 64
 // columns. Per product the tensor core runs 8 score MMAs of N = 128 and 8
@@ -119,7 +120,7 @@ struct TcLayout {
   static constexpr int kQBytes = Geo::kColBlocks * 128 * 128;  // one 128-row Q tile, bf16
   // stages: what is left of 227 KB after Q, 512 bytes of barriers and the
   // 1024-byte alignment slack, a multiple of TPS, at most 8 (P lives in TMEM)
-  static constexpr int kFitStages = (232448 - 1024 - 512 - MT * kQBytes) / Geo::kStageBytes;
+  static constexpr int kFitStages = (232448 - 1024 - 512 - 1536 - MT * kQBytes) / Geo::kStageBytes;
   static constexpr int kStages = (kFitStages < 8 ? kFitStages : 8) / TPS * TPS;
   static_assert(kStages >= 2 * TPS, "at least two score products in the ring");
   static constexpr int kVOff = kStages * Geo::kTileBytes;       // V tiles after the K tiles
@@ -127,10 +128,15 @@ struct TcLayout {
   static constexpr int kPOff = kQOff + MT * kQBytes;  // end of the ring and Q tiles
   static constexpr int kBarOff = kPOff;
   // k_full[st], v_full[st], k_empty[st], v_empty[st], s_full[2], s_free[2], p_full[kPBufs], o_done[kPBufs],
-  // q_ready, q_full, drain, o_fin, tmem slot
-  static constexpr int kNumBars = 4 * kStages + 4 + 2 * kPBufs + 4;
-  static constexpr int kBytes = kBarOff + kNumBars * 8 + 16;
+  // q_ready, q_full, drain, o_fin, xm_full[2], tmem slot
+  static constexpr int kNumBars = 4 * kStages + 4 + 2 * kPBufs + 4 + 2;
   static_assert(kNumBars * 8 + 16 <= 512, "barrier reserve");
+  // two softmax groups: each row's score max per group, truncated to 24 bits
+  // (high 16 bits [2][group][TMEM lane], then the next 8 bits, same order),
+  // exchanged every step (two buffers by step parity)
+  static constexpr int kXmOff = kBarOff + 512;
+  static constexpr int kXmLoOff = kXmOff + 2 * 2 * 128 * 2;
+  static constexpr int kBytes = kXmLoOff + 2 * 2 * 128;
   static_assert(kBytes + 1024 <= 232448, "shared memory per CTA");
   static constexpr int kMergeRows = 128 * MT;
   static constexpr int kLseOff = kMergeRows * merge_pitch<D>();
@@ -203,7 +209,10 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
   // once, after the last). With one group every softmax warp waits on the
   // last o_done phase.
   uint64_t* o_fin = drain + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_fin + 1);
+  // xm_full[b] (two softmax groups): every softmax warp has written its rows'
+  // score maxima of the step with parity b
+  uint64_t* xm_full = o_fin + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(xm_full + 2);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -238,7 +247,11 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
     mbar_init(q_ready, Cfg::kSmWarps);
     mbar_init(q_full, 1);
     mbar_init(drain, 1);
-    if (CG == 2) mbar_init(o_fin, 1);
+    if (CG == 2) {
+      mbar_init(o_fin, 1);
+      mbar_init(&xm_full[0], Cfg::kSmWarps);
+      mbar_init(&xm_full[1], Cfg::kSmWarps);
+    }
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
@@ -610,9 +623,9 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
     if constexpr (CG == 2) {
       // Two softmax groups over every score product j: group c takes tile
       // 2j + c. The row max of a step is taken over both tiles of the product
-      // by each group (the other tile's columns are read for the max only),
-      // so the two groups hold the same running max and accumulate into one
-      // shared O; each keeps the sum of its own tiles. P_j goes to P buffer
+      // (each group's tile max, exchanged through shared memory), so the two
+      // groups hold the same running max and accumulate into one shared O;
+      // each keeps the sum of its own tiles. P_j goes to P buffer
       // j % 2 once the PV products of product j - 2 (which read that buffer)
       // have completed; every warp waits for that before it hands product j
       // over, so no warp is ever two products ahead on p_full. The empty
@@ -626,14 +639,12 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
         const int k = 2 * j + cg;        // this group's tile
         const bool has = k < ntiles;     // warp-uniform (the last product may hold one tile)
         const int t_own = t_begin + k * kTileTok;
-        const int t_oth = t_begin + (2 * j + 1 - cg) * kTileTok;
         if (!warp_wait(&s_full[j & 1], (j >> 1) & 1)) {
           ok = false;
           break;
         }
         tc_fence_after();
         float s[kTileTok];
-        float pm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
         constexpr uint64_t kAll = ~0ull;
         auto vis_of = [&](int col0) -> uint64_t {
           if constexpr (MASKED) {
@@ -643,34 +654,21 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
             return nv >= 64 ? ~0ull : nv <= 0 ? 0ull : (1ull << nv) - 1ull;
           }
         };
-        if (warp_rows) {
-          const uint32_t ts = tS(0, j & 1) + lane_off;
-          if (has) tmem_ld64(ts + static_cast<uint32_t>(cg * kTileTok), s);
-          // The other tile, for the max only, 32 columns at a time.
-          const uint64_t vo = vis_of(t_oth);
-          const bool all_o = __all_sync(0xffffffffu, vo == kAll);
-#pragma unroll
-          for (int cc = 0; cc < 2; ++cc) {
-            float x[32];
-            tmem_ld32(ts + static_cast<uint32_t>((1 - cg) * kTileTok + cc * 32), x);
-            if (!all_o) {
-              const uint32_t bits = static_cast<uint32_t>(vo >> (32 * cc));
-#pragma unroll
-              for (int e = 0; e < 32; ++e) x[e] = ((bits >> e) & 1u) ? x[e] : -INFINITY;
-            }
-#pragma unroll
-            for (int e = 0; e < 32; e += 8) {
-#pragma unroll
-              for (int q = 0; q < 4; ++q) pm[q] = fmax3(pm[q], x[e + 2 * q], x[e + 2 * q + 1]);
-            }
-          }
-        }
+        if (warp_rows && has) tmem_ld64(tS(0, j & 1) + lane_off + static_cast<uint32_t>(cg * kTileTok), s);
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&s_free[j & 1]);
 
-        float alpha = 1.f;
-        bool rescale = false;
+        // The row max of the product: this group's tile max, truncated to 24
+        // bits (toward zero: relative error below 2^-15), exchanged with the
+        // other group through shared memory; both groups take the max of the
+        // two truncated values, so they agree exactly. The max only offsets
+        // the exponent: the largest P is 2^d with d below 2^-15 of the
+        // scaled max, which rounds to exactly 1 in bf16 while the scaled max
+        // is below ~90, as with the untruncated max.
+        uint16_t* xm = reinterpret_cast<uint16_t*>(smem + Lay::kXmOff) + (j & 1) * 256;  // [group][TMEM lane]
+        uint8_t* xm_lo = smem + Lay::kXmLoOff + (j & 1) * 256;
+        float own = -INFINITY;
         if (warp_rows) {
           if (has) {
             const uint64_t vis = vis_of(t_own);
@@ -678,13 +676,31 @@ __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
 #pragma unroll
               for (int e = 0; e < kTileTok; ++e) s[e] = ((vis >> e) & 1ull) ? s[e] : -INFINITY;
             }
+            float pm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
             for (int e = 0; e < kTileTok; e += 8) {
 #pragma unroll
               for (int q = 0; q < 4; ++q) pm[q] = fmax3(pm[q], s[e + 2 * q], s[e + 2 * q + 1]);
             }
+            own = fmax3(pm[0], pm[1], fmaxf(pm[2], pm[3]));
           }
-          const float mx = fmax3(pm[0], pm[1], fmaxf(pm[2], pm[3])) * scl;  // base-2 units, both tiles
+          const uint32_t own_t = __float_as_uint(own) & 0xFFFFFF00u;
+          own = __uint_as_float(own_t);
+          xm[cg * 128 + r_loc] = static_cast<uint16_t>(own_t >> 16);
+          xm_lo[cg * 128 + r_loc] = static_cast<uint8_t>(own_t >> 8);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&xm_full[j & 1]);
+        if (!warp_wait(&xm_full[j & 1], (j >> 1) & 1)) {
+          ok = false;
+          break;
+        }
+        float alpha = 1.f;
+        bool rescale = false;
+        if (warp_rows) {
+          const float oth = __uint_as_float((static_cast<uint32_t>(xm[(1 - cg) * 128 + r_loc]) << 16) |
+                                            (static_cast<uint32_t>(xm_lo[(1 - cg) * 128 + r_loc]) << 8));
+          const float mx = fmaxf(own, oth) * scl;  // base-2 units, both tiles
           if (m_run == -INFINITY) {
             m_run = mx;
           } else if (mx > m_run + kRescaleLog2) {
