@@ -31,18 +31,19 @@
 //             in the freed K/V ring in 128-byte-swizzled boxes, which one
 //             thread writes with tiled TMA stores (the bf16 output or bf16
 //             split partials, in packed row order).
-//             With at most 64 (32) packed rows, Q is replicated into the idle
-//             lane quadrants (REP = 2 or 4): each copy of a row takes a 64/REP-
-//             token slice of every tile with its own running max and sum, so
-//             every softmax warp works and each does 1/REP of the exponentials;
-//             the copies are merged once, each finalising 1/REP of the columns.
-//             With 65..128 rows (CG = 2) two groups of four softmax warps
-//             share the TMEM lanes: group c takes tile 2j + c of score
-//             product j. Both take the row max over both tiles (the groups'
-//             tile maxima exchanged through shared memory), so they hold the same
-//             running max and accumulate into one O; P has two TMEM buffers
-//             of its own, so a score product waits only for the softmax to
-//             have read the S buffer it overwrites, never for a PV product.
+//             With 33..64 packed rows, Q is replicated into the idle lane
+//             quadrants (REP = 2): each copy of a row takes a 32-token slice
+//             of every tile with its own running max and sum, so every
+//             softmax warp works and each does half of the exponentials; the
+//             copies are merged once, each finalising half of the columns.
+//             With up to 32 or 65..128 rows (CG = 2) two groups of four
+//             softmax warps share the TMEM lanes: group c takes tile 2j + c
+//             of score product j. Both take the row max over both tiles (the
+//             groups' tile maxima exchanged through shared memory), so they
+//             hold the same running max and accumulate into one O; P has two
+//             TMEM buffers of its own, so a score product waits only for the
+//             softmax to have read the S buffer it overwrites, never for a
+//             PV product.
 // When the KV range of a (sequence, KV head) is split over a thread-block
 // cluster, the CTAs stage their normalised rows in shared memory and merge
 // them through distributed shared memory (a cluster barrier, then each CTA
@@ -173,7 +174,7 @@ __device__ __noinline__ int sequence_by_length_rank(const AttnArgs& a, int* scra
 template <int D, int MT, int REP, int TPS, bool MASKED, bool ORDERED, int CG>
 __global__ void __launch_bounds__(TcCfg<MT, TPS, CG>::kThreads, 1)
     block_attn_tc_kernel(const __grid_constant__ TmaMaps maps, const AttnArgs a) {
-  static_assert(REP == 1 || REP == 2 || REP == 4, "replication of 1, 2 or 4");
+  static_assert(REP == 1 || REP == 2, "replication of 1 or 2 (up to 32 rows run on two softmax groups)");
   static_assert(MT == 1 || REP == 1, "replication only with one M tile");
   static_assert(CG == 1 || REP == 1, "softmax groups without row copies");
   using Geo = TileGeom<D>;
@@ -1351,26 +1352,30 @@ int max_active_clusters_t(int csize) {
 
 // Copies of each Q row in the 128 TMEM lanes of one M tile: 4 for up to 32
 // packed rows, 2 for up to 64, else 1 (and 1 with two M tiles).
-int tc_replication(int rows) { return rows <= 32 ? 4 : rows <= 64 ? 2 : 1; }
+// Row copies of the one-group kernel: 33..64 rows take two copies; up to
+// 32 rows and 65..128 rows run on the two-group kernel (1).
+int tc_replication(int rows) { return rows > 32 && rows <= 64 ? 2 : 1; }
 
 template <int D>
 int max_active_clusters_d(int csize, int rows) {
   if (rows > 128) return max_active_clusters_t<D, 2, 1, 1, 1>(csize);
   switch (tc_replication(rows)) {
-    case 4: return max_active_clusters_t<D, 1, 4, 1, 1>(csize);
     case 2: return max_active_clusters_t<D, 1, 2, 1, 1>(csize);
     default: return max_active_clusters_t<D, 1, 1, 2, 2>(csize);
   }
 }
 
-// One M tile: rows copied 4 or 2 times (up to 64 rows), with paired score
-// products when a split fits in the ring whole (it is then latency-bound:
-// fewer, wider steps help) and single tiles when it streams; 65..128 rows
-// take paired products and two softmax groups, streaming or not.
+// One M tile: 33..64 rows copied twice, with paired score products when a
+// split fits in the ring whole (it is then latency-bound: fewer, wider steps
+// help; the 8B shape's 64 rows measured 7.12 us per launch against 7.32 on
+// the two-group kernel) and single tiles when it streams; up to 32 and
+// 65..128 rows take paired products and two softmax groups, streaming or
+// not (32-row batches measured 50/75/87 -> 55/86/95% of peak at B = 8, 32,
+// 128 against four row copies: the score products run ahead of the PV
+// products there, and each tile takes 8 MMAs instead of 12).
 template <int D, int TPS, bool MASKED>
 cudaError_t launch_tc_rep(const AttnArgs& a, const TmaMaps& maps, cudaStream_t stream) {
   switch (tc_replication(a.R)) {
-    case 4: return launch_tc_t<D, 1, 4, TPS, MASKED>(a, maps, stream);
     case 2: return launch_tc_t<D, 1, 2, TPS, MASKED>(a, maps, stream);
     default: return launch_tc_t<D, 1, 1, 2, MASKED, 2>(a, maps, stream);
   }

@@ -56,10 +56,11 @@ def _lib():
     assert nld.nld_device_error(clear=True) == 0, "a kernel flagged a device error"
 
 
-# name, B, Hq, Hkv, D, P, bl, prefix lengths; packed rows G*bl set the row
-# copies (<= 32 rows: 4 copies, <= 64: 2, <= 128: 1) or two M tiles (> 128)
+# name, B, Hq, Hkv, D, P, bl, prefix lengths; packed rows G*bl set the
+# kernel: two softmax groups (<= 32 and 65..128 rows), two row copies
+# (33..64) or two M tiles (> 128)
 SHAPES = [
-    ("rows32_rep4_d64", 1, 4, 1, 64, 16, 8, [700]),
+    ("rows32_cg2_d64", 1, 4, 1, 64, 16, 8, [700]),
     ("rows64_rep2_d128", 1, 32, 8, 128, 16, 16, [1500]),
     ("rows96_rep1_d128", 2, 6, 2, 128, 16, 32, [900, 400]),
     ("rows160_mt2_d128", 1, 10, 2, 128, 16, 32, [1200]),
